@@ -1,0 +1,96 @@
+"""Brute-force K-VEC selection in NumPy, for tiny inputs only.
+
+An implementation independent of the C oracle, written from the K-VEC paper:
+it materialises the full causal attention tensor A[h, q, t] for *every* query
+position of a short sequence (Algorithm 1's input), slices the last O / O'
+query rows as Eq. 1 states, and resolves every top-k with a full sort.  It is
+used only to pin the oracle.
+"""
+from __future__ import annotations
+
+import math
+from typing import Dict
+
+import numpy as np
+
+
+def causal_attention(q_full: np.ndarray, k: np.ndarray, scale: float) -> np.ndarray:
+    """q_full [T][Hq][d], k [T][Hkv][d] (float64) -> A [Hq][T][T] with A[h, i, j] = 0 for j > i."""
+    T, Hq, _ = q_full.shape
+    Hkv = k.shape[1]
+    g = Hq // Hkv
+    A = np.zeros((Hq, T, T))
+    mask = np.triu(np.ones((T, T), bool), 1)
+    for hq in range(Hq):
+        s = scale * (q_full[:, hq, :] @ k[:, hq // g, :].T)
+        s[mask] = -np.inf
+        s = s - s.max(axis=1, keepdims=True)
+        e = np.exp(s)
+        A[hq] = e / e.sum(axis=1, keepdims=True)
+    return A
+
+
+def _ranked(score: np.ndarray, positions: np.ndarray) -> np.ndarray:
+    """positions sorted by descending score, ascending position on ties."""
+    order = np.lexsort((positions, -score[positions]))
+    return positions[order]
+
+
+def select(q_full, k, *, num_kv_heads, window, obs_window, ext_window, pool_kernel,
+           num_ext_heads, lam, beta, budget, n_counts, layers_done, scale=None) -> Dict[str, np.ndarray]:
+    """Algorithm 1 followed by per-head top-B for one sequence of length T = q_full.shape[0]."""
+    T, Hq, d = q_full.shape
+    Hkv = num_kv_heads
+    g = Hq // Hkv
+    w, O, Oe = window, obs_window, ext_window
+    scale = 1.0 / math.sqrt(d) if scale is None else scale
+    A = causal_attention(q_full, k, scale)
+    Akv = A.reshape(Hkv, g, T, T).sum(axis=1)               # KV-head attention (GQA group sum)
+
+    # Eq. 1 over the last O (and O') query rows; I: mean over the last O rows of the head-max.
+    P_O_raw = Akv[:, T - O:, :].mean(axis=1)
+    P_Oe_raw = Akv[:, T - Oe:, :].mean(axis=1)
+    I_raw = Akv[:, T - O:, :].max(axis=0).mean(axis=0)
+
+    Lc = T - w
+    r = pool_kernel // 2
+
+    def pool(x):
+        return np.array([x[max(0, t - r):min(Lc, t + r + 1)].max() for t in range(Lc)])
+
+    PO = np.stack([pool(P_O_raw[h]) for h in range(Hkv)]) if Lc > 0 else np.zeros((Hkv, 0))
+    POe = np.stack([pool(P_Oe_raw[h]) for h in range(Hkv)]) if Lc > 0 else np.zeros((Hkv, 0))
+    I = pool(I_raw) if Lc > 0 else np.zeros(0)
+
+    sigma = PO.std(axis=1, ddof=1) if Lc >= 2 else np.zeros(Hkv)
+    head_order = np.lexsort((np.arange(Hkv), sigma))
+    htop = np.zeros(Hkv, bool)
+    htop[head_order[:num_ext_heads]] = True
+    P = np.where(htop[:, None], POe, PO)
+
+    coverage = n_counts[:Lc].astype(np.float64) / (layers_done + 1)
+    Pprime = P + lam * (I * (1.0 - coverage))[None, :]
+    Kp = min(int(math.floor(beta * budget)), budget - w)
+    cand = np.arange(Lc)
+    keep = np.zeros((Hkv, T), bool)
+    pres = np.zeros((Hkv, max(Lc, 0)), bool)
+    if T <= budget:
+        keep[:] = True
+    else:
+        for h in range(Hkv):
+            top = _ranked(P[h], cand)[:Kp]
+            pres[h, top] = True
+            rest = cand[~pres[h]]
+            fill = _ranked(Pprime[h], rest)[:budget - w - Kp]
+            keep[h, top] = True
+            keep[h, fill] = True
+            keep[h, Lc:] = True
+    out_idx = np.full((Hkv, budget), -1, np.int64)
+    for h in range(Hkv):
+        sel = np.flatnonzero(keep[h])
+        out_idx[h, :sel.size] = sel
+    union = keep.any(axis=0)
+    n_new = n_counts[:T].astype(np.int64) + union
+    return dict(A=A, P_O_raw=P_O_raw, P_Oext_raw=P_Oe_raw, I_raw=I_raw, P_O=PO, P_Oext=POe, I=I,
+                sigma=sigma, htop=htop, P=P, Pprime=Pprime, pres=pres, out_idx=out_idx,
+                union=union, n=n_new)

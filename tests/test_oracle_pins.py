@@ -1,0 +1,311 @@
+"""Pins of the fp64 CPU oracle against things other than itself.
+
+* an independent NumPy brute force (full T x T causal attention, full sorts);
+* closed forms (all-zero keys give a uniform causal softmax);
+* invariants that the K-VEC paper's definitions fix (Eq. 1 mass, Section 4.2
+  coverage counting, budget bookkeeping);
+* special cases that reduce K-VEC to plain window-score top-B (SnapKV).
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from bruteforce import select as bf_select
+from paper_2606_29563_gb300 import synth
+
+
+def _f64(x: torch.Tensor) -> np.ndarray:
+    return x.to(torch.float64).numpy()
+
+
+def _run_oracle(params, q_obs, k, v, state, budget, cu=None, ml=None):
+    if cu is None:
+        cu = [0, k.shape[0]]
+    return oracle.select_layer(params, cu, q_obs, k, v, state, budget, max_seqlen=ml)
+
+
+TINY_CASES = [
+    # (seed, T, Hq, Hkv, d, w, O, O', pool, delta, lam, beta, B)
+    (1, 14, 2, 1, 8, 4, 2, 4, 3, 1, 1.0, 0.25, 8),
+    (2, 16, 4, 2, 8, 6, 3, 5, 3, 1, 1.0, 0.5, 10),
+    (3, 16, 8, 4, 4, 5, 2, 5, 1, 2, 0.5, 0.34, 9),
+    (4, 12, 4, 4, 8, 3, 2, 3, 5, 3, 2.0, 0.25, 6),
+    (5, 16, 6, 3, 8, 4, 2, 4, 3, 0, 1.0, 0.25, 8),
+    (6, 15, 4, 2, 6, 6, 6, 6, 3, 2, 1.0, 1.0, 11),
+    (7, 16, 2, 2, 8, 2, 1, 2, 7, 1, 1.0, 0.0, 5),
+    (8, 10, 4, 2, 8, 4, 2, 4, 3, 1, 1.0, 0.25, 12),   # L <= B: keep everything
+]
+
+
+@pytest.mark.parametrize("case", TINY_CASES)
+def test_oracle_matches_bruteforce_over_layers(case):
+    seed, T, Hq, Hkv, d, w, O, Oe, pool, delta, lam, beta, B = case
+    params = oracle.OracleParams(num_q_heads=Hq, num_kv_heads=Hkv, head_dim=d, window=w,
+                                 obs_window=O, ext_window=Oe, pool_kernel=pool,
+                                 num_ext_heads=delta, lam=lam, beta=beta)
+    state = oracle.new_state(1, T)
+    n_bf = np.zeros(T, np.int64)
+    for layer in range(3):
+        x = synth.tiny_full_inputs(seed * 100 + layer, T, Hq, Hkv, d)
+        q_obs = x["q_full"][T - w:].reshape(1, w, Hq, d)
+        r = _run_oracle(params, q_obs, x["k"], x["v"], state, B)
+        bf = bf_select(_f64(x["q_full"]), _f64(x["k"]), num_kv_heads=Hkv, window=w, obs_window=O,
+                       ext_window=Oe, pool_kernel=pool, num_ext_heads=delta, lam=lam, beta=beta,
+                       budget=B, n_counts=n_bf, layers_done=layer)
+        Lc = T - w
+        np.testing.assert_allclose(r["P_O_raw"][0, :, :T], bf["P_O_raw"], rtol=1e-12, atol=1e-15)
+        np.testing.assert_allclose(r["P_Oext_raw"][0, :, :T], bf["P_Oext_raw"], rtol=1e-12, atol=1e-15)
+        np.testing.assert_allclose(r["I_raw"][0, :T], bf["I_raw"], rtol=1e-12, atol=1e-15)
+        np.testing.assert_allclose(r["P_O"][0, :, :Lc], bf["P_O"], rtol=1e-12, atol=1e-15)
+        np.testing.assert_allclose(r["P_Oext"][0, :, :Lc], bf["P_Oext"], rtol=1e-12, atol=1e-15)
+        np.testing.assert_allclose(r["I"][0, :Lc], bf["I"], rtol=1e-12, atol=1e-15)
+        np.testing.assert_allclose(r["sigma"][0], bf["sigma"], rtol=1e-9, atol=1e-15)
+        assert (r["htop"][0].astype(bool) == bf["htop"]).all()
+        np.testing.assert_allclose(r["P"][0, :, :Lc], bf["P"], rtol=1e-12, atol=1e-15)
+        np.testing.assert_allclose(r["Pprime"][0, :, :Lc], bf["Pprime"], rtol=1e-12, atol=1e-15)
+        if T > B:
+            assert (r["pres"][0, :, :Lc].astype(bool) == bf["pres"]).all()
+        assert (r["out_idx"][0] == bf["out_idx"]).all()
+        n_bf = bf["n"]
+        f = oracle.state_fields(state, T)
+        assert (f["n"][0].astype(np.int64) == n_bf).all()
+        assert f["layers_done"][0] == layer + 1
+
+
+def test_softmax_rows_sum_to_one_and_eq1_mass():
+    wl = synth.small_workload(seqlens=(257,), num_q_heads=8, num_kv_heads=2)
+    x = synth.make_layer(wl, 0)
+    p = oracle.OracleParams.from_workload(wl)
+    r = oracle.select_layer(p, wl.cu_seqlens, x["q_obs"], x["k"], x["v"], oracle.new_state(1, 257), wl.budget)
+    np.testing.assert_allclose(r["row_sums"], 1.0, atol=1e-12)
+    # Eq. 1 averages O rows that each sum to 1, summed over the g heads of a group: mass g.
+    g = wl.group
+    np.testing.assert_allclose(r["P_O_raw"][0].sum(axis=1), g, rtol=1e-12)
+    np.testing.assert_allclose(r["P_Oext_raw"][0].sum(axis=1), g, rtol=1e-12)
+    # I averages a max over KV heads: between the mean (mass g) and the sum over heads (mass Hq).
+    mass_I = r["I_raw"][0].sum()
+    assert g - 1e-12 <= mass_I <= wl.num_q_heads + 1e-12
+
+
+def test_uniform_keys_closed_form_two_layers():
+    """K = 0: every visible key gets 1/(p+1); all candidates tie, so lower positions win.
+
+    Layer 0 keeps [0, B-w) plus the window.  At layer 1 those tokens have
+    coverage 1/2, so the fill (not the preserved part) moves to [B-w, ...).
+    """
+    T, Hq, Hkv, d, w, O, Oe, B = 64, 4, 2, 8, 8, 4, 8, 24
+    params = oracle.OracleParams(num_q_heads=Hq, num_kv_heads=Hkv, head_dim=d, window=w,
+                                 obs_window=O, ext_window=Oe, pool_kernel=3, num_ext_heads=1,
+                                 lam=1.0, beta=0.25)
+    g = Hq // Hkv
+    x = synth.tiny_full_inputs(3, T, Hq, Hkv, d)
+    q_obs = x["q_full"][T - w:].reshape(1, w, Hq, d)
+    k = torch.zeros(T, Hkv, d, dtype=torch.bfloat16)
+    v = x["v"]
+    state = oracle.new_state(1, T)
+    r = _run_oracle(params, q_obs, k, v, state, B)
+    Lc = T - w
+    expect_PO = g / O * sum(1.0 / (T - w + q + 1) for q in range(w - O, w))
+    expect_POe = g / Oe * sum(1.0 / (T - w + q + 1) for q in range(w - Oe, w))
+    expect_I = 1.0 / O * sum(g / (T - w + q + 1) for q in range(w - O, w))
+    np.testing.assert_allclose(r["P_O"][0, :, :Lc], expect_PO, rtol=1e-13)
+    np.testing.assert_allclose(r["P_Oext"][0, :, :Lc], expect_POe, rtol=1e-13)
+    np.testing.assert_allclose(r["I"][0, :Lc], expect_I, rtol=1e-13)
+    # Window rows: key t in the window is visible only to rows q with L-w+q >= t.
+    t = T - 1
+    np.testing.assert_allclose(r["P_O_raw"][0, 0, t], g / O * (1.0 / T), rtol=1e-13)
+    assert np.all(r["sigma"][0] < 1e-15) and r["sigma"][0, 0] == r["sigma"][0, 1]
+    assert list(r["htop"][0]) == [1, 0]          # equal sigma: the lower head index wins
+    Kp = int(math.floor(0.25 * B))
+    layer0 = list(range(B - w)) + list(range(T - w, T))
+    assert (r["out_idx"][0] == np.array(layer0)).all()
+    r1 = _run_oracle(params, q_obs, k, v, state, B)
+    layer1 = list(range(Kp)) + list(range(B - w, B - w + (B - w - Kp))) + list(range(T - w, T))
+    assert (r1["out_idx"][0] == np.array(sorted(layer1))).all()
+    f = oracle.state_fields(state, T)
+    expect_n = np.zeros(T, np.int64)
+    for sel in (layer0, layer1):
+        expect_n[sel] += 1
+    assert (f["n"][0] == expect_n).all()
+    assert r1["coverage"][0] == np.count_nonzero(expect_n)
+
+
+def test_lowest_sigma_head_gets_extended_window():
+    """A head whose keys are all zero attends uniformly: its sigma is the smallest (Section 4.1)."""
+    T, Hq, Hkv, d, w, B = 96, 4, 4, 16, 16, 40
+    x = synth.tiny_full_inputs(11, T, Hq, Hkv, d, key_scale=2.0)
+    k = x["k"].clone()
+    k[:, 2, :] = 0
+    params = oracle.OracleParams(num_q_heads=Hq, num_kv_heads=Hkv, head_dim=d, window=w, obs_window=8,
+                                 ext_window=16, pool_kernel=3, num_ext_heads=1, lam=0.0, beta=0.25)
+    q_obs = x["q_full"][T - w:].reshape(1, w, Hq, d)
+    r = _run_oracle(params, q_obs, k, x["v"], oracle.new_state(1, T), B)
+    assert int(np.argmin(r["sigma"][0])) == 2
+    assert list(r["htop"][0]) == [0, 0, 1, 0]
+    Lc = T - w
+    np.testing.assert_array_equal(r["P"][0, 2, :Lc], r["P_Oext"][0, 2, :Lc])
+    np.testing.assert_array_equal(r["P"][0, 0, :Lc], r["P_O"][0, 0, :Lc])
+
+
+def _top_positions(score_row, k):
+    order = np.lexsort((np.arange(score_row.size), -score_row))
+    return np.sort(order[:k])
+
+
+def _wl_layers(wl, layers):
+    return synth.make_layers(wl, layers)
+
+
+def test_no_coverage_reduces_to_window_score_topB():
+    """delta = 0 and lambda = 0: K-VEC is plain top-(B-w) of pooled P_O plus the window."""
+    wl = synth.small_workload(seqlens=(400,), num_ext_heads=0, lam=0.0, budget=72)
+    p = oracle.OracleParams.from_workload(wl)
+    st = oracle.new_state(1, 400)
+    Lc = 400 - wl.window
+    for layer, x in enumerate(_wl_layers(wl, 2)):
+        r = oracle.select_layer(p, wl.cu_seqlens, x["q_obs"], x["k"], x["v"], st, wl.budget)
+        for h in range(wl.num_kv_heads):
+            expect = np.concatenate([_top_positions(r["P_O"][0, h, :Lc], wl.budget - wl.window),
+                                     np.arange(Lc, 400)])
+            assert (r["out_idx"][0, h] == expect).all()
+
+
+def test_equal_windows_disable_cross_head():
+    wl = synth.small_workload(seqlens=(350,), ext_window=16, obs_window=16)
+    a = oracle.OracleParams.from_workload(wl)
+    b = oracle.OracleParams.from_workload(wl, num_ext_heads=0)
+    x = synth.make_layer(wl, 0)
+    ra = oracle.select_layer(a, wl.cu_seqlens, x["q_obs"], x["k"], x["v"], oracle.new_state(1, 350), wl.budget)
+    rb = oracle.select_layer(b, wl.cu_seqlens, x["q_obs"], x["k"], x["v"], oracle.new_state(1, 350), wl.budget)
+    assert (ra["out_idx"] == rb["out_idx"]).all()
+
+
+def test_lambda_zero_makes_preservation_a_no_op():
+    wl = synth.small_workload(seqlens=(330,), lam=0.0)
+    x = synth.make_layer(wl, 0)
+    outs = []
+    for beta in (0.0, 0.25, 1.0):
+        p = oracle.OracleParams.from_workload(wl, beta=beta)
+        outs.append(oracle.select_layer(p, wl.cu_seqlens, x["q_obs"], x["k"], x["v"],
+                                        oracle.new_state(1, 330), wl.budget)["out_idx"])
+    assert (outs[0] == outs[1]).all() and (outs[1] == outs[2]).all()
+
+
+def test_full_preservation_ignores_coverage():
+    """beta = 1 preserves B - w tokens by P alone: the state has no effect."""
+    wl = synth.small_workload(seqlens=(330,), beta=1.0)
+    x = synth.make_layer(wl, 0)
+    p = oracle.OracleParams.from_workload(wl)
+    st = oracle.new_state(1, 330)
+    st[0, 16:16 + 330] = 3                       # pretend every token was kept 3 times
+    st[0, 0] = 5                                 # ... over 5 layers
+    r1 = oracle.select_layer(p, wl.cu_seqlens, x["q_obs"], x["k"], x["v"], st, wl.budget)
+    r0 = oracle.select_layer(oracle.OracleParams.from_workload(wl, lam=0.0), wl.cu_seqlens, x["q_obs"],
+                             x["k"], x["v"], oracle.new_state(1, 330), wl.budget)
+    assert (r1["out_idx"] == r0["out_idx"]).all()
+
+
+def test_layer0_focus_is_global_importance():
+    wl = synth.small_workload(seqlens=(310,), lam=0.5)
+    x = synth.make_layer(wl, 0)
+    r = oracle.select_layer(oracle.OracleParams.from_workload(wl), wl.cu_seqlens, x["q_obs"], x["k"],
+                            x["v"], oracle.new_state(1, 310), wl.budget)
+    Lc = 310 - wl.window
+    np.testing.assert_allclose(r["Pprime"][0, :, :Lc] - r["P"][0, :, :Lc],
+                               np.broadcast_to(0.5 * r["I"][0, :Lc], (wl.num_kv_heads, Lc)),
+                               rtol=1e-10, atol=1e-18)
+
+
+def test_pool_width_one_is_identity():
+    wl = synth.small_workload(seqlens=(300,), pool_kernel=1)
+    x = synth.make_layer(wl, 0)
+    r = oracle.select_layer(oracle.OracleParams.from_workload(wl), wl.cu_seqlens, x["q_obs"], x["k"],
+                            x["v"], oracle.new_state(1, 300), wl.budget)
+    Lc = 300 - wl.window
+    np.testing.assert_array_equal(r["P_O"][0, :, :Lc], r["P_O_raw"][0, :, :Lc])
+    np.testing.assert_array_equal(r["I"][0, :Lc], r["I_raw"][0, :Lc])
+
+
+def test_multilayer_state_and_budget_invariants():
+    wl = synth.small_workload(seqlens=(300, 180, 420), budget=64, layers=4)
+    p = oracle.OracleParams.from_workload(wl)
+    st = oracle.new_state(wl.batch, wl.max_seqlen)
+    n_expect = np.zeros((wl.batch, wl.max_seqlen), np.int64)
+    cu = wl.cu_seqlens
+    for layer, x in enumerate(_wl_layers(wl, 4)):
+        r = oracle.select_layer(p, cu, x["q_obs"], x["k"], x["v"], st, wl.budget, max_seqlen=wl.max_seqlen)
+        k_np = x["k"].view(torch.int16).numpy().view(np.uint16)
+        v_np = x["v"].view(torch.int16).numpy().view(np.uint16)
+        f = oracle.state_fields(st, wl.max_seqlen)
+        for b, L in enumerate(wl.seqlens):
+            union = np.zeros(wl.max_seqlen, bool)
+            for h in range(wl.num_kv_heads):
+                idx = r["out_idx"][b, h]
+                sel = idx[idx >= 0]
+                assert sel.size == min(L, wl.budget)
+                assert np.all(np.diff(sel) > 0)
+                assert set(range(L - wl.window, L)) <= set(sel.tolist())
+                pres = np.flatnonzero(r["pres"][b, h])
+                assert set(pres.tolist()) <= set(sel.tolist())
+                assert pres.size == min(int(math.floor(wl.beta * wl.budget)), wl.budget - wl.window)
+                np.testing.assert_array_equal(r["out_k"][b, h, :sel.size], k_np[cu[b] + sel, h])
+                np.testing.assert_array_equal(r["out_v"][b, h, :sel.size], v_np[cu[b] + sel, h])
+                assert np.all(r["out_k"][b, h, sel.size:] == 0)
+                union[sel] = True
+            n_expect[b] += union
+            bits = np.unpackbits(f["last_union"][b].view(np.uint8), bitorder="little")[:wl.max_seqlen]
+            assert (bits.astype(bool) == union).all()
+            assert r["coverage"][b] == np.count_nonzero(n_expect[b])
+        assert (f["n"].astype(np.int64) == n_expect).all()
+        assert (f["layers_done"] == layer + 1).all()
+        assert (f["seqlen"] == np.array(wl.seqlens)).all()
+        assert np.all(f["n"] <= layer + 1)
+
+
+def test_keep_all_when_sequence_fits_budget():
+    wl = synth.small_workload(seqlens=(50,), budget=64)
+    x = synth.make_layer(wl, 0)
+    st = oracle.new_state(1, 50)
+    r = oracle.select_layer(oracle.OracleParams.from_workload(wl), wl.cu_seqlens, x["q_obs"], x["k"],
+                            x["v"], st, wl.budget)
+    for h in range(wl.num_kv_heads):
+        assert (r["out_idx"][0, h, :50] == np.arange(50)).all()
+        assert (r["out_idx"][0, h, 50:] == -1).all()
+    assert (oracle.state_fields(st, 50)["n"][0] == 1).all()
+
+
+def test_cross_layer_coverage_grows_when_layers_repeat():
+    """Section 4.2: with the same scores in every layer, SnapKV keeps the same tokens (coverage flat)
+    while the (1 - coverage) focus term pushes K-VEC to new tokens (coverage grows)."""
+    wl = synth.small_workload(seqlens=(1200,), num_q_heads=8, num_kv_heads=4, budget=96,
+                              salient=30, p_share=0.8, num_ext_heads=2, lam=1.0)
+    x = synth.make_layer(wl, 0)
+    cov = {}
+    for name, over in (("kvec", {}), ("snapkv", dict(num_ext_heads=0, lam=0.0))):
+        p = oracle.OracleParams.from_workload(wl, **over)
+        st = oracle.new_state(1, 1200)
+        cov[name] = []
+        for _ in range(4):
+            r = oracle.select_layer(p, wl.cu_seqlens, x["q_obs"], x["k"], x["v"], st, wl.budget)
+            cov[name].append(int(r["coverage"][0]))
+    assert cov["snapkv"] == [cov["snapkv"][0]] * 4
+    assert cov["kvec"][3] > cov["kvec"][0]
+    assert cov["kvec"][3] > cov["snapkv"][3]
+
+
+@pytest.mark.parametrize("bad", [
+    dict(num_kv_heads=3), dict(obs_window=40), dict(pool_kernel=4), dict(num_ext_heads=5),
+    dict(beta=1.5), dict(window=0),
+])
+def test_oracle_rejects_bad_parameters(bad):
+    kw = dict(num_q_heads=8, num_kv_heads=4, head_dim=8, window=8, obs_window=4, ext_window=8,
+              pool_kernel=3, num_ext_heads=1, lam=1.0, beta=0.25)
+    kw.update(bad)
+    p = oracle.OracleParams(**kw)
+    x = synth.tiny_full_inputs(0, 32, 8, 4, 8)
+    with pytest.raises(ValueError):
+        oracle.select_layer(p, [0, 32], x["q_full"][24:].reshape(1, 8, 8, 8), x["k"], x["v"],
+                            oracle.new_state(1, 32), 16)

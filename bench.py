@@ -1,0 +1,409 @@
+"""Benchmark of the K-VEC eviction-selection hot path on GB300.
+
+One step = one end-of-prefill eviction pass over every layer of a synthetic
+prompt batch: reset the coverage state, then kvec_select_layers over all layers
+(window scores, softmax, window sums, pooling, cross-head and cross-layer
+coverage, per-KV-head top-B, K/V gather).  The metric is prefix tokens evicted
+per second: sum over layers, sequences and KV heads of (L_s - B).
+
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                       [--workload NAME] [--budget B]
+Under torchrun every rank runs its own batch (weak scaling, no collective on the
+data path); rank 0 prints one JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "prefix tokens evicted/sec (all layers, device-timed) and % of HBM roofline"
+DEFAULT_WORKLOAD = "llama8b_l8192_b512"
+FALLBACK_HBM_GBS = 6800.0
+KERNEL_SOURCES = {"score": "paper_2606_29563_gb300/csrc/score_kernel.cu"}
+
+
+# ----------------------------------------------------------------------------- distributed plumbing
+
+def dist_env():
+    return (int(os.environ.get("RANK", "0")), int(os.environ.get("WORLD_SIZE", "1")),
+            int(os.environ.get("LOCAL_RANK", "0")))
+
+
+def init_dist(backend: str):
+    import torch.distributed as dist
+    rank, world, _ = dist_env()
+    if world > 1 and not dist.is_initialized():
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        os.environ.setdefault("MASTER_PORT", "29511")
+        dist.init_process_group(backend=backend, rank=rank, world_size=world)
+    return rank, world
+
+
+def barrier():
+    import torch.distributed as dist
+    if dist.is_initialized():
+        dist.barrier()
+
+
+def max_over_ranks(x: float, device=None) -> float:
+    """Largest value of x across ranks (x itself on a single process)."""
+    import torch
+    import torch.distributed as dist
+    if not dist.is_initialized():
+        return float(x)
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ----------------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """Samples nvidia-smi SM clocks and throttle reasons in the background."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int, interval_ms: int = 50):
+        self.samples = []
+        self.proc = None
+        self.cmd = ["nvidia-smi", "-i", str(gpu_index), f"--query-gpu={self.FIELDS}",
+                    "--format=csv,noheader,nounits", f"--loop-ms={interval_ms}"]
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(self.cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, ValueError):
+            self.proc = None
+            return self
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.samples.append((time.perf_counter(), line.strip()))
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.thread.join(timeout=5)
+
+    def summary(self, t0: float, t1: float):
+        rows = [s for t, s in self.samples if t0 <= t <= t1]
+        window = "timed region"
+        if not rows:
+            rows = [s for _, s in self.samples]
+            window = "whole run (no sample fell inside the timed region)"
+        mhz, mx, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for r in rows:
+            parts = [p.strip() for p in r.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                mhz.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[4:8]):
+                if val.lower() == "active":
+                    reasons.add(name)
+        if not mhz:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0, "window": "unavailable"}
+        return {"sm_mhz": statistics.median(mhz), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(mhz), "window": window}
+
+
+# ----------------------------------------------------------------------------- helpers
+
+def measured_hbm_gbs():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            v = float(json.load(f)["hbm_gbs"])
+        return v, "measured"
+    except (OSError, ValueError, KeyError):
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def committed_traffic(kernel: str, workload: str):
+    """dram read+write bytes per launch from a committed ncu summary, if the kernel is unchanged."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            data = json.load(f)
+        entry = data[kernel][workload]
+        src = open(os.path.join(ROOT, KERNEL_SOURCES[kernel]), "rb").read()
+        if entry.get("source_sha256") != hashlib.sha256(src).hexdigest():
+            return None
+        return float(entry["bytes_per_launch"])
+    except (OSError, ValueError, KeyError, TypeError):
+        return None
+
+
+def workload_bytes(wl):
+    """Algorithmic HBM bytes of one layer: K read once, q_obs read, gathered K/V read, cache and indices written."""
+    d = wl.head_dim
+    k_read = wl.total_tokens * wl.num_kv_heads * d * 2
+    q_read = wl.batch * wl.window * wl.num_q_heads * d * 2
+    kept = sum(min(L, wl.budget) for L in wl.seqlens) * wl.num_kv_heads
+    gather_rw = 2 * 2 * kept * d * 2              # K and V rows, read + written
+    idx = wl.batch * wl.num_kv_heads * wl.budget * 4
+    return {"k_read": k_read, "q_read": q_read, "gather": gather_rw, "idx": idx,
+            "layer_total": k_read + q_read + gather_rw + idx, "score_launch": k_read + q_read}
+
+
+def oracle_baseline(wl, budget_s: float = 15.0, max_layers: int = 8):
+    """Times the fp64 CPU oracle on a bounded sample (leading layers) of the workload."""
+    import numpy as np
+    import oracle
+    from paper_2606_29563_gb300 import synth
+    p = oracle.OracleParams.from_workload(wl)
+    st = oracle.new_state(wl.batch, wl.max_seqlen)
+    structure = [synth.salient_structure(wl, b, max_layers) for b in range(wl.batch)]
+    spent, layers, evicted = 0.0, 0, 0
+    for l in range(min(max_layers, wl.layers)):
+        x = synth.make_layer(wl, l, "cpu", structure)
+        t0 = time.perf_counter()
+        oracle.select_layer(p, wl.cu_seqlens, x["q_obs"], x["k"], x["v"], st, wl.budget,
+                            max_seqlen=wl.max_seqlen, debug=False)
+        spent += time.perf_counter() - t0
+        layers += 1
+        evicted += wl.evicted_per_layer()
+        if spent >= budget_s:
+            break
+    return {"value": evicted / spent, "unit": "tokens/s", "cores": oracle.num_threads(), "kind": "oracle",
+            "sample": f"first {layers} of {wl.layers} layers of {wl.name} (fp64 C oracle, OpenMP), "
+                      f"{spent:.1f} s of CPU work"}
+
+
+# ----------------------------------------------------------------------------- our arm
+
+def run_ours(args, wl):
+    import torch
+    from paper_2606_29563_gb300 import build as kbuild
+    from paper_2606_29563_gb300 import kvec, synth
+
+    rank, world = init_dist("nccl" if args.gpus > 1 else "gloo")
+    _, _, local = dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    kbuild.build()
+    kvec.load()
+
+    L_layers = wl.layers
+    params = kvec.params_from_workload(wl)
+    sel = kvec.KvecSelector(params)
+    cu_host = torch.tensor(wl.cu_seqlens, dtype=torch.int32).pin_memory()
+    cu_dev = cu_host.to(dev)
+    structure = [synth.salient_structure(wl, b, L_layers) for b in range(wl.batch)]
+    # Each rank draws its own batch (seed offset by rank): weak scaling.
+    wl_rank = wl.replace(seed=wl.seed + 1000 * rank)
+    layers = [synth.make_layer(wl_rank, l, dev, structure) for l in range(L_layers)]
+    qs, ks, vs = [x["q_obs"] for x in layers], [x["k"] for x in layers], [x["v"] for x in layers]
+    outs = [sel.alloc_outputs(wl.batch, wl.budget, dev) for _ in range(L_layers)]
+    state = sel.new_state(wl.batch, dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        kvec.kvec_reset(sel.handle, state.data_ptr(), wl.batch, stream.cuda_stream)
+        sel.select_layers(cu_host, cu_dev, qs, ks, vs, state, wl.budget, outs, stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    kvec.kvec_sync_status(sel.handle)
+
+    clocks = ClockSampler(local).start()
+    time.sleep(0.3)
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier()
+    torch.cuda.synchronize()
+    t_host0 = time.perf_counter()
+    start.record(stream)
+    for _ in range(args.steps):
+        step()
+    stop.record(stream)
+    torch.cuda.synchronize()
+    t_host1 = time.perf_counter()
+    barrier()
+    elapsed_ms = max_over_ranks(start.elapsed_time(stop), dev)
+    time.sleep(0.1)
+    clocks.stop()
+    kvec.kvec_sync_status(sel.handle)
+
+    evicted_per_step = wl.evicted_per_layer() * L_layers
+    value = world * evicted_per_step * args.steps / (elapsed_ms / 1e3)
+    ms_per_step = elapsed_ms / args.steps
+
+    # Per-kernel device time (CUDA events recorded by the library on the launching stream).
+    kvec.kvec_set_profiling(sel.handle, True)
+    for _ in range(args.steps):
+        step()
+    torch.cuda.synchronize()
+    ktimes = {}
+    for i, name in enumerate(kvec.KERNEL_NAMES):
+        ms, n = kvec.kvec_kernel_time(sel.handle, i)
+        ktimes[name] = {"ms_per_launch": ms / n if n else None, "launches": n,
+                        "share": None}
+    total_k = sum(v["ms_per_launch"] * v["launches"] for v in ktimes.values() if v["ms_per_launch"])
+    for v in ktimes.values():
+        if v["ms_per_launch"]:
+            v["share"] = v["ms_per_launch"] * v["launches"] / total_k
+    kvec.kvec_set_profiling(sel.handle, False)
+    peak, peak_kind = measured_hbm_gbs()
+    by = workload_bytes(wl)
+    score_ms = ktimes["score"]["ms_per_launch"]
+    achieved = by["score_launch"] / (score_ms / 1e3) / 1e9
+    traffic = committed_traffic("score", wl.name)
+    path_gbs = by["layer_total"] * L_layers / (ms_per_step / 1e3) / 1e9
+
+    # End to end through the public API: pinned host inputs copied in, indices and state copied out.
+    e2e = run_e2e(args, wl, sel, layers, outs, state, cu_host, cu_dev, dev, stream) if args.e2e else None
+
+    gpu_launches = args.steps * L_layers * len(kvec.KERNEL_NAMES)   # six kernels per layer
+    sel.close()
+    result = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": wl.name, "layers": L_layers, "batch": wl.batch, "seqlens": list(wl.seqlens)[:8],
+                   "q_heads": wl.num_q_heads, "kv_heads": wl.num_kv_heads, "head_dim": wl.head_dim,
+                   "window": wl.window, "budget": wl.budget, "parallelism": f"replicas{world}",
+                   "l2": f"inputs larger than L2 ({(by['k_read'] * 2 + by['q_read']) * L_layers / 1e9:.2f} GB per step)",
+                   "precision": "bf16 inputs, fp32 accumulation and scores"},
+        "roofline": {"bound": "hbm", "kernel": "score", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": traffic, "peak_source": peak_kind,
+                     "bytes_per_launch": by["score_launch"]},
+        "path_roofline": {"achieved": path_gbs, "peak": peak, "unit": "GB/s", "frac": path_gbs / peak,
+                          "bytes_per_step": by["layer_total"] * L_layers},
+        "kernels": ktimes,
+        "clocks": {k: v for k, v in clocks.summary(t_host0, t_host1).items()},
+        "gpu_launches": gpu_launches,
+        "e2e": e2e,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        result["cpu_baseline"] = oracle_baseline(wl)
+    return rank, result
+
+
+def run_e2e(args, wl, sel, layers, outs, state, cu_host, cu_dev, dev, stream):
+    import torch
+    from paper_2606_29563_gb300 import kvec
+    host = [{k: v.cpu().pin_memory() for k, v in x.items()} for x in layers]
+    dev_in = [{k: torch.empty_like(v) for k, v in x.items()} for x in layers]
+    host_idx = [torch.empty(o[0].shape, dtype=o[0].dtype).pin_memory() for o in outs]
+    host_state = torch.empty(state.shape, dtype=state.dtype).pin_memory()
+    h2d = sum(t.numel() * t.element_size() for x in host for t in x.values())
+    d2h = sum(t.numel() * t.element_size() for t in host_idx) + host_state.numel()
+
+    def step():
+        for src, dst in zip(host, dev_in):
+            for k in src:
+                dst[k].copy_(src[k], non_blocking=True)
+        kvec.kvec_reset(sel.handle, state.data_ptr(), wl.batch, stream.cuda_stream)
+        sel.select_layers(cu_host, cu_dev, [x["q_obs"] for x in dev_in], [x["k"] for x in dev_in],
+                          [x["v"] for x in dev_in], state, wl.budget, outs, stream)
+        for o, h in zip(outs, host_idx):
+            h.copy_(o[0], non_blocking=True)
+        host_state.copy_(state, non_blocking=True)
+
+    for _ in range(max(1, args.warmup)):
+        step()
+    torch.cuda.synchronize()
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier()
+    start.record(stream)
+    n = max(1, args.steps)
+    for _ in range(n):
+        step()
+    stop.record(stream)
+    torch.cuda.synchronize()
+    ms = max_over_ranks(start.elapsed_time(stop), dev)
+    _, world, _ = dist_env()
+    value = world * wl.evicted_per_layer() * wl.layers * n / (ms / 1e3)
+    return {"value": value, "unit": "tokens/s", "ms_per_step": ms / n, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h}
+
+
+# ----------------------------------------------------------------------------- reference arm (the oracle)
+
+def run_reference(args, wl):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return rank, None
+    import oracle
+    from paper_2606_29563_gb300 import synth
+    oracle.build()
+    p = oracle.OracleParams.from_workload(wl)
+    structure = [synth.salient_structure(wl, b, 1) for b in range(wl.batch)]
+    x = synth.make_layer(wl, 0, "cpu", structure)
+    # A bounded sample per step: the first layer of the workload, from a fresh state.
+    def step():
+        st = oracle.new_state(wl.batch, wl.max_seqlen)
+        oracle.select_layer(p, wl.cu_seqlens, x["q_obs"], x["k"], x["v"], st, wl.budget,
+                            max_seqlen=wl.max_seqlen, debug=False)
+
+    for _ in range(args.warmup):
+        step()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    dt = time.perf_counter() - t0
+    value = wl.evicted_per_layer() * args.steps / dt
+    sample = f"layer 0 of {wl.name} per step (fp64 C oracle, OpenMP, {oracle.num_threads()} threads)"
+    return rank, {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3 / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": wl.name, "layers_per_step": 1, "batch": wl.batch, "budget": wl.budget},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": oracle.num_threads(), "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--budget", type=int, default=None)
+    ap.add_argument("--layers", type=int, default=None, help="run only the first N layers (not a bench line)")
+    ap.add_argument("--no-e2e", dest="e2e", action="store_false")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    if args.warmup < 3 and args.impl == "ours":
+        args.warmup = 3
+    from paper_2606_29563_gb300 import synth
+    wl = synth.WORKLOADS[args.workload]
+    if args.budget:
+        wl = wl.replace(budget=args.budget, name=f"{wl.name.rsplit('_b', 1)[0]}_b{args.budget}")
+    if args.layers:
+        wl = wl.replace(layers=args.layers)
+    rank, result = (run_reference if args.impl == "reference" else run_ours)(args, wl)
+    if rank == 0 and result is not None:
+        print(json.dumps(result), flush=True)
+
+
+if __name__ == "__main__":
+    main()

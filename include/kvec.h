@@ -1,0 +1,169 @@
+/*
+ * kvec.h -- C ABI of the GB300 (sm_103a) K-VEC eviction-selection library.
+ *
+ * K-VEC ("KV cache Eviction with Coverage") decides, at the end of prefill and
+ * layer by layer, which B tokens each KV head keeps in its cache:
+ *   - window scores: Eq. 1, the mean attention of the last O queries (O' for
+ *     the cross-head heads), summed over the query heads of a GQA group;
+ *   - cross-head coverage (Section 4.1): the delta KV heads whose scores have
+ *     the lowest standard deviation use the extended window O';
+ *   - cross-layer coverage (Section 4.2): P' = P + lambda * I * (1 - n_t/(l+1)),
+ *     with I the head-max importance and n_t the number of earlier layers that
+ *     kept token t; the top floor(beta*B) tokens by P are preserved;
+ *   - per-KV-head top-B (Section 4.1, "each head selects the top-B tokens"),
+ *     then the gather of the selected K/V rows into the budget-sized cache.
+ * Algorithm 1 of the paper lists the same steps.
+ *
+ * Conventions shared by every entry point:
+ *   - Pointers marked "device" are CUDA device memory owned by the caller
+ *     (torch tensors, cudaMalloc, ...).  The library never frees them.
+ *   - Work is asynchronous and stream ordered on the stream argument; results
+ *     are valid once that stream reaches the call.  Host-side validation runs
+ *     first and a rejected call launches nothing.
+ *   - Errors are returned as kvec_status; kvec_last_error() gives a message
+ *     for the calling thread.  No C++ exception crosses this boundary.
+ *   - A handle is used from one host thread at a time.
+ *   - bf16 tensors are raw IEEE bfloat16 (2 bytes per element).
+ */
+#ifndef KVEC_H
+#define KVEC_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define KVEC_API __attribute__((visibility("default")))
+#else
+#define KVEC_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    KVEC_OK = 0,
+    KVEC_ERR_INVALID_ARG = 1,     /* a pointer, size or parameter is out of range */
+    KVEC_ERR_UNSUPPORTED = 2,     /* valid per the paper, not supported by these kernels */
+    KVEC_ERR_CUDA = 3,            /* a CUDA runtime call failed (message has the CUDA error) */
+    KVEC_ERR_DEVICE_TIMEOUT = 4,  /* a bounded device-side wait gave up; outputs are invalid */
+    KVEC_ERR_OOM = 5              /* workspace allocation in kvec_create failed */
+} kvec_status;
+
+typedef struct kvec_handle kvec_handle;
+/* Same object as cudaStream_t; declared here so the header needs no CUDA include. */
+typedef struct CUstream_st* kvec_stream_t;
+
+/* Hyper-parameters (names follow Algorithm 1) and workspace sizing. */
+typedef struct {
+    int   num_q_heads;    /* H_q query heads */
+    int   num_kv_heads;   /* H_kv KV heads; query head hq uses KV head hq / (H_q/H_kv) */
+    int   head_dim;       /* d; these kernels support 128 */
+    int   window;         /* w: observation query rows given per sequence; the last w
+                             tokens are always kept and count toward the budget */
+    int   obs_window;     /* O of Eq. 1 (paper: "e.g., 16"), 1 <= O <= w */
+    int   ext_window;     /* O' of Section 4.1 (paper default 32), 1 <= O' <= w */
+    int   pool_kernel;    /* odd width of the 1-D max-pool over candidate scores, 1..15 */
+    int   num_ext_heads;  /* delta of Section 4.1 (paper default 3), 0..H_kv */
+    float lambda;         /* lambda of Section 4.2 (paper default 1.0), finite */
+    float beta;           /* beta of Section 4.2 (paper's best 0.25), 0..1 */
+    float softmax_scale;  /* <= 0 selects 1/sqrt(head_dim) */
+    int   max_batch;      /* largest batch a call may pass */
+    int   max_seqlen;     /* largest prefix length L a call may pass (<= 131072) */
+    int   max_layers;     /* layers one coverage state may see (<= 255; n_t is 8-bit) */
+} kvec_params;
+
+/* Creates a handle and allocates its device workspace on the current device.
+ * Returns INVALID_ARG / UNSUPPORTED for bad parameters (nothing allocated),
+ * OOM or CUDA on allocation failure.  *out is NULL on failure. */
+KVEC_API kvec_status kvec_create(const kvec_params* params, kvec_handle** out);
+
+/* Frees the workspace; waits for the handle's pending work first. */
+KVEC_API kvec_status kvec_destroy(kvec_handle* h);
+
+/* Bytes of coverage state per sequence (Section 4.2's counters n_t).  The
+ * caller allocates batch * kvec_state_bytes(max_seqlen) bytes of device memory.
+ * Layout of one sequence's state (little endian, 16-byte aligned):
+ *   u32 layers_done   layers processed so far (l in coverage = n_t/(l+1))
+ *   u32 seqlen        L of the last call
+ *   u32 reserved[2]   zero
+ *   u8  n[round_up(max_seqlen, 16)]      n_t: layers that kept token t
+ *   u32 last_union[ceil(max_seqlen/32)]  bit t set if any head kept t in the last layer
+ * padded to a multiple of 16 bytes.  Copying it is a checkpoint. */
+KVEC_API size_t kvec_state_bytes(int max_seqlen);
+
+/* Zeroes `batch` consecutive states (a new prompt starts at layer 0). */
+KVEC_API kvec_status kvec_reset(kvec_handle* h, void* coverage_state, int batch, kvec_stream_t stream);
+
+/* One layer of eviction selection for a varlen-packed batch (Algorithm 1 followed
+ * by per-KV-head top-B and the K/V gather).
+ *   cu_seqlens_host [batch+1] host, cu_seqlens_dev [batch+1] device: same values,
+ *       cu[0] = 0, L_s = cu[s+1] - cu[s] with w <= L_s <= max_seqlen.
+ *   q_obs  device bf16 [batch][w][H_q][d]: the last w query rows of every sequence
+ *          (post-RoPE, as the attention saw them).
+ *   k, v   device bf16 [cu[batch]][H_kv][d]: the layer's prefix keys and values.
+ *   coverage_state  device, batch states (kvec_state_bytes each); read and updated.
+ *   budget B: tokens kept per KV head, the w window tokens included; B >= w.
+ *   out_idx device int32 [batch][H_kv][B]: kept positions (0-based within the
+ *          sequence), ascending; -1 after the last one when L_s < B.
+ *   out_k, out_v device bf16 [batch][H_kv][B][d]: gathered rows, zero padded.
+ * When L_s <= B every token is kept.  All device pointers must be 16-byte aligned. */
+KVEC_API kvec_status kvec_select_layer(kvec_handle* h, int batch,
+                              const int32_t* cu_seqlens_host, const int32_t* cu_seqlens_dev,
+                              const void* q_obs, const void* k, const void* v,
+                              void* coverage_state, int budget,
+                              int32_t* out_idx, void* out_k, void* out_v,
+                              kvec_stream_t stream);
+
+/* num_layers consecutive layers of one prefill (same batch, lengths and state),
+ * as if kvec_select_layer were called for layer 0, 1, ... in order.  Each array
+ * holds num_layers device pointers with the per-layer meaning above.  The
+ * library overlaps the score work of later layers with the coverage-dependent
+ * selection of earlier ones; the results are identical to the layer-by-layer
+ * calls.  num_layers must not exceed max_layers. */
+KVEC_API kvec_status kvec_select_layers(kvec_handle* h, int num_layers, int batch,
+                               const int32_t* cu_seqlens_host, const int32_t* cu_seqlens_dev,
+                               const void* const* q_obs, const void* const* k, const void* const* v,
+                               void* coverage_state, int budget,
+                               int32_t* const* out_idx, void* const* out_k, void* const* out_v,
+                               kvec_stream_t stream);
+
+/* Device views of the last processed layer's intermediates (valid until the
+ * next call on the handle; read after synchronising the stream).  Strides use
+ * the handle's max_seqlen (ML).  Only candidate positions t < L_s - w hold
+ * scores. */
+typedef struct {
+    const float*    P_O;        /* [max_batch][H_kv][ML]  Eq. 1 with O, max-pooled */
+    const float*    P_Oext;     /* [max_batch][H_kv][ML]  Eq. 1 with O', max-pooled */
+    const float*    I;          /* [max_batch][ML]        Section 4.2 importance, max-pooled */
+    const float*    sigma;      /* [max_batch][H_kv]      std of pooled P_O over candidates */
+    const int32_t*  htop;       /* [max_batch][H_kv]      1 if the head uses O' */
+    const uint32_t* pres_bits;  /* [max_batch][H_kv][ceil(ML/32)] preserved top-K tokens */
+    const float*    Pprime;     /* [max_batch][H_kv][ML]  P + lambda * focus */
+    const float*    row_stats;  /* [max_batch][H_kv][g*w][2]  softmax row max (log2 units)
+                                   and denominator; row r = q*g + j is query head
+                                   h*g + j at window row q */
+    int max_seqlen;
+    int words_per_row;          /* ceil(ML/32) */
+} kvec_debug_view;
+
+KVEC_API kvec_status kvec_debug_scores(kvec_handle* h, kvec_debug_view* out);
+
+/* Synchronises the handle's streams and reports a device-side error recorded
+ * by a bounded wait (KVEC_ERR_DEVICE_TIMEOUT), then clears it. */
+KVEC_API kvec_status kvec_sync_status(kvec_handle* h);
+
+/* Per-kernel device time recorded since the last kvec_set_profiling(h, 1)
+ * call, from CUDA events on the launching stream.  kernel: 0 score (QK^T +
+ * softmax partials), 1 row-stat merge, 2 window sums + pooling, 3 cross-head
+ * + preserve, 4 coverage select, 5 gather.  Synchronises. */
+KVEC_API kvec_status kvec_set_profiling(kvec_handle* h, int enable);
+KVEC_API kvec_status kvec_kernel_time(kvec_handle* h, int kernel, double* total_ms, int* launches);
+
+KVEC_API const char* kvec_status_string(kvec_status s);
+KVEC_API const char* kvec_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

@@ -1,0 +1,73 @@
+"""Teacher-forced parity run of the CUDA path against the oracle (TEST INFRASTRUCTURE ONLY).
+
+For every layer: run the GPU layer, copy the GPU's state from *before* that layer
+into the oracle, run the oracle on the same inputs, and compare (oracle.compare).
+Errors therefore never compound across layers.
+"""
+from __future__ import annotations
+
+import math
+from typing import Dict, List, Optional
+
+import numpy as np
+import torch
+
+import oracle
+from oracle import compare
+from paper_2606_29563_gb300 import kvec, synth
+
+
+def _bits(x: torch.Tensor) -> np.ndarray:
+    return x.detach().cpu().contiguous().view(torch.int16).numpy().view(np.uint16)
+
+
+def gpu_debug_numpy(sel: kvec.KvecSelector, batch: int, max_seqlen: int) -> Dict[str, np.ndarray]:
+    d = {k: v.cpu().numpy() for k, v in sel.debug().items()}
+    words = d["pres_bits"][:batch]
+    pres = np.unpackbits(words.view(np.uint8), axis=-1, bitorder="little")[..., :max_seqlen]
+    return {"P_O": d["P_O"][:batch], "P_Oext": d["P_Oext"][:batch], "I": d["I"][:batch],
+            "sigma": d["sigma"][:batch], "htop": d["htop"][:batch], "pres": pres,
+            "Pprime": d["Pprime"][:batch], "row_stats": d["row_stats"][:batch]}
+
+
+def run_parity(wl: synth.Workload, layers: Optional[int] = None, device: str = "cuda", budget: Optional[int] = None,
+               tol: float = compare.TOL, verbose: bool = False) -> List[str]:
+    """Returns every mismatch over `layers` layers of `wl` (empty list = parity)."""
+    layers = layers or wl.layers
+    budget = budget or wl.budget
+    ML = wl.max_seqlen
+    params = kvec.params_from_workload(wl, max_layers=max(layers, 1))
+    sel = kvec.KvecSelector(params)
+    oparams = oracle.OracleParams.from_workload(wl)
+    Kp = min(int(math.floor(float(np.float32(wl.beta)) * budget)), budget - wl.window)
+    cu_host = torch.tensor(wl.cu_seqlens, dtype=torch.int32)
+    cu_dev = cu_host.to(device)
+    state = sel.new_state(wl.batch, device)
+    errs: List[str] = []
+    inputs = synth.make_layers(wl, layers, device="cpu")
+    dev_inputs = [{k: v.to(device) for k, v in x.items()} for x in inputs]
+    for l in range(layers):
+        before = state.cpu().numpy().copy()
+        out_idx, out_k, out_v = sel.select_layer(cu_host, cu_dev, dev_inputs[l]["q_obs"], dev_inputs[l]["k"],
+                                                 dev_inputs[l]["v"], state, budget)
+        torch.cuda.synchronize()
+        kvec.kvec_sync_status(sel.handle)
+        gdbg = gpu_debug_numpy(sel, wl.batch, ML)
+        after = state.cpu().numpy()
+        ostate = before.copy()
+        r = oracle.select_layer(oparams, wl.cu_seqlens, inputs[l]["q_obs"], inputs[l]["k"], inputs[l]["v"], ostate,
+                                budget, max_seqlen=ML)
+        g = dict(gdbg)
+        g["out_idx"] = out_idx.cpu().numpy()
+        layer_errs = compare.check_layer(g, r, wl.seqlens, wl.window, budget, Kp, wl.num_ext_heads, tol)
+        layer_errs += compare.check_state_and_gather(
+            g["out_idx"], _bits(out_k), _bits(out_v), _bits(inputs[l]["k"]), _bits(inputs[l]["v"]), wl.cu_seqlens,
+            oracle.state_fields(before, ML), oracle.state_fields(after, ML))
+        if np.array_equal(g["out_idx"], r["out_idx"]) and not np.array_equal(after, ostate):
+            layer_errs.append("same indices as the oracle but a different coverage state")
+        errs += [f"layer {l}: {e}" for e in layer_errs]
+        if verbose:
+            same = np.mean(g["out_idx"] == r["out_idx"])
+            print(f"layer {l}: {len(layer_errs)} mismatches, index agreement {same:.5f}")
+    sel.close()
+    return errs

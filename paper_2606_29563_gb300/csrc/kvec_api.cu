@@ -1,0 +1,450 @@
+// C ABI of the K-VEC eviction-selection library: validation, workspace, launch
+// sequence.  Declarations and the meaning of every argument are in kvec.h.
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <string>
+#include <vector>
+
+#include "../../include/kvec.h"
+#include "kvec_internal.cuh"
+
+using namespace kvec;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+kvec_status fail(kvec_status s, const char* fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    g_last_error = buf;
+    return s;
+}
+
+kvec_status cuda_fail(cudaError_t e, const char* what) {
+    return fail(KVEC_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+constexpr int kKernelKinds = 6;
+
+struct TimedLaunch {
+    int kind;
+    cudaEvent_t start, stop;
+};
+
+}  // namespace
+
+struct kvec_handle {
+    kvec_params p;
+    int device = 0;
+    int g = 1, R = 0, words = 0;
+    size_t state_stride = 0, n_off = 16, union_off = 0;
+    void* ws = nullptr;
+    size_t ws_bytes = 0;
+    Scratch sc{};
+    Slot slot{};
+    int last_batch = 0;
+    bool profiling = false;
+    std::vector<TimedLaunch> timed;
+    std::vector<cudaEvent_t> event_pool;
+};
+
+namespace {
+
+cudaEvent_t take_event(kvec_handle* h) {
+    if (!h->event_pool.empty()) {
+        cudaEvent_t e = h->event_pool.back();
+        h->event_pool.pop_back();
+        return e;
+    }
+    cudaEvent_t e = nullptr;
+    cudaEventCreate(&e);
+    return e;
+}
+
+void recycle_timed(kvec_handle* h) {
+    for (auto& t : h->timed) {
+        h->event_pool.push_back(t.start);
+        h->event_pool.push_back(t.stop);
+    }
+    h->timed.clear();
+}
+
+template <class F>
+void timed_launch(kvec_handle* h, int kind, cudaStream_t st, F&& launch) {
+    if (!h->profiling) {
+        launch();
+        return;
+    }
+    TimedLaunch t{kind, take_event(h), take_event(h)};
+    cudaEventRecord(t.start, st);
+    launch();
+    cudaEventRecord(t.stop, st);
+    h->timed.push_back(t);
+}
+
+kvec_status validate_params(const kvec_params* p) {
+    if (!p) return fail(KVEC_ERR_INVALID_ARG, "params is NULL");
+    if (p->num_kv_heads < 1 || p->num_q_heads < p->num_kv_heads || p->num_q_heads % p->num_kv_heads)
+        return fail(KVEC_ERR_INVALID_ARG, "num_q_heads (%d) must be a positive multiple of num_kv_heads (%d)",
+                    p->num_q_heads, p->num_kv_heads);
+    if (p->num_kv_heads > 32) return fail(KVEC_ERR_UNSUPPORTED, "num_kv_heads > 32 is not supported");
+    if (p->head_dim != kHeadDim) return fail(KVEC_ERR_UNSUPPORTED, "head_dim must be %d", kHeadDim);
+    if (p->window < 1) return fail(KVEC_ERR_INVALID_ARG, "window must be >= 1");
+    if (p->obs_window < 1 || p->obs_window > p->window || p->ext_window < 1 || p->ext_window > p->window)
+        return fail(KVEC_ERR_INVALID_ARG, "need 1 <= obs_window, ext_window <= window");
+    const int g = p->num_q_heads / p->num_kv_heads;
+    if ((g * p->window) % 8 != 0 || g * p->window > 256)
+        return fail(KVEC_ERR_UNSUPPORTED, "rows per KV head (group %d x window %d) must be a multiple of 8 and <= 256",
+                    g, p->window);
+    if (p->pool_kernel < 1 || p->pool_kernel > kMaxPool || p->pool_kernel % 2 == 0)
+        return fail(KVEC_ERR_INVALID_ARG, "pool_kernel must be odd and in [1, %d]", kMaxPool);
+    if (p->num_ext_heads < 0 || p->num_ext_heads > p->num_kv_heads)
+        return fail(KVEC_ERR_INVALID_ARG, "num_ext_heads must be in [0, num_kv_heads]");
+    if (!(p->beta >= 0.f && p->beta <= 1.f)) return fail(KVEC_ERR_INVALID_ARG, "beta must be in [0, 1]");
+    if (!isfinite(p->lambda)) return fail(KVEC_ERR_INVALID_ARG, "lambda must be finite");
+    if (!isfinite(p->softmax_scale)) return fail(KVEC_ERR_INVALID_ARG, "softmax_scale must be finite");
+    if (p->max_batch < 1 || p->max_seqlen < 1 || p->max_seqlen > 131072)
+        return fail(KVEC_ERR_INVALID_ARG, "need max_batch >= 1 and 1 <= max_seqlen <= 131072");
+    if (p->max_layers < 1 || p->max_layers > 255)
+        return fail(KVEC_ERR_INVALID_ARG, "max_layers must be in [1, 255]");
+    return KVEC_OK;
+}
+
+kvec_status set_device(kvec_handle* h, int* prev) {
+    cudaError_t e = cudaGetDevice(prev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if (*prev != h->device) {
+        e = cudaSetDevice(h->device);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaSetDevice");
+    }
+    return KVEC_OK;
+}
+
+struct DeviceGuard {
+    int prev, dev;
+    ~DeviceGuard() {
+        if (prev != dev) cudaSetDevice(prev);
+    }
+};
+
+kvec_status validate_call(kvec_handle* h, int batch, const int32_t* cu_host, const int32_t* cu_dev, int budget,
+                          int* total_tiles, int* total_chunks) {
+    if (!h) return fail(KVEC_ERR_INVALID_ARG, "handle is NULL");
+    if (batch < 1 || batch > h->p.max_batch)
+        return fail(KVEC_ERR_INVALID_ARG, "batch %d outside [1, max_batch=%d]", batch, h->p.max_batch);
+    if (!cu_host || !cu_dev) return fail(KVEC_ERR_INVALID_ARG, "cu_seqlens pointers must not be NULL");
+    if (cu_host[0] != 0) return fail(KVEC_ERR_INVALID_ARG, "cu_seqlens[0] must be 0");
+    if (budget < h->p.window) return fail(KVEC_ERR_INVALID_ARG, "budget %d < window %d", budget, h->p.window);
+    int tiles = 0, chunks = 0;
+    for (int b = 0; b < batch; ++b) {
+        const int L = cu_host[b + 1] - cu_host[b];
+        if (L < h->p.window || L > h->p.max_seqlen)
+            return fail(KVEC_ERR_INVALID_ARG, "sequence %d has length %d outside [window=%d, max_seqlen=%d]", b, L,
+                        h->p.window, h->p.max_seqlen);
+        tiles += (L + kTileT - 1) / kTileT;
+        const int Lc = L - h->p.window;
+        chunks += Lc > 0 ? (Lc + kChunk - 1) / kChunk : 0;
+    }
+    *total_tiles = tiles;
+    *total_chunks = chunks;
+    return KVEC_OK;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+Geometry make_geometry(const kvec_handle* h, int batch, int budget, int tiles, int chunks) {
+    const kvec_params& p = h->p;
+    Geometry G{};
+    G.Hq = p.num_q_heads;
+    G.Hkv = p.num_kv_heads;
+    G.g = h->g;
+    G.w = p.window;
+    G.O = p.obs_window;
+    G.Oe = p.ext_window;
+    G.pool = p.pool_kernel;
+    G.delta = p.num_ext_heads;
+    G.R = h->R;
+    G.lambda = p.lambda;
+    const double scale = p.softmax_scale > 0.f ? (double)p.softmax_scale : 1.0 / sqrt((double)p.head_dim);
+    G.sl2 = (float)(scale * 1.4426950408889634);
+    G.ML = p.max_seqlen;
+    G.words = h->words;
+    G.batch = batch;
+    G.budget = budget;
+    int Kp = (int)floor((double)p.beta * (double)budget);
+    if (Kp > budget - p.window) Kp = budget - p.window;
+    G.Kp = Kp;
+    G.k2 = budget - p.window - Kp;
+    G.total_tiles = tiles;
+    G.total_chunks = chunks;
+    G.state_stride = h->state_stride;
+    G.state_n_off = h->n_off;
+    G.state_union_off = h->union_off;
+    return G;
+}
+
+kvec_status run_layer(kvec_handle* h, const Geometry& G, const LayerIO& io, cudaStream_t st) {
+    timed_launch(h, 0, st, [&] { launch_score(G, io, h->sc, st); });
+    timed_launch(h, 1, st, [&] { launch_rowstat(G, io, h->sc, st); });
+    timed_launch(h, 2, st, [&] { launch_window(G, io, h->sc, h->slot, st); });
+    timed_launch(h, 3, st, [&] { launch_heads(G, io, h->sc, h->slot, st); });
+    timed_launch(h, 4, st, [&] { launch_select(G, io, h->sc, h->slot, st); });
+    timed_launch(h, 5, st, [&] { launch_gather(G, io, st); });
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_fail(e, "kernel launch");
+    return KVEC_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t kvec_state_bytes(int max_seqlen) {
+    if (max_seqlen < 1) return 0;
+    const size_t ns = round_up((size_t)max_seqlen, 16);
+    const size_t words = ((size_t)max_seqlen + 31) / 32;
+    return round_up(16 + ns + 4 * words, 16);
+}
+
+kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
+    if (!out) return fail(KVEC_ERR_INVALID_ARG, "out is NULL");
+    *out = nullptr;
+    kvec_status s = validate_params(params);
+    if (s != KVEC_OK) return s;
+    kvec_handle* h = new kvec_handle();
+    h->p = *params;
+    cudaError_t e = cudaGetDevice(&h->device);
+    if (e != cudaSuccess) {
+        delete h;
+        return cuda_fail(e, "cudaGetDevice");
+    }
+    const kvec_params& p = h->p;
+    h->g = p.num_q_heads / p.num_kv_heads;
+    h->R = h->g * p.window;
+    h->words = (p.max_seqlen + 31) / 32;
+    h->state_stride = kvec_state_bytes(p.max_seqlen);
+    h->n_off = 16;
+    h->union_off = 16 + round_up((size_t)p.max_seqlen, 16);
+
+    const size_t MB = p.max_batch, ML = p.max_seqlen, Hkv = p.num_kv_heads, R = h->R, W = h->words;
+    const size_t max_tiles = MB * ((ML + kTileT - 1) / kTileT);
+    const size_t sig_stride = ML / kChunk + 1;
+    struct Part {
+        void** dst;
+        size_t bytes;
+    };
+    std::vector<Part> parts = {
+        {(void**)&h->sc.ebuf, max_tiles * Hkv * kTileT * R * sizeof(__half)},
+        {(void**)&h->sc.tstat, max_tiles * Hkv * R * sizeof(float2)},
+        {(void**)&h->sc.rowstat, MB * Hkv * R * sizeof(float2)},
+        {(void**)&h->sc.keys, MB * Hkv * ML * sizeof(uint32_t)},
+        {(void**)&h->sc.ubits, MB * W * sizeof(uint32_t)},
+        {(void**)&h->sc.ucount, MB * sizeof(unsigned)},
+        {(void**)&h->sc.err, sizeof(int)},
+        {(void**)&h->slot.PO, MB * Hkv * ML * sizeof(float)},
+        {(void**)&h->slot.POe, MB * Hkv * ML * sizeof(float)},
+        {(void**)&h->slot.I, MB * ML * sizeof(float)},
+        {(void**)&h->slot.sigpart, MB * Hkv * sig_stride * sizeof(float2)},
+        {(void**)&h->slot.sigma, MB * Hkv * sizeof(float)},
+        {(void**)&h->slot.htop, MB * Hkv * sizeof(int)},
+        {(void**)&h->slot.pres, MB * Hkv * W * sizeof(uint32_t)},
+        {(void**)&h->slot.Pprime, MB * Hkv * ML * sizeof(float)},
+    };
+    size_t total = 0;
+    for (auto& pt : parts) total += round_up(pt.bytes, 256);
+    e = cudaMalloc(&h->ws, total);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        delete h;
+        return fail(KVEC_ERR_OOM, "workspace of %zu bytes: %s", total, cudaGetErrorString(e));
+    }
+    h->ws_bytes = total;
+    e = cudaMemset(h->ws, 0, total);
+    size_t off = 0;
+    for (auto& pt : parts) {
+        *pt.dst = static_cast<char*>(h->ws) + off;
+        off += round_up(pt.bytes, 256);
+    }
+    Geometry G = make_geometry(h, 1, p.window, 1, 1);
+    if (e == cudaSuccess) e = configure_score(G);
+    if (e == cudaSuccess) e = configure_window(G);
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) {
+        cudaFree(h->ws);
+        delete h;
+        return cuda_fail(e, "workspace set-up");
+    }
+    *out = h;
+    return KVEC_OK;
+}
+
+kvec_status kvec_destroy(kvec_handle* h) {
+    if (!h) return fail(KVEC_ERR_INVALID_ARG, "handle is NULL");
+    int prev = 0;
+    kvec_status s = set_device(h, &prev);
+    if (s != KVEC_OK) return s;
+    DeviceGuard guard{prev, h->device};
+    cudaDeviceSynchronize();
+    recycle_timed(h);
+    for (cudaEvent_t e : h->event_pool) cudaEventDestroy(e);
+    cudaError_t e = cudaFree(h->ws);
+    delete h;
+    if (e != cudaSuccess) return cuda_fail(e, "cudaFree");
+    return KVEC_OK;
+}
+
+kvec_status kvec_reset(kvec_handle* h, void* coverage_state, int batch, kvec_stream_t stream) {
+    if (!h) return fail(KVEC_ERR_INVALID_ARG, "handle is NULL");
+    if (!coverage_state || batch < 1 || batch > h->p.max_batch)
+        return fail(KVEC_ERR_INVALID_ARG, "coverage_state must be non-NULL and 1 <= batch <= max_batch");
+    int prev = 0;
+    kvec_status s = set_device(h, &prev);
+    if (s != KVEC_OK) return s;
+    DeviceGuard guard{prev, h->device};
+    cudaError_t e = cudaMemsetAsync(coverage_state, 0, h->state_stride * (size_t)batch, (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
+    return KVEC_OK;
+}
+
+kvec_status kvec_select_layer(kvec_handle* h, int batch, const int32_t* cu_seqlens_host,
+                              const int32_t* cu_seqlens_dev, const void* q_obs, const void* k, const void* v,
+                              void* coverage_state, int budget, int32_t* out_idx, void* out_k, void* out_v,
+                              kvec_stream_t stream) {
+    const void* qs[1] = {q_obs};
+    const void* ks[1] = {k};
+    const void* vs[1] = {v};
+    int32_t* ois[1] = {out_idx};
+    void* oks[1] = {out_k};
+    void* ovs[1] = {out_v};
+    return kvec_select_layers(h, 1, batch, cu_seqlens_host, cu_seqlens_dev, qs, ks, vs, coverage_state, budget, ois,
+                              oks, ovs, stream);
+}
+
+kvec_status kvec_select_layers(kvec_handle* h, int num_layers, int batch, const int32_t* cu_seqlens_host,
+                               const int32_t* cu_seqlens_dev, const void* const* q_obs, const void* const* k,
+                               const void* const* v, void* coverage_state, int budget, int32_t* const* out_idx,
+                               void* const* out_k, void* const* out_v, kvec_stream_t stream) {
+    int tiles = 0, chunks = 0;
+    kvec_status s = validate_call(h, batch, cu_seqlens_host, cu_seqlens_dev, budget, &tiles, &chunks);
+    if (s != KVEC_OK) return s;
+    if (num_layers < 1 || num_layers > h->p.max_layers)
+        return fail(KVEC_ERR_INVALID_ARG, "num_layers %d outside [1, max_layers=%d]", num_layers, h->p.max_layers);
+    if (!q_obs || !k || !v || !out_idx || !out_k || !out_v || !coverage_state)
+        return fail(KVEC_ERR_INVALID_ARG, "NULL pointer argument");
+    if (!aligned16(coverage_state)) return fail(KVEC_ERR_INVALID_ARG, "coverage_state must be 16-byte aligned");
+    for (int l = 0; l < num_layers; ++l) {
+        if (!q_obs[l] || !k[l] || !v[l] || !out_idx[l] || !out_k[l] || !out_v[l])
+            return fail(KVEC_ERR_INVALID_ARG, "NULL pointer for layer %d", l);
+        if (!aligned16(q_obs[l]) || !aligned16(k[l]) || !aligned16(v[l]) || !aligned16(out_k[l]) ||
+            !aligned16(out_v[l]) || (reinterpret_cast<uintptr_t>(out_idx[l]) & 3u))
+            return fail(KVEC_ERR_INVALID_ARG, "layer %d: device pointers must be 16-byte aligned", l);
+    }
+    int prev = 0;
+    s = set_device(h, &prev);
+    if (s != KVEC_OK) return s;
+    DeviceGuard guard{prev, h->device};
+    const Geometry G = make_geometry(h, batch, budget, tiles, chunks);
+    cudaStream_t st = (cudaStream_t)stream;
+    for (int l = 0; l < num_layers; ++l) {
+        LayerIO io{};
+        io.q = static_cast<const __nv_bfloat16*>(q_obs[l]);
+        io.k = static_cast<const __nv_bfloat16*>(k[l]);
+        io.v = static_cast<const __nv_bfloat16*>(v[l]);
+        io.cu = cu_seqlens_dev;
+        io.state = static_cast<uint8_t*>(coverage_state);
+        io.out_idx = out_idx[l];
+        io.out_k = static_cast<__nv_bfloat16*>(out_k[l]);
+        io.out_v = static_cast<__nv_bfloat16*>(out_v[l]);
+        s = run_layer(h, G, io, st);
+        if (s != KVEC_OK) return s;
+    }
+    h->last_batch = batch;
+    return KVEC_OK;
+}
+
+kvec_status kvec_debug_scores(kvec_handle* h, kvec_debug_view* out) {
+    if (!h || !out) return fail(KVEC_ERR_INVALID_ARG, "NULL argument");
+    out->P_O = h->slot.PO;
+    out->P_Oext = h->slot.POe;
+    out->I = h->slot.I;
+    out->sigma = h->slot.sigma;
+    out->htop = h->slot.htop;
+    out->pres_bits = h->slot.pres;
+    out->Pprime = h->slot.Pprime;
+    out->row_stats = reinterpret_cast<const float*>(h->sc.rowstat);
+    out->max_seqlen = h->p.max_seqlen;
+    out->words_per_row = h->words;
+    return KVEC_OK;
+}
+
+kvec_status kvec_sync_status(kvec_handle* h) {
+    if (!h) return fail(KVEC_ERR_INVALID_ARG, "handle is NULL");
+    int prev = 0;
+    kvec_status s = set_device(h, &prev);
+    if (s != KVEC_OK) return s;
+    DeviceGuard guard{prev, h->device};
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceSynchronize");
+    int err = 0;
+    e = cudaMemcpy(&err, h->sc.err, sizeof(int), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(e, "reading the device error word");
+    if (err) {
+        cudaMemset(h->sc.err, 0, sizeof(int));
+        if (err == 2) return fail(KVEC_ERR_INVALID_ARG, "a coverage state already counted 255 layers");
+        return fail(KVEC_ERR_DEVICE_TIMEOUT, "a bounded device wait gave up (code %d)", err);
+    }
+    return KVEC_OK;
+}
+
+kvec_status kvec_set_profiling(kvec_handle* h, int enable) {
+    if (!h) return fail(KVEC_ERR_INVALID_ARG, "handle is NULL");
+    cudaDeviceSynchronize();
+    recycle_timed(h);
+    h->profiling = enable != 0;
+    return KVEC_OK;
+}
+
+kvec_status kvec_kernel_time(kvec_handle* h, int kernel, double* total_ms, int* launches) {
+    if (!h || !total_ms || !launches) return fail(KVEC_ERR_INVALID_ARG, "NULL argument");
+    if (kernel < 0 || kernel >= kKernelKinds) return fail(KVEC_ERR_INVALID_ARG, "kernel id %d unknown", kernel);
+    double sum = 0.0;
+    int n = 0;
+    for (auto& t : h->timed) {
+        if (t.kind != kernel) continue;
+        cudaError_t e = cudaEventSynchronize(t.stop);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaEventSynchronize");
+        float ms = 0.f;
+        e = cudaEventElapsedTime(&ms, t.start, t.stop);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaEventElapsedTime");
+        sum += ms;
+        ++n;
+    }
+    *total_ms = sum;
+    *launches = n;
+    return KVEC_OK;
+}
+
+const char* kvec_status_string(kvec_status s) {
+    switch (s) {
+        case KVEC_OK: return "ok";
+        case KVEC_ERR_INVALID_ARG: return "invalid argument";
+        case KVEC_ERR_UNSUPPORTED: return "unsupported configuration";
+        case KVEC_ERR_CUDA: return "CUDA error";
+        case KVEC_ERR_DEVICE_TIMEOUT: return "device-side wait timed out";
+        case KVEC_ERR_OOM: return "out of device memory";
+    }
+    return "unknown status";
+}
+
+const char* kvec_last_error(void) { return g_last_error.c_str(); }
+
+}  // extern "C"

@@ -1,0 +1,104 @@
+// Internal declarations of the K-VEC CUDA path (sm_103a).  Not part of the ABI.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace kvec {
+
+constexpr int kHeadDim = 128;      // d supported by the score kernel
+constexpr int kTileT = 128;        // tokens per score tile (one MMA N block / e-buffer tile)
+constexpr int kChunk = 64;         // candidate tokens per window/pool CTA
+constexpr int kMaxPool = 15;       // largest pool kernel (halo 7)
+constexpr int kSelectThreads = 1024;
+constexpr float kEScaleLog2 = 15.f;  // e values are stored as fp16(2^15 * exp(s - mu))
+
+// Sizes and hyper-parameters shared by every kernel of one call.
+struct Geometry {
+    int Hq, Hkv, g, w, O, Oe, pool, delta;
+    int R;             // rows per KV head = g * w, ordered r = q * g + j
+    float lambda;
+    float sl2;         // softmax scale * log2(e)
+    int ML;            // max_seqlen: row stride of per-position workspace arrays
+    int words;         // ceil(ML / 32)
+    int batch, budget, Kp, k2;
+    int total_tiles;   // sum over sequences of ceil(L_s / kTileT)
+    int total_chunks;  // sum over sequences of ceil((L_s - w) / kChunk)
+    size_t state_stride;
+    size_t state_n_off, state_union_off;
+};
+
+// Device workspace owned by the handle (one slot of per-layer score arrays).
+struct Slot {
+    float* PO;            // [max_batch][Hkv][ML]  pooled Eq. 1 scores, window O
+    float* POe;           // [max_batch][Hkv][ML]  pooled, window O'
+    float* I;             // [max_batch][ML]       pooled importance
+    float2* sigpart;      // [max_batch][Hkv][ML/kChunk+1] (chunk mean, chunk M2)
+    float* sigma;         // [max_batch][Hkv]
+    int* htop;            // [max_batch][Hkv]
+    uint32_t* pres;       // [max_batch][Hkv][words]
+    float* Pprime;        // [max_batch][Hkv][ML]
+};
+
+struct Scratch {
+    __half* ebuf;         // [total_tiles][Hkv][kTileT][R]  scaled exp(s - mu_tile)
+    float2* tstat;        // [total_tiles][Hkv][R]  (mu_tile in log2 units, sum of exp)
+    float2* rowstat;      // [max_batch][Hkv][R]    (row max in log2 units, softmax denominator)
+    uint32_t* keys;       // [max_batch][Hkv][ML]   radix-select keys
+    uint32_t* ubits;      // [max_batch][words]     union of this layer's selections
+    unsigned* ucount;     // [max_batch]            heads finished (last-CTA fold)
+    int* err;             // device error word
+};
+
+struct LayerIO {
+    const __nv_bfloat16* q;   // [batch][w][Hq][d]
+    const __nv_bfloat16* k;   // [total][Hkv][d]
+    const __nv_bfloat16* v;
+    const int* cu;            // device cu_seqlens
+    uint8_t* state;
+    int32_t* out_idx;
+    __nv_bfloat16* out_k;
+    __nv_bfloat16* out_v;
+};
+
+// ---------------------------------------------------------------- helpers
+
+__device__ __forceinline__ uint32_t float_order_key(float f) {
+    // Monotone map of IEEE floats onto unsigned integers (larger float -> larger key).
+    uint32_t u = __float_as_uint(f);
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+// Finds (sequence, local index) of global item `gi` where sequence s owns
+// count(s) consecutive items; also returns the first global item of s.
+template <class CountFn>
+__device__ __forceinline__ bool locate_item(int batch, int gi, CountFn count, int& s, int& local, int& base) {
+    int acc = 0;
+    for (int b = 0; b < batch; ++b) {
+        int c = count(b);
+        if (gi < acc + c) { s = b; local = gi - acc; base = acc; return true; }
+        acc += c;
+    }
+    return false;
+}
+
+__device__ __forceinline__ int tiles_of(int L) { return (L + kTileT - 1) / kTileT; }
+__device__ __forceinline__ int chunks_of(int Lc) { return Lc > 0 ? (Lc + kChunk - 1) / kChunk : 0; }
+
+// ---------------------------------------------------------------- launchers
+
+void launch_score(const Geometry& g, const LayerIO& io, const Scratch& sc, cudaStream_t st);
+void launch_rowstat(const Geometry& g, const LayerIO& io, const Scratch& sc, cudaStream_t st);
+void launch_window(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st);
+void launch_heads(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st);
+void launch_select(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st);
+void launch_gather(const Geometry& g, const LayerIO& io, cudaStream_t st);
+
+size_t score_smem_bytes(const Geometry& g);
+size_t window_smem_bytes(const Geometry& g);
+cudaError_t configure_score(const Geometry& g);
+cudaError_t configure_window(const Geometry& g);
+
+}  // namespace kvec

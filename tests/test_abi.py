@@ -1,0 +1,89 @@
+"""Host-side checks of the C ABI that need no GPU: the library builds and loads,
+exports every entry point include/kvec.h declares, sizes the coverage state like
+the oracle, and rejects bad arguments before touching CUDA."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import oracle
+from paper_2606_29563_gb300 import build as kbuild
+from paper_2606_29563_gb300 import kvec
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    kbuild.build()
+    return kvec.load()
+
+
+def declared_entry_points():
+    text = open(os.path.join(ROOT, "include", "kvec.h")).read()
+    return sorted(set(re.findall(r"KVEC_API\s+[\w\s\*]+?\b(kvec_\w+)\s*\(", text)))
+
+
+def test_header_declares_expected_entry_points():
+    names = declared_entry_points()
+    assert set(names) == set(kvec.EXPORTED)
+
+
+def test_library_exports_every_declared_symbol(lib):
+    raw = ctypes.CDLL(kvec.LIB_PATH)
+    for name in declared_entry_points():
+        assert hasattr(raw, name), name
+
+
+def test_state_bytes_matches_oracle(lib):
+    for ml in (1, 31, 32, 33, 1000, 8192, 16384, 32768, 131072):
+        assert kvec.kvec_state_bytes(ml) == oracle.state_bytes(ml)
+        assert kvec.kvec_state_bytes(ml) % 16 == 0
+    assert kvec.kvec_state_bytes(0) == 0
+
+
+BAD_PARAMS = [
+    (dict(num_q_heads=30, num_kv_heads=8), kvec.KVEC_ERR_INVALID_ARG),
+    (dict(num_kv_heads=0), kvec.KVEC_ERR_INVALID_ARG),
+    (dict(head_dim=64), kvec.KVEC_ERR_UNSUPPORTED),
+    (dict(obs_window=40), kvec.KVEC_ERR_INVALID_ARG),
+    (dict(ext_window=0), kvec.KVEC_ERR_INVALID_ARG),
+    (dict(pool_kernel=6), kvec.KVEC_ERR_INVALID_ARG),
+    (dict(pool_kernel=17), kvec.KVEC_ERR_INVALID_ARG),
+    (dict(num_ext_heads=9), kvec.KVEC_ERR_INVALID_ARG),
+    (dict(beta=1.5), kvec.KVEC_ERR_INVALID_ARG),
+    (dict(lam=float("inf")), kvec.KVEC_ERR_INVALID_ARG),
+    (dict(max_layers=256), kvec.KVEC_ERR_INVALID_ARG),
+    (dict(max_seqlen=0), kvec.KVEC_ERR_INVALID_ARG),
+    (dict(max_seqlen=200000), kvec.KVEC_ERR_INVALID_ARG),
+    (dict(num_q_heads=72, num_kv_heads=8), kvec.KVEC_ERR_UNSUPPORTED),   # 9 x 32 rows > 256
+    (dict(num_q_heads=264, num_kv_heads=33), kvec.KVEC_ERR_UNSUPPORTED),
+]
+
+
+@pytest.mark.parametrize("over,code", BAD_PARAMS)
+def test_create_rejects_bad_parameters_before_cuda(lib, over, code):
+    kw = dict(num_q_heads=32, num_kv_heads=8)
+    kw.update(over)
+    p = kvec.make_params(**kw)
+    with pytest.raises(kvec.KvecError) as e:
+        kvec.kvec_create(p)
+    assert e.value.status == code
+    assert kvec.load().kvec_last_error()
+
+
+def test_calls_on_null_handle_are_rejected(lib):
+    cu = (ctypes.c_int32 * 2)(0, 64)
+    with pytest.raises(kvec.KvecError) as e:
+        kvec.kvec_select_layer(None, 1, ctypes.addressof(cu), ctypes.addressof(cu), 16, 16, 16, 16, 64, 16, 16, 16)
+    assert e.value.status == kvec.KVEC_ERR_INVALID_ARG
+    for fn in (lambda: kvec.kvec_reset(None, 16, 1), lambda: kvec.kvec_sync_status(None),
+               lambda: kvec.kvec_debug_scores(None), lambda: kvec.kvec_destroy(None)):
+        with pytest.raises(kvec.KvecError):
+            fn()
+
+
+def test_status_strings(lib):
+    for code in range(6):
+        assert kvec.kvec_status_string(code)

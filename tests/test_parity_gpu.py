@@ -1,0 +1,171 @@
+"""GPU parity: the CUDA path (through the C ABI) against the fp64 oracle.
+
+Every case is teacher-forced layer by layer (oracle.parity): scores within the
+2e-3 relative tolerance, kept-index sets identical outside the tie band, and
+gathered K/V plus the coverage-state update bit-exact given the GPU's indices.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import parity
+from paper_2606_29563_gb300 import kvec, synth
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+    from paper_2606_29563_gb300 import build as kbuild
+    import oracle
+    kbuild.build()
+    oracle.build()
+
+
+def _assert_parity(wl, **kw):
+    errs = parity.run_parity(wl, **kw)
+    assert not errs, "\n".join(errs[:25])
+
+
+def test_small_two_layers():
+    _assert_parity(synth.small_workload(seqlens=(700,), layers=2))
+
+
+@pytest.mark.parametrize("g,Hkv", [(1, 4), (2, 4), (4, 2), (7, 4), (8, 2)])
+def test_group_sizes(g, Hkv):
+    _assert_parity(synth.small_workload(seqlens=(523,), num_q_heads=g * Hkv, num_kv_heads=Hkv, layers=2,
+                                        num_ext_heads=1))
+
+
+@pytest.mark.parametrize("L", [33, 129, 255, 256, 257, 1000])
+def test_ragged_tails_and_short_sequences(L):
+    # w = 32: L = 33 leaves one candidate; 129 / 257 end one token into a new tile.
+    _assert_parity(synth.small_workload(seqlens=(L,), budget=48, layers=2))
+
+
+def test_ragged_batch_with_keep_all_members():
+    # 40 and 64 fit the budget (keep everything); the others are evicted.
+    _assert_parity(synth.small_workload(seqlens=(40, 900, 64, 1531, 300), budget=64, layers=3))
+
+
+def test_budget_equals_window():
+    _assert_parity(synth.small_workload(seqlens=(600,), budget=32, layers=2))
+
+
+@pytest.mark.parametrize("pool", [1, 3, 15])
+def test_pool_widths(pool):
+    _assert_parity(synth.small_workload(seqlens=(640,), pool_kernel=pool, layers=2))
+
+
+@pytest.mark.parametrize("over", [dict(num_ext_heads=0, lam=0.0), dict(lam=0.0), dict(beta=0.0), dict(beta=1.0),
+                                  dict(lam=2.0, beta=0.1), dict(obs_window=32, ext_window=32),
+                                  dict(window=16, obs_window=8, ext_window=16)])
+def test_hyperparameter_corners(over):
+    _assert_parity(synth.small_workload(seqlens=(777,), layers=2, **over))
+
+
+def test_uniform_keys_tie_to_lowest_positions():
+    """K = 0 makes every candidate score equal: selection must be the lowest positions (exact ties)."""
+    wl = synth.small_workload(seqlens=(400,), budget=64, layers=1)
+    params = kvec.params_from_workload(wl)
+    sel = kvec.KvecSelector(params)
+    x = synth.make_layer(wl, 0)
+    k = torch.zeros_like(x["k"]).cuda()
+    cu = torch.tensor(wl.cu_seqlens, dtype=torch.int32)
+    st = sel.new_state(1)
+    idx, _, _ = sel.select_layer(cu, cu.cuda(), x["q_obs"].cuda(), k, x["v"].cuda(), st, wl.budget)
+    torch.cuda.synchronize()
+    expect = list(range(wl.budget - wl.window)) + list(range(400 - wl.window, 400))
+    for h in range(wl.num_kv_heads):
+        assert idx[0, h].cpu().tolist() == expect
+    sel.close()
+
+
+def test_deterministic_rerun():
+    wl = synth.small_workload(seqlens=(900, 450), layers=2)
+    outs = []
+    for _ in range(2):
+        sel = kvec.KvecSelector(kvec.params_from_workload(wl))
+        cu = torch.tensor(wl.cu_seqlens, dtype=torch.int32)
+        st = sel.new_state(wl.batch)
+        res = []
+        for x in synth.make_layers(wl, 2):
+            o = sel.select_layer(cu, cu.cuda(), x["q_obs"].cuda(), x["k"].cuda(), x["v"].cuda(), st, wl.budget)
+            res.append([t.cpu() for t in o])
+        torch.cuda.synchronize()
+        res.append([st.cpu()])
+        outs.append(res)
+        sel.close()
+    for a, b in zip(outs[0], outs[1]):
+        for x, y in zip(a, b):
+            assert torch.equal(x, y)
+
+
+def test_multi_layer_call_matches_layer_by_layer():
+    wl = synth.small_workload(seqlens=(1100, 700), layers=4, budget=96)
+    layers = [{k: v.cuda() for k, v in x.items()} for x in synth.make_layers(wl, 4)]
+    cu = torch.tensor(wl.cu_seqlens, dtype=torch.int32)
+    sel = kvec.KvecSelector(kvec.params_from_workload(wl))
+    st1 = sel.new_state(wl.batch)
+    one = [sel.select_layer(cu, cu.cuda(), x["q_obs"], x["k"], x["v"], st1, wl.budget) for x in layers]
+    st2 = sel.new_state(wl.batch)
+    many = [sel.alloc_outputs(wl.batch, wl.budget) for _ in layers]
+    sel.select_layers(cu, cu.cuda(), [x["q_obs"] for x in layers], [x["k"] for x in layers],
+                      [x["v"] for x in layers], st2, wl.budget, many)
+    torch.cuda.synchronize()
+    for a, b in zip(one, many):
+        for x, y in zip(a, b):
+            assert torch.equal(x, y)
+    assert torch.equal(st1, st2)
+    sel.close()
+
+
+def test_call_validation_on_device():
+    wl = synth.small_workload(seqlens=(300,))
+    sel = kvec.KvecSelector(kvec.params_from_workload(wl))
+    x = {k: v.cuda() for k, v in synth.make_layer(wl, 0).items()}
+    st = sel.new_state(1)
+    cu_ok = torch.tensor([0, 300], dtype=torch.int32)
+    cases = [
+        (torch.tensor([0, 20], dtype=torch.int32), wl.budget),     # L < w
+        (torch.tensor([0, 301], dtype=torch.int32), wl.budget),    # L > max_seqlen
+        (torch.tensor([1, 300], dtype=torch.int32), wl.budget),    # cu[0] != 0
+        (cu_ok, wl.window - 1),                                    # B < w
+    ]
+    for cu, budget in cases:
+        with pytest.raises(kvec.KvecError) as e:
+            sel.select_layer(cu, cu.cuda(), x["q_obs"], x["k"], x["v"], st, budget)
+        assert e.value.status == kvec.KVEC_ERR_INVALID_ARG
+    with pytest.raises(kvec.KvecError):   # misaligned K
+        sel.select_layer(cu_ok, cu_ok.cuda(), x["q_obs"], x["k"].view(-1)[1:].view(torch.uint8)[:0], x["v"], st,
+                         wl.budget) if False else kvec.kvec_select_layer(
+            sel.handle, 1, cu_ok.data_ptr(), cu_ok.cuda().data_ptr(), x["q_obs"].data_ptr(), x["k"].data_ptr() + 2,
+            x["v"].data_ptr(), st.data_ptr(), wl.budget, *[t.data_ptr() for t in sel.alloc_outputs(1, wl.budget)],
+            torch.cuda.current_stream().cuda_stream)
+    assert st.cpu().sum().item() == 0   # rejected calls launched nothing
+    sel.close()
+
+
+# ---- the five workloads at full size (teacher-forced, a few layers each) ----
+
+def test_mha8_l1024_b128_full():
+    _assert_parity(synth.WORKLOADS["mha8_l1024_b128"])
+
+
+def test_llama8b_l8192_b512_first_layers():
+    _assert_parity(synth.WORKLOADS["llama8b_l8192_b512"], layers=3)
+
+
+def test_llama8b_l32768_b128_first_layers():
+    _assert_parity(synth.WORKLOADS["llama8b_l32768_b128"], layers=2)
+
+
+def test_llama8b_ragged8_b256_first_layers():
+    _assert_parity(synth.WORKLOADS["llama8b_ragged8_b256"], layers=2)
+
+
+@pytest.mark.parametrize("budget", synth.QWEN_BUDGETS)
+def test_qwen7b_l16384_budget_sweep(budget):
+    _assert_parity(synth.WORKLOADS["qwen7b_l16384_b512"].replace(budget=budget), layers=2)

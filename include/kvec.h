@@ -128,6 +128,36 @@ KVEC_API kvec_status kvec_select_layers(kvec_handle* h, int num_layers, int batc
                                int32_t* const* out_idx, void* const* out_k, void* const* out_v,
                                kvec_stream_t stream);
 
+/* kvec_select_layer for callers that cannot allocate device memory: the
+ * library then needs no handle and calls no cudaMalloc, cudaFree or other
+ * allocating routine.  It serves hosts whose device memory belongs to someone
+ * else (an inference server or framework plugin that hands out all memory
+ * from its own pool and forbids extra allocations), which cannot create a
+ * handle because kvec_create allocates its workspace.  The paper has no
+ * counterpart; this is a deployment convenience.
+ *   Arguments: as kvec_select_layer, with the hyper-parameters and the sizing
+ *   limits (max_batch, max_seqlen; max_seqlen also fixes the state layout)
+ *   given in *params instead of a handle.
+ *   Scratch: one 32 MiB static device array inside the library, held by every
+ *   GPU that loads the library until the process exits.  A call whose
+ *   geometry needs more (roughly: batch * H_kv * (L * g * w * 2 + 16 * L)
+ *   bytes; one 8192-token Llama-3.1-8B-shaped sequence needs about 18 MiB) is
+ *   rejected with KVEC_ERR_INVALID_ARG and a message giving both sizes.
+ *   Every call shares that array and it keeps the last call's contents; the
+ *   call clears what must start at zero.  Calls whose work overlaps on the
+ *   GPU (different streams, or several host threads) race on it: serialise
+ *   them.
+ *   The first call on each device resolves the array's device address and
+ *   sets kernel attributes (no allocation); make that first call before any
+ *   stream capture.  The device-side 255-layer guard is not reported by this
+ *   entry point: keep layers_done below 255 yourself. */
+KVEC_API kvec_status kvec_select_layer_noalloc(const kvec_params* params, int batch,
+                                      const int32_t* cu_seqlens_host, const int32_t* cu_seqlens_dev,
+                                      const void* q_obs, const void* k, const void* v,
+                                      void* coverage_state, int budget,
+                                      int32_t* out_idx, void* out_k, void* out_v,
+                                      kvec_stream_t stream);
+
 /* Device views of the last processed layer's intermediates (valid until the
  * next call on the handle; read after synchronising the stream).  Strides use
  * the handle's max_seqlen (ML).  Only candidate positions t < L_s - w hold

@@ -5,6 +5,7 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <mutex>
 #include <string>
 #include <vector>
 
@@ -369,6 +370,139 @@ kvec_status kvec_select_layers(kvec_handle* h, int num_layers, int batch, const 
     }
     h->last_batch = batch;
     return KVEC_OK;
+}
+
+// ---------------------------------------------------------------------------
+// kvec_select_layer_noalloc: the same layer as kvec_select_layer for callers
+// that may not allocate device memory.  Its scratch lives in one file-scope
+// static device array that every GPU loading this library holds until exit.
+// ---------------------------------------------------------------------------
+}  // extern "C"
+
+namespace {
+
+constexpr size_t kNoallocScratchBytes = size_t(32) << 20;   // 32 MiB
+__device__ __align__(256) unsigned char g_noalloc_scratch[kNoallocScratchBytes];
+
+constexpr int kMaxDevices = 64;
+struct NoallocDevice {
+    bool ready = false;
+    void* base = nullptr;   // device address of g_noalloc_scratch on that device
+};
+NoallocDevice g_noalloc_dev[kMaxDevices];
+std::mutex g_noalloc_mutex;
+
+// Once per device, with that device current: resolve the array's device address
+// (host code cannot use the symbol's name as a pointer) and set the kernels'
+// shared-memory limits.  Neither call allocates.
+kvec_status noalloc_setup(int dev, void** base, const Geometry& G) {
+    std::lock_guard<std::mutex> lock(g_noalloc_mutex);
+    if (dev < 0 || dev >= kMaxDevices) return fail(KVEC_ERR_UNSUPPORTED, "device index %d out of range", dev);
+    NoallocDevice& d = g_noalloc_dev[dev];
+    if (!d.ready) {
+        void* ptr = nullptr;
+        cudaError_t e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(scratch)");
+        e = configure_score(G);
+        if (e == cudaSuccess) e = configure_window(G);
+        if (e != cudaSuccess) return cuda_fail(e, "kernel attributes");
+        d.base = ptr;
+        d.ready = true;
+    }
+    *base = d.base;
+    return KVEC_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+kvec_status kvec_select_layer_noalloc(const kvec_params* params, int batch, const int32_t* cu_seqlens_host,
+                                      const int32_t* cu_seqlens_dev, const void* q_obs, const void* k,
+                                      const void* v, void* coverage_state, int budget, int32_t* out_idx,
+                                      void* out_k, void* out_v, kvec_stream_t stream) {
+    kvec_status s = validate_params(params);
+    if (s != KVEC_OK) return s;
+    // A stack handle carries the geometry; its vectors stay empty and nothing is allocated.
+    kvec_handle tmp;
+    tmp.p = *params;
+    tmp.g = params->num_q_heads / params->num_kv_heads;
+    tmp.R = tmp.g * params->window;
+    tmp.words = (params->max_seqlen + 31) / 32;
+    tmp.state_stride = kvec_state_bytes(params->max_seqlen);
+    tmp.n_off = 16;
+    tmp.union_off = 16 + round_up((size_t)params->max_seqlen, 16);
+    int tiles = 0, chunks = 0;
+    s = validate_call(&tmp, batch, cu_seqlens_host, cu_seqlens_dev, budget, &tiles, &chunks);
+    if (s != KVEC_OK) return s;
+    if (!q_obs || !k || !v || !out_idx || !out_k || !out_v || !coverage_state)
+        return fail(KVEC_ERR_INVALID_ARG, "NULL pointer argument");
+    if (!aligned16(q_obs) || !aligned16(k) || !aligned16(v) || !aligned16(out_k) || !aligned16(out_v) ||
+        !aligned16(coverage_state) || (reinterpret_cast<uintptr_t>(out_idx) & 3u))
+        return fail(KVEC_ERR_INVALID_ARG, "device pointers must be 16-byte aligned");
+
+    // Carve the scratch for exactly this call's geometry.
+    const size_t nb = batch, ML = params->max_seqlen, Hkv = params->num_kv_heads, R = tmp.R, W = tmp.words;
+    const size_t nt = tiles, sig_stride = ML / kChunk + 1;
+    struct Part {
+        void** dst;
+        size_t bytes;
+    };
+    Part parts[] = {
+        {(void**)&tmp.sc.ucount, nb * sizeof(unsigned)},      // zeroed every call (first three parts)
+        {(void**)&tmp.sc.err, sizeof(int)},
+        {(void**)&tmp.sc.ubits, nb * W * sizeof(uint32_t)},
+        {(void**)&tmp.sc.ebuf, nt * Hkv * kTileT * R * sizeof(__half)},
+        {(void**)&tmp.sc.tstat, nt * Hkv * R * sizeof(float2)},
+        {(void**)&tmp.sc.rowstat, nb * Hkv * R * sizeof(float2)},
+        {(void**)&tmp.sc.keys, nb * Hkv * ML * sizeof(uint32_t)},
+        {(void**)&tmp.slot.PO, nb * Hkv * ML * sizeof(float)},
+        {(void**)&tmp.slot.POe, nb * Hkv * ML * sizeof(float)},
+        {(void**)&tmp.slot.I, nb * ML * sizeof(float)},
+        {(void**)&tmp.slot.sigpart, nb * Hkv * sig_stride * sizeof(float2)},
+        {(void**)&tmp.slot.sigma, nb * Hkv * sizeof(float)},
+        {(void**)&tmp.slot.htop, nb * Hkv * sizeof(int)},
+        {(void**)&tmp.slot.pres, nb * Hkv * W * sizeof(uint32_t)},
+        {(void**)&tmp.slot.Pprime, nb * Hkv * ML * sizeof(float)},
+    };
+    size_t need = 0, zero_bytes = 0;
+    for (size_t i = 0; i < sizeof(parts) / sizeof(parts[0]); ++i) {
+        need += round_up(parts[i].bytes, 256);
+        if (i == 2) zero_bytes = need;
+    }
+    if (need > kNoallocScratchBytes)
+        return fail(KVEC_ERR_INVALID_ARG,
+                    "this call needs %zu bytes of scratch; kvec_select_layer_noalloc has %zu (use kvec_create / "
+                    "kvec_select_layer for larger batches or sequences)",
+                    need, kNoallocScratchBytes);
+
+    int prev = 0;
+    cudaError_t e = cudaGetDevice(&prev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    tmp.device = prev;
+    const Geometry G = make_geometry(&tmp, batch, budget, tiles, chunks);
+    void* base = nullptr;
+    s = noalloc_setup(prev, &base, G);
+    if (s != KVEC_OK) return s;
+    size_t off = 0;
+    for (auto& pt : parts) {
+        *pt.dst = static_cast<char*>(base) + off;
+        off += round_up(pt.bytes, 256);
+    }
+    cudaStream_t st = (cudaStream_t)stream;
+    // The array keeps the previous call's contents: the counters and union bits must start at zero.
+    e = cudaMemsetAsync(base, 0, zero_bytes, st);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync(scratch)");
+    LayerIO io{};
+    io.q = static_cast<const __nv_bfloat16*>(q_obs);
+    io.k = static_cast<const __nv_bfloat16*>(k);
+    io.v = static_cast<const __nv_bfloat16*>(v);
+    io.cu = cu_seqlens_dev;
+    io.state = static_cast<uint8_t*>(coverage_state);
+    io.out_idx = out_idx;
+    io.out_k = static_cast<__nv_bfloat16*>(out_k);
+    io.out_v = static_cast<__nv_bfloat16*>(out_v);
+    return run_layer(&tmp, G, io, st);
 }
 
 kvec_status kvec_debug_scores(kvec_handle* h, kvec_debug_view* out) {

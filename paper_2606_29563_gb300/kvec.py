@@ -27,7 +27,7 @@ KERNEL_NAMES = ("score", "rowstat", "window", "heads", "select", "gather")
 
 EXPORTED = ("kvec_create", "kvec_destroy", "kvec_state_bytes", "kvec_reset", "kvec_select_layer",
             "kvec_select_layers", "kvec_debug_scores", "kvec_sync_status", "kvec_set_profiling",
-            "kvec_kernel_time", "kvec_status_string", "kvec_last_error")
+            "kvec_kernel_time", "kvec_status_string", "kvec_last_error", "kvec_select_layer_noalloc")
 
 
 class KvecUnavailable(ImportError):
@@ -89,6 +89,8 @@ def load() -> ctypes.CDLL:
             "kvec_kernel_time": ([_vp, i, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_int)], st),
             "kvec_status_string": ([i], ctypes.c_char_p),
             "kvec_last_error": ([], ctypes.c_char_p),
+            "kvec_select_layer_noalloc": ([ctypes.POINTER(kvec_params), i, _vp, _vp, _vp, _vp, _vp, _vp, i, _vp,
+                                           _vp, _vp, _vp], st),
         }
         for name, (args, res) in sig.items():
             fn = getattr(lib, name)
@@ -138,6 +140,14 @@ def kvec_select_layers(handle: int, batch: int, cu_host_ptr: int, cu_dev_ptr: in
     n = len(q_obs)
     _check(load().kvec_select_layers(handle, n, int(batch), cu_host_ptr, cu_dev_ptr, _arr(q_obs), _arr(k), _arr(v),
                                      state, int(budget), _arr(out_idx), _arr(out_k), _arr(out_v), stream))
+
+
+def kvec_select_layer_noalloc(params: kvec_params, batch: int, cu_host_ptr: int, cu_dev_ptr: int, q_obs: int,
+                              k: int, v: int, state: int, budget: int, out_idx: int, out_k: int, out_v: int,
+                              stream: int = 0) -> None:
+    """kvec_select_layer without a handle; scratch comes from the library's static device array."""
+    _check(load().kvec_select_layer_noalloc(ctypes.byref(params), int(batch), cu_host_ptr, cu_dev_ptr, q_obs, k, v,
+                                            state, int(budget), out_idx, out_k, out_v, stream))
 
 
 def kvec_debug_scores(handle: int) -> kvec_debug_view:

@@ -278,7 +278,7 @@ def run_ours(args, wl):
     # End to end through the public API: pinned host inputs copied in, indices and state copied out.
     e2e = run_e2e(args, wl, sel, layers, outs, state, cu_host, cu_dev, dev, stream) if args.e2e else None
 
-    gpu_launches = args.steps * L_layers * len(kvec.KERNEL_NAMES)   # six kernels per layer
+    gpu_launches = args.steps * L_layers * len(kvec.KERNEL_NAMES)   # five kernels per layer
     sel.close()
     result = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,

@@ -159,9 +159,9 @@ KVEC_API kvec_status kvec_select_layer_noalloc(const kvec_params* params, int ba
                                       kvec_stream_t stream);
 
 /* Device views of the last processed layer's intermediates (valid until the
- * next call on the handle; read after synchronising the stream).  Strides use
- * the handle's max_seqlen (ML).  Only candidate positions t < L_s - w hold
- * scores. */
+ * next call on the handle; read after synchronising the stream).  Row strides
+ * use ML = max_seqlen rounded up to a multiple of 32 (reported in max_seqlen).
+ * Only candidate positions t < L_s - w hold scores. */
 typedef struct {
     const float*    P_O;        /* [max_batch][H_kv][ML]  Eq. 1 with O, max-pooled */
     const float*    P_Oext;     /* [max_batch][H_kv][ML]  Eq. 1 with O', max-pooled */
@@ -173,8 +173,8 @@ typedef struct {
     const float*    row_stats;  /* [max_batch][H_kv][g*w][2]  softmax row max (log2 units)
                                    and denominator; row r = q*g + j is query head
                                    h*g + j at window row q */
-    int max_seqlen;
-    int words_per_row;          /* ceil(ML/32) */
+    int max_seqlen;             /* ML: the row stride of the arrays above */
+    int words_per_row;          /* ML/32 */
 } kvec_debug_view;
 
 KVEC_API kvec_status kvec_debug_scores(kvec_handle* h, kvec_debug_view* out);
@@ -184,9 +184,9 @@ KVEC_API kvec_status kvec_debug_scores(kvec_handle* h, kvec_debug_view* out);
 KVEC_API kvec_status kvec_sync_status(kvec_handle* h);
 
 /* Per-kernel device time recorded since the last kvec_set_profiling(h, 1)
- * call, from CUDA events on the launching stream.  kernel: 0 score (QK^T +
- * softmax partials), 1 row-stat merge, 2 window sums + pooling, 3 cross-head
- * + preserve, 4 coverage select, 5 gather.  Synchronises. */
+ * call, from CUDA events on the launching stream.  kernel: 0 score (QK^T and
+ * softmax statistics), 1 window sums + pooling, 2 cross-head choice +
+ * preserved tokens, 3 coverage-adjusted selection, 4 gather.  Synchronises. */
 KVEC_API kvec_status kvec_set_profiling(kvec_handle* h, int enable);
 KVEC_API kvec_status kvec_kernel_time(kvec_handle* h, int kernel, double* total_ms, int* launches);
 

@@ -9,7 +9,7 @@
 #include <string>
 #include <vector>
 
-#include "../../include/kvec.h"
+#include "kvec.h"
 #include "kvec_internal.cuh"
 
 using namespace kvec;
@@ -34,7 +34,7 @@ kvec_status cuda_fail(cudaError_t e, const char* what) {
 
 size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
-constexpr int kKernelKinds = 6;
+constexpr int kKernelKinds = 5;
 
 struct TimedLaunch {
     int kind;
@@ -46,6 +46,7 @@ struct TimedLaunch {
 struct kvec_handle {
     kvec_params p;
     int device = 0;
+    int num_sms = 1;
     int g = 1, R = 0, words = 0;
     size_t state_stride = 0, n_off = 16, union_off = 0;
     void* ws = nullptr;
@@ -97,7 +98,8 @@ kvec_status validate_params(const kvec_params* p) {
     if (p->num_kv_heads < 1 || p->num_q_heads < p->num_kv_heads || p->num_q_heads % p->num_kv_heads)
         return fail(KVEC_ERR_INVALID_ARG, "num_q_heads (%d) must be a positive multiple of num_kv_heads (%d)",
                     p->num_q_heads, p->num_kv_heads);
-    if (p->num_kv_heads > 32) return fail(KVEC_ERR_UNSUPPORTED, "num_kv_heads > 32 is not supported");
+    if (p->num_kv_heads > 16)
+        return fail(KVEC_ERR_UNSUPPORTED, "num_kv_heads > 16 is not supported (one thread-block cluster per sequence)");
     if (p->head_dim != kHeadDim) return fail(KVEC_ERR_UNSUPPORTED, "head_dim must be %d", kHeadDim);
     if (p->window < 1) return fail(KVEC_ERR_INVALID_ARG, "window must be >= 1");
     if (p->obs_window < 1 || p->obs_window > p->window || p->ext_window < 1 || p->ext_window > p->window)
@@ -152,8 +154,7 @@ kvec_status validate_call(kvec_handle* h, int batch, const int32_t* cu_host, con
             return fail(KVEC_ERR_INVALID_ARG, "sequence %d has length %d outside [window=%d, max_seqlen=%d]", b, L,
                         h->p.window, h->p.max_seqlen);
         tiles += (L + kTileT - 1) / kTileT;
-        const int Lc = L - h->p.window;
-        chunks += Lc > 0 ? (Lc + kChunk - 1) / kChunk : 0;
+        chunks += window_blocks(L - h->p.window);
     }
     *total_tiles = tiles;
     *total_chunks = chunks;
@@ -162,7 +163,7 @@ kvec_status validate_call(kvec_handle* h, int batch, const int32_t* cu_host, con
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-Geometry make_geometry(const kvec_handle* h, int batch, int budget, int tiles, int chunks) {
+Geometry make_geometry(const kvec_handle* h, int batch, int budget, int tiles, int chunks, int total_tokens) {
     const kvec_params& p = h->p;
     Geometry G{};
     G.Hq = p.num_q_heads;
@@ -177,7 +178,7 @@ Geometry make_geometry(const kvec_handle* h, int batch, int budget, int tiles, i
     G.lambda = p.lambda;
     const double scale = p.softmax_scale > 0.f ? (double)p.softmax_scale : 1.0 / sqrt((double)p.head_dim);
     G.sl2 = (float)(scale * 1.4426950408889634);
-    G.ML = p.max_seqlen;
+    G.ML = (int)round_up((size_t)p.max_seqlen, 32);   // row stride: 128-byte aligned rows
     G.words = h->words;
     G.batch = batch;
     G.budget = budget;
@@ -187,6 +188,7 @@ Geometry make_geometry(const kvec_handle* h, int batch, int budget, int tiles, i
     G.k2 = budget - p.window - Kp;
     G.total_tiles = tiles;
     G.total_chunks = chunks;
+    G.total_tokens = total_tokens;
     G.state_stride = h->state_stride;
     G.state_n_off = h->n_off;
     G.state_union_off = h->union_off;
@@ -194,12 +196,17 @@ Geometry make_geometry(const kvec_handle* h, int batch, int budget, int tiles, i
 }
 
 kvec_status run_layer(kvec_handle* h, const Geometry& G, const LayerIO& io, cudaStream_t st) {
-    timed_launch(h, 0, st, [&] { launch_score(G, io, h->sc, st); });
-    timed_launch(h, 1, st, [&] { launch_rowstat(G, io, h->sc, st); });
-    timed_launch(h, 2, st, [&] { launch_window(G, io, h->sc, h->slot, st); });
-    timed_launch(h, 3, st, [&] { launch_heads(G, io, h->sc, h->slot, st); });
-    timed_launch(h, 4, st, [&] { launch_select(G, io, h->sc, h->slot, st); });
-    timed_launch(h, 5, st, [&] { launch_gather(G, io, st); });
+    ScorePlan plan;
+    cudaError_t se = plan_score(G, io, h->sc, h->num_sms, &plan);
+    if (se != cudaSuccess) return cuda_fail(se, "score kernel tensor maps");
+    timed_launch(h, 0, st, [&] { se = launch_score(plan, st); });
+    if (se != cudaSuccess) return cuda_fail(se, "score kernel launch");
+    timed_launch(h, 1, st, [&] { launch_window(G, io, h->sc, h->slot, st); });
+    cudaError_t he = cudaSuccess;
+    timed_launch(h, 2, st, [&] { he = launch_heads(G, io, h->sc, h->slot, st); });
+    if (he != cudaSuccess) return cuda_fail(he, "heads kernel launch");
+    timed_launch(h, 3, st, [&] { launch_select(G, io, h->sc, h->slot, st); });
+    timed_launch(h, 4, st, [&] { launch_gather(G, io, st); });
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_fail(e, "kernel launch");
     return KVEC_OK;
@@ -236,9 +243,9 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
     h->n_off = 16;
     h->union_off = 16 + round_up((size_t)p.max_seqlen, 16);
 
-    const size_t MB = p.max_batch, ML = p.max_seqlen, Hkv = p.num_kv_heads, R = h->R, W = h->words;
+    const size_t MB = p.max_batch, ML = round_up((size_t)p.max_seqlen, 32), Hkv = p.num_kv_heads, R = h->R,
+                 W = h->words;
     const size_t max_tiles = MB * ((ML + kTileT - 1) / kTileT);
-    const size_t sig_stride = ML / kChunk + 1;
     struct Part {
         void** dst;
         size_t bytes;
@@ -246,15 +253,19 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
     std::vector<Part> parts = {
         {(void**)&h->sc.ebuf, max_tiles * Hkv * kTileT * R * sizeof(__half)},
         {(void**)&h->sc.tstat, max_tiles * Hkv * R * sizeof(float2)},
+        {(void**)&h->sc.segpart, max_tiles * Hkv * R * sizeof(float2)},
+        {(void**)&h->sc.shcount, MB * Hkv * sizeof(unsigned)},
         {(void**)&h->sc.rowstat, MB * Hkv * R * sizeof(float2)},
         {(void**)&h->sc.keys, MB * Hkv * ML * sizeof(uint32_t)},
         {(void**)&h->sc.ubits, MB * W * sizeof(uint32_t)},
         {(void**)&h->sc.ucount, MB * sizeof(unsigned)},
         {(void**)&h->sc.err, sizeof(int)},
+        {(void**)&h->slot.rawO, MB * Hkv * ML * sizeof(float)},
+        {(void**)&h->slot.rawOe, MB * Hkv * ML * sizeof(float)},
+        {(void**)&h->slot.rawI, MB * ML * sizeof(float)},
         {(void**)&h->slot.PO, MB * Hkv * ML * sizeof(float)},
         {(void**)&h->slot.POe, MB * Hkv * ML * sizeof(float)},
         {(void**)&h->slot.I, MB * ML * sizeof(float)},
-        {(void**)&h->slot.sigpart, MB * Hkv * sig_stride * sizeof(float2)},
         {(void**)&h->slot.sigma, MB * Hkv * sizeof(float)},
         {(void**)&h->slot.htop, MB * Hkv * sizeof(int)},
         {(void**)&h->slot.pres, MB * Hkv * W * sizeof(uint32_t)},
@@ -275,9 +286,11 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
         *pt.dst = static_cast<char*>(h->ws) + off;
         off += round_up(pt.bytes, 256);
     }
-    Geometry G = make_geometry(h, 1, p.window, 1, 1);
+    Geometry G = make_geometry(h, 1, p.window, 1, 1, p.window);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device);
     if (e == cudaSuccess) e = configure_score(G);
     if (e == cudaSuccess) e = configure_window(G);
+    if (e == cudaSuccess) e = configure_select();
     if (e == cudaSuccess) e = cudaDeviceSynchronize();
     if (e != cudaSuccess) {
         cudaFree(h->ws);
@@ -353,7 +366,8 @@ kvec_status kvec_select_layers(kvec_handle* h, int num_layers, int batch, const 
     s = set_device(h, &prev);
     if (s != KVEC_OK) return s;
     DeviceGuard guard{prev, h->device};
-    const Geometry G = make_geometry(h, batch, budget, tiles, chunks);
+    Geometry G = make_geometry(h, batch, budget, tiles, chunks, cu_seqlens_host[batch]);
+    G.cu_host = cu_seqlens_host;
     cudaStream_t st = (cudaStream_t)stream;
     for (int l = 0; l < num_layers; ++l) {
         LayerIO io{};
@@ -405,6 +419,7 @@ kvec_status noalloc_setup(int dev, void** base, const Geometry& G) {
         if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(scratch)");
         e = configure_score(G);
         if (e == cudaSuccess) e = configure_window(G);
+        if (e == cudaSuccess) e = configure_select();
         if (e != cudaSuccess) return cuda_fail(e, "kernel attributes");
         d.base = ptr;
         d.ready = true;
@@ -442,24 +457,29 @@ kvec_status kvec_select_layer_noalloc(const kvec_params* params, int batch, cons
         return fail(KVEC_ERR_INVALID_ARG, "device pointers must be 16-byte aligned");
 
     // Carve the scratch for exactly this call's geometry.
-    const size_t nb = batch, ML = params->max_seqlen, Hkv = params->num_kv_heads, R = tmp.R, W = tmp.words;
-    const size_t nt = tiles, sig_stride = ML / kChunk + 1;
+    const size_t nb = batch, ML = round_up((size_t)params->max_seqlen, 32), Hkv = params->num_kv_heads, R = tmp.R,
+                 W = tmp.words;
+    const size_t nt = tiles;
     struct Part {
         void** dst;
         size_t bytes;
     };
     Part parts[] = {
-        {(void**)&tmp.sc.ucount, nb * sizeof(unsigned)},      // zeroed every call (first three parts)
+        {(void**)&tmp.sc.ucount, nb * sizeof(unsigned)},      // zeroed every call (first four parts)
         {(void**)&tmp.sc.err, sizeof(int)},
         {(void**)&tmp.sc.ubits, nb * W * sizeof(uint32_t)},
+        {(void**)&tmp.sc.shcount, nb * Hkv * sizeof(unsigned)},
+        {(void**)&tmp.sc.segpart, nt * Hkv * R * sizeof(float2)},
         {(void**)&tmp.sc.ebuf, nt * Hkv * kTileT * R * sizeof(__half)},
         {(void**)&tmp.sc.tstat, nt * Hkv * R * sizeof(float2)},
         {(void**)&tmp.sc.rowstat, nb * Hkv * R * sizeof(float2)},
         {(void**)&tmp.sc.keys, nb * Hkv * ML * sizeof(uint32_t)},
+        {(void**)&tmp.slot.rawO, nb * Hkv * ML * sizeof(float)},
+        {(void**)&tmp.slot.rawOe, nb * Hkv * ML * sizeof(float)},
+        {(void**)&tmp.slot.rawI, nb * ML * sizeof(float)},
         {(void**)&tmp.slot.PO, nb * Hkv * ML * sizeof(float)},
         {(void**)&tmp.slot.POe, nb * Hkv * ML * sizeof(float)},
         {(void**)&tmp.slot.I, nb * ML * sizeof(float)},
-        {(void**)&tmp.slot.sigpart, nb * Hkv * sig_stride * sizeof(float2)},
         {(void**)&tmp.slot.sigma, nb * Hkv * sizeof(float)},
         {(void**)&tmp.slot.htop, nb * Hkv * sizeof(int)},
         {(void**)&tmp.slot.pres, nb * Hkv * W * sizeof(uint32_t)},
@@ -468,7 +488,7 @@ kvec_status kvec_select_layer_noalloc(const kvec_params* params, int batch, cons
     size_t need = 0, zero_bytes = 0;
     for (size_t i = 0; i < sizeof(parts) / sizeof(parts[0]); ++i) {
         need += round_up(parts[i].bytes, 256);
-        if (i == 2) zero_bytes = need;
+        if (i == 3) zero_bytes = need;
     }
     if (need > kNoallocScratchBytes)
         return fail(KVEC_ERR_INVALID_ARG,
@@ -480,7 +500,10 @@ kvec_status kvec_select_layer_noalloc(const kvec_params* params, int batch, cons
     cudaError_t e = cudaGetDevice(&prev);
     if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
     tmp.device = prev;
-    const Geometry G = make_geometry(&tmp, batch, budget, tiles, chunks);
+    Geometry G = make_geometry(&tmp, batch, budget, tiles, chunks, cu_seqlens_host[batch]);
+    G.cu_host = cu_seqlens_host;
+    e = cudaDeviceGetAttribute(&tmp.num_sms, cudaDevAttrMultiProcessorCount, prev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
     void* base = nullptr;
     s = noalloc_setup(prev, &base, G);
     if (s != KVEC_OK) return s;
@@ -515,7 +538,7 @@ kvec_status kvec_debug_scores(kvec_handle* h, kvec_debug_view* out) {
     out->pres_bits = h->slot.pres;
     out->Pprime = h->slot.Pprime;
     out->row_stats = reinterpret_cast<const float*>(h->sc.rowstat);
-    out->max_seqlen = h->p.max_seqlen;
+    out->max_seqlen = (int)round_up((size_t)h->p.max_seqlen, 32);
     out->words_per_row = h->words;
     return KVEC_OK;
 }

@@ -3,6 +3,7 @@
 
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -10,7 +11,6 @@ namespace kvec {
 
 constexpr int kHeadDim = 128;      // d supported by the score kernel
 constexpr int kTileT = 128;        // tokens per score tile (one MMA N block / e-buffer tile)
-constexpr int kChunk = 64;         // candidate tokens per window/pool CTA
 constexpr int kMaxPool = 15;       // largest pool kernel (halo 7)
 constexpr int kSelectThreads = 1024;
 constexpr float kEScaleLog2 = 15.f;  // e values are stored as fp16(2^15 * exp(s - mu))
@@ -25,17 +25,21 @@ struct Geometry {
     int words;         // ceil(ML / 32)
     int batch, budget, Kp, k2;
     int total_tiles;   // sum over sequences of ceil(L_s / kTileT)
-    int total_chunks;  // sum over sequences of ceil((L_s - w) / kChunk)
+    int total_chunks;  // window-kernel blocks: sum over sequences of window_blocks(L_s - w)
+    int total_tokens;  // cu_seqlens[batch]
+    const int* cu_host;  // host copy of cu_seqlens (host-side planning only; not for device code)
     size_t state_stride;
     size_t state_n_off, state_union_off;
 };
 
 // Device workspace owned by the handle (one slot of per-layer score arrays).
 struct Slot {
+    float* rawO;          // [max_batch][Hkv][ML]  Eq. 1 scores, window O, before pooling
+    float* rawOe;         // [max_batch][Hkv][ML]  window O', before pooling
+    float* rawI;          // [max_batch][ML]       importance, before pooling
     float* PO;            // [max_batch][Hkv][ML]  pooled Eq. 1 scores, window O
     float* POe;           // [max_batch][Hkv][ML]  pooled, window O'
     float* I;             // [max_batch][ML]       pooled importance
-    float2* sigpart;      // [max_batch][Hkv][ML/kChunk+1] (chunk mean, chunk M2)
     float* sigma;         // [max_batch][Hkv]
     int* htop;            // [max_batch][Hkv]
     uint32_t* pres;       // [max_batch][Hkv][words]
@@ -43,8 +47,10 @@ struct Slot {
 };
 
 struct Scratch {
-    __half* ebuf;         // [total_tiles][Hkv][kTileT][R]  scaled exp(s - mu_tile)
+    __half* ebuf;         // [total_tiles][Hkv][R][kTileT]  scaled exp(s - mu_tile), row-major
     float2* tstat;        // [total_tiles][Hkv][R]  (mu_tile in log2 units, sum of exp)
+    float2* segpart;      // [total_tiles * Hkv][R] per-CTA segment (max, sum) keyed by first item
+    unsigned* shcount;    // [max_batch][Hkv]       tiles finished per (sequence, KV head)
     float2* rowstat;      // [max_batch][Hkv][R]    (row max in log2 units, softmax denominator)
     uint32_t* keys;       // [max_batch][Hkv][ML]   radix-select keys
     uint32_t* ubits;      // [max_batch][words]     union of this layer's selections
@@ -85,20 +91,28 @@ __device__ __forceinline__ bool locate_item(int batch, int gi, CountFn count, in
 }
 
 __device__ __forceinline__ int tiles_of(int L) { return (L + kTileT - 1) / kTileT; }
-__device__ __forceinline__ int chunks_of(int Lc) { return Lc > 0 ? (Lc + kChunk - 1) / kChunk : 0; }
 
 // ---------------------------------------------------------------- launchers
 
-void launch_score(const Geometry& g, const LayerIO& io, const Scratch& sc, cudaStream_t st);
-void launch_rowstat(const Geometry& g, const LayerIO& io, const Scratch& sc, cudaStream_t st);
+// Host-side launch description of the score kernel (tensor maps encoded ahead of the launch).
+struct ScorePlan {
+    CUtensorMap kmap, qmap, emap;
+    alignas(16) unsigned char args[512];
+    int grid, threads;
+    size_t smem;
+};
+cudaError_t plan_score(const Geometry& g, const LayerIO& io, const Scratch& sc, int num_sms, ScorePlan* plan);
+cudaError_t launch_score(const ScorePlan& plan, cudaStream_t st);
 void launch_window(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st);
-void launch_heads(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st);
+cudaError_t launch_heads(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st);
 void launch_select(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st);
 void launch_gather(const Geometry& g, const LayerIO& io, cudaStream_t st);
 
 size_t score_smem_bytes(const Geometry& g);
 size_t window_smem_bytes(const Geometry& g);
+int window_blocks(int Lc);
 cudaError_t configure_score(const Geometry& g);
 cudaError_t configure_window(const Geometry& g);
+cudaError_t configure_select();
 
 }  // namespace kvec

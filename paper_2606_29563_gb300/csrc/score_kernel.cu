@@ -1,219 +1,534 @@
-// Window-query scores against every prefix key: s = <q_obs, k_t> for the w
-// observation rows of each query head (Eq. 1's A before normalisation), with the
-// softmax split into per-tile partials (Section 4.1 needs A normalised over all
-// visible keys, so the normalisation is finished by rowstat_kernel).
+// Window-query scores against every prefix key, s = <q_obs, k_t> (the logits of
+// the attention A that Eq. 1 averages), and the softmax over every visible key,
+// split into tile partials that are merged in the same launch.
 //
-// One CTA per (128-token tile, KV head).  The g*w query rows of the KV head
-// (r = q*g + j) form the M side of bf16 tensor-core MMAs, the tile's keys the
-// N side; every accumulator row stays inside one warp, so the tile max and the
-// partial sum need only quad shuffles.  The kernel writes
-//   ebuf[tile][h][t][r] = fp16(2^15 * exp(s - mu_tile,r))   (token-major)
-//   tstat[tile][h][r]   = (mu_tile,r in log2 units, sum_t exp(s - mu_tile,r))
+// Persistent, warp-specialised, one CTA per SM; a CTA walks a contiguous range
+// of work items (sequence s, KV head h, 128-token tile j):
+//   warp 0      TMA producer: the KV head's g*w query rows (once per (s,h)) and
+//               a 3-stage ring of 128-token K tiles, both 128-byte swizzled;
+//   warp 1      one thread issues tcgen05.mma (M = 128 query rows per M-block,
+//               N = 128 tokens, K = 128 = d) into TMEM accumulators;
+//   warps 2..   epilogue, one thread per (query row, half of the tile's
+//               columns): tcgen05.ld of 64 logits, the row's tile max mu (the
+//               two halves exchange partial maxima), e = exp(s - mu) and row
+//               sums; e is packed to fp16(2^15 e), staged row-major in a
+//               128-byte-swizzled tile and written by a TMA tiled store.
+// Outputs: ebuf[tile][h][r][t], tstat[tile][h][r] = (mu in log2 units, sum e),
+// and rowstat[s][h][r] = (row max, softmax denominator) merged from per-CTA
+// segment partials by the last CTA to finish a (s, h).
+#include <cudaTypedefs.h>
+
 #include "kvec_internal.cuh"
+#include "sm100_ptx.cuh"
 
 namespace kvec {
 
 namespace {
 
-constexpr int kRowBytes = 272;  // 128 bf16 + 16 B pad: conflict-free ldmatrix rows
+constexpr int kKStages = 3;                           // deepest K ring (2 when shared memory is short)
+constexpr int kMaxSmem = 232448;                      // opt-in shared memory per CTA on sm_103
+constexpr int kKStageBytes = kTileT * kHeadDim * 2;   // 32 KB: two 64-column swizzled halves
+constexpr int kKHalfBytes = kTileT * 128;             // 16 KB
+constexpr uint32_t kTmemCols = 512;
 
-__device__ __forceinline__ void cp_async16(void* smem, const void* gmem, int src_bytes) {
-    uint32_t s = static_cast<uint32_t>(__cvta_generic_to_shared(smem));
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(s), "l"(gmem), "r"(src_bytes));
-}
+struct ItemPos {
+    int s, h, j, gt, ibase, ntiles;  // ibase: first item of (s, h)
+};
 
-__device__ __forceinline__ void ldmatrix_x4(uint32_t* r, const void* p) {
-    uint32_t a = static_cast<uint32_t>(__cvta_generic_to_shared(p));
-    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
-                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-                 : "r"(a));
-}
-
-__device__ __forceinline__ void mma_bf16_16816(float* c, const uint32_t* a, uint32_t b0, uint32_t b1) {
-    asm volatile(
-        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
-        "{%0,%1,%2,%3};\n"
-        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
-
-__global__ void __launch_bounds__(512, 1) score_kernel(Geometry G, LayerIO io, Scratch sc) {
-    extern __shared__ __align__(128) uint8_t smem[];
-    const int h = blockIdx.y;
-    const int gt = blockIdx.x;
-    int s, j, tbase;
-    if (!locate_item(G.batch, gt, [&](int b) { return tiles_of(io.cu[b + 1] - io.cu[b]); }, s, j, tbase))
-        return;
-    const int L = io.cu[s + 1] - io.cu[s];
-    const int t0 = j * kTileT;
-    const int R = G.R;
-    const int R16 = (R + 15) & ~15;
-    uint8_t* sQ = smem;
-    uint8_t* sK = smem + (size_t)R16 * kRowBytes;
-    const int tid = threadIdx.x, nthr = blockDim.x;
-
-    for (int i = tid; i < R16 * 16; i += nthr) {
-        const int r = i >> 4, c = i & 15;
-        const __nv_bfloat16* src = io.q;
-        int bytes = 0;
-        if (r < R) {
-            const int q = r / G.g, jj = r - q * G.g;
-            src = io.q + (((size_t)s * G.w + q) * G.Hq + h * G.g + jj) * kHeadDim + c * 8;
-            bytes = 16;
+// Items are ordered (s, h, j); sequence s owns ntiles(s) * Hkv consecutive items.
+template <class Cu>
+__device__ __forceinline__ ItemPos decode_item(const Cu& cu, int batch, int Hkv, int i) {
+    ItemPos p{};
+    int ibase = 0, tbase = 0;
+    for (int b = 0; b < batch; ++b) {
+        const int nt = tiles_of(cu[b + 1] - cu[b]);
+        if (i < ibase + nt * Hkv) {
+            const int local = i - ibase;
+            p.s = b;
+            p.h = local / nt;
+            p.j = local - p.h * nt;
+            p.gt = tbase + p.j;
+            p.ibase = ibase + p.h * nt;
+            p.ntiles = nt;
+            return p;
         }
-        cp_async16(sQ + r * kRowBytes + c * 16, src, bytes);
+        ibase += nt * Hkv;
+        tbase += nt;
     }
-    for (int i = tid; i < kTileT * 16; i += nthr) {
-        const int t = i >> 4, c = i & 15;
-        const __nv_bfloat16* src = io.k;
-        int bytes = 0;
-        if (t0 + t < L) {
-            src = io.k + (((size_t)io.cu[s] + t0 + t) * G.Hkv + h) * kHeadDim + c * 8;
-            bytes = 16;
+    return p;
+}
+
+// CTA b of G owns items [start(b), start(b+1)) with start(b) = b*q + min(b, r), W = q*G + r.
+__device__ __forceinline__ int range_start(int b, int W, int G) {
+    const int q = W / G, r = W % G;
+    return b * q + min(b, r);
+}
+
+constexpr int kMaxCuParam = 64;   // sequences whose offsets travel in the kernel parameters
+
+struct ScoreArgs {
+    Geometry G;
+    const int* cu;                 // device cu_seqlens
+    int cuv[kMaxCuParam + 1];      // the same offsets (when batch <= kMaxCuParam)
+    const uint8_t* kbytes;         // the layer's K, for the L2 prefetch
+    long long kbytes_total;
+    Scratch sc;
+    int W;        // total work items
+    int MB;       // 128-row M-blocks per KV head (1 or 2)
+    int Rpad;     // 128 * MB
+    int ebufs;    // e staging buffers (2 when MB == 1)
+    int kst;      // K ring depth
+};
+
+struct __align__(8) Barriers {
+    uint64_t k_full[kKStages], k_empty[kKStages];
+    uint64_t q_full, q_empty;
+    uint64_t acc_full[4], acc_empty[4];
+    uint64_t mma_done;
+    uint32_t tmem_base;
+    volatile int abort_flag;
+    volatile int last_flag;
+    volatile int go;
+    float zhalf[256];          // row sums of the second column half
+    float pmax[2][256];        // per-half row maxima of the current tile
+};
+
+__device__ __forceinline__ void raise_abort(Barriers* bars, int* err) {
+    bars->abort_flag = 1;
+    atomicExch(err, 3);
+}
+
+__global__ void __launch_bounds__(576, 1)
+    score_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap qmap,
+                 const __grid_constant__ CUtensorMap emap, const __grid_constant__ ScoreArgs A) {
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    // 1024-byte alignment for the swizzled operand tiles.
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const Geometry& G = A.G;
+    const int MB = A.MB, Rpad = A.Rpad, R = G.R;
+    uint8_t* sQ = smem;                                   // 2 halves x Rpad rows x 128 B
+    uint8_t* sK = sQ + 2 * Rpad * 128;                    // A.kst x 32 KB
+    uint8_t* sE = sK + A.kst * kKStageBytes;           // ebufs x 2 halves x R rows x 128 B (swizzled)
+    const int ebytes = kTileT * R * 2;
+    Barriers* bars = reinterpret_cast<Barriers*>(sE + A.ebufs * ebytes);
+
+    const bool cu_param = G.batch <= kMaxCuParam;
+    auto cu = [&](int b) { return cu_param ? A.cuv[b] : A.cu[b]; };
+    struct CuView {
+        decltype(cu)& f;
+        __device__ int operator[](int b) const { return f(b); }
+    } cuview{cu};
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int nepi = 8 * MB * 32;                          // epilogue threads: 2 column halves x MB x 4 quads
+    const int NB = 4 / MB;                                 // TMEM accumulator buffers
+    const int Gc = gridDim.x;
+    const int i0 = range_start(blockIdx.x, A.W, Gc), i1 = range_start(blockIdx.x + 1, A.W, Gc);
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < A.kst; ++s) {
+            ptx::mbar_init(&bars->k_full[s], 1);
+            ptx::mbar_init(&bars->k_empty[s], 1);
         }
-        cp_async16(sK + t * kRowBytes + c * 16, src, bytes);
+        ptx::mbar_init(&bars->q_full, 1);
+        ptx::mbar_init(&bars->q_empty, 1);
+        for (int b = 0; b < 4; ++b) {
+            ptx::mbar_init(&bars->acc_full[b], 1);
+            ptx::mbar_init(&bars->acc_empty[b], 8 * MB);  // one arrival per epilogue warp
+        }
+        ptx::mbar_init(&bars->mma_done, 1);
+        bars->abort_flag = 0;
+        ptx::fence_barrier_init();
     }
-    asm volatile("cp.async.commit_group;\n");
-    asm volatile("cp.async.wait_all;\n" ::: "memory");
+    if (warp == 1) {
+        ptx::tmem_alloc(&bars->tmem_base, kTmemCols);
+        ptx::tmem_relinquish();
+    }
+    if (warp == 0 && lane == 0) {
+        ptx::prefetch_tensormap(&kmap);
+        ptx::prefetch_tensormap(&qmap);
+        ptx::prefetch_tensormap(&emap);
+    }
+    ptx::tc_fence_before();
     __syncthreads();
+    ptx::tc_fence_after();
+    const uint32_t tmem = bars->tmem_base;
 
-    const int warp = tid >> 5, lane = tid & 31;
-    const int r0 = warp * 16;
-    uint32_t a[8][4];
-#pragma unroll
-    for (int ks = 0; ks < 8; ++ks)
-        ldmatrix_x4(a[ks], sQ + (r0 + (lane & 7) + ((lane >> 3) & 1) * 8) * kRowBytes + (ks * 16 + (lane >> 4) * 8) * 2);
-
-    float acc[16][4];
-#pragma unroll
-    for (int n = 0; n < 16; ++n) acc[n][0] = acc[n][1] = acc[n][2] = acc[n][3] = 0.f;
-#pragma unroll
-    for (int np = 0; np < 8; ++np) {
-#pragma unroll
-        for (int ks = 0; ks < 8; ++ks) {
-            uint32_t b[4];
-            ldmatrix_x4(b, sK + (np * 16 + (lane & 7) + (lane >> 4) * 8) * kRowBytes +
-                               (ks * 16 + ((lane >> 3) & 1) * 8) * 2);
-            mma_bf16_16816(acc[2 * np], a[ks], b[0], b[1]);
-            mma_bf16_16816(acc[2 * np + 1], a[ks], b[2], b[3]);
-        }
-    }
-    __syncthreads();  // Q and K tiles are dead: the e-tile reuses their shared memory
-
-    const int gid = lane >> 2, tq = lane & 3;
-    const int rA = r0 + gid, rB = rA + 8;
-    // Last key visible to a row: causal for the window part (row q sits at L - w + q).
-    const int lastA = rA < R ? min(L - 1, L - G.w + rA / G.g) : -1;
-    const int lastB = rB < R ? min(L - 1, L - G.w + rB / G.g) : -1;
-    float mA = -INFINITY, mB = -INFINITY;
-#pragma unroll
-    for (int n = 0; n < 16; ++n)
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-            const int tok = t0 + n * 8 + 2 * tq + e;
-            if (tok <= lastA) mA = fmaxf(mA, acc[n][e]);
-            if (tok <= lastB) mB = fmaxf(mB, acc[n][2 + e]);
-        }
-    mA = fmaxf(mA, __shfl_xor_sync(0xffffffffu, mA, 1));
-    mA = fmaxf(mA, __shfl_xor_sync(0xffffffffu, mA, 2));
-    mB = fmaxf(mB, __shfl_xor_sync(0xffffffffu, mB, 1));
-    mB = fmaxf(mB, __shfl_xor_sync(0xffffffffu, mB, 2));
-    const float muA = mA * G.sl2, muB = mB * G.sl2;  // -inf when no key of the tile is visible
-    __half* sE = reinterpret_cast<__half*>(smem);    // [kTileT][R]
-    float zA = 0.f, zB = 0.f;
-#pragma unroll
-    for (int n = 0; n < 16; ++n)
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-            const int tl = n * 8 + 2 * tq + e;
-            const int tok = t0 + tl;
-            const float eA = tok <= lastA ? exp2f(fmaf(acc[n][e], G.sl2, -muA)) : 0.f;
-            const float eB = tok <= lastB ? exp2f(fmaf(acc[n][2 + e], G.sl2, -muB)) : 0.f;
-            zA += eA;
-            zB += eB;
-            if (rA < R) sE[tl * R + rA] = __float2half_rn(eA * 32768.f);
-            if (rB < R) sE[tl * R + rB] = __float2half_rn(eB * 32768.f);
-        }
-    zA += __shfl_xor_sync(0xffffffffu, zA, 1);
-    zA += __shfl_xor_sync(0xffffffffu, zA, 2);
-    zB += __shfl_xor_sync(0xffffffffu, zB, 1);
-    zB += __shfl_xor_sync(0xffffffffu, zB, 2);
-    float2* ts = sc.tstat + ((size_t)gt * G.Hkv + h) * R;
-    if (tq == 0) {
-        if (rA < R) ts[rA] = make_float2(muA, zA);
-        if (rB < R) ts[rB] = make_float2(muB, zB);
-    }
-    __syncthreads();
-    const uint4* src = reinterpret_cast<const uint4*>(sE);
-    uint4* dst = reinterpret_cast<uint4*>(sc.ebuf + ((size_t)gt * G.Hkv + h) * kTileT * R);
-    const int n16 = kTileT * R / 8;
-    for (int i = tid; i < n16; i += nthr) dst[i] = src[i];
-}
-
-// Merges the per-tile (mu, z) partials of every window row into the row's
-// softmax max and denominator.  Grid (ceil(R/32), Hkv, batch), 256 threads:
-// a lane owns a row, the 8 warps stride over tiles, shared memory combines them.
-__global__ void __launch_bounds__(256) rowstat_kernel(Geometry G, LayerIO io, Scratch sc) {
-    __shared__ float2 part[8][32];
-    const int s = blockIdx.z, h = blockIdx.y;
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int r = blockIdx.x * 32 + lane;
-    int tbase = 0;
-    for (int b = 0; b < s; ++b) tbase += tiles_of(io.cu[b + 1] - io.cu[b]);
-    const int nt = tiles_of(io.cu[s + 1] - io.cu[s]);
-    float m = -INFINITY, z = 0.f;
-    if (r < G.R) {
-        for (int jt = warp; jt < nt; jt += 8) {
-            const float2 t = sc.tstat[((size_t)(tbase + jt) * G.Hkv + h) * G.R + r];
-            if (t.x == -INFINITY) continue;
-            if (t.x > m) {
-                z = z * exp2f(m - t.x) + t.y;
-                m = t.x;
-            } else {
-                z += t.y * exp2f(t.x - m);
+    if (warp == 0) {
+        // ------------------------------------------------------------ TMA producer
+        if (lane == 0) {
+            // Stream this CTA's contiguous slice of the layer's K into L2 first: DRAM then
+            // sees sequential reads, and the strided per-head tiles below hit in L2.
+            {
+                const long long per = ((A.kbytes_total / Gc) + 15) & ~15LL;
+                long long lo = per * blockIdx.x, hi = lo + per;
+                if (hi > A.kbytes_total) hi = A.kbytes_total;
+                for (long long o = lo; o < hi; o += 32768) {
+                    const long long n = hi - o < 32768 ? hi - o : 32768;
+                    ptx::prefetch_l2_bulk(A.kbytes + o, (uint32_t)(n & ~15LL));
+                }
             }
+            const uint64_t policy = ptx::policy_evict_first();
+            int prev_sh = -1, qloads = 0;
+            int fills[kKStages] = {0, 0, 0};
+            for (int i = i0, it = 0; i < i1 && !bars->abort_flag; ++i, ++it) {
+                const ItemPos p = decode_item(cuview, G.batch, G.Hkv, i);
+                const int sh = p.s * G.Hkv + p.h;
+                if (sh != prev_sh) {
+                    if (qloads > 0 && !ptx::mbar_wait(&bars->q_empty, (qloads - 1) & 1)) {
+                        raise_abort(bars, A.sc.err);
+                        break;
+                    }
+                    ptx::mbar_arrive_expect_tx(&bars->q_full, 2u * R * 128u);
+                    ptx::tma_load_4d(sQ, &qmap, &bars->q_full, 0, p.h * G.g, 0, p.s);
+                    ptx::tma_load_4d(sQ + Rpad * 128, &qmap, &bars->q_full, 64, p.h * G.g, 0, p.s);
+                    ++qloads;
+                    prev_sh = sh;
+                }
+                const int st = it % A.kst, n = it / A.kst;
+                if (n > 0 && !ptx::mbar_wait(&bars->k_empty[st], (n - 1) & 1)) {
+                    raise_abort(bars, A.sc.err);
+                    break;
+                }
+                uint8_t* dst = sK + st * kKStageBytes;
+                const int row = cu(p.s) + p.j * kTileT;
+                ptx::mbar_arrive_expect_tx(&bars->k_full[st], (uint32_t)kKStageBytes);
+                ptx::tma_load_3d(dst, &kmap, &bars->k_full[st], 0, p.h, row, policy);
+                ptx::tma_load_3d(dst + kKHalfBytes, &kmap, &bars->k_full[st], 64, p.h, row, policy);
+                ++fills[st];
+            }
+            // Drain: every issued copy lands before the CTA may exit.
+            for (int st = 0; st < A.kst; ++st)
+                if (fills[st] > 0) ptx::mbar_wait(&bars->k_full[st], (fills[st] - 1) & 1, 50000000ull);
+            if (qloads > 0) ptx::mbar_wait(&bars->q_full, (qloads - 1) & 1, 50000000ull);
         }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            const uint32_t idesc = ptx::idesc_bf16_f32(128, kTileT);
+            const uint32_t sQa = ptx::smem_u32(sQ), sKa = ptx::smem_u32(sK);
+            int prev_sh = -1, qk = 0;
+            for (int i = i0, it = 0; i < i1 && !bars->abort_flag; ++i, ++it) {
+                const ItemPos p = decode_item(cuview, G.batch, G.Hkv, i);
+                const int sh = p.s * G.Hkv + p.h;
+                if (sh != prev_sh) {
+                    if (!ptx::mbar_wait(&bars->q_full, qk & 1)) {
+                        raise_abort(bars, A.sc.err);
+                        break;
+                    }
+                    ++qk;
+                    prev_sh = sh;
+                }
+                const int st = it % A.kst, n = it / A.kst;
+                const int buf = it % NB, nb = it / NB;
+                if (!ptx::mbar_wait(&bars->k_full[st], n & 1) ||
+                    (nb > 0 && !ptx::mbar_wait(&bars->acc_empty[buf], (nb - 1) & 1))) {
+                    raise_abort(bars, A.sc.err);
+                    break;
+                }
+                ptx::tc_fence_after();
+                const uint32_t kst = sKa + st * kKStageBytes;
+                for (int m = 0; m < MB; ++m) {
+                    const uint32_t d = tmem + (uint32_t)(buf * 128 * MB + m * 128);
+#pragma unroll
+                    for (int kk = 0; kk < 8; ++kk) {
+                        const int half = kk >> 2, kin = kk & 3;
+                        const uint64_t ad = ptx::smem_desc_k_sw128(sQa + half * Rpad * 128 + m * 16384 + kin * 32);
+                        const uint64_t bd = ptx::smem_desc_k_sw128(kst + half * kKHalfBytes + kin * 32);
+                        ptx::mma_bf16(d, ad, bd, idesc, kk > 0 ? 1u : 0u);
+                    }
+                }
+                ptx::mma_commit(&bars->k_empty[st]);
+                ptx::mma_commit(&bars->acc_full[buf]);
+                bool q_done = i + 1 >= i1;
+                if (!q_done) {
+                    const ItemPos nx = decode_item(cuview, G.batch, G.Hkv, i + 1);
+                    q_done = nx.s * G.Hkv + nx.h != sh;
+                }
+                if (q_done) ptx::mma_commit(&bars->q_empty);
+            }
+            ptx::mma_commit(&bars->mma_done);
+        }
+    } else if (warp < 2 + 8 * MB) {
+        // ------------------------------------------------------------ epilogue
+        const int epi = threadIdx.x - 64;                   // 0 .. nepi-1
+        const int ew = warp - 2;
+        const int m = (ew >> 2) % MB;                       // M-block of this warp
+        const int half = (ew >> 2) / MB;                    // column half: tokens [64*half, 64*half + 64)
+        const int quad = warp & 3;                          // TMEM lanes 32*quad .. +31
+        const int row = m * 128 + quad * 32 + lane;
+        const bool vrow = row < R;
+        const int q = vrow ? row / G.g : 0;
+        const bool issuer = epi == 0;
+        bool aborted = false;
+        float seg_m = -INFINITY, seg_z = 0.f;
+        int cur_sh = -1, seg_first = 0, seg_n = 0, seg_s = 0, seg_h = 0, seg_ibase = 0, seg_nt = 0;
+
+        auto flush_segment = [&]() {
+            if (vrow && half == 0) A.sc.segpart[(size_t)seg_first * R + row] = make_float2(seg_m, seg_z);
+            ptx::named_bar_sync(1, nepi);
+            if (issuer) {
+                // The barrier orders the CTA's writes before this thread's fence (cumulativity).
+                __threadfence();
+                const unsigned old = atomicAdd(&A.sc.shcount[seg_s * G.Hkv + seg_h], (unsigned)seg_n);
+                __threadfence();
+                bars->last_flag = old + (unsigned)seg_n == (unsigned)seg_nt;
+            }
+            ptx::named_bar_sync(1, nepi);
+            if (bars->last_flag && half == 0) {
+                // Gather the segment starts of (s, h), then load them in independent batches.
+                float M = -INFINITY, Z = 0.f;
+                // Segment starts of (s, h): its first item and every CTA range start after it.
+                const int qW = A.W / Gc, rW = A.W % Gc;
+                const int iend = seg_ibase + seg_nt;
+                auto cta_of = [&](int i) { return i < rW * (qW + 1) ? i / (qW + 1) : rW + (i - rW * (qW + 1)) / qW; };
+                int b = cta_of(seg_ibase) + 1;
+                int next = seg_ibase;
+                while (next < iend) {
+                    float2 pz[16];
+                    int n = 0;
+#pragma unroll
+                    for (int k = 0; k < 16; ++k) {
+                        pz[k] = make_float2(-INFINITY, 0.f);
+                        if (next < iend) {
+                            if (vrow) pz[k] = __ldcg(&A.sc.segpart[(size_t)next * R + row]);
+                            next = b * qW + min(b, rW);
+                            ++b;
+                            ++n;
+                        }
+                    }
+#pragma unroll
+                    for (int k = 0; k < 16; ++k) {
+                        if (pz[k].x == -INFINITY) continue;
+                        if (pz[k].x > M) {
+                            Z = Z * ptx::ex2(M - pz[k].x) + pz[k].y;
+                            M = pz[k].x;
+                        } else {
+                            Z += pz[k].y * ptx::ex2(pz[k].x - M);
+                        }
+                    }
+                }
+                if (vrow) A.sc.rowstat[((size_t)seg_s * G.Hkv + seg_h) * R + row] = make_float2(M, Z);
+                if (issuer) A.sc.shcount[seg_s * G.Hkv + seg_h] = 0u;
+            }
+        };
+
+        for (int i = i0, it = 0; i < i1; ++i, ++it) {
+            const ItemPos p = decode_item(cuview, G.batch, G.Hkv, i);
+            const int sh = p.s * G.Hkv + p.h;
+            if (sh != cur_sh) {
+                if (cur_sh >= 0) flush_segment();
+                cur_sh = sh;
+                seg_m = -INFINITY;
+                seg_z = 0.f;
+                seg_first = i;
+                seg_n = 0;
+                seg_s = p.s;
+                seg_h = p.h;
+                seg_ibase = p.ibase;
+                seg_nt = p.ntiles;
+            }
+            const int buf = it % NB, nb = it / NB;
+            // One thread waits for the accumulator and for the staging buffer, then
+            // publishes the outcome; every epilogue thread takes the same branch.
+            if (issuer) {
+                const bool ok = !bars->abort_flag && ptx::mbar_wait(&bars->acc_full[buf], nb & 1);
+                if (!ok) raise_abort(bars, A.sc.err);
+                if (A.ebufs == 2)
+                    asm volatile("cp.async.bulk.wait_group.read 1;\n" ::: "memory");
+                else
+                    ptx::bulk_wait_read_all();
+                bars->go = ok ? 1 : 0;
+            }
+            ptx::named_bar_sync(1, nepi);
+            if (!bars->go) {
+                aborted = true;
+                break;
+            }
+            ptx::tc_fence_after();
+            const uint32_t taddr = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(buf * 128 * MB + m * 128);
+            const int L = cu(p.s + 1) - cu(p.s);
+            const int t0 = p.j * kTileT;
+            const int last = vrow ? min(L - 1, L - G.w + q) : -1;   // causal on the window part
+            const int nvalid = max(0, min(kTileT, last - t0 + 1));
+            // This warp's 64 columns of the accumulator; the row max is combined across the halves.
+            const int c0 = half * 64;
+            float v[64];
+            ptx::tmem_ld32(taddr + c0, v);
+            ptx::tmem_ld32(taddr + c0 + 32, v + 32);
+            ptx::tmem_wait_ld();
+            ptx::tc_fence_before();
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(&bars->acc_empty[buf]);
+            const int lim = nvalid - c0;
+            float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+            if (lim >= 64) {
+#pragma unroll
+                for (int c = 0; c < 64; ++c) m4[c & 3] = fmaxf(m4[c & 3], v[c]);
+            } else {
+#pragma unroll
+                for (int c = 0; c < 64; ++c)
+                    if (c < lim) m4[c & 3] = fmaxf(m4[c & 3], v[c]);
+            }
+            bars->pmax[half][row] = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
+            ptx::named_bar_sync(1, nepi);
+            const float mx = fmaxf(bars->pmax[0][row], bars->pmax[1][row]);
+            const float mu = mx * G.sl2;                           // -inf when nothing is visible
+            const float bias = kEScaleLog2 - mu;                   // stores 2^15 * exp(s - mu)
+            const int eb = A.ebufs == 2 ? (it & 1) : 0;
+            // Row-major staging [half][row][64 tokens], 16-byte chunk k of a row at chunk k ^ (row % 8)
+            // (the tensor map's 128-byte swizzle).
+            const uint32_t srow = ptx::smem_u32(sE + eb * ebytes + half * (R * 128)) + (uint32_t)(row * 128);
+            float z4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                float e[8];
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const int c = k * 8 + i;
+                    e[i] = (lim >= 64 || c < lim) ? ptx::ex2(fmaf(v[c], G.sl2, bias)) : 0.f;
+                    z4[i & 3] += e[i];
+                }
+                if (vrow)
+                    ptx::st_shared_v4(srow + (uint32_t)((k ^ (row & 7)) * 16), ptx::pack_half2(e[0], e[1]),
+                                      ptx::pack_half2(e[2], e[3]), ptx::pack_half2(e[4], e[5]),
+                                      ptx::pack_half2(e[6], e[7]));
+            }
+            float z = ((z4[0] + z4[1]) + (z4[2] + z4[3])) * (1.f / 32768.f);
+            if (half == 1) bars->zhalf[row] = z;
+            ptx::fence_proxy_async_smem();
+            ptx::named_bar_sync(1, nepi);
+            if (issuer) {
+                const int erow0 = (p.gt * G.Hkv + p.h) * R;
+                ptx::tma_store_2d(&emap, sE + eb * ebytes, 0, erow0);
+                ptx::tma_store_2d(&emap, sE + eb * ebytes + R * 128, 64, erow0);
+                ptx::bulk_commit();
+            }
+            if (half == 1) continue;                               // sums and statistics live in half 0
+            z += bars->zhalf[row];
+            if (vrow) A.sc.tstat[((size_t)p.gt * G.Hkv + p.h) * R + row] = make_float2(mu, z);
+            if (mu != -INFINITY) {
+                if (mu > seg_m) {
+                    seg_z = seg_z * ptx::ex2(seg_m - mu) + z;
+                    seg_m = mu;
+                } else {
+                    seg_z += z * ptx::ex2(mu - seg_m);
+                }
+            }
+            ++seg_n;
+        }
+        if (cur_sh >= 0 && !aborted) flush_segment();
+        if (issuer) ptx::bulk_wait_all();
     }
-    part[warp][lane] = make_float2(m, z);
+
+    // ---------------------------------------------------------------- teardown
+    if (warp == 1 && lane == 0) ptx::mbar_wait(&bars->mma_done, 0, 50000000ull);
+    ptx::tc_fence_before();
     __syncthreads();
-    if (warp == 0 && r < G.R) {
-        float M = -INFINITY;
-        for (int w8 = 0; w8 < 8; ++w8) M = fmaxf(M, part[w8][lane].x);
-        float Z = 0.f;
-        for (int w8 = 0; w8 < 8; ++w8)
-            if (part[w8][lane].x != -INFINITY) Z += part[w8][lane].y * exp2f(part[w8][lane].x - M);
-        sc.rowstat[((size_t)s * G.Hkv + h) * G.R + r] = make_float2(M, Z);
-    }
+    ptx::tc_fence_after();
+    if (warp == 1) ptx::tmem_dealloc(tmem, kTmemCols);
 }
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    if (!fn) {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    }
+    return fn;
+}
+
+int mblocks(const Geometry& g) { return g.R > 128 ? 2 : 1; }
+
+size_t smem_bytes_with(const Geometry& g, int kst) {
+    const int MB = mblocks(g);
+    const int ebufs = MB == 1 ? 2 : 1;
+    return 1024 + 2 * (size_t)MB * 128 * 128 + (size_t)kst * kKStageBytes + (size_t)ebufs * kTileT * g.R * 2 +
+           sizeof(Barriers);
+}
+
+int kstages_for(const Geometry& g) { return smem_bytes_with(g, kKStages) <= (size_t)kMaxSmem ? kKStages : 2; }
+
+size_t smem_bytes_for(const Geometry& g) { return smem_bytes_with(g, kstages_for(g)); }
 
 }  // namespace
 
-size_t score_smem_bytes(const Geometry& g) {
-    const int R16 = (g.R + 15) & ~15;
-    size_t mma = (size_t)(R16 + kTileT) * kRowBytes;
-    size_t etile = (size_t)kTileT * g.R * sizeof(__half);
-    return mma > etile ? mma : etile;
-}
+size_t score_smem_bytes(const Geometry& g) { return smem_bytes_for(g); }
 
 cudaError_t configure_score(const Geometry& g) {
-    // The attribute is per function, shared by every handle: request the largest
-    // size any supported geometry (rows per KV head <= 256) can need.
-    Geometry widest = g;
-    widest.R = 256;
-    size_t need = score_smem_bytes(widest);
-    if (score_smem_bytes(g) > need) need = score_smem_bytes(g);
+    // Per-function attribute shared by every handle: the largest supported geometry.
+    size_t need = 0;
+    for (int R = 8; R <= 256; R += 8) {
+        Geometry gr = g;
+        gr.R = R;
+        if (smem_bytes_for(gr) > need) need = smem_bytes_for(gr);
+    }
     return cudaFuncSetAttribute(score_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)need);
 }
 
-void launch_score(const Geometry& g, const LayerIO& io, const Scratch& sc, cudaStream_t st) {
-    const int R16 = (g.R + 15) & ~15;
-    dim3 grid(g.total_tiles, g.Hkv);
-    score_kernel<<<grid, (R16 / 16) * 32, score_smem_bytes(g), st>>>(g, io, sc);
+cudaError_t plan_score(const Geometry& g, const LayerIO& io, const Scratch& sc, int num_sms, ScorePlan* plan) {
+    PFN_cuTensorMapEncodeTiled_v12000 enc = encode_fn();
+    if (!enc) return cudaErrorNotSupported;
+    CUtensorMap& kmap = plan->kmap;
+    CUtensorMap& qmap = plan->qmap;
+    {
+        cuuint64_t dims[3] = {(cuuint64_t)kHeadDim, (cuuint64_t)g.Hkv, (cuuint64_t)g.total_tokens};
+        cuuint64_t strides[2] = {(cuuint64_t)kHeadDim * 2, (cuuint64_t)g.Hkv * kHeadDim * 2};
+        cuuint32_t box[3] = {64, 1, (cuuint32_t)kTileT};
+        cuuint32_t es[3] = {1, 1, 1};
+        if (enc(&kmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<__nv_bfloat16*>(io.k), dims, strides, box, es,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+    }
+    {
+        cuuint64_t dims[4] = {(cuuint64_t)kHeadDim, (cuuint64_t)g.Hq, (cuuint64_t)g.w, (cuuint64_t)g.batch};
+        cuuint64_t strides[3] = {(cuuint64_t)kHeadDim * 2, (cuuint64_t)g.Hq * kHeadDim * 2,
+                                 (cuuint64_t)g.w * g.Hq * kHeadDim * 2};
+        cuuint32_t box[4] = {64, (cuuint32_t)g.g, (cuuint32_t)g.w, 1};
+        cuuint32_t es[4] = {1, 1, 1, 1};
+        if (enc(&qmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<__nv_bfloat16*>(io.q), dims, strides, box, es,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+    }
+    {
+        cuuint64_t dims[2] = {(cuuint64_t)kTileT, (cuuint64_t)g.total_tiles * g.Hkv * g.R};
+        cuuint64_t strides[1] = {(cuuint64_t)kTileT * 2};
+        cuuint32_t box[2] = {64, (cuuint32_t)g.R};
+        cuuint32_t es[2] = {1, 1};
+        if (enc(&plan->emap, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, sc.ebuf, dims, strides, box, es,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+    }
+    ScoreArgs& a = *reinterpret_cast<ScoreArgs*>(plan->args);
+    static_assert(sizeof(ScoreArgs) <= sizeof(plan->args), "ScorePlan::args too small");
+    a = ScoreArgs{};
+    a.G = g;
+    a.cu = io.cu;
+    for (int b = 0; b <= g.batch && b <= kMaxCuParam; ++b) a.cuv[b] = g.cu_host ? g.cu_host[b] : 0;
+    a.kbytes = reinterpret_cast<const uint8_t*>(io.k);
+    a.kbytes_total = (long long)g.total_tokens * g.Hkv * kHeadDim * 2;
+    a.sc = sc;
+    a.W = g.total_tiles * g.Hkv;
+    a.MB = mblocks(g);
+    a.Rpad = 128 * a.MB;
+    a.ebufs = a.MB == 1 ? 2 : 1;
+    a.kst = kstages_for(g);
+    plan->grid = a.W < num_sms ? a.W : num_sms;
+    plan->threads = 32 * (2 + 8 * a.MB);
+    plan->smem = smem_bytes_for(g);
+    return cudaSuccess;
 }
 
-void launch_rowstat(const Geometry& g, const LayerIO& io, const Scratch& sc, cudaStream_t st) {
-    dim3 grid((g.R + 31) / 32, g.Hkv, g.batch);
-    rowstat_kernel<<<grid, 256, 0, st>>>(g, io, sc);
+cudaError_t launch_score(const ScorePlan& plan, cudaStream_t st) {
+    score_kernel<<<plan.grid, plan.threads, plan.smem, st>>>(plan.kmap, plan.qmap, plan.emap,
+                                                              *reinterpret_cast<const ScoreArgs*>(plan.args));
+    return cudaGetLastError();
 }
 
 }  // namespace kvec

@@ -5,11 +5,19 @@
 // Top-k is an exact block-wide MSB radix select over order-preserving uint32
 // keys (11/11/10-bit digits, shared-memory histograms, block scans built from
 // warp shuffles and ballots).  Ties at the threshold go to the lower position.
+#include <cooperative_groups.h>
+
 #include "kvec_internal.cuh"
+
+namespace cg = cooperative_groups;
 
 namespace kvec {
 
 namespace {
+
+constexpr int kSmemKeys = 40960;   // positions whose keys fit in shared memory (160 KB)
+
+__host__ __device__ inline bool keys_in_smem(int ML) { return ML <= kSmemKeys; }
 
 struct TopkShared {
     int hist[2048];
@@ -125,60 +133,118 @@ __device__ __forceinline__ uint32_t range_bits(int word, int lo, int hi) {
     return upto & ~((1u << a) - 1u);
 }
 
-// Section 4.1: sigma of every head (Chan merge of chunk statistics), the delta
-// lowest-sigma heads take the O' scores; then the top-K preserved tokens by P
-// (Section 4.2).  Grid (Hkv, batch).
+// Max-pool width `2*halo+1` over [0, Lc) of one row: the output positions
+// [c0, c0+n) are staged with their halo in shared memory first.
+__device__ void pool_chunk(const float* __restrict__ raw, float* __restrict__ out, int c0, int n, int Lc, int halo,
+                           float* stage) {
+    const int lo = max(c0 - halo, 0), hi = min(c0 + n + halo, Lc);
+    for (int t = lo + threadIdx.x; t < hi; t += blockDim.x) stage[t - lo] = __ldcg(raw + t);
+    __syncthreads();
+    for (int t = c0 + threadIdx.x; t < c0 + n; t += blockDim.x) {
+        const int a = max(t - halo, 0) - lo, b = min(t + halo, Lc - 1) - lo;
+        float m = stage[a];
+        for (int x = a + 1; x <= b; ++x) m = fmaxf(m, stage[x]);
+        out[t] = m;
+    }
+    __syncthreads();
+}
+
+__device__ double block_sum(double v, double* red) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    for (int off = 16; off; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+    if (lane == 0) red[warp] = v;
+    __syncthreads();
+    double t = 0.0;
+    for (int i = 0; i < nw; ++i) t += red[i];
+    __syncthreads();
+    return t;
+}
+
+constexpr int kPoolChunk = 4096;
+
+// Section 4.1 and the preserved tokens of Section 4.2.  One thread-block
+// cluster per sequence, one CTA per KV head (cluster rank = head):
+//   pool the head's P_O and P_O' rows and a slice of I (max-pool, inherited
+//   from SnapKV), sigma_h = sample std of pooled P_O over the candidates (two
+//   passes, fp64 sums), exchange sigma through distributed shared memory, the
+//   delta lowest-sigma heads take the O' scores, then the top-K preserved
+//   tokens of the chosen row by radix select.
 __global__ void __launch_bounds__(kSelectThreads) heads_kernel(Geometry G, LayerIO io, Scratch sc, Slot sl) {
+    cg::cluster_group cluster = cg::this_cluster();
     __shared__ TopkShared sm;
-    __shared__ double sig[32];
+    __shared__ double red[32];
+    __shared__ float sig_self;
     extern __shared__ uint32_t bits[];
-    const int h = blockIdx.x, s = blockIdx.y;
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int h = (int)cluster.block_rank(), s = blockIdx.y;
+    const int tid = threadIdx.x, NT = blockDim.x;
     const int L = io.cu[s + 1] - io.cu[s];
     const int Lc = L - G.w;
-    const int nch = chunks_of(Lc);
-    const int stride = G.ML / kChunk + 1;
-    if (warp < G.Hkv) {
-        const float2* part = sl.sigpart + ((size_t)s * G.Hkv + warp) * stride;
-        double cnt = 0.0, sx = 0.0;
-        for (int c = lane; c < nch; c += 32) {
-            const int nc = min(kChunk, Lc - c * kChunk);
-            cnt += nc;
-            sx += nc * (double)part[c].x;
-        }
-        for (int off = 16; off; off >>= 1) {
-            cnt += __shfl_xor_sync(0xffffffffu, cnt, off);
-            sx += __shfl_xor_sync(0xffffffffu, sx, off);
-        }
-        const double mean = cnt > 0.0 ? sx / cnt : 0.0;
-        double m2 = 0.0;
-        for (int c = lane; c < nch; c += 32) {
-            const int nc = min(kChunk, Lc - c * kChunk);
-            const double dm = (double)part[c].x - mean;
-            m2 += (double)part[c].y + nc * dm * dm;
-        }
-        for (int off = 16; off; off >>= 1) m2 += __shfl_xor_sync(0xffffffffu, m2, off);
-        if (lane == 0) sig[warp] = cnt >= 2.0 ? sqrt(m2 / (cnt - 1.0)) : 0.0;
+    const int halo = G.pool / 2;
+    const size_t row = (size_t)s * G.Hkv + h;
+    float* stage = reinterpret_cast<float*>(bits + G.words + (keys_in_smem(G.ML) ? G.ML : 0));
+
+    // Pool P_O and P_O' of this head; sum of pooled P_O for the mean.
+    double sum = 0.0;
+    for (int c0 = 0; c0 < Lc; c0 += kPoolChunk) {
+        const int n = min(kPoolChunk, Lc - c0);
+        pool_chunk(sl.rawO + row * G.ML, sl.PO + row * G.ML, c0, n, Lc, halo, stage);
+        pool_chunk(sl.rawOe + row * G.ML, sl.POe + row * G.ML, c0, n, Lc, halo, stage);
+        for (int t = c0 + tid; t < c0 + n; t += NT) sum += sl.PO[row * G.ML + t];
     }
-    for (int wd = tid; wd < G.words; wd += blockDim.x) bits[wd] = 0u;
-    __syncthreads();
+    // Pool this CTA's slice of I.
+    {
+        const int per = (Lc + G.Hkv - 1) / G.Hkv;
+        const int a = min(h * per, Lc), b = min(a + per, Lc);
+        for (int c0 = a; c0 < b; c0 += kPoolChunk)
+            pool_chunk(sl.rawI + (size_t)s * G.ML, sl.I + (size_t)s * G.ML, c0, min(kPoolChunk, b - c0), Lc, halo,
+                       stage);
+    }
+    const double mean = Lc > 0 ? block_sum(sum, red) / Lc : 0.0;
+    double m2 = 0.0;
+    for (int t = tid; t < Lc; t += NT) {
+        const double d = (double)sl.PO[row * G.ML + t] - mean;
+        m2 += d * d;
+    }
+    m2 = block_sum(m2, red);
+    const float sigma = Lc >= 2 ? (float)sqrt(m2 / (double)(Lc - 1)) : 0.f;
+    if (tid == 0) sig_self = sigma;
+    for (int wd = tid; wd < G.words; wd += NT) bits[wd] = 0u;
+    cluster.sync();
     int rank = 0;
-    for (int o = 0; o < G.Hkv; ++o)
-        if (sig[o] < sig[h] || (sig[o] == sig[h] && o < h)) ++rank;
+    for (int o = 0; o < G.Hkv; ++o) {
+        const float so = *cluster.map_shared_rank(&sig_self, o);
+        if (so < sigma || (so == sigma && o < h)) ++rank;
+    }
     const int top = rank < G.delta;
     if (tid == 0) {
-        sl.sigma[(size_t)s * G.Hkv + h] = (float)sig[h];
-        sl.htop[(size_t)s * G.Hkv + h] = top;
+        sl.sigma[row] = sigma;
+        sl.htop[row] = top;
     }
     if (L > G.budget && G.Kp > 0) {
-        const float* P = (top ? sl.POe : sl.PO) + ((size_t)s * G.Hkv + h) * G.ML;
-        uint32_t* keys = sc.keys + ((size_t)s * G.Hkv + h) * G.ML;
-        for (int t = tid; t < Lc; t += blockDim.x) keys[t] = float_order_key(P[t]);
+        const float* __restrict__ P = (top ? sl.POe : sl.PO) + row * G.ML;
+        uint32_t* keys = keys_in_smem(G.ML) ? bits + G.words : sc.keys + row * G.ML;
+        for (int b0 = 4 * tid; b0 < Lc; b0 += 16 * NT) {
+            float4 pv[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int t4 = b0 + 4 * u * NT;
+                pv[u] = t4 < Lc ? __ldcg(reinterpret_cast<const float4*>(P + t4)) : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int t4 = b0 + 4 * u * NT;
+                const float x[4] = {pv[u].x, pv[u].y, pv[u].z, pv[u].w};
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+                    if (t4 + i < Lc) keys[t4 + i] = float_order_key(x[i]);
+            }
+        }
         __syncthreads();
         block_topk(keys, Lc, G.Kp, bits, sm);
     }
-    uint32_t* pres = sl.pres + ((size_t)s * G.Hkv + h) * G.words;
-    for (int wd = tid; wd < G.words; wd += blockDim.x) pres[wd] = bits[wd];
+    uint32_t* pres = sl.pres + row * G.words;
+    for (int wd = tid; wd < G.words; wd += NT) pres[wd] = bits[wd];
+    cluster.sync();   // peers may still read sig_self
 }
 
 // Section 4.2: P' = P + lambda * I * (1 - n_t / (l + 1)); the preserved tokens
@@ -210,14 +276,41 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
         const float* I = sl.I + (size_t)s * G.ML;
         const uint32_t* pres = sl.pres + row * G.words;
         float* Pp = sl.Pprime + row * G.ML;
-        uint32_t* keys = sc.keys + row * G.ML;
+        uint32_t* keys = keys_in_smem(G.ML) ? bits + G.words : sc.keys + row * G.ML;
         const float denom = (float)(ell + 1u);
-        for (int t = tid; t < Lc; t += NT) {
-            const float coverage = (float)ncount[t] / denom;
-            const float pp = P[t] + G.lambda * (I[t] * (1.f - coverage));
-            Pp[t] = pp;
-            const bool kept = (pres[t >> 5] >> (t & 31)) & 1u;
-            keys[t] = kept ? 0u : float_order_key(pp);
+        for (int b0 = 4 * tid; b0 < Lc; b0 += 8 * NT) {
+            float4 pv[2], iv[2];
+            uchar4 nv[2];
+            uint32_t pw[2];
+#pragma unroll
+            for (int u = 0; u < 2; ++u) {
+                const int t4 = b0 + 4 * u * NT;
+                if (t4 < Lc) {
+                    pv[u] = *reinterpret_cast<const float4*>(P + t4);
+                    iv[u] = *reinterpret_cast<const float4*>(I + t4);
+                    nv[u] = *reinterpret_cast<const uchar4*>(ncount + t4);
+                    pw[u] = pres[t4 >> 5];
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < 2; ++u) {
+                const int t4 = b0 + 4 * u * NT;
+                if (t4 >= Lc) continue;
+                const float p4[4] = {pv[u].x, pv[u].y, pv[u].z, pv[u].w};
+                const float i4[4] = {iv[u].x, iv[u].y, iv[u].z, iv[u].w};
+                const uint8_t n4[4] = {nv[u].x, nv[u].y, nv[u].z, nv[u].w};
+                float out[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int t = t4 + i;
+                    const float coverage = (float)n4[i] / denom;
+                    const float pp = p4[i] + G.lambda * (i4[i] * (1.f - coverage));
+                    out[i] = pp;
+                    const bool kept = (pw[u] >> (t & 31)) & 1u;
+                    if (t < Lc) keys[t] = kept ? 0u : float_order_key(pp);
+                }
+                *reinterpret_cast<float4*>(Pp + t4) = make_float4(out[0], out[1], out[2], out[3]);
+            }
         }
         __syncthreads();
         block_topk(keys, Lc, G.k2, bits, sm);
@@ -256,9 +349,14 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
     __syncthreads();
     if (!last_head) return;
     __threadfence();
-    for (int t = tid; t < L; t += NT) {
-        const uint32_t wv = __ldcg(&ub[t >> 5]);
-        if ((wv >> (t & 31)) & 1u) ncount[t] = (uint8_t)(ncount[t] + 1u);
+    for (int t4 = 4 * tid; t4 < L; t4 += 4 * NT) {
+        const uint32_t wv = __ldcg(&ub[t4 >> 5]) >> (t4 & 31);
+        uchar4 n4 = *reinterpret_cast<uchar4*>(ncount + t4);
+        n4.x = (uint8_t)(n4.x + (wv & 1u));
+        if (t4 + 1 < L) n4.y = (uint8_t)(n4.y + ((wv >> 1) & 1u));
+        if (t4 + 2 < L) n4.z = (uint8_t)(n4.z + ((wv >> 2) & 1u));
+        if (t4 + 3 < L) n4.w = (uint8_t)(n4.w + ((wv >> 3) & 1u));
+        *reinterpret_cast<uchar4*>(ncount + t4) = n4;
     }
     __syncthreads();
     uint32_t* last_union = reinterpret_cast<uint32_t*>(st + G.state_union_off);
@@ -295,12 +393,42 @@ __global__ void __launch_bounds__(256) gather_kernel(Geometry G, LayerIO io) {
 
 }  // namespace
 
-void launch_heads(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st) {
-    heads_kernel<<<dim3(g.Hkv, g.batch), kSelectThreads, g.words * sizeof(uint32_t), st>>>(g, io, sc, sl);
+size_t select_smem_bytes(const Geometry& g) {
+    return sizeof(uint32_t) * ((size_t)g.words + (keys_in_smem(g.ML) ? (size_t)g.ML : 0));
+}
+
+size_t heads_smem_bytes(const Geometry& g) {
+    return select_smem_bytes(g) + sizeof(float) * (kPoolChunk + 2 * (kMaxPool / 2));
+}
+
+cudaError_t configure_select() {
+    const int need = (int)(sizeof(uint32_t) * (kSmemKeys + kSmemKeys / 32));
+    cudaError_t e = cudaFuncSetAttribute(heads_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         need + (int)sizeof(float) * (kPoolChunk + 2 * (kMaxPool / 2)));
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(heads_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, need);
+    return e;
+}
+
+cudaError_t launch_heads(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(g.Hkv, g.batch);
+    cfg.blockDim = dim3(kSelectThreads);
+    cfg.dynamicSmemBytes = heads_smem_bytes(g);
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = g.Hkv;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, heads_kernel, g, io, sc, sl);
 }
 
 void launch_select(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st) {
-    select_kernel<<<dim3(g.Hkv, g.batch), kSelectThreads, g.words * sizeof(uint32_t), st>>>(g, io, sc, sl);
+    select_kernel<<<dim3(g.Hkv, g.batch), kSelectThreads, select_smem_bytes(g), st>>>(g, io, sc, sl);
 }
 
 void launch_gather(const Geometry& g, const LayerIO& io, cudaStream_t st) {

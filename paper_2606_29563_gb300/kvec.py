@@ -23,7 +23,7 @@ KVEC_ERR_DEVICE_TIMEOUT = 4
 KVEC_ERR_OOM = 5
 
 # kernel ids of kvec_kernel_time
-KERNEL_NAMES = ("score", "rowstat", "window", "heads", "select", "gather")
+KERNEL_NAMES = ("score", "window", "heads", "select", "gather")
 
 EXPORTED = ("kvec_create", "kvec_destroy", "kvec_state_bytes", "kvec_reset", "kvec_select_layer",
             "kvec_select_layers", "kvec_debug_scores", "kvec_sync_status", "kvec_set_profiling",

@@ -160,7 +160,7 @@ KVEC_API kvec_status kvec_select_layer_noalloc(const kvec_params* params, int ba
 
 /* Device views of the last processed layer's intermediates (valid until the
  * next call on the handle; read after synchronising the stream).  Row strides
- * use ML = max_seqlen rounded up to a multiple of 32 (reported in max_seqlen).
+ * use ML = max_seqlen + 4 rounded up to a multiple of 32 (reported in max_seqlen).
  * Only candidate positions t < L_s - w hold scores. */
 typedef struct {
     const float*    P_O;        /* [max_batch][H_kv][ML]  Eq. 1 with O, max-pooled */
@@ -174,7 +174,7 @@ typedef struct {
                                    and denominator; row r = q*g + j is query head
                                    h*g + j at window row q */
     int max_seqlen;             /* ML: the row stride of the arrays above */
-    int words_per_row;          /* ML/32 */
+    int words_per_row;          /* ceil(max_seqlen/32): words of pres_bits per row */
 } kvec_debug_view;
 
 KVEC_API kvec_status kvec_debug_scores(kvec_handle* h, kvec_debug_view* out);

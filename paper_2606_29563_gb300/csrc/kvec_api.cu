@@ -34,6 +34,10 @@ kvec_status cuda_fail(cudaError_t e, const char* what) {
 
 size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
+// Row stride of per-position workspace arrays: 128-byte aligned rows with room for
+// a float4 access that starts at the last position of a row.
+size_t row_stride(int max_seqlen) { return round_up((size_t)max_seqlen + 4, 32); }
+
 constexpr int kKernelKinds = 5;
 
 struct TimedLaunch {
@@ -42,6 +46,8 @@ struct TimedLaunch {
 };
 
 }  // namespace
+
+constexpr int kSlots = 4;   // per-layer score arrays in flight between the score and select stages
 
 struct kvec_handle {
     kvec_params p;
@@ -52,11 +58,19 @@ struct kvec_handle {
     void* ws = nullptr;
     size_t ws_bytes = 0;
     Scratch sc{};
-    Slot slot{};
+    Slot slots[kSlots]{};
+    int last_slot = 0;
     int last_batch = 0;
     bool profiling = false;
     std::vector<TimedLaunch> timed;
     std::vector<cudaEvent_t> event_pool;
+    // Streams of the layer pipeline: score + window | heads | coverage select | gather.
+    cudaStream_t s_score = nullptr, s_heads = nullptr, s_chain = nullptr, s_gather = nullptr, s_cap = nullptr;
+    std::vector<cudaEvent_t> ev_win, ev_heads, ev_sel;
+    cudaEvent_t ev_fork = nullptr, ev_join[3] = {nullptr, nullptr, nullptr};
+    // CUDA graph of the last repeated multi-layer call.
+    cudaGraphExec_t gexec = nullptr;
+    std::vector<uint64_t> gkey, pending_key;
 };
 
 namespace {
@@ -178,7 +192,7 @@ Geometry make_geometry(const kvec_handle* h, int batch, int budget, int tiles, i
     G.lambda = p.lambda;
     const double scale = p.softmax_scale > 0.f ? (double)p.softmax_scale : 1.0 / sqrt((double)p.head_dim);
     G.sl2 = (float)(scale * 1.4426950408889634);
-    G.ML = (int)round_up((size_t)p.max_seqlen, 32);   // row stride: 128-byte aligned rows
+    G.ML = (int)row_stride(p.max_seqlen);
     G.words = h->words;
     G.batch = batch;
     G.budget = budget;
@@ -195,21 +209,98 @@ Geometry make_geometry(const kvec_handle* h, int batch, int budget, int tiles, i
     return G;
 }
 
-kvec_status run_layer(kvec_handle* h, const Geometry& G, const LayerIO& io, cudaStream_t st) {
+// One layer, every kernel on one stream with one slot (used without a handle).
+kvec_status run_layer_sequential(kvec_handle* h, const Geometry& G, const LayerIO& io, cudaStream_t st) {
     ScorePlan plan;
     cudaError_t se = plan_score(G, io, h->sc, h->num_sms, &plan);
     if (se != cudaSuccess) return cuda_fail(se, "score kernel tensor maps");
-    timed_launch(h, 0, st, [&] { se = launch_score(plan, st); });
+    se = launch_score(plan, st);
     if (se != cudaSuccess) return cuda_fail(se, "score kernel launch");
-    timed_launch(h, 1, st, [&] { launch_window(G, io, h->sc, h->slot, st); });
-    cudaError_t he = cudaSuccess;
-    timed_launch(h, 2, st, [&] { he = launch_heads(G, io, h->sc, h->slot, st); });
-    if (he != cudaSuccess) return cuda_fail(he, "heads kernel launch");
-    timed_launch(h, 3, st, [&] { launch_select(G, io, h->sc, h->slot, st); });
-    timed_launch(h, 4, st, [&] { launch_gather(G, io, st); });
+    launch_window(G, io, h->sc, h->slots[0], st);
+    se = launch_heads(G, io, h->sc, h->slots[0], st);
+    if (se != cudaSuccess) return cuda_fail(se, "heads kernel launch");
+    launch_select(G, io, h->sc, h->slots[0], st);
+    launch_gather(G, io, st);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_fail(e, "kernel launch");
     return KVEC_OK;
+}
+
+#define KV_CHECK(call)                                        \
+    do {                                                      \
+        cudaError_t e_ = (call);                              \
+        if (e_ != cudaSuccess) return cuda_fail(e_, #call);   \
+    } while (0)
+
+// Layers 0..n-1 as a four-stream pipeline.  Only the coverage-adjusted select is
+// serial across layers (it carries n_t); the score, window and heads work of
+// later layers runs ahead of it, bounded by the kSlots ring of score arrays.
+kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* ios, int n, cudaStream_t origin) {
+    KV_CHECK(cudaEventRecord(h->ev_fork, origin));
+    for (cudaStream_t st : {h->s_score, h->s_heads, h->s_chain, h->s_gather})
+        KV_CHECK(cudaStreamWaitEvent(st, h->ev_fork, 0));
+    for (int l = 0; l < n; ++l) {
+        const Slot& sl = h->slots[l % kSlots];
+        const LayerIO& io = ios[l];
+        if (l >= kSlots) KV_CHECK(cudaStreamWaitEvent(h->s_score, h->ev_sel[l - kSlots], 0));
+        ScorePlan plan;
+        cudaError_t se = plan_score(G, io, h->sc, h->num_sms, &plan);
+        if (se != cudaSuccess) return cuda_fail(se, "score kernel tensor maps");
+        timed_launch(h, 0, h->s_score, [&] { se = launch_score(plan, h->s_score); });
+        if (se != cudaSuccess) return cuda_fail(se, "score kernel launch");
+        timed_launch(h, 1, h->s_score, [&] { launch_window(G, io, h->sc, sl, h->s_score); });
+        KV_CHECK(cudaEventRecord(h->ev_win[l], h->s_score));
+        KV_CHECK(cudaStreamWaitEvent(h->s_heads, h->ev_win[l], 0));
+        timed_launch(h, 2, h->s_heads, [&] { se = launch_heads(G, io, h->sc, sl, h->s_heads); });
+        if (se != cudaSuccess) return cuda_fail(se, "heads kernel launch");
+        KV_CHECK(cudaEventRecord(h->ev_heads[l], h->s_heads));
+        KV_CHECK(cudaStreamWaitEvent(h->s_chain, h->ev_heads[l], 0));
+        timed_launch(h, 3, h->s_chain, [&] { launch_select(G, io, h->sc, sl, h->s_chain); });
+        KV_CHECK(cudaEventRecord(h->ev_sel[l], h->s_chain));
+        KV_CHECK(cudaStreamWaitEvent(h->s_gather, h->ev_sel[l], 0));
+        timed_launch(h, 4, h->s_gather, [&] { launch_gather(G, io, h->s_gather); });
+    }
+    KV_CHECK(cudaGetLastError());
+    KV_CHECK(cudaEventRecord(h->ev_join[0], h->s_score));
+    KV_CHECK(cudaEventRecord(h->ev_join[1], h->s_heads));
+    KV_CHECK(cudaEventRecord(h->ev_join[2], h->s_gather));
+    KV_CHECK(cudaStreamWaitEvent(origin, h->ev_sel[n - 1], 0));
+    for (cudaEvent_t e : h->ev_join) KV_CHECK(cudaStreamWaitEvent(origin, e, 0));
+    h->last_slot = (n - 1) % kSlots;
+    return KVEC_OK;
+}
+
+std::vector<uint64_t> graph_key(int n, int batch, int budget, const int32_t* cu_host, const int32_t* cu_dev,
+                                const LayerIO* ios) {
+    std::vector<uint64_t> k = {(uint64_t)n, (uint64_t)batch, (uint64_t)budget, (uint64_t)(uintptr_t)cu_dev};
+    for (int b = 0; b <= batch; ++b) k.push_back((uint64_t)cu_host[b]);
+    for (int l = 0; l < n; ++l) {
+        const LayerIO& io = ios[l];
+        for (const void* ptr : {(const void*)io.q, (const void*)io.k, (const void*)io.v, (const void*)io.state,
+                                (const void*)io.out_idx, (const void*)io.out_k, (const void*)io.out_v})
+            k.push_back((uint64_t)(uintptr_t)ptr);
+    }
+    return k;
+}
+
+}  // namespace
+
+namespace {
+
+void release_handle(kvec_handle* h) {
+    if (h->gexec) cudaGraphExecDestroy(h->gexec);
+    for (cudaStream_t st : {h->s_score, h->s_heads, h->s_chain, h->s_gather, h->s_cap})
+        if (st) cudaStreamDestroy(st);
+    for (auto* v : {&h->ev_win, &h->ev_heads, &h->ev_sel})
+        for (cudaEvent_t ev : *v)
+            if (ev) cudaEventDestroy(ev);
+    if (h->ev_fork) cudaEventDestroy(h->ev_fork);
+    for (cudaEvent_t ev : h->ev_join)
+        if (ev) cudaEventDestroy(ev);
+    recycle_timed(h);
+    for (cudaEvent_t ev : h->event_pool) cudaEventDestroy(ev);
+    if (h->ws) cudaFree(h->ws);
+    delete h;
 }
 
 }  // namespace
@@ -243,7 +334,7 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
     h->n_off = 16;
     h->union_off = 16 + round_up((size_t)p.max_seqlen, 16);
 
-    const size_t MB = p.max_batch, ML = round_up((size_t)p.max_seqlen, 32), Hkv = p.num_kv_heads, R = h->R,
+    const size_t MB = p.max_batch, ML = row_stride(p.max_seqlen), Hkv = p.num_kv_heads, R = h->R,
                  W = h->words;
     const size_t max_tiles = MB * ((ML + kTileT - 1) / kTileT);
     struct Part {
@@ -260,17 +351,19 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
         {(void**)&h->sc.ubits, MB * W * sizeof(uint32_t)},
         {(void**)&h->sc.ucount, MB * sizeof(unsigned)},
         {(void**)&h->sc.err, sizeof(int)},
-        {(void**)&h->slot.rawO, MB * Hkv * ML * sizeof(float)},
-        {(void**)&h->slot.rawOe, MB * Hkv * ML * sizeof(float)},
-        {(void**)&h->slot.rawI, MB * ML * sizeof(float)},
-        {(void**)&h->slot.PO, MB * Hkv * ML * sizeof(float)},
-        {(void**)&h->slot.POe, MB * Hkv * ML * sizeof(float)},
-        {(void**)&h->slot.I, MB * ML * sizeof(float)},
-        {(void**)&h->slot.sigma, MB * Hkv * sizeof(float)},
-        {(void**)&h->slot.htop, MB * Hkv * sizeof(int)},
-        {(void**)&h->slot.pres, MB * Hkv * W * sizeof(uint32_t)},
-        {(void**)&h->slot.Pprime, MB * Hkv * ML * sizeof(float)},
+        {(void**)&h->sc.keys_sel, MB * Hkv * ML * sizeof(uint32_t)},
     };
+    for (int k = 0; k < kSlots; ++k) {
+        Slot& sl = h->slots[k];
+        std::vector<Part> sp = {
+            {(void**)&sl.rawO, MB * Hkv * ML * sizeof(float)},  {(void**)&sl.rawOe, MB * Hkv * ML * sizeof(float)},
+            {(void**)&sl.rawI, MB * ML * sizeof(float)},        {(void**)&sl.PO, MB * Hkv * ML * sizeof(float)},
+            {(void**)&sl.POe, MB * Hkv * ML * sizeof(float)},   {(void**)&sl.I, MB * ML * sizeof(float)},
+            {(void**)&sl.sigma, MB * Hkv * sizeof(float)},      {(void**)&sl.htop, MB * Hkv * sizeof(int)},
+            {(void**)&sl.pres, MB * Hkv * W * sizeof(uint32_t)}, {(void**)&sl.Pprime, MB * Hkv * ML * sizeof(float)},
+        };
+        parts.insert(parts.end(), sp.begin(), sp.end());
+    }
     size_t total = 0;
     for (auto& pt : parts) total += round_up(pt.bytes, 256);
     e = cudaMalloc(&h->ws, total);
@@ -291,10 +384,20 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
     if (e == cudaSuccess) e = configure_score(G);
     if (e == cudaSuccess) e = configure_window(G);
     if (e == cudaSuccess) e = configure_select();
+    for (cudaStream_t* st : {&h->s_score, &h->s_heads, &h->s_chain, &h->s_gather, &h->s_cap})
+        if (e == cudaSuccess) e = cudaStreamCreateWithFlags(st, cudaStreamNonBlocking);
+    h->ev_win.assign(p.max_layers, nullptr);
+    h->ev_heads.assign(p.max_layers, nullptr);
+    h->ev_sel.assign(p.max_layers, nullptr);
+    for (auto* v : {&h->ev_win, &h->ev_heads, &h->ev_sel})
+        for (auto& ev : *v)
+            if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming);
+    for (auto& ev : h->ev_join)
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
     if (e == cudaSuccess) e = cudaDeviceSynchronize();
     if (e != cudaSuccess) {
-        cudaFree(h->ws);
-        delete h;
+        release_handle(h);
         return cuda_fail(e, "workspace set-up");
     }
     *out = h;
@@ -307,12 +410,9 @@ kvec_status kvec_destroy(kvec_handle* h) {
     kvec_status s = set_device(h, &prev);
     if (s != KVEC_OK) return s;
     DeviceGuard guard{prev, h->device};
-    cudaDeviceSynchronize();
-    recycle_timed(h);
-    for (cudaEvent_t e : h->event_pool) cudaEventDestroy(e);
-    cudaError_t e = cudaFree(h->ws);
-    delete h;
-    if (e != cudaSuccess) return cuda_fail(e, "cudaFree");
+    cudaError_t e = cudaDeviceSynchronize();
+    release_handle(h);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceSynchronize");
     return KVEC_OK;
 }
 
@@ -369,8 +469,9 @@ kvec_status kvec_select_layers(kvec_handle* h, int num_layers, int batch, const 
     Geometry G = make_geometry(h, batch, budget, tiles, chunks, cu_seqlens_host[batch]);
     G.cu_host = cu_seqlens_host;
     cudaStream_t st = (cudaStream_t)stream;
+    std::vector<LayerIO> ios(num_layers);
     for (int l = 0; l < num_layers; ++l) {
-        LayerIO io{};
+        LayerIO& io = ios[l];
         io.q = static_cast<const __nv_bfloat16*>(q_obs[l]);
         io.k = static_cast<const __nv_bfloat16*>(k[l]);
         io.v = static_cast<const __nv_bfloat16*>(v[l]);
@@ -379,9 +480,41 @@ kvec_status kvec_select_layers(kvec_handle* h, int num_layers, int batch, const 
         io.out_idx = out_idx[l];
         io.out_k = static_cast<__nv_bfloat16*>(out_k[l]);
         io.out_v = static_cast<__nv_bfloat16*>(out_v[l]);
-        s = run_layer(h, G, io, st);
-        if (s != KVEC_OK) return s;
     }
+    if (!h->profiling && num_layers >= 2) {
+        // A call repeated with the same arguments replays a captured graph of the pipeline.
+        std::vector<uint64_t> key = graph_key(num_layers, batch, budget, cu_seqlens_host, cu_seqlens_dev, ios.data());
+        if (h->gexec && key == h->gkey) {
+            KV_CHECK(cudaGraphLaunch(h->gexec, st));
+            h->last_slot = (num_layers - 1) % kSlots;
+            h->last_batch = batch;
+            return KVEC_OK;
+        }
+        if (key == h->pending_key) {
+            cudaGraph_t graph = nullptr;
+            KV_CHECK(cudaStreamBeginCapture(h->s_cap, cudaStreamCaptureModeThreadLocal));
+            s = launch_pipeline(h, G, ios.data(), num_layers, h->s_cap);
+            cudaError_t ce = cudaStreamEndCapture(h->s_cap, &graph);
+            if (s != KVEC_OK) {
+                if (graph) cudaGraphDestroy(graph);
+                return s;
+            }
+            if (ce != cudaSuccess) return cuda_fail(ce, "cudaStreamEndCapture");
+            cudaGraphExec_t exec = nullptr;
+            ce = cudaGraphInstantiate(&exec, graph, 0);
+            cudaGraphDestroy(graph);
+            if (ce != cudaSuccess) return cuda_fail(ce, "cudaGraphInstantiate");
+            if (h->gexec) cudaGraphExecDestroy(h->gexec);
+            h->gexec = exec;
+            h->gkey = key;
+            KV_CHECK(cudaGraphLaunch(h->gexec, st));
+            h->last_batch = batch;
+            return KVEC_OK;
+        }
+        h->pending_key = key;
+    }
+    s = launch_pipeline(h, G, ios.data(), num_layers, st);
+    if (s != KVEC_OK) return s;
     h->last_batch = batch;
     return KVEC_OK;
 }
@@ -457,7 +590,7 @@ kvec_status kvec_select_layer_noalloc(const kvec_params* params, int batch, cons
         return fail(KVEC_ERR_INVALID_ARG, "device pointers must be 16-byte aligned");
 
     // Carve the scratch for exactly this call's geometry.
-    const size_t nb = batch, ML = round_up((size_t)params->max_seqlen, 32), Hkv = params->num_kv_heads, R = tmp.R,
+    const size_t nb = batch, ML = row_stride(params->max_seqlen), Hkv = params->num_kv_heads, R = tmp.R,
                  W = tmp.words;
     const size_t nt = tiles;
     struct Part {
@@ -474,16 +607,17 @@ kvec_status kvec_select_layer_noalloc(const kvec_params* params, int batch, cons
         {(void**)&tmp.sc.tstat, nt * Hkv * R * sizeof(float2)},
         {(void**)&tmp.sc.rowstat, nb * Hkv * R * sizeof(float2)},
         {(void**)&tmp.sc.keys, nb * Hkv * ML * sizeof(uint32_t)},
-        {(void**)&tmp.slot.rawO, nb * Hkv * ML * sizeof(float)},
-        {(void**)&tmp.slot.rawOe, nb * Hkv * ML * sizeof(float)},
-        {(void**)&tmp.slot.rawI, nb * ML * sizeof(float)},
-        {(void**)&tmp.slot.PO, nb * Hkv * ML * sizeof(float)},
-        {(void**)&tmp.slot.POe, nb * Hkv * ML * sizeof(float)},
-        {(void**)&tmp.slot.I, nb * ML * sizeof(float)},
-        {(void**)&tmp.slot.sigma, nb * Hkv * sizeof(float)},
-        {(void**)&tmp.slot.htop, nb * Hkv * sizeof(int)},
-        {(void**)&tmp.slot.pres, nb * Hkv * W * sizeof(uint32_t)},
-        {(void**)&tmp.slot.Pprime, nb * Hkv * ML * sizeof(float)},
+        {(void**)&tmp.sc.keys_sel, nb * Hkv * ML * sizeof(uint32_t)},
+        {(void**)&tmp.slots[0].rawO, nb * Hkv * ML * sizeof(float)},
+        {(void**)&tmp.slots[0].rawOe, nb * Hkv * ML * sizeof(float)},
+        {(void**)&tmp.slots[0].rawI, nb * ML * sizeof(float)},
+        {(void**)&tmp.slots[0].PO, nb * Hkv * ML * sizeof(float)},
+        {(void**)&tmp.slots[0].POe, nb * Hkv * ML * sizeof(float)},
+        {(void**)&tmp.slots[0].I, nb * ML * sizeof(float)},
+        {(void**)&tmp.slots[0].sigma, nb * Hkv * sizeof(float)},
+        {(void**)&tmp.slots[0].htop, nb * Hkv * sizeof(int)},
+        {(void**)&tmp.slots[0].pres, nb * Hkv * W * sizeof(uint32_t)},
+        {(void**)&tmp.slots[0].Pprime, nb * Hkv * ML * sizeof(float)},
     };
     size_t need = 0, zero_bytes = 0;
     for (size_t i = 0; i < sizeof(parts) / sizeof(parts[0]); ++i) {
@@ -525,20 +659,21 @@ kvec_status kvec_select_layer_noalloc(const kvec_params* params, int batch, cons
     io.out_idx = out_idx;
     io.out_k = static_cast<__nv_bfloat16*>(out_k);
     io.out_v = static_cast<__nv_bfloat16*>(out_v);
-    return run_layer(&tmp, G, io, st);
+    return run_layer_sequential(&tmp, G, io, st);
 }
 
 kvec_status kvec_debug_scores(kvec_handle* h, kvec_debug_view* out) {
     if (!h || !out) return fail(KVEC_ERR_INVALID_ARG, "NULL argument");
-    out->P_O = h->slot.PO;
-    out->P_Oext = h->slot.POe;
-    out->I = h->slot.I;
-    out->sigma = h->slot.sigma;
-    out->htop = h->slot.htop;
-    out->pres_bits = h->slot.pres;
-    out->Pprime = h->slot.Pprime;
+    const Slot& sl = h->slots[h->last_slot];
+    out->P_O = sl.PO;
+    out->P_Oext = sl.POe;
+    out->I = sl.I;
+    out->sigma = sl.sigma;
+    out->htop = sl.htop;
+    out->pres_bits = sl.pres;
+    out->Pprime = sl.Pprime;
     out->row_stats = reinterpret_cast<const float*>(h->sc.rowstat);
-    out->max_seqlen = (int)round_up((size_t)h->p.max_seqlen, 32);
+    out->max_seqlen = (int)row_stride(h->p.max_seqlen);
     out->words_per_row = h->words;
     return KVEC_OK;
 }

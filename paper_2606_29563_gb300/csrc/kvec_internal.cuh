@@ -52,7 +52,8 @@ struct Scratch {
     float2* segpart;      // [total_tiles * Hkv][R] per-CTA segment (max, sum) keyed by first item
     unsigned* shcount;    // [max_batch][Hkv]       tiles finished per (sequence, KV head)
     float2* rowstat;      // [max_batch][Hkv][R]    (row max in log2 units, softmax denominator)
-    uint32_t* keys;       // [max_batch][Hkv][ML]   radix-select keys
+    uint32_t* keys;       // [max_batch][Hkv][ML]   radix-select keys of the heads kernel
+    uint32_t* keys_sel;   // [max_batch][Hkv][ML]   radix-select keys of the select kernel
     uint32_t* ubits;      // [max_batch][words]     union of this layer's selections
     unsigned* ucount;     // [max_batch]            heads finished (last-CTA fold)
     int* err;             // device error word

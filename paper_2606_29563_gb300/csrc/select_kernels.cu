@@ -133,46 +133,89 @@ __device__ __forceinline__ uint32_t range_bits(int word, int lo, int hi) {
     return upto & ~((1u << a) - 1u);
 }
 
-// Max-pool width `2*halo+1` over [0, Lc) of one row: the output positions
-// [c0, c0+n) are staged with their halo in shared memory first.
-__device__ void pool_chunk(const float* __restrict__ raw, float* __restrict__ out, int c0, int n, int Lc, int halo,
-                           float* stage) {
-    const int lo = max(c0 - halo, 0), hi = min(c0 + n + halo, Lc);
-    for (int t = lo + threadIdx.x; t < hi; t += blockDim.x) stage[t - lo] = __ldcg(raw + t);
-    __syncthreads();
-    for (int t = c0 + threadIdx.x; t < c0 + n; t += blockDim.x) {
-        const int a = max(t - halo, 0) - lo, b = min(t + halo, Lc - 1) - lo;
-        float m = stage[a];
-        for (int x = a + 1; x <= b; ++x) m = fmaxf(m, stage[x]);
-        out[t] = m;
+// Max-pool (width 2*halo+1, stride 1, neighbours outside [0, Lc) ignored) of
+// the four positions [t4, t4+4) of a row: the raw values [t4-8, t4+12) arrive
+// as five float4 loads issued together.
+struct Pooled4 {
+    float v[4];
+};
+
+__device__ __forceinline__ Pooled4 pool4(const float* __restrict__ raw, int t4, int Lc, int halo) {
+    float x[20];
+#pragma unroll
+    for (int b = 0; b < 5; ++b) {
+        const int p = t4 - 8 + 4 * b;
+        float4 f = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+        if (p >= 0 && p < Lc) f = __ldcg(reinterpret_cast<const float4*>(raw + p));
+        x[4 * b] = p < Lc ? f.x : -INFINITY;
+        x[4 * b + 1] = p + 1 < Lc ? f.y : -INFINITY;
+        x[4 * b + 2] = p + 2 < Lc ? f.z : -INFINITY;
+        x[4 * b + 3] = p + 3 < Lc ? f.w : -INFINITY;
     }
-    __syncthreads();
+    Pooled4 out;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        float m = x[8 + i];
+#pragma unroll
+        for (int d = 1; d <= kMaxPool / 2; ++d)
+            if (d <= halo) m = fmaxf(m, fmaxf(x[8 + i - d], x[8 + i + d]));
+        out.v[i] = m;
+    }
+    return out;
 }
 
-__device__ double block_sum(double v, double* red) {
+// Running (count, mean, sum of squared deviations); merge() is Chan et al.'s
+// pairwise update, stable in fp32 (no cancellation of sum(x^2) - n*mean^2).
+struct Moments {
+    float n, mean, m2;
+    __device__ void add(float x) {
+        n += 1.f;
+        const float d = x - mean;
+        mean += d / n;
+        m2 += d * (x - mean);
+    }
+    __device__ void merge(float nb, float meanb, float m2b) {
+        if (nb == 0.f) return;
+        if (n == 0.f) {
+            n = nb;
+            mean = meanb;
+            m2 = m2b;
+            return;
+        }
+        const float nt = n + nb, d = meanb - mean;
+        mean += d * (nb / nt);
+        m2 += m2b + d * d * (n * nb / nt);
+        n = nt;
+    }
+};
+
+__device__ Moments block_moments(Moments v, float3* red) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
-    for (int off = 16; off; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-    if (lane == 0) red[warp] = v;
+    for (int off = 16; off; off >>= 1)
+        v.merge(__shfl_xor_sync(0xffffffffu, v.n, off), __shfl_xor_sync(0xffffffffu, v.mean, off),
+                __shfl_xor_sync(0xffffffffu, v.m2, off));
+    if (lane == 0) red[warp] = make_float3(v.n, v.mean, v.m2);
     __syncthreads();
-    double t = 0.0;
-    for (int i = 0; i < nw; ++i) t += red[i];
+    Moments t{0.f, 0.f, 0.f};
+    if (lane < nw) t = Moments{red[lane].x, red[lane].y, red[lane].z};
+    for (int off = 16; off; off >>= 1)
+        t.merge(__shfl_xor_sync(0xffffffffu, t.n, off), __shfl_xor_sync(0xffffffffu, t.mean, off),
+                __shfl_xor_sync(0xffffffffu, t.m2, off));
     __syncthreads();
     return t;
 }
 
-constexpr int kPoolChunk = 4096;
-
 // Section 4.1 and the preserved tokens of Section 4.2.  One thread-block
 // cluster per sequence, one CTA per KV head (cluster rank = head):
 //   pool the head's P_O and P_O' rows and a slice of I (max-pool, inherited
-//   from SnapKV), sigma_h = sample std of pooled P_O over the candidates (two
-//   passes, fp64 sums), exchange sigma through distributed shared memory, the
+//   from SnapKV), sigma_h = sample std of pooled P_O over the candidates
+//   (Welford/Chan moments in fp32), exchange sigma through distributed shared memory, the
 //   delta lowest-sigma heads take the O' scores, then the top-K preserved
 //   tokens of the chosen row by radix select.
 __global__ void __launch_bounds__(kSelectThreads) heads_kernel(Geometry G, LayerIO io, Scratch sc, Slot sl) {
     cg::cluster_group cluster = cg::this_cluster();
     __shared__ TopkShared sm;
-    __shared__ double red[32];
+    __shared__ float3 red[32];
     __shared__ float sig_self;
     extern __shared__ uint32_t bits[];
     const int h = (int)cluster.block_rank(), s = blockIdx.y;
@@ -181,41 +224,44 @@ __global__ void __launch_bounds__(kSelectThreads) heads_kernel(Geometry G, Layer
     const int Lc = L - G.w;
     const int halo = G.pool / 2;
     const size_t row = (size_t)s * G.Hkv + h;
-    float* stage = reinterpret_cast<float*>(bits + G.words + (keys_in_smem(G.ML) ? G.ML : 0));
-
-    // Pool P_O and P_O' of this head; sum of pooled P_O for the mean.
-    double sum = 0.0;
-    for (int c0 = 0; c0 < Lc; c0 += kPoolChunk) {
-        const int n = min(kPoolChunk, Lc - c0);
-        pool_chunk(sl.rawO + row * G.ML, sl.PO + row * G.ML, c0, n, Lc, halo, stage);
-        pool_chunk(sl.rawOe + row * G.ML, sl.POe + row * G.ML, c0, n, Lc, halo, stage);
-        for (int t = c0 + tid; t < c0 + n; t += NT) sum += sl.PO[row * G.ML + t];
+    // Pool P_O and P_O' of this head (four positions per thread per step) and
+    // accumulate the sums of pooled P_O and of its squares in fp64.
+    Moments mom{0.f, 0.f, 0.f};
+    const float* rO = sl.rawO + row * G.ML;
+    const float* rOe = sl.rawOe + row * G.ML;
+    for (int t4 = 4 * tid; t4 < Lc; t4 += 4 * NT) {
+        const Pooled4 a = pool4(rO, t4, Lc, halo);
+        const Pooled4 b = pool4(rOe, t4, Lc, halo);
+        *reinterpret_cast<float4*>(sl.PO + row * G.ML + t4) = make_float4(a.v[0], a.v[1], a.v[2], a.v[3]);
+        *reinterpret_cast<float4*>(sl.POe + row * G.ML + t4) = make_float4(b.v[0], b.v[1], b.v[2], b.v[3]);
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+            if (t4 + i < Lc) mom.add(a.v[i]);
     }
-    // Pool this CTA's slice of I.
+    // This CTA's slice of pooled I.
     {
-        const int per = (Lc + G.Hkv - 1) / G.Hkv;
-        const int a = min(h * per, Lc), b = min(a + per, Lc);
-        for (int c0 = a; c0 < b; c0 += kPoolChunk)
-            pool_chunk(sl.rawI + (size_t)s * G.ML, sl.I + (size_t)s * G.ML, c0, min(kPoolChunk, b - c0), Lc, halo,
-                       stage);
+        const int per = ((Lc + G.Hkv - 1) / G.Hkv + 3) & ~3;
+        const int a0 = min(h * per, Lc), b0 = min(a0 + per, Lc);
+        const float* rI = sl.rawI + (size_t)s * G.ML;
+        for (int t4 = a0 + 4 * tid; t4 < b0; t4 += 4 * NT) {
+            const Pooled4 c = pool4(rI, t4, Lc, halo);
+            *reinterpret_cast<float4*>(sl.I + (size_t)s * G.ML + t4) = make_float4(c.v[0], c.v[1], c.v[2], c.v[3]);
+        }
     }
-    const double mean = Lc > 0 ? block_sum(sum, red) / Lc : 0.0;
-    double m2 = 0.0;
-    for (int t = tid; t < Lc; t += NT) {
-        const double d = (double)sl.PO[row * G.ML + t] - mean;
-        m2 += d * d;
-    }
-    m2 = block_sum(m2, red);
-    const float sigma = Lc >= 2 ? (float)sqrt(m2 / (double)(Lc - 1)) : 0.f;
+    mom = block_moments(mom, red);
+    const float sigma = Lc >= 2 ? sqrtf(fmaxf(mom.m2, 0.f) / (float)(Lc - 1)) : 0.f;
     if (tid == 0) sig_self = sigma;
     for (int wd = tid; wd < G.words; wd += NT) bits[wd] = 0u;
     cluster.sync();
-    int rank = 0;
-    for (int o = 0; o < G.Hkv; ++o) {
-        const float so = *cluster.map_shared_rank(&sig_self, o);
-        if (so < sigma || (so == sigma && o < h)) ++rank;
+    __shared__ int top_flag;
+    if (tid < 32) {
+        const float so = tid < G.Hkv ? *cluster.map_shared_rank(&sig_self, tid) : INFINITY;
+        const bool before = tid < G.Hkv && (so < sigma || (so == sigma && tid < h));
+        const int rank = __popc(__ballot_sync(0xffffffffu, before));
+        if (tid == 0) top_flag = rank < G.delta;
     }
-    const int top = rank < G.delta;
+    __syncthreads();
+    const int top = top_flag;
     if (tid == 0) {
         sl.sigma[row] = sigma;
         sl.htop[row] = top;
@@ -276,7 +322,7 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
         const float* I = sl.I + (size_t)s * G.ML;
         const uint32_t* pres = sl.pres + row * G.words;
         float* Pp = sl.Pprime + row * G.ML;
-        uint32_t* keys = keys_in_smem(G.ML) ? bits + G.words : sc.keys + row * G.ML;
+        uint32_t* keys = keys_in_smem(G.ML) ? bits + G.words : sc.keys_sel + row * G.ML;
         const float denom = (float)(ell + 1u);
         for (int b0 = 4 * tid; b0 < Lc; b0 += 8 * NT) {
             float4 pv[2], iv[2];
@@ -397,14 +443,11 @@ size_t select_smem_bytes(const Geometry& g) {
     return sizeof(uint32_t) * ((size_t)g.words + (keys_in_smem(g.ML) ? (size_t)g.ML : 0));
 }
 
-size_t heads_smem_bytes(const Geometry& g) {
-    return select_smem_bytes(g) + sizeof(float) * (kPoolChunk + 2 * (kMaxPool / 2));
-}
+size_t heads_smem_bytes(const Geometry& g) { return select_smem_bytes(g); }
 
 cudaError_t configure_select() {
     const int need = (int)(sizeof(uint32_t) * (kSmemKeys + kSmemKeys / 32));
-    cudaError_t e = cudaFuncSetAttribute(heads_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         need + (int)sizeof(float) * (kPoolChunk + 2 * (kMaxPool / 2)));
+    cudaError_t e = cudaFuncSetAttribute(heads_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, need);
     if (e == cudaSuccess) e = cudaFuncSetAttribute(heads_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (e == cudaSuccess)
         e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, need);

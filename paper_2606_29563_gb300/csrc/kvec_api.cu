@@ -58,16 +58,18 @@ struct kvec_handle {
     void* ws = nullptr;
     size_t ws_bytes = 0;
     Scratch sc{};
+    Scratch score_buf[2]{};   // e-buffer, tile/segment/row statistics, counters: one per layer parity
     Slot slots[kSlots]{};
-    int last_slot = 0;
+    int last_slot = 0, last_parity = 0;
     int last_batch = 0;
     bool profiling = false;
     std::vector<TimedLaunch> timed;
     std::vector<cudaEvent_t> event_pool;
-    // Streams of the layer pipeline: score + window | heads | coverage select | gather.
-    cudaStream_t s_score = nullptr, s_heads = nullptr, s_chain = nullptr, s_gather = nullptr, s_cap = nullptr;
-    std::vector<cudaEvent_t> ev_win, ev_heads, ev_sel;
-    cudaEvent_t ev_fork = nullptr, ev_join[3] = {nullptr, nullptr, nullptr};
+    // Streams of the layer pipeline: score | window | heads | coverage select | gather.
+    cudaStream_t s_score = nullptr, s_win = nullptr, s_heads = nullptr, s_chain = nullptr, s_gather = nullptr,
+                 s_cap = nullptr;
+    std::vector<cudaEvent_t> ev_score, ev_win, ev_heads, ev_sel;
+    cudaEvent_t ev_fork = nullptr, ev_join[4] = {nullptr, nullptr, nullptr, nullptr};
     // CUDA graph of the last repeated multi-layer call.
     cudaGraphExec_t gexec = nullptr;
     std::vector<uint64_t> gkey, pending_key;
@@ -232,41 +234,48 @@ kvec_status run_layer_sequential(kvec_handle* h, const Geometry& G, const LayerI
         if (e_ != cudaSuccess) return cuda_fail(e_, #call);   \
     } while (0)
 
-// Layers 0..n-1 as a four-stream pipeline.  Only the coverage-adjusted select is
-// serial across layers (it carries n_t); the score, window and heads work of
-// later layers runs ahead of it, bounded by the kSlots ring of score arrays.
+// Layers 0..n-1 as a five-stream pipeline.  Only the coverage-adjusted select
+// is serial across layers (it carries n_t); the score, window and heads work of
+// later layers runs ahead of it, bounded by the double-buffered score scratch
+// and by the kSlots ring of per-layer score arrays.
 kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* ios, int n, cudaStream_t origin) {
     KV_CHECK(cudaEventRecord(h->ev_fork, origin));
-    for (cudaStream_t st : {h->s_score, h->s_heads, h->s_chain, h->s_gather})
+    for (cudaStream_t st : {h->s_score, h->s_win, h->s_heads, h->s_chain, h->s_gather})
         KV_CHECK(cudaStreamWaitEvent(st, h->ev_fork, 0));
     for (int l = 0; l < n; ++l) {
         const Slot& sl = h->slots[l % kSlots];
+        const Scratch& sc = h->score_buf[l & 1];
         const LayerIO& io = ios[l];
-        if (l >= kSlots) KV_CHECK(cudaStreamWaitEvent(h->s_score, h->ev_sel[l - kSlots], 0));
+        if (l >= 2) KV_CHECK(cudaStreamWaitEvent(h->s_score, h->ev_win[l - 2], 0));
         ScorePlan plan;
-        cudaError_t se = plan_score(G, io, h->sc, h->num_sms, &plan);
+        cudaError_t se = plan_score(G, io, sc, h->num_sms, &plan);
         if (se != cudaSuccess) return cuda_fail(se, "score kernel tensor maps");
         timed_launch(h, 0, h->s_score, [&] { se = launch_score(plan, h->s_score); });
         if (se != cudaSuccess) return cuda_fail(se, "score kernel launch");
-        timed_launch(h, 1, h->s_score, [&] { launch_window(G, io, h->sc, sl, h->s_score); });
-        KV_CHECK(cudaEventRecord(h->ev_win[l], h->s_score));
+        KV_CHECK(cudaEventRecord(h->ev_score[l], h->s_score));
+        KV_CHECK(cudaStreamWaitEvent(h->s_win, h->ev_score[l], 0));
+        if (l >= kSlots) KV_CHECK(cudaStreamWaitEvent(h->s_win, h->ev_sel[l - kSlots], 0));
+        timed_launch(h, 1, h->s_win, [&] { launch_window(G, io, sc, sl, h->s_win); });
+        KV_CHECK(cudaEventRecord(h->ev_win[l], h->s_win));
         KV_CHECK(cudaStreamWaitEvent(h->s_heads, h->ev_win[l], 0));
-        timed_launch(h, 2, h->s_heads, [&] { se = launch_heads(G, io, h->sc, sl, h->s_heads); });
+        timed_launch(h, 2, h->s_heads, [&] { se = launch_heads(G, io, sc, sl, h->s_heads); });
         if (se != cudaSuccess) return cuda_fail(se, "heads kernel launch");
         KV_CHECK(cudaEventRecord(h->ev_heads[l], h->s_heads));
         KV_CHECK(cudaStreamWaitEvent(h->s_chain, h->ev_heads[l], 0));
-        timed_launch(h, 3, h->s_chain, [&] { launch_select(G, io, h->sc, sl, h->s_chain); });
+        timed_launch(h, 3, h->s_chain, [&] { launch_select(G, io, sc, sl, h->s_chain); });
         KV_CHECK(cudaEventRecord(h->ev_sel[l], h->s_chain));
         KV_CHECK(cudaStreamWaitEvent(h->s_gather, h->ev_sel[l], 0));
         timed_launch(h, 4, h->s_gather, [&] { launch_gather(G, io, h->s_gather); });
     }
     KV_CHECK(cudaGetLastError());
     KV_CHECK(cudaEventRecord(h->ev_join[0], h->s_score));
-    KV_CHECK(cudaEventRecord(h->ev_join[1], h->s_heads));
-    KV_CHECK(cudaEventRecord(h->ev_join[2], h->s_gather));
+    KV_CHECK(cudaEventRecord(h->ev_join[1], h->s_win));
+    KV_CHECK(cudaEventRecord(h->ev_join[2], h->s_heads));
+    KV_CHECK(cudaEventRecord(h->ev_join[3], h->s_gather));
     KV_CHECK(cudaStreamWaitEvent(origin, h->ev_sel[n - 1], 0));
     for (cudaEvent_t e : h->ev_join) KV_CHECK(cudaStreamWaitEvent(origin, e, 0));
     h->last_slot = (n - 1) % kSlots;
+    h->last_parity = (n - 1) & 1;
     return KVEC_OK;
 }
 
@@ -289,9 +298,9 @@ namespace {
 
 void release_handle(kvec_handle* h) {
     if (h->gexec) cudaGraphExecDestroy(h->gexec);
-    for (cudaStream_t st : {h->s_score, h->s_heads, h->s_chain, h->s_gather, h->s_cap})
+    for (cudaStream_t st : {h->s_score, h->s_win, h->s_heads, h->s_chain, h->s_gather, h->s_cap})
         if (st) cudaStreamDestroy(st);
-    for (auto* v : {&h->ev_win, &h->ev_heads, &h->ev_sel})
+    for (auto* v : {&h->ev_score, &h->ev_win, &h->ev_heads, &h->ev_sel})
         for (cudaEvent_t ev : *v)
             if (ev) cudaEventDestroy(ev);
     if (h->ev_fork) cudaEventDestroy(h->ev_fork);
@@ -342,17 +351,24 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
         size_t bytes;
     };
     std::vector<Part> parts = {
-        {(void**)&h->sc.ebuf, max_tiles * Hkv * kTileT * R * sizeof(__half)},
-        {(void**)&h->sc.tstat, max_tiles * Hkv * R * sizeof(float2)},
-        {(void**)&h->sc.segpart, max_tiles * Hkv * R * sizeof(float2)},
-        {(void**)&h->sc.shcount, MB * Hkv * sizeof(unsigned)},
-        {(void**)&h->sc.rowstat, MB * Hkv * R * sizeof(float2)},
+
         {(void**)&h->sc.keys, MB * Hkv * ML * sizeof(uint32_t)},
         {(void**)&h->sc.ubits, MB * W * sizeof(uint32_t)},
         {(void**)&h->sc.ucount, MB * sizeof(unsigned)},
         {(void**)&h->sc.err, sizeof(int)},
         {(void**)&h->sc.keys_sel, MB * Hkv * ML * sizeof(uint32_t)},
     };
+    for (int k = 0; k < 2; ++k) {
+        Scratch& b = h->score_buf[k];
+        std::vector<Part> sp = {
+            {(void**)&b.ebuf, max_tiles * Hkv * kTileT * R * sizeof(__half)},
+            {(void**)&b.tstat, max_tiles * Hkv * R * sizeof(float2)},
+            {(void**)&b.segpart, max_tiles * Hkv * R * sizeof(float2)},
+            {(void**)&b.shcount, MB * Hkv * sizeof(unsigned)},
+            {(void**)&b.rowstat, MB * Hkv * R * sizeof(float2)},
+        };
+        parts.insert(parts.end(), sp.begin(), sp.end());
+    }
     for (int k = 0; k < kSlots; ++k) {
         Slot& sl = h->slots[k];
         std::vector<Part> sp = {
@@ -379,17 +395,25 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
         *pt.dst = static_cast<char*>(h->ws) + off;
         off += round_up(pt.bytes, 256);
     }
+    for (Scratch& b : h->score_buf) {
+        b.keys = h->sc.keys;
+        b.keys_sel = h->sc.keys_sel;
+        b.ubits = h->sc.ubits;
+        b.ucount = h->sc.ucount;
+        b.err = h->sc.err;
+    }
     Geometry G = make_geometry(h, 1, p.window, 1, 1, p.window);
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device);
     if (e == cudaSuccess) e = configure_score(G);
     if (e == cudaSuccess) e = configure_window(G);
     if (e == cudaSuccess) e = configure_select();
-    for (cudaStream_t* st : {&h->s_score, &h->s_heads, &h->s_chain, &h->s_gather, &h->s_cap})
+    for (cudaStream_t* st : {&h->s_score, &h->s_win, &h->s_heads, &h->s_chain, &h->s_gather, &h->s_cap})
         if (e == cudaSuccess) e = cudaStreamCreateWithFlags(st, cudaStreamNonBlocking);
+    h->ev_score.assign(p.max_layers, nullptr);
     h->ev_win.assign(p.max_layers, nullptr);
     h->ev_heads.assign(p.max_layers, nullptr);
     h->ev_sel.assign(p.max_layers, nullptr);
-    for (auto* v : {&h->ev_win, &h->ev_heads, &h->ev_sel})
+    for (auto* v : {&h->ev_score, &h->ev_win, &h->ev_heads, &h->ev_sel})
         for (auto& ev : *v)
             if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
     if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming);
@@ -487,6 +511,7 @@ kvec_status kvec_select_layers(kvec_handle* h, int num_layers, int batch, const 
         if (h->gexec && key == h->gkey) {
             KV_CHECK(cudaGraphLaunch(h->gexec, st));
             h->last_slot = (num_layers - 1) % kSlots;
+            h->last_parity = (num_layers - 1) & 1;
             h->last_batch = batch;
             return KVEC_OK;
         }
@@ -672,7 +697,7 @@ kvec_status kvec_debug_scores(kvec_handle* h, kvec_debug_view* out) {
     out->htop = sl.htop;
     out->pres_bits = sl.pres;
     out->Pprime = sl.Pprime;
-    out->row_stats = reinterpret_cast<const float*>(h->sc.rowstat);
+    out->row_stats = reinterpret_cast<const float*>(h->score_buf[h->last_parity].rowstat);
     out->max_seqlen = (int)row_stride(h->p.max_seqlen);
     out->words_per_row = h->words;
     return KVEC_OK;

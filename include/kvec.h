@@ -61,7 +61,7 @@ typedef struct {
     int   head_dim;       /* d; these kernels support 128 */
     int   window;         /* w: observation query rows given per sequence; the last w
                              tokens are always kept and count toward the budget */
-    int   obs_window;     /* O of Eq. 1 (paper: "e.g., 16"), 1 <= O <= w */
+    int   obs_window;     /* O of Eq. 1 (paper: "e.g., 16"), 1 <= O <= min(w, 64) */
     int   ext_window;     /* O' of Section 4.1 (paper default 32), 1 <= O' <= w */
     int   pool_kernel;    /* odd width of the 1-D max-pool over candidate scores, 1..15 */
     int   num_ext_heads;  /* delta of Section 4.1 (paper default 3), 0..H_kv */

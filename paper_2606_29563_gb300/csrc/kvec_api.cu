@@ -65,11 +65,15 @@ struct kvec_handle {
     bool profiling = false;
     std::vector<TimedLaunch> timed;
     std::vector<cudaEvent_t> event_pool;
-    // Streams of the layer pipeline: score | window | heads | coverage select | gather.
-    cudaStream_t s_score = nullptr, s_win = nullptr, s_heads = nullptr, s_chain = nullptr, s_gather = nullptr,
-                 s_cap = nullptr;
+    // Streams of the layer pipeline: score | window | heads (two, alternating by
+    // layer, so consecutive layers' head passes overlap) | coverage select | gather.
+    cudaStream_t s_score = nullptr, s_win = nullptr, s_heads = nullptr, s_heads2 = nullptr, s_chain = nullptr,
+                 s_gather = nullptr, s_cap = nullptr;
     std::vector<cudaEvent_t> ev_score, ev_win, ev_heads, ev_sel;
-    cudaEvent_t ev_fork = nullptr, ev_join[4] = {nullptr, nullptr, nullptr, nullptr};
+    cudaEvent_t ev_fork = nullptr, ev_join[5] = {nullptr, nullptr, nullptr, nullptr, nullptr};
+    // Scheduling priorities: the heads and coverage-select kernels (the serial
+    // chain of the pipeline) take SMs before the score, window and gather kernels.
+    int prio_hi = 0, prio_lo = 0;
     // CUDA graph of the last repeated multi-layer call.
     cudaGraphExec_t gexec = nullptr;
     std::vector<uint64_t> gkey, pending_key;
@@ -114,12 +118,14 @@ kvec_status validate_params(const kvec_params* p) {
     if (p->num_kv_heads < 1 || p->num_q_heads < p->num_kv_heads || p->num_q_heads % p->num_kv_heads)
         return fail(KVEC_ERR_INVALID_ARG, "num_q_heads (%d) must be a positive multiple of num_kv_heads (%d)",
                     p->num_q_heads, p->num_kv_heads);
-    if (p->num_kv_heads > 16)
-        return fail(KVEC_ERR_UNSUPPORTED, "num_kv_heads > 16 is not supported (one thread-block cluster per sequence)");
+    if (p->num_kv_heads > 32)
+        return fail(KVEC_ERR_UNSUPPORTED, "num_kv_heads > 32 is not supported (a token's KV heads share one warp)");
     if (p->head_dim != kHeadDim) return fail(KVEC_ERR_UNSUPPORTED, "head_dim must be %d", kHeadDim);
     if (p->window < 1) return fail(KVEC_ERR_INVALID_ARG, "window must be >= 1");
     if (p->obs_window < 1 || p->obs_window > p->window || p->ext_window < 1 || p->ext_window > p->window)
         return fail(KVEC_ERR_INVALID_ARG, "need 1 <= obs_window, ext_window <= window");
+    if (p->obs_window > kMaxObsWindow)
+        return fail(KVEC_ERR_UNSUPPORTED, "obs_window > %d is not supported", kMaxObsWindow);
     const int g = p->num_q_heads / p->num_kv_heads;
     if ((g * p->window) % 8 != 0 || g * p->window > 256)
         return fail(KVEC_ERR_UNSUPPORTED, "rows per KV head (group %d x window %d) must be a multiple of 8 and <= 256",
@@ -156,7 +162,7 @@ struct DeviceGuard {
 };
 
 kvec_status validate_call(kvec_handle* h, int batch, const int32_t* cu_host, const int32_t* cu_dev, int budget,
-                          int* total_tiles, int* total_chunks) {
+                          int* total_tiles, int* total_win_tiles) {
     if (!h) return fail(KVEC_ERR_INVALID_ARG, "handle is NULL");
     if (batch < 1 || batch > h->p.max_batch)
         return fail(KVEC_ERR_INVALID_ARG, "batch %d outside [1, max_batch=%d]", batch, h->p.max_batch);
@@ -170,10 +176,10 @@ kvec_status validate_call(kvec_handle* h, int batch, const int32_t* cu_host, con
             return fail(KVEC_ERR_INVALID_ARG, "sequence %d has length %d outside [window=%d, max_seqlen=%d]", b, L,
                         h->p.window, h->p.max_seqlen);
         tiles += (L + kTileT - 1) / kTileT;
-        chunks += window_blocks(L - h->p.window);
+        chunks += (L - h->p.window + kTileT - 1) / kTileT;   // candidate tiles of the window kernel
     }
     *total_tiles = tiles;
-    *total_chunks = chunks;
+    *total_win_tiles = chunks;
     return KVEC_OK;
 }
 
@@ -203,7 +209,9 @@ Geometry make_geometry(const kvec_handle* h, int batch, int budget, int tiles, i
     G.Kp = Kp;
     G.k2 = budget - p.window - Kp;
     G.total_tiles = tiles;
-    G.total_chunks = chunks;
+    G.win_tiles = chunks;
+    G.HG = p.num_kv_heads < kWinHeadsPerCta ? p.num_kv_heads : kWinHeadsPerCta;
+    G.NG = (p.num_kv_heads + G.HG - 1) / G.HG;
     G.total_tokens = total_tokens;
     G.state_stride = h->state_stride;
     G.state_n_off = h->n_off;
@@ -218,10 +226,12 @@ kvec_status run_layer_sequential(kvec_handle* h, const Geometry& G, const LayerI
     if (se != cudaSuccess) return cuda_fail(se, "score kernel tensor maps");
     se = launch_score(plan, st);
     if (se != cudaSuccess) return cuda_fail(se, "score kernel launch");
-    launch_window(G, io, h->sc, h->slots[0], st);
-    se = launch_heads(G, io, h->sc, h->slots[0], st);
+    se = launch_window(plan, G, io, h->sc, h->slots[0], st);
+    if (se != cudaSuccess) return cuda_fail(se, "window kernel launch");
+    se = launch_heads(G, io, h->sc, h->slots[0], st, h->prio_hi);
     if (se != cudaSuccess) return cuda_fail(se, "heads kernel launch");
-    launch_select(G, io, h->sc, h->slots[0], st);
+    se = launch_select(G, io, h->sc, h->slots[0], st, h->prio_hi);
+    if (se != cudaSuccess) return cuda_fail(se, "select kernel launch");
     launch_gather(G, io, st);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_fail(e, "kernel launch");
@@ -240,7 +250,7 @@ kvec_status run_layer_sequential(kvec_handle* h, const Geometry& G, const LayerI
 // and by the kSlots ring of per-layer score arrays.
 kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* ios, int n, cudaStream_t origin) {
     KV_CHECK(cudaEventRecord(h->ev_fork, origin));
-    for (cudaStream_t st : {h->s_score, h->s_win, h->s_heads, h->s_chain, h->s_gather})
+    for (cudaStream_t st : {h->s_score, h->s_win, h->s_heads, h->s_heads2, h->s_chain, h->s_gather})
         KV_CHECK(cudaStreamWaitEvent(st, h->ev_fork, 0));
     for (int l = 0; l < n; ++l) {
         const Slot& sl = h->slots[l % kSlots];
@@ -255,14 +265,17 @@ kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* io
         KV_CHECK(cudaEventRecord(h->ev_score[l], h->s_score));
         KV_CHECK(cudaStreamWaitEvent(h->s_win, h->ev_score[l], 0));
         if (l >= kSlots) KV_CHECK(cudaStreamWaitEvent(h->s_win, h->ev_sel[l - kSlots], 0));
-        timed_launch(h, 1, h->s_win, [&] { launch_window(G, io, sc, sl, h->s_win); });
+        timed_launch(h, 1, h->s_win, [&] { se = launch_window(plan, G, io, sc, sl, h->s_win); });
+        if (se != cudaSuccess) return cuda_fail(se, "window kernel launch");
         KV_CHECK(cudaEventRecord(h->ev_win[l], h->s_win));
-        KV_CHECK(cudaStreamWaitEvent(h->s_heads, h->ev_win[l], 0));
-        timed_launch(h, 2, h->s_heads, [&] { se = launch_heads(G, io, sc, sl, h->s_heads); });
+        cudaStream_t s_h = (l & 1) ? h->s_heads2 : h->s_heads;
+        KV_CHECK(cudaStreamWaitEvent(s_h, h->ev_win[l], 0));
+        timed_launch(h, 2, s_h, [&] { se = launch_heads(G, io, sc, sl, s_h, h->prio_hi); });
         if (se != cudaSuccess) return cuda_fail(se, "heads kernel launch");
-        KV_CHECK(cudaEventRecord(h->ev_heads[l], h->s_heads));
+        KV_CHECK(cudaEventRecord(h->ev_heads[l], s_h));
         KV_CHECK(cudaStreamWaitEvent(h->s_chain, h->ev_heads[l], 0));
-        timed_launch(h, 3, h->s_chain, [&] { launch_select(G, io, sc, sl, h->s_chain); });
+        timed_launch(h, 3, h->s_chain, [&] { se = launch_select(G, io, sc, sl, h->s_chain, h->prio_hi); });
+        if (se != cudaSuccess) return cuda_fail(se, "select kernel launch");
         KV_CHECK(cudaEventRecord(h->ev_sel[l], h->s_chain));
         KV_CHECK(cudaStreamWaitEvent(h->s_gather, h->ev_sel[l], 0));
         timed_launch(h, 4, h->s_gather, [&] { launch_gather(G, io, h->s_gather); });
@@ -272,6 +285,7 @@ kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* io
     KV_CHECK(cudaEventRecord(h->ev_join[1], h->s_win));
     KV_CHECK(cudaEventRecord(h->ev_join[2], h->s_heads));
     KV_CHECK(cudaEventRecord(h->ev_join[3], h->s_gather));
+    KV_CHECK(cudaEventRecord(h->ev_join[4], h->s_heads2));
     KV_CHECK(cudaStreamWaitEvent(origin, h->ev_sel[n - 1], 0));
     for (cudaEvent_t e : h->ev_join) KV_CHECK(cudaStreamWaitEvent(origin, e, 0));
     h->last_slot = (n - 1) % kSlots;
@@ -298,7 +312,7 @@ namespace {
 
 void release_handle(kvec_handle* h) {
     if (h->gexec) cudaGraphExecDestroy(h->gexec);
-    for (cudaStream_t st : {h->s_score, h->s_win, h->s_heads, h->s_chain, h->s_gather, h->s_cap})
+    for (cudaStream_t st : {h->s_score, h->s_win, h->s_heads, h->s_heads2, h->s_chain, h->s_gather, h->s_cap})
         if (st) cudaStreamDestroy(st);
     for (auto* v : {&h->ev_score, &h->ev_win, &h->ev_heads, &h->ev_sel})
         for (cudaEvent_t ev : *v)
@@ -346,6 +360,8 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
     const size_t MB = p.max_batch, ML = row_stride(p.max_seqlen), Hkv = p.num_kv_heads, R = h->R,
                  W = h->words;
     const size_t max_tiles = MB * ((ML + kTileT - 1) / kTileT);
+    const size_t HGmax = Hkv < (size_t)kWinHeadsPerCta ? Hkv : (size_t)kWinHeadsPerCta;
+    const size_t NGmax = (Hkv + HGmax - 1) / HGmax;
     struct Part {
         void** dst;
         size_t bytes;
@@ -361,9 +377,7 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
     for (int k = 0; k < 2; ++k) {
         Scratch& b = h->score_buf[k];
         std::vector<Part> sp = {
-            {(void**)&b.ebuf, max_tiles * Hkv * kTileT * R * sizeof(__half)},
-            {(void**)&b.tstat, max_tiles * Hkv * R * sizeof(float2)},
-            {(void**)&b.segpart, max_tiles * Hkv * R * sizeof(float2)},
+            {(void**)&b.segpart, max_tiles * Hkv * 2 * R * sizeof(float2)},
             {(void**)&b.shcount, MB * Hkv * sizeof(unsigned)},
             {(void**)&b.rowstat, MB * Hkv * R * sizeof(float2)},
         };
@@ -377,6 +391,7 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
             {(void**)&sl.POe, MB * Hkv * ML * sizeof(float)},   {(void**)&sl.I, MB * ML * sizeof(float)},
             {(void**)&sl.sigma, MB * Hkv * sizeof(float)},      {(void**)&sl.htop, MB * Hkv * sizeof(int)},
             {(void**)&sl.pres, MB * Hkv * W * sizeof(uint32_t)}, {(void**)&sl.Pprime, MB * Hkv * ML * sizeof(float)},
+            {(void**)&sl.wpart, max_tiles * NGmax * p.obs_window * kTileT * sizeof(float)},
         };
         parts.insert(parts.end(), sp.begin(), sp.end());
     }
@@ -407,8 +422,11 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
     if (e == cudaSuccess) e = configure_score(G);
     if (e == cudaSuccess) e = configure_window(G);
     if (e == cudaSuccess) e = configure_select();
-    for (cudaStream_t* st : {&h->s_score, &h->s_win, &h->s_heads, &h->s_chain, &h->s_gather, &h->s_cap})
-        if (e == cudaSuccess) e = cudaStreamCreateWithFlags(st, cudaStreamNonBlocking);
+    if (e == cudaSuccess) e = cudaDeviceGetStreamPriorityRange(&h->prio_lo, &h->prio_hi);
+    for (cudaStream_t* st : {&h->s_score, &h->s_win, &h->s_gather, &h->s_cap})
+        if (e == cudaSuccess) e = cudaStreamCreateWithPriority(st, cudaStreamNonBlocking, h->prio_lo);
+    for (cudaStream_t* st : {&h->s_heads, &h->s_heads2, &h->s_chain})
+        if (e == cudaSuccess) e = cudaStreamCreateWithPriority(st, cudaStreamNonBlocking, h->prio_hi);
     h->ev_score.assign(p.max_layers, nullptr);
     h->ev_win.assign(p.max_layers, nullptr);
     h->ev_heads.assign(p.max_layers, nullptr);
@@ -526,7 +544,7 @@ kvec_status kvec_select_layers(kvec_handle* h, int num_layers, int batch, const 
             }
             if (ce != cudaSuccess) return cuda_fail(ce, "cudaStreamEndCapture");
             cudaGraphExec_t exec = nullptr;
-            ce = cudaGraphInstantiate(&exec, graph, 0);
+            ce = cudaGraphInstantiateWithFlags(&exec, graph, cudaGraphInstantiateFlagUseNodePriority);
             cudaGraphDestroy(graph);
             if (ce != cudaSuccess) return cuda_fail(ce, "cudaGraphInstantiate");
             if (h->gexec) cudaGraphExecDestroy(h->gexec);
@@ -622,14 +640,15 @@ kvec_status kvec_select_layer_noalloc(const kvec_params* params, int batch, cons
         void** dst;
         size_t bytes;
     };
+    const size_t HGv = Hkv < (size_t)kWinHeadsPerCta ? Hkv : (size_t)kWinHeadsPerCta;
+    const size_t NGv = (Hkv + HGv - 1) / HGv;
     Part parts[] = {
         {(void**)&tmp.sc.ucount, nb * sizeof(unsigned)},      // zeroed every call (first four parts)
         {(void**)&tmp.sc.err, sizeof(int)},
         {(void**)&tmp.sc.ubits, nb * W * sizeof(uint32_t)},
         {(void**)&tmp.sc.shcount, nb * Hkv * sizeof(unsigned)},
-        {(void**)&tmp.sc.segpart, nt * Hkv * R * sizeof(float2)},
-        {(void**)&tmp.sc.ebuf, nt * Hkv * kTileT * R * sizeof(__half)},
-        {(void**)&tmp.sc.tstat, nt * Hkv * R * sizeof(float2)},
+        {(void**)&tmp.sc.segpart, nt * Hkv * 2 * R * sizeof(float2)},
+        {(void**)&tmp.slots[0].wpart, nt * NGv * (size_t)params->obs_window * kTileT * sizeof(float)},
         {(void**)&tmp.sc.rowstat, nb * Hkv * R * sizeof(float2)},
         {(void**)&tmp.sc.keys, nb * Hkv * ML * sizeof(uint32_t)},
         {(void**)&tmp.sc.keys_sel, nb * Hkv * ML * sizeof(uint32_t)},

@@ -10,10 +10,11 @@
 namespace kvec {
 
 constexpr int kHeadDim = 128;      // d supported by the score kernel
-constexpr int kTileT = 128;        // tokens per score tile (one MMA N block / e-buffer tile)
+constexpr int kTileT = 128;        // tokens per score / window tile (one MMA N or M block)
 constexpr int kMaxPool = 15;       // largest pool kernel (halo 7)
-constexpr int kSelectThreads = 1024;
-constexpr float kEScaleLog2 = 15.f;  // e values are stored as fp16(2^15 * exp(s - mu))
+constexpr int kSelectThreads = 512;
+constexpr int kMaxObsWindow = 64;  // largest O: the window kernel keeps O x 128 head maxima in shared memory
+constexpr int kWinHeadsPerCta = 4; // KV heads one window CTA processes
 
 // Sizes and hyper-parameters shared by every kernel of one call.
 struct Geometry {
@@ -25,7 +26,8 @@ struct Geometry {
     int words;         // ceil(ML / 32)
     int batch, budget, Kp, k2;
     int total_tiles;   // sum over sequences of ceil(L_s / kTileT)
-    int total_chunks;  // window-kernel blocks: sum over sequences of window_blocks(L_s - w)
+    int win_tiles;     // sum over sequences of ceil((L_s - w) / kTileT): candidate tiles
+    int HG, NG;        // KV heads per window CTA, window CTAs per candidate tile
     int total_tokens;  // cu_seqlens[batch]
     const int* cu_host;  // host copy of cu_seqlens (host-side planning only; not for device code)
     size_t state_stride;
@@ -44,12 +46,11 @@ struct Slot {
     int* htop;            // [max_batch][Hkv]
     uint32_t* pres;       // [max_batch][Hkv][words]
     float* Pprime;        // [max_batch][Hkv][ML]
+    float* wpart;         // [win_tiles][NG][O][kTileT] per-group head maxima of G_h[q][t] (NG > 1)
 };
 
 struct Scratch {
-    __half* ebuf;         // [total_tiles][Hkv][R][kTileT]  scaled exp(s - mu_tile), row-major
-    float2* tstat;        // [total_tiles][Hkv][R]  (mu_tile in log2 units, sum of exp)
-    float2* segpart;      // [total_tiles * Hkv][R] per-CTA segment (max, sum) keyed by first item
+    float2* segpart;      // [total_tiles * Hkv][2][R] per-CTA segment (max, sum) per column half, keyed by first item
     unsigned* shcount;    // [max_batch][Hkv]       tiles finished per (sequence, KV head)
     float2* rowstat;      // [max_batch][Hkv][R]    (row max in log2 units, softmax denominator)
     uint32_t* keys;       // [max_batch][Hkv][ML]   radix-select keys of the heads kernel
@@ -97,21 +98,46 @@ __device__ __forceinline__ int tiles_of(int L) { return (L + kTileT - 1) / kTile
 
 // Host-side launch description of the score kernel (tensor maps encoded ahead of the launch).
 struct ScorePlan {
-    CUtensorMap kmap, qmap, emap;
+    CUtensorMap kmap, qmap;
     alignas(16) unsigned char args[512];
     int grid, threads;
     size_t smem;
 };
 cudaError_t plan_score(const Geometry& g, const LayerIO& io, const Scratch& sc, int num_sms, ScorePlan* plan);
 cudaError_t launch_score(const ScorePlan& plan, cudaStream_t st);
-void launch_window(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st);
-cudaError_t launch_heads(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st);
-void launch_select(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st);
+cudaError_t launch_window(const ScorePlan& sp, const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl,
+                          cudaStream_t st);
+// Launches kernel<<<grid, block, smem, st>>> with a scheduling priority (lower
+// numbers first; the range comes from cudaDeviceGetStreamPriorityRange) and,
+// with `programmatic`, as a programmatic dependent of the stream's previous
+// kernel: it may start once that grid triggers launch_dependents and must
+// execute griddepcontrol.wait before it reads what that grid writes.
+template <class... KArgs, class... Args>
+cudaError_t launch_prio(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st, int priority,
+                        bool programmatic, Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributePriority;
+    attr[0].val.priority = priority;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = programmatic ? 2 : 1;
+    return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
+cudaError_t launch_heads(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st,
+                         int priority);
+cudaError_t launch_select(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st,
+                          int priority);
 void launch_gather(const Geometry& g, const LayerIO& io, cudaStream_t st);
 
 size_t score_smem_bytes(const Geometry& g);
 size_t window_smem_bytes(const Geometry& g);
-int window_blocks(int Lc);
 cudaError_t configure_score(const Geometry& g);
 cudaError_t configure_window(const Geometry& g);
 cudaError_t configure_select();

@@ -1,21 +1,21 @@
-// Window-query scores against every prefix key, s = <q_obs, k_t> (the logits of
-// the attention A that Eq. 1 averages), and the softmax over every visible key,
-// split into tile partials that are merged in the same launch.
+// Softmax statistics of the window queries' attention over every visible key
+// (the denominators of the attention A that Eq. 1 averages): for each query
+// row r of KV head h, the row max m_r of s = <q_r, k_t> * scale (log2 units)
+// and Z_r = sum_t 2^(s_rt - m_r), causal on the window part.
 //
 // Persistent, warp-specialised, one CTA per SM; a CTA walks a contiguous range
 // of work items (sequence s, KV head h, 128-token tile j):
 //   warp 0      TMA producer: the KV head's g*w query rows (once per (s,h)) and
-//               a 3-stage ring of 128-token K tiles, both 128-byte swizzled;
+//               a ring of 128-token K tiles, both 128-byte swizzled;
 //   warp 1      one thread issues tcgen05.mma (M = 128 query rows per M-block,
 //               N = 128 tokens, K = 128 = d) into TMEM accumulators;
 //   warps 2..   epilogue, one thread per (query row, half of the tile's
-//               columns): tcgen05.ld of 64 logits, the row's tile max mu (the
-//               two halves exchange partial maxima), e = exp(s - mu) and row
-//               sums; e is packed to fp16(2^15 e), staged row-major in a
-//               128-byte-swizzled tile and written by a TMA tiled store.
-// Outputs: ebuf[tile][h][r][t], tstat[tile][h][r] = (mu in log2 units, sum e),
-// and rowstat[s][h][r] = (row max, softmax denominator) merged from per-CTA
-// segment partials by the last CTA to finish a (s, h).
+//               columns): tcgen05.ld of 64 logits, their max and sum of
+//               2^(s - max), merged online into the thread's running
+//               (max, sum) of the CTA's contiguous segment of (s, h).
+// Each CTA writes one (max, sum) partial per segment, row and column half; the
+// last CTA to finish a (s, h) merges them into rowstat[s][h][r] = (m_r, Z_r).
+// The window kernel recomputes the logits with these statistics.
 #include <cudaTypedefs.h>
 
 #include "kvec_internal.cuh"
@@ -25,7 +25,7 @@ namespace kvec {
 
 namespace {
 
-constexpr int kKStages = 3;                           // deepest K ring (2 when shared memory is short)
+constexpr int kKStages = 4;                           // deepest K ring (fewer when shared memory is short)
 constexpr int kMaxSmem = 232448;                      // opt-in shared memory per CTA on sm_103
 constexpr int kKStageBytes = kTileT * kHeadDim * 2;   // 32 KB: two 64-column swizzled halves
 constexpr int kKHalfBytes = kTileT * 128;             // 16 KB
@@ -64,7 +64,8 @@ __device__ __forceinline__ int range_start(int b, int W, int G) {
     return b * q + min(b, r);
 }
 
-constexpr int kMaxCuParam = 64;   // sequences whose offsets travel in the kernel parameters
+constexpr int kMaxCuParam = 64;          // sequences whose offsets travel in the kernel parameters
+constexpr int kScoreReserveSms = 8;      // SMs a score launch leaves to the other kernels
 
 struct ScoreArgs {
     Geometry G;
@@ -76,7 +77,6 @@ struct ScoreArgs {
     int W;        // total work items
     int MB;       // 128-row M-blocks per KV head (1 or 2)
     int Rpad;     // 128 * MB
-    int ebufs;    // e staging buffers (2 when MB == 1)
     int kst;      // K ring depth
 };
 
@@ -89,8 +89,7 @@ struct __align__(8) Barriers {
     volatile int abort_flag;
     volatile int last_flag;
     volatile int go;
-    float zhalf[256];          // row sums of the second column half
-    float pmax[2][256];        // per-half row maxima of the current tile
+    float2 xfer[256];          // merged (max, sum) of the second column half, last CTA only
 };
 
 __device__ __forceinline__ void raise_abort(Barriers* bars, int* err) {
@@ -100,7 +99,7 @@ __device__ __forceinline__ void raise_abort(Barriers* bars, int* err) {
 
 __global__ void __launch_bounds__(576, 1)
     score_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap qmap,
-                 const __grid_constant__ CUtensorMap emap, const __grid_constant__ ScoreArgs A) {
+                 const __grid_constant__ ScoreArgs A) {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     // 1024-byte alignment for the swizzled operand tiles.
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -108,9 +107,7 @@ __global__ void __launch_bounds__(576, 1)
     const int MB = A.MB, Rpad = A.Rpad, R = G.R;
     uint8_t* sQ = smem;                                   // 2 halves x Rpad rows x 128 B
     uint8_t* sK = sQ + 2 * Rpad * 128;                    // A.kst x 32 KB
-    uint8_t* sE = sK + A.kst * kKStageBytes;           // ebufs x 2 halves x R rows x 128 B (swizzled)
-    const int ebytes = kTileT * R * 2;
-    Barriers* bars = reinterpret_cast<Barriers*>(sE + A.ebufs * ebytes);
+    Barriers* bars = reinterpret_cast<Barriers*>(sK + A.kst * kKStageBytes);
 
     const bool cu_param = G.batch <= kMaxCuParam;
     auto cu = [&](int b) { return cu_param ? A.cuv[b] : A.cu[b]; };
@@ -146,7 +143,6 @@ __global__ void __launch_bounds__(576, 1)
     if (warp == 0 && lane == 0) {
         ptx::prefetch_tensormap(&kmap);
         ptx::prefetch_tensormap(&qmap);
-        ptx::prefetch_tensormap(&emap);
     }
     ptx::tc_fence_before();
     __syncthreads();
@@ -167,9 +163,9 @@ __global__ void __launch_bounds__(576, 1)
                     ptx::prefetch_l2_bulk(A.kbytes + o, (uint32_t)(n & ~15LL));
                 }
             }
-            const uint64_t policy = ptx::policy_evict_first();
+            const uint64_t policy = ptx::policy_evict_normal();   // the window kernel reads K again
             int prev_sh = -1, qloads = 0;
-            int fills[kKStages] = {0, 0, 0};
+            int fills[kKStages] = {0, 0, 0, 0};
             for (int i = i0, it = 0; i < i1 && !bars->abort_flag; ++i, ++it) {
                 const ItemPos p = decode_item(cuview, G.batch, G.Hkv, i);
                 const int sh = p.s * G.Hkv + p.h;
@@ -264,7 +260,7 @@ __global__ void __launch_bounds__(576, 1)
         int cur_sh = -1, seg_first = 0, seg_n = 0, seg_s = 0, seg_h = 0, seg_ibase = 0, seg_nt = 0;
 
         auto flush_segment = [&]() {
-            if (vrow && half == 0) A.sc.segpart[(size_t)seg_first * R + row] = make_float2(seg_m, seg_z);
+            if (vrow) A.sc.segpart[((size_t)seg_first * 2 + half) * R + row] = make_float2(seg_m, seg_z);
             ptx::named_bar_sync(1, nepi);
             if (issuer) {
                 // The barrier orders the CTA's writes before this thread's fence (cumulativity).
@@ -274,10 +270,11 @@ __global__ void __launch_bounds__(576, 1)
                 bars->last_flag = old + (unsigned)seg_n == (unsigned)seg_nt;
             }
             ptx::named_bar_sync(1, nepi);
-            if (bars->last_flag && half == 0) {
-                // Gather the segment starts of (s, h), then load them in independent batches.
+            if (bars->last_flag) {
+                // Merge the partials of (s, h): each half its own column half, every
+                // segment start (the first item, then each CTA range start after it)
+                // loaded in independent batches; then the halves combine.
                 float M = -INFINITY, Z = 0.f;
-                // Segment starts of (s, h): its first item and every CTA range start after it.
                 const int qW = A.W / Gc, rW = A.W % Gc;
                 const int iend = seg_ibase + seg_nt;
                 auto cta_of = [&](int i) { return i < rW * (qW + 1) ? i / (qW + 1) : rW + (i - rW * (qW + 1)) / qW; };
@@ -285,15 +282,13 @@ __global__ void __launch_bounds__(576, 1)
                 int next = seg_ibase;
                 while (next < iend) {
                     float2 pz[16];
-                    int n = 0;
 #pragma unroll
                     for (int k = 0; k < 16; ++k) {
                         pz[k] = make_float2(-INFINITY, 0.f);
                         if (next < iend) {
-                            if (vrow) pz[k] = __ldcg(&A.sc.segpart[(size_t)next * R + row]);
+                            if (vrow) pz[k] = __ldcg(&A.sc.segpart[((size_t)next * 2 + half) * R + row]);
                             next = b * qW + min(b, rW);
                             ++b;
-                            ++n;
                         }
                     }
 #pragma unroll
@@ -307,7 +302,20 @@ __global__ void __launch_bounds__(576, 1)
                         }
                     }
                 }
-                if (vrow) A.sc.rowstat[((size_t)seg_s * G.Hkv + seg_h) * R + row] = make_float2(M, Z);
+                if (half == 1) bars->xfer[row] = make_float2(M, Z);
+                ptx::named_bar_sync(1, nepi);
+                if (half == 0) {
+                    const float2 o = bars->xfer[row];
+                    if (o.x != -INFINITY) {
+                        if (o.x > M) {
+                            Z = Z * ptx::ex2(M - o.x) + o.y;
+                            M = o.x;
+                        } else {
+                            Z += o.y * ptx::ex2(o.x - M);
+                        }
+                    }
+                    if (vrow) A.sc.rowstat[((size_t)seg_s * G.Hkv + seg_h) * R + row] = make_float2(M, Z);
+                }
                 if (issuer) A.sc.shcount[seg_s * G.Hkv + seg_h] = 0u;
             }
         };
@@ -328,15 +336,11 @@ __global__ void __launch_bounds__(576, 1)
                 seg_nt = p.ntiles;
             }
             const int buf = it % NB, nb = it / NB;
-            // One thread waits for the accumulator and for the staging buffer, then
-            // publishes the outcome; every epilogue thread takes the same branch.
+            // One thread waits for the accumulator and publishes the outcome; every
+            // epilogue thread takes the same branch.
             if (issuer) {
                 const bool ok = !bars->abort_flag && ptx::mbar_wait(&bars->acc_full[buf], nb & 1);
                 if (!ok) raise_abort(bars, A.sc.err);
-                if (A.ebufs == 2)
-                    asm volatile("cp.async.bulk.wait_group.read 1;\n" ::: "memory");
-                else
-                    ptx::bulk_wait_read_all();
                 bars->go = ok ? 1 : 0;
             }
             ptx::named_bar_sync(1, nepi);
@@ -350,7 +354,7 @@ __global__ void __launch_bounds__(576, 1)
             const int t0 = p.j * kTileT;
             const int last = vrow ? min(L - 1, L - G.w + q) : -1;   // causal on the window part
             const int nvalid = max(0, min(kTileT, last - t0 + 1));
-            // This warp's 64 columns of the accumulator; the row max is combined across the halves.
+            // This warp's 64 columns of the accumulator.
             const int c0 = half * 64;
             float v[64];
             ptx::tmem_ld32(taddr + c0, v);
@@ -360,6 +364,10 @@ __global__ void __launch_bounds__(576, 1)
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&bars->acc_empty[buf]);
             const int lim = nvalid - c0;
+            if (lim <= 0) {
+                ++seg_n;
+                continue;
+            }
             float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
             if (lim >= 64) {
 #pragma unroll
@@ -369,55 +377,26 @@ __global__ void __launch_bounds__(576, 1)
                 for (int c = 0; c < 64; ++c)
                     if (c < lim) m4[c & 3] = fmaxf(m4[c & 3], v[c]);
             }
-            bars->pmax[half][row] = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
-            ptx::named_bar_sync(1, nepi);
-            const float mx = fmaxf(bars->pmax[0][row], bars->pmax[1][row]);
-            const float mu = mx * G.sl2;                           // -inf when nothing is visible
-            const float bias = kEScaleLog2 - mu;                   // stores 2^15 * exp(s - mu)
-            const int eb = A.ebufs == 2 ? (it & 1) : 0;
-            // Row-major staging [half][row][64 tokens], 16-byte chunk k of a row at chunk k ^ (row % 8)
-            // (the tensor map's 128-byte swizzle).
-            const uint32_t srow = ptx::smem_u32(sE + eb * ebytes + half * (R * 128)) + (uint32_t)(row * 128);
+            const float mu = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * G.sl2;
             float z4[4] = {0.f, 0.f, 0.f, 0.f};
+            if (lim >= 64) {
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
-                float e[8];
+                for (int c = 0; c < 64; ++c) z4[c & 3] += ptx::ex2(fmaf(v[c], G.sl2, -mu));
+            } else {
 #pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const int c = k * 8 + i;
-                    e[i] = (lim >= 64 || c < lim) ? ptx::ex2(fmaf(v[c], G.sl2, bias)) : 0.f;
-                    z4[i & 3] += e[i];
-                }
-                if (vrow)
-                    ptx::st_shared_v4(srow + (uint32_t)((k ^ (row & 7)) * 16), ptx::pack_half2(e[0], e[1]),
-                                      ptx::pack_half2(e[2], e[3]), ptx::pack_half2(e[4], e[5]),
-                                      ptx::pack_half2(e[6], e[7]));
+                for (int c = 0; c < 64; ++c)
+                    if (c < lim) z4[c & 3] += ptx::ex2(fmaf(v[c], G.sl2, -mu));
             }
-            float z = ((z4[0] + z4[1]) + (z4[2] + z4[3])) * (1.f / 32768.f);
-            if (half == 1) bars->zhalf[row] = z;
-            ptx::fence_proxy_async_smem();
-            ptx::named_bar_sync(1, nepi);
-            if (issuer) {
-                const int erow0 = (p.gt * G.Hkv + p.h) * R;
-                ptx::tma_store_2d(&emap, sE + eb * ebytes, 0, erow0);
-                ptx::tma_store_2d(&emap, sE + eb * ebytes + R * 128, 64, erow0);
-                ptx::bulk_commit();
-            }
-            if (half == 1) continue;                               // sums and statistics live in half 0
-            z += bars->zhalf[row];
-            if (vrow) A.sc.tstat[((size_t)p.gt * G.Hkv + p.h) * R + row] = make_float2(mu, z);
-            if (mu != -INFINITY) {
-                if (mu > seg_m) {
-                    seg_z = seg_z * ptx::ex2(seg_m - mu) + z;
-                    seg_m = mu;
-                } else {
-                    seg_z += z * ptx::ex2(mu - seg_m);
-                }
+            const float z = (z4[0] + z4[1]) + (z4[2] + z4[3]);
+            if (mu > seg_m) {
+                seg_z = seg_z * ptx::ex2(seg_m - mu) + z;
+                seg_m = mu;
+            } else {
+                seg_z += z * ptx::ex2(mu - seg_m);
             }
             ++seg_n;
         }
         if (cur_sh >= 0 && !aborted) flush_segment();
-        if (issuer) ptx::bulk_wait_all();
     }
 
     // ---------------------------------------------------------------- teardown
@@ -445,12 +424,14 @@ int mblocks(const Geometry& g) { return g.R > 128 ? 2 : 1; }
 
 size_t smem_bytes_with(const Geometry& g, int kst) {
     const int MB = mblocks(g);
-    const int ebufs = MB == 1 ? 2 : 1;
-    return 1024 + 2 * (size_t)MB * 128 * 128 + (size_t)kst * kKStageBytes + (size_t)ebufs * kTileT * g.R * 2 +
-           sizeof(Barriers);
+    return 1024 + 2 * (size_t)MB * 128 * 128 + (size_t)kst * kKStageBytes + sizeof(Barriers);
 }
 
-int kstages_for(const Geometry& g) { return smem_bytes_with(g, kKStages) <= (size_t)kMaxSmem ? kKStages : 2; }
+int kstages_for(const Geometry& g) {
+    int kst = kKStages;
+    while (kst > 2 && smem_bytes_with(g, kst) > (size_t)kMaxSmem) --kst;
+    return kst;
+}
 
 size_t smem_bytes_for(const Geometry& g) { return smem_bytes_with(g, kstages_for(g)); }
 
@@ -495,16 +476,6 @@ cudaError_t plan_score(const Geometry& g, const LayerIO& io, const Scratch& sc, 
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return cudaErrorInvalidValue;
     }
-    {
-        cuuint64_t dims[2] = {(cuuint64_t)kTileT, (cuuint64_t)g.total_tiles * g.Hkv * g.R};
-        cuuint64_t strides[1] = {(cuuint64_t)kTileT * 2};
-        cuuint32_t box[2] = {64, (cuuint32_t)g.R};
-        cuuint32_t es[2] = {1, 1};
-        if (enc(&plan->emap, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, sc.ebuf, dims, strides, box, es,
-                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
-                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
-            return cudaErrorInvalidValue;
-    }
     ScoreArgs& a = *reinterpret_cast<ScoreArgs*>(plan->args);
     static_assert(sizeof(ScoreArgs) <= sizeof(plan->args), "ScorePlan::args too small");
     a = ScoreArgs{};
@@ -517,16 +488,20 @@ cudaError_t plan_score(const Geometry& g, const LayerIO& io, const Scratch& sc, 
     a.W = g.total_tiles * g.Hkv;
     a.MB = mblocks(g);
     a.Rpad = 128 * a.MB;
-    a.ebufs = a.MB == 1 ? 2 : 1;
     a.kst = kstages_for(g);
-    plan->grid = a.W < num_sms ? a.W : num_sms;
+    // As few CTAs as give the same items per CTA on all but kScoreReserveSms SMs:
+    // the SMs left free run the window, heads and selection kernels of other
+    // layers, which cannot share an SM with a score CTA.
+    const int usable = num_sms > 2 * kScoreReserveSms ? num_sms - kScoreReserveSms : num_sms;
+    const int per_cta = (a.W + usable - 1) / usable;
+    plan->grid = (a.W + per_cta - 1) / per_cta;
     plan->threads = 32 * (2 + 8 * a.MB);
     plan->smem = smem_bytes_for(g);
     return cudaSuccess;
 }
 
 cudaError_t launch_score(const ScorePlan& plan, cudaStream_t st) {
-    score_kernel<<<plan.grid, plan.threads, plan.smem, st>>>(plan.kmap, plan.qmap, plan.emap,
+    score_kernel<<<plan.grid, plan.threads, plan.smem, st>>>(plan.kmap, plan.qmap,
                                                               *reinterpret_cast<const ScoreArgs*>(plan.args));
     return cudaGetLastError();
 }

@@ -2,14 +2,11 @@
 // coverage-state update (Section 4.1, Section 4.2, Algorithm 1), plus the K/V
 // gather into the budget-sized cache.
 //
-// Top-k is an exact block-wide MSB radix select over order-preserving uint32
-// keys (11/11/10-bit digits, shared-memory histograms, block scans built from
-// warp shuffles and ballots).  Ties at the threshold go to the lower position.
-#include <cooperative_groups.h>
-
+// Top-k is an exact MSB radix select over order-preserving uint32 keys (bits
+// shared by all keys skipped, 4-bit digits counted in registers, one barrier
+// per digit, small threshold buckets compacted and ranked directly).  Ties at
+// the threshold go to the lower position.
 #include "kvec_internal.cuh"
-
-namespace cg = cooperative_groups;
 
 namespace kvec {
 
@@ -19,10 +16,30 @@ constexpr int kSmemKeys = 40960;   // positions whose keys fit in shared memory 
 
 __host__ __device__ inline bool keys_in_smem(int ML) { return ML <= kSmemKeys; }
 
+// Key rows are stored transposed, key t at keys[(t & 31) * kw + (t >> 5)]: a lane
+// that owns the 32 positions of one bits word then reads them from consecutive
+// words of its warp's neighbours (an odd stride keeps the writers' banks apart).
+__host__ __device__ inline int key_stride(const Geometry& g) { return keys_in_smem(g.ML) ? (g.words | 1) : g.words; }
+__device__ __forceinline__ int key_index(int t, int kw) { return (t & 31) * kw + (t >> 5); }
+
+constexpr int kIChunk = 2048;                  // positions of raw I combined per pass in the heads kernel
+constexpr int kTopkWarps = 8;                  // warps that run the radix select
+constexpr int kTopkThreads = 32 * kTopkWarps;
+constexpr int kTopkSeg = 1024;                 // positions per warp segment (32 per lane)
+constexpr int kTopkBarrier = 1;                // named barrier of the select warps
+constexpr int kTopkCap = 1792;                 // keys a compacted candidate list holds (7 per thread)
+constexpr int kTopkFew = 32;                   // a threshold bucket this small is ranked directly
+
 struct TopkShared {
-    int hist[2048];
+    int wcnt[2][kTopkWarps][16];   // per-warp digit counts, double-buffered across passes
+    uint32_t wor[kTopkWarps], wand[kTopkWarps];
+    int weq[kTopkWarps];
     int wsum[32];
-    int bcast[4];
+    int fcount;
+    uint32_t fkey[kTopkFew];
+    int fpos[kTopkFew];
+    uint32_t ckey[kTopkCap];       // compacted candidates: key and position
+    int cpos[kTopkCap];
 };
 
 // Exclusive prefix sum over the block (blockDim.x a multiple of 32, <= 1024).
@@ -52,74 +69,355 @@ __device__ int block_exclusive_sum(int v, int* wsum, int& total) {
     return before + x - v;
 }
 
-// ORs into bits[] (shared, one bit per position) the k largest keys of keys[0, n).
-// Key 0 marks an ineligible position; the caller guarantees k <= #eligible.
-__device__ void block_topk(const uint32_t* __restrict__ keys, int n, int k, uint32_t* bits, TopkShared& sm) {
-    if (k <= 0 || n <= 0) return;
-    const int tid = threadIdx.x, NT = blockDim.x;
-    uint32_t prefix = 0, mask = 0;
-    int kk = k;
-    bool whole_bin = false;
-    for (int pass = 0; pass < 3; ++pass) {
-        const int sh = pass == 0 ? 21 : (pass == 1 ? 10 : 0);
-        const int nb = pass == 2 ? 1024 : 2048;
-        for (int i = tid; i < nb; i += NT) sm.hist[i] = 0;
-        __syncthreads();
-        for (int t = tid; t < n; t += NT) {
-            const uint32_t u = keys[t];
-            if (u != 0u && (u & mask) == prefix) atomicAdd(&sm.hist[(u >> sh) & (nb - 1)], 1);
-        }
-        __syncthreads();
-        // Thread i owns the i-th block of bins counted from the top.
-        const int bpt = (nb + NT - 1) / NT;
-        const int hi = nb - tid * bpt, lo = max(hi - bpt, 0);
-        int mine = 0;
-        for (int b = lo; b < hi; ++b) mine += sm.hist[b];
-        int total;
-        const int above_me = block_exclusive_sum(mine, sm.wsum, total);
-        if (hi > 0 && above_me < kk && above_me + mine >= kk) {
-            int acc = above_me;
-            for (int b = hi - 1; b >= lo; --b) {
-                if (acc + sm.hist[b] >= kk) {
-                    sm.bcast[0] = b;
-                    sm.bcast[1] = acc;
-                    sm.bcast[2] = sm.hist[b];
-                    break;
+__device__ __forceinline__ void topk_bar() {
+    asm volatile("bar.sync %0, %1;" ::"n"(kTopkBarrier), "n"(kTopkThreads) : "memory");
+}
+
+// Digit counting without divergent branches: a key adds 1 << (4 d) to a 64-bit
+// accumulator of sixteen 4-bit counters (at most 15 keys per accumulator),
+// which is then spread into byte counters of the even and odd digits.
+__device__ __forceinline__ unsigned long long digit_nibble(uint32_t u, uint32_t mask, uint32_t prefix, int lo,
+                                                           uint32_t wmask) {
+    const uint32_t m = (u != 0u && (u & mask) == prefix) ? 1u : 0u;
+    return (unsigned long long)m << (((u >> lo) & wmask) << 2);
+}
+
+struct DigitBytes {
+    unsigned long long ev = 0ull, od = 0ull;   // byte j: count of digit 2j / 2j + 1
+    __device__ __forceinline__ void add(unsigned long long nib) {
+        ev += nib & 0x0F0F0F0F0F0F0F0Full;
+        od += (nib >> 4) & 0x0F0F0F0F0F0F0F0Full;
+    }
+    // pair[j] += count(2j) | count(2j + 1) << 16
+    __device__ __forceinline__ void to_pairs(uint32_t* pair) const {
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+            pair[j] += (uint32_t)((ev >> (8 * j)) & 255ull) | ((uint32_t)((od >> (8 * j)) & 255ull) << 16);
+    }
+};
+
+// Lane d < 16 receives the warp's count of digit d.
+__device__ __forceinline__ int warp_digit_counts(const uint32_t* pair, int lane) {
+    int mine = 0;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        const uint32_t t = __reduce_add_sync(0xffffffffu, pair[j]);
+        mine = lane == 2 * j ? (int)(t & 0xffffu) : mine;
+        mine = lane == 2 * j + 1 ? (int)(t >> 16) : mine;
+    }
+    return mine;
+}
+
+// ORs into bits[] (shared, one bit per position) the k largest keys of a row of
+// n keys stored transposed with stride kw; every thread of the block calls it
+// and the bits are complete on return.  Key 0 marks an ineligible position;
+// the caller guarantees k <= #eligible.
+//
+// MSB radix select run by kTopkWarps warps.  Warp w owns a contiguous run of
+// 1024-position segments; in a segment lane l owns the 32 positions of bits
+// word 32 s + l, which stay in registers when one segment covers the warp's
+// share.  A first reduction of OR and AND over the eligible keys fixes the bits
+// they all share; each pass then resolves the next (up to) 4 bits that differ:
+// threads count digits in registers, warps add the counts with the hardware
+// warp reduction, and after one barrier every warp scans the 16 bucket totals
+// from the top to find the digit that holds the k-th key.  Once the threshold
+// bucket holds at most kTopkCap keys they are compacted (key and position) so
+// later passes read only them; once it holds at most kTopkFew keys one warp
+// ranks them directly (larger key first, then lower position).  If more equal
+// keys than that straddle the threshold they are ranked by position.
+template <bool kCached>
+__device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ keys, int kw, int n, int k, uint32_t* bits,
+                                                TopkShared& sm) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, tid = threadIdx.x;
+    {
+        const int nwords = (n + 31) >> 5;
+        const int nseg = (n + kTopkSeg - 1) / kTopkSeg;
+        const int spw = (nseg + kTopkWarps - 1) / kTopkWarps;   // segments per warp
+        const int seg0 = min(warp * spw, nseg), seg1 = min(seg0 + spw, nseg);
+        auto fetch = [&](int sg, uint32_t* v) {
+            const int wd = sg * 32 + lane;
+#pragma unroll
+            for (int j = 0; j < 32; ++j) v[j] = (wd < nwords && wd * 32 + j < n) ? keys[j * kw + wd] : 0u;
+        };
+        // With one segment per warp (kCached) a lane's 32 keys stay in registers.
+        uint32_t ureg[kCached ? 32 : 1];
+        if (kCached) fetch(seg0 < seg1 ? seg0 : nseg, ureg);
+        auto load_seg = [&](int sg, uint32_t* v) {
+            if (kCached) {
+#pragma unroll
+                for (int j = 0; j < 32; ++j) v[j] = ureg[kCached ? j : 0];
+            } else {
+                fetch(sg, v);
+            }
+        };
+
+        // Bits shared by every eligible key.
+        {
+            uint32_t kor = 0u, kand = 0xffffffffu;
+            for (int sg = seg0; sg < seg1; ++sg) {
+                uint32_t v[32];
+                load_seg(sg, v);
+#pragma unroll
+                for (int j = 0; j < 32; ++j) {
+                    kor |= v[j];
+                    kand &= v[j] != 0u ? v[j] : 0xffffffffu;
                 }
-                acc += sm.hist[b];
+            }
+            kor = __reduce_or_sync(0xffffffffu, kor);
+            kand = __reduce_and_sync(0xffffffffu, kand);
+            if (lane == 0) {
+                sm.wor[warp] = kor;
+                sm.wand[warp] = kand;
+            }
+            if (tid == 0) sm.fcount = 0;
+        }
+        topk_bar();
+        uint32_t gor = 0u, gand = 0xffffffffu;
+#pragma unroll
+        for (int x = 0; x < kTopkWarps; ++x) {
+            gor |= sm.wor[x];
+            gand &= sm.wand[x];
+        }
+        const uint32_t gdiff = gor ^ gand;   // bits on which eligible keys differ
+
+        uint32_t prefix = 0u, mask = 0u;
+        int kk = k;
+        int cnt = 0x7fffffff;   // keys matching the prefix (unknown before the first pass)
+        int mlist = -1;         // length of the compacted list, -1 while counting all keys
+        bool whole_bin = false;
+        int lo = 32;            // lowest bit resolved so far
+        for (int pass = 0;; ++pass) {
+            // Fix the bits below lo that every eligible key shares, then take up
+            // to 4 bits down from the highest differing one.
+            const uint32_t below = lo == 32 ? 0xffffffffu : ((1u << lo) - 1u);
+            const uint32_t diff = gdiff & below;
+            if (diff == 0u) {
+                prefix |= gand & below;
+                mask |= below;
+                break;
+            }
+            const int hb = 31 - __clz(diff);
+            const uint32_t fixed = below & ~((2u << hb) - 1u);   // bits (hb, lo), none when hb = 31
+            prefix |= gand & fixed;
+            mask |= fixed;
+            lo = max(hb - 3, 0);
+            const uint32_t wmask = (1u << (hb - lo + 1)) - 1u;
+
+            int mine;   // lane d < 16: this warp's count of digit d
+            if (mlist < 0) {
+                uint32_t pair[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
+                for (int sg = seg0; sg < seg1; ++sg) {
+                    uint32_t v[32];
+                    load_seg(sg, v);
+                    DigitBytes db;
+#pragma unroll
+                    for (int j0 = 0; j0 < 32; j0 += 15) {
+                        unsigned long long nib = 0ull;
+#pragma unroll
+                        for (int j = j0; j < j0 + 15 && j < 32; ++j) nib += digit_nibble(v[j], mask, prefix, lo, wmask);
+                        db.add(nib);
+                    }
+                    db.to_pairs(pair);
+                }
+                mine = warp_digit_counts(pair, lane);
+            } else {
+                // At most 7 list entries per thread: a warp's count of a digit fits a byte.
+                unsigned long long nib = 0ull;
+#pragma unroll
+                for (int r = 0; r < kTopkCap / kTopkThreads; ++r) {
+                    const int j = tid + r * kTopkThreads;
+                    nib += digit_nibble(j < mlist ? sm.ckey[j] : 0u, mask, prefix, lo, wmask);
+                }
+                DigitBytes db;
+                db.add(nib);
+                mine = 0;
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    // quad q: bytes (digit 4q, 4q + 2) from ev, (4q + 1, 4q + 3) from od
+                    const uint32_t e = (uint32_t)(db.ev >> (16 * q)) & 0xffffu, o = (uint32_t)(db.od >> (16 * q)) & 0xffffu;
+                    const uint32_t quad = (e & 0xffu) | ((o & 0xffu) << 8) | ((e >> 8) << 16) | ((o >> 8) << 24);
+                    const uint32_t t = __reduce_add_sync(0xffffffffu, quad);
+#pragma unroll
+                    for (int b = 0; b < 4; ++b) mine = lane == 4 * q + b ? (int)((t >> (8 * b)) & 0xffu) : mine;
+                }
+            }
+            const int buf = pass & 1;
+            if (lane < 16) sm.wcnt[buf][warp][lane] = mine;
+            topk_bar();
+            // Every warp finds the threshold digit itself (no second barrier; the
+            // counts are double-buffered so the next pass cannot overwrite them early).
+            int tot = 0;
+            if (lane < 16) {
+#pragma unroll
+                for (int x = 0; x < kTopkWarps; ++x) tot += sm.wcnt[buf][x][lane];
+            }
+            int suf = tot;   // count of digits >= lane
+#pragma unroll
+            for (int off = 1; off < 16; off <<= 1) {
+                const int y = __shfl_down_sync(0xffffffffu, suf, off);
+                if (lane + off < 16) suf += y;
+            }
+            const int above_l = suf - tot;
+            const unsigned hit = __ballot_sync(0xffffffffu, lane < 16 && above_l < kk && kk <= suf);
+            const int D = hit ? __ffs(hit) - 1 : 0;
+            const int above = __shfl_sync(0xffffffffu, above_l, D);
+            cnt = __shfl_sync(0xffffffffu, tot, D);
+            prefix |= (uint32_t)D << lo;
+            mask |= wmask << lo;
+            kk -= above;
+            if (cnt == kk) {
+                whole_bin = true;
+                break;
+            }
+            if (lo == 0 || cnt <= kTopkFew) break;
+            if (mlist < 0 && cnt <= kTopkCap) {
+                // Compact the keys of the threshold bucket.  Warp w's share starts
+                // after the bucket counts of warps 0..w-1, a lane's after the
+                // matches of its segment's lower lanes and earlier segments.
+                int off = 0;
+                for (int x = 0; x < warp; ++x) off += sm.wcnt[buf][x][D];
+                for (int sg = seg0; sg < seg1; ++sg) {
+                    uint32_t v[32];
+                    load_seg(sg, v);
+                    int mc = 0;
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) mc += (v[j] != 0u && (v[j] & mask) == prefix) ? 1 : 0;
+                    int incl = mc;
+#pragma unroll
+                    for (int o = 1; o < 32; o <<= 1) {
+                        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+                        if (lane >= o) incl += y;
+                    }
+                    int at = off + incl - mc;
+                    const int pos0 = (sg * 32 + lane) * 32;
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        const bool m = v[j] != 0u && (v[j] & mask) == prefix;
+                        if (m && at < kTopkCap) {
+                            sm.ckey[at] = v[j];
+                            sm.cpos[at] = pos0 + j;
+                        }
+                        at += m ? 1 : 0;
+                    }
+                    off += __shfl_sync(0xffffffffu, incl, 31);
+                }
+                mlist = cnt;
+                topk_bar();
             }
         }
-        __syncthreads();
-        const int D = sm.bcast[0], above = sm.bcast[1], cnt = sm.bcast[2];
-        __syncthreads();
-        prefix |= (uint32_t)D << sh;
-        mask |= (uint32_t)(nb - 1) << sh;
-        kk -= above;
-        if (cnt == kk) {
-            whole_bin = true;
-            break;
+
+        const bool few = !whole_bin && cnt <= kTopkFew;
+        if (few) {
+            // Gather the bucket's keys with their positions.
+            if (mlist >= 0) {
+#pragma unroll
+                for (int r = 0; r < kTopkCap / kTopkThreads; ++r) {
+                    const int j = tid + r * kTopkThreads;
+                    if (j < mlist && (sm.ckey[j] & mask) == prefix) {
+                        const int slot = atomicAdd(&sm.fcount, 1);
+                        if (slot < kTopkFew) {
+                            sm.fkey[slot] = sm.ckey[j];
+                            sm.fpos[slot] = sm.cpos[j];
+                        }
+                    }
+                }
+            } else {
+                for (int sg = seg0; sg < seg1; ++sg) {
+                    uint32_t v[32];
+                    load_seg(sg, v);
+                    const int pos0 = (sg * 32 + lane) * 32;
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        if (v[j] != 0u && (v[j] & mask) == prefix) {
+                            const int slot = atomicAdd(&sm.fcount, 1);
+                            if (slot < kTopkFew) {
+                                sm.fkey[slot] = v[j];
+                                sm.fpos[slot] = pos0 + j;
+                            }
+                        }
+                    }
+                }
+            }
+        }
+        const bool ties = !whole_bin && !few;
+        if (ties) {
+            // More equal keys straddle the threshold than kTopkFew: rank by position.
+            int eqc = 0;
+            for (int sg = seg0; sg < seg1; ++sg) {
+                uint32_t v[32];
+                load_seg(sg, v);
+#pragma unroll
+                for (int j = 0; j < 32; ++j) eqc += (v[j] != 0u && (v[j] & mask) == prefix) ? 1 : 0;
+            }
+            eqc = __reduce_add_sync(0xffffffffu, eqc);
+            if (lane == 0) sm.weq[warp] = eqc;
+        }
+        topk_bar();
+        int base = 0;   // equal keys at lower positions (ties only)
+        if (ties)
+            for (int x = 0; x < warp; ++x) base += sm.weq[x];
+        // Mark the keys above the threshold prefix (all of the bucket when it is
+        // taken whole; with ties, the equal keys at the kk lowest positions).
+        for (int sg = seg0; sg < seg1; ++sg) {
+            uint32_t v[32];
+            load_seg(sg, v);
+            uint32_t word = 0u;
+            if (!ties) {
+#pragma unroll
+                for (int j = 0; j < 32; ++j) {
+                    const uint32_t um = v[j] & mask;
+                    const bool sel = v[j] != 0u && (um > prefix || (whole_bin && um == prefix));
+                    word |= (sel ? 1u : 0u) << j;
+                }
+            } else {
+                int ec = 0;
+#pragma unroll
+                for (int j = 0; j < 32; ++j) ec += (v[j] != 0u && (v[j] & mask) == prefix) ? 1 : 0;
+                int incl = ec;
+#pragma unroll
+                for (int o = 1; o < 32; o <<= 1) {
+                    const int y = __shfl_up_sync(0xffffffffu, incl, o);
+                    if (lane >= o) incl += y;
+                }
+                int rank = base + incl - ec;
+#pragma unroll
+                for (int j = 0; j < 32; ++j) {
+                    const uint32_t um = v[j] & mask;
+                    const bool eq = v[j] != 0u && um == prefix;
+                    const bool sel = (v[j] != 0u && um > prefix) || (eq && rank < kk);
+                    rank += eq ? 1 : 0;
+                    word |= (sel ? 1u : 0u) << j;
+                }
+                base += __shfl_sync(0xffffffffu, incl, 31);
+            }
+            const int wd = sg * 32 + lane;
+            if (wd < nwords && word) bits[wd] |= word;
+        }
+        if (few) {
+            topk_bar();   // the sweep's plain stores are done before warp 0 adds bits
+            if (warp == 0) {
+                const int m = min(sm.fcount, kTopkFew);
+                const uint32_t key = lane < m ? sm.fkey[lane] : 0u;
+                const int pos = lane < m ? sm.fpos[lane] : 0x7fffffff;
+                int rank = 0;
+                for (int j = 0; j < m; ++j) {
+                    const uint32_t kj = __shfl_sync(0xffffffffu, key, j);
+                    const int pj = __shfl_sync(0xffffffffu, pos, j);
+                    rank += (kj > key || (kj == key && pj < pos)) ? 1 : 0;
+                }
+                if (lane < m && rank < kk && pos < n) atomicOr(&bits[pos >> 5], 1u << (pos & 31));
+            }
         }
     }
-    // Positions strictly above the threshold prefix are in; positions equal to it
-    // are in either all together or, when equal keys exceed the need, lowest first.
-    const int nchunks = (n + NT - 1) / NT;
-    int taken = 0;
-    for (int ch = 0; ch < nchunks; ++ch) {
-        const int t = ch * NT + tid;
-        const uint32_t u = t < n ? keys[t] : 0u;
-        const bool above = u != 0u && (u & mask) > prefix;
-        const bool eq = u != 0u && (u & mask) == prefix;
-        bool sel;
-        if (whole_bin) {
-            sel = above || eq;
-        } else {
-            int tot;
-            const int r = block_exclusive_sum(eq ? 1 : 0, sm.wsum, tot);
-            sel = above || (eq && taken + r < kk);
-            taken += tot;
-        }
-        const unsigned bal = __ballot_sync(0xffffffffu, sel);
-        if ((tid & 31) == 0 && bal) bits[(ch * NT + (tid & ~31)) >> 5] |= bal;
+}
+
+__device__ void block_topk(const uint32_t* __restrict__ keys, int kw, int n, int k, uint32_t* bits, TopkShared& sm) {
+    if (k > 0 && n > 0 && (threadIdx.x >> 5) < kTopkWarps) {
+        const int nseg = (n + kTopkSeg - 1) / kTopkSeg;
+        if (nseg <= kTopkWarps)
+            block_topk_impl<true>(keys, kw, n, k, bits, sm);
+        else
+            block_topk_impl<false>(keys, kw, n, k, bits, sm);
     }
     __syncthreads();
 }
@@ -205,27 +503,21 @@ __device__ Moments block_moments(Moments v, float3* red) {
     return t;
 }
 
-// Section 4.1 and the preserved tokens of Section 4.2.  One thread-block
-// cluster per sequence, one CTA per KV head (cluster rank = head):
-//   pool the head's P_O and P_O' rows and a slice of I (max-pool, inherited
-//   from SnapKV), sigma_h = sample std of pooled P_O over the candidates
-//   (Welford/Chan moments in fp32), exchange sigma through distributed shared memory, the
-//   delta lowest-sigma heads take the O' scores, then the top-K preserved
-//   tokens of the chosen row by radix select.
-__global__ void __launch_bounds__(kSelectThreads) heads_kernel(Geometry G, LayerIO io, Scratch sc, Slot sl) {
-    cg::cluster_group cluster = cg::this_cluster();
-    __shared__ TopkShared sm;
+// Section 4.1, first half.  One CTA per (KV head, sequence): pool the head's
+// P_O and P_O' rows and a slice of I (max-pool, inherited from SnapKV) and
+// sigma_h = sample std of pooled P_O over the candidates (Welford/Chan moments
+// in fp32).
+__global__ void __launch_bounds__(kSelectThreads) heads_pool_kernel(Geometry G, LayerIO io, Scratch sc, Slot sl) {
     __shared__ float3 red[32];
-    __shared__ float sig_self;
-    extern __shared__ uint32_t bits[];
-    const int h = (int)cluster.block_rank(), s = blockIdx.y;
+    __shared__ float ibuf[kIChunk + 2 * (kMaxPool / 2)];
+    const int h = blockIdx.x, s = blockIdx.y;
     const int tid = threadIdx.x, NT = blockDim.x;
     const int L = io.cu[s + 1] - io.cu[s];
     const int Lc = L - G.w;
     const int halo = G.pool / 2;
     const size_t row = (size_t)s * G.Hkv + h;
     // Pool P_O and P_O' of this head (four positions per thread per step) and
-    // accumulate the sums of pooled P_O and of its squares in fp64.
+    // accumulate the moments of pooled P_O.
     Moments mom{0.f, 0.f, 0.f};
     const float* rO = sl.rawO + row * G.ML;
     const float* rOe = sl.rawOe + row * G.ML;
@@ -242,33 +534,83 @@ __global__ void __launch_bounds__(kSelectThreads) heads_kernel(Geometry G, Layer
     {
         const int per = ((Lc + G.Hkv - 1) / G.Hkv + 3) & ~3;
         const int a0 = min(h * per, Lc), b0 = min(a0 + per, Lc);
-        const float* rI = sl.rawI + (size_t)s * G.ML;
-        for (int t4 = a0 + 4 * tid; t4 < b0; t4 += 4 * NT) {
-            const Pooled4 c = pool4(rI, t4, Lc, halo);
-            *reinterpret_cast<float4*>(sl.I + (size_t)s * G.ML + t4) = make_float4(c.v[0], c.v[1], c.v[2], c.v[3]);
+        if (G.NG == 1) {
+            const float* rI = sl.rawI + (size_t)s * G.ML;
+            for (int t4 = a0 + 4 * tid; t4 < b0; t4 += 4 * NT) {
+                const Pooled4 c = pool4(rI, t4, Lc, halo);
+                *reinterpret_cast<float4*>(sl.I + (size_t)s * G.ML + t4) = make_float4(c.v[0], c.v[1], c.v[2], c.v[3]);
+            }
+        } else {
+            // The window kernel left, per head group, the maxima over its KV heads of
+            // G_h[q][t]: raw I is the sum over q of the maxima over the groups, built
+            // chunk by chunk (with the pool halo) in shared memory, then pooled.
+            int tbase = 0;
+            for (int b = 0; b < s; ++b) {
+                const int lb = io.cu[b + 1] - io.cu[b] - G.w;
+                tbase += lb > 0 ? (lb + kTileT - 1) / kTileT : 0;
+            }
+            const float invO = 1.f / (float)G.O;
+            const size_t n_el = (size_t)G.O * kTileT;
+            for (int c = a0; c < b0; c += kIChunk) {
+                const int ce = min(c + kIChunk, b0);
+                const int lo = max(c - halo, 0), hi = min(ce + halo, Lc);
+                for (int t = lo + tid; t < hi; t += NT) {
+                    const float* wt = sl.wpart + (size_t)(tbase + (t >> 7)) * G.NG * n_el + (t & (kTileT - 1));
+                    float sum = 0.f;
+                    for (int qi = 0; qi < G.O; ++qi) {
+                        float m = __ldcg(wt + (size_t)qi * kTileT);
+                        for (int gg = 1; gg < G.NG; ++gg) m = fmaxf(m, __ldcg(wt + ((size_t)gg * G.O + qi) * kTileT));
+                        sum += m;
+                    }
+                    ibuf[t - lo] = sum * invO;
+                }
+                __syncthreads();
+                for (int t = c + tid; t < ce; t += NT) {
+                    float m = ibuf[t - lo];
+                    for (int d = 1; d <= halo; ++d) {
+                        if (t - d >= 0) m = fmaxf(m, ibuf[t - d - lo]);
+                        if (t + d < Lc) m = fmaxf(m, ibuf[t + d - lo]);
+                    }
+                    sl.I[(size_t)s * G.ML + t] = m;
+                }
+                __syncthreads();
+            }
         }
     }
     mom = block_moments(mom, red);
-    const float sigma = Lc >= 2 ? sqrtf(fmaxf(mom.m2, 0.f) / (float)(Lc - 1)) : 0.f;
-    if (tid == 0) sig_self = sigma;
-    for (int wd = tid; wd < G.words; wd += NT) bits[wd] = 0u;
-    cluster.sync();
+    if (tid == 0) sl.sigma[row] = Lc >= 2 ? sqrtf(fmaxf(mom.m2, 0.f) / (float)(Lc - 1)) : 0.f;
+}
+
+// Section 4.1, second half, and the preserved tokens of Section 4.2.  One CTA
+// per (KV head, sequence), launched after heads_pool_kernel: every CTA ranks the
+// sequence's sigmas the same way, the delta lowest-sigma heads take the O'
+// scores, then the top-K preserved tokens of the chosen row by radix select.
+__global__ void __launch_bounds__(kSelectThreads) heads_topk_kernel(Geometry G, LayerIO io, Scratch sc, Slot sl) {
+    __shared__ TopkShared sm;
     __shared__ int top_flag;
+    extern __shared__ uint32_t bits[];
+    const int h = blockIdx.x, s = blockIdx.y;
+    const int tid = threadIdx.x, NT = blockDim.x;
+    const int L = io.cu[s + 1] - io.cu[s];
+    const int Lc = L - G.w;
+    const size_t row = (size_t)s * G.Hkv + h;
+    for (int wd = tid; wd < G.words; wd += NT) bits[wd] = 0u;
     if (tid < 32) {
-        const float so = tid < G.Hkv ? *cluster.map_shared_rank(&sig_self, tid) : INFINITY;
+        const float sigma = __ldcg(&sl.sigma[row]);
+        const float so = tid < G.Hkv ? __ldcg(&sl.sigma[(size_t)s * G.Hkv + tid]) : INFINITY;
         const bool before = tid < G.Hkv && (so < sigma || (so == sigma && tid < h));
         const int rank = __popc(__ballot_sync(0xffffffffu, before));
-        if (tid == 0) top_flag = rank < G.delta;
+        if (tid == 0) {
+            top_flag = rank < G.delta;
+            sl.htop[row] = rank < G.delta;
+        }
     }
     __syncthreads();
     const int top = top_flag;
-    if (tid == 0) {
-        sl.sigma[row] = sigma;
-        sl.htop[row] = top;
-    }
     if (L > G.budget && G.Kp > 0) {
         const float* __restrict__ P = (top ? sl.POe : sl.PO) + row * G.ML;
         uint32_t* keys = keys_in_smem(G.ML) ? bits + G.words : sc.keys + row * G.ML;
+        const int kw = key_stride(G);
         for (int b0 = 4 * tid; b0 < Lc; b0 += 16 * NT) {
             float4 pv[4];
 #pragma unroll
@@ -282,15 +624,14 @@ __global__ void __launch_bounds__(kSelectThreads) heads_kernel(Geometry G, Layer
                 const float x[4] = {pv[u].x, pv[u].y, pv[u].z, pv[u].w};
 #pragma unroll
                 for (int i = 0; i < 4; ++i)
-                    if (t4 + i < Lc) keys[t4 + i] = float_order_key(x[i]);
+                    if (t4 + i < Lc) keys[key_index(t4 + i, kw)] = float_order_key(x[i]);
             }
         }
         __syncthreads();
-        block_topk(keys, Lc, G.Kp, bits, sm);
+        block_topk(keys, kw, Lc, G.Kp, bits, sm);
     }
     uint32_t* pres = sl.pres + row * G.words;
     for (int wd = tid; wd < G.words; wd += NT) pres[wd] = bits[wd];
-    cluster.sync();   // peers may still read sig_self
 }
 
 // Section 4.2: P' = P + lambda * I * (1 - n_t / (l + 1)); the preserved tokens
@@ -306,6 +647,11 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
     const int L = io.cu[s + 1] - io.cu[s];
     const int Lc = L - G.w;
     const int wordsL = (L + 31) >> 5;
+    for (int wd = tid; wd < G.words; wd += NT) bits[wd] = 0u;
+    // Launched as a programmatic dependent of the previous layer's selection:
+    // everything above overlaps its tail; the coverage state is read only after
+    // that grid has completed and its writes are visible.
+    asm volatile("griddepcontrol.wait;\n" ::: "memory");
     uint8_t* st = io.state + (size_t)s * G.state_stride;
     const uint32_t ell = reinterpret_cast<const uint32_t*>(st)[0];
     uint8_t* ncount = st + G.state_n_off;
@@ -313,7 +659,6 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
         if (tid == 0) atomicExch(sc.err, 2);
         return;
     }
-    for (int wd = tid; wd < G.words; wd += NT) bits[wd] = 0u;
     __syncthreads();
     if (L > G.budget) {
         const size_t row = (size_t)s * G.Hkv + h;
@@ -323,6 +668,7 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
         const uint32_t* pres = sl.pres + row * G.words;
         float* Pp = sl.Pprime + row * G.ML;
         uint32_t* keys = keys_in_smem(G.ML) ? bits + G.words : sc.keys_sel + row * G.ML;
+        const int kw = key_stride(G);
         const float denom = (float)(ell + 1u);
         for (int b0 = 4 * tid; b0 < Lc; b0 += 8 * NT) {
             float4 pv[2], iv[2];
@@ -353,13 +699,15 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
                     const float pp = p4[i] + G.lambda * (i4[i] * (1.f - coverage));
                     out[i] = pp;
                     const bool kept = (pw[u] >> (t & 31)) & 1u;
-                    if (t < Lc) keys[t] = kept ? 0u : float_order_key(pp);
+                    if (t < Lc) keys[key_index(t, kw)] = kept ? 0u : float_order_key(pp);
                 }
                 *reinterpret_cast<float4*>(Pp + t4) = make_float4(out[0], out[1], out[2], out[3]);
             }
         }
         __syncthreads();
-        block_topk(keys, Lc, G.k2, bits, sm);
+        block_topk(keys, kw, Lc, G.k2, bits, sm);
+        // The next layer's selection may be scheduled now (it waits for this grid).
+        asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
         for (int wd = tid; wd < wordsL; wd += NT) bits[wd] |= pres[wd] | range_bits(wd, Lc, L);
     } else {
         for (int wd = tid; wd < wordsL; wd += NT) bits[wd] = range_bits(wd, 0, L);
@@ -440,38 +788,33 @@ __global__ void __launch_bounds__(256) gather_kernel(Geometry G, LayerIO io) {
 }  // namespace
 
 size_t select_smem_bytes(const Geometry& g) {
-    return sizeof(uint32_t) * ((size_t)g.words + (keys_in_smem(g.ML) ? (size_t)g.ML : 0));
+    return sizeof(uint32_t) * ((size_t)g.words + (keys_in_smem(g.ML) ? 32 * (size_t)key_stride(g) : 0));
 }
 
 size_t heads_smem_bytes(const Geometry& g) { return select_smem_bytes(g); }
 
 cudaError_t configure_select() {
-    const int need = (int)(sizeof(uint32_t) * (kSmemKeys + kSmemKeys / 32));
-    cudaError_t e = cudaFuncSetAttribute(heads_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, need);
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(heads_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    const int need = (int)(sizeof(uint32_t) * (kSmemKeys / 32 + 32 * ((kSmemKeys / 32) | 1)));
+    cudaError_t e = cudaFuncSetAttribute(heads_topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, need);
     if (e == cudaSuccess)
         e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, need);
     return e;
 }
 
-cudaError_t launch_heads(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st) {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(g.Hkv, g.batch);
-    cfg.blockDim = dim3(kSelectThreads);
-    cfg.dynamicSmemBytes = heads_smem_bytes(g);
-    cfg.stream = st;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = g.Hkv;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, heads_kernel, g, io, sc, sl);
+cudaError_t launch_heads(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st,
+                         int priority) {
+    const dim3 grid(g.Hkv, g.batch);
+    cudaError_t e = launch_prio(heads_pool_kernel, grid, dim3(kSelectThreads), 0, st, priority, false, g, io, sc, sl);
+    if (e == cudaSuccess)
+        e = launch_prio(heads_topk_kernel, grid, dim3(kSelectThreads), heads_smem_bytes(g), st, priority, false, g, io,
+                        sc, sl);
+    return e;
 }
 
-void launch_select(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st) {
-    select_kernel<<<dim3(g.Hkv, g.batch), kSelectThreads, select_smem_bytes(g), st>>>(g, io, sc, sl);
+cudaError_t launch_select(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st,
+                          int priority) {
+    return launch_prio(select_kernel, dim3(g.Hkv, g.batch), dim3(kSelectThreads), select_smem_bytes(g), st, priority,
+                       /*programmatic=*/true, g, io, sc, sl);
 }
 
 void launch_gather(const Geometry& g, const LayerIO& io, cudaStream_t st) {

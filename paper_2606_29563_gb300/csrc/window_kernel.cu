@@ -1,247 +1,401 @@
-// Eq. 1 window scores and the Section 4.2 importance I (before pooling).
+// Eq. 1 window scores and the Section 4.2 importance I (before pooling), from
+// the window queries' attention over the candidate tokens, recomputed on the
+// tensor cores with the softmax statistics (m_r, Z_r) of the score kernel.
 //
-// One CTA per (sequence, 32-token block of candidates).  The score kernel left
-// e[tile][h][r][t] = fp16(2^15 exp(s - mu)) row-major; with the row factors
-// c_r = 2^(mu_tile,r - m_r - 15) / Z_r the normalised attention is c_r * e.
-// A thread owns (8-token group, KV head, subset of window rows q) and issues
-// all of its 16-byte row loads before consuming them:
-//   G_h[q][t] = sum_j c * e[rows (q, j) of head h][t]     (GQA group sum)
+// One CTA per (sequence s, 128-token tile of candidates, group of KV heads).
+// For each KV head h of the group the CTA computes S^T = K_tile Q_h^T with
+// tcgen05.mma (M = 128 tokens, N = g*w query rows padded to 16, K = d) into
+// TMEM, so one epilogue thread owns one token and every query row of it:
+//   A[r][t]   = 2^(s_rt * scale * log2(e) - m_r) / Z_r   (softmax over all visible keys)
+//   G_h[q][t] = sum_j A[(q, j)][t]                       (GQA group sum, r = q * g + j)
 //   P_O[h,t]  = (1/O)  sum_{q >= w-O}  G_h[q][t]
 //   P_O'[h,t] = (1/O') sum_{q >= w-O'} G_h[q][t]
 //   I[t]      = (1/O)  sum_{q >= w-O}  max_h G_h[q][t]
-// The HP (next power of two >= Hkv) lanes of a group are adjacent, so the head
-// max is an xor-shuffle; row subsets are summed through shared memory.  The
-// raw rows go to the slot arrays; pooling happens in the heads kernel.
+// Warp 0 streams K_h and Q_h with TMA, warp 1 issues the MMAs into one or two
+// TMEM accumulators, warps 2..17 are the epilogue: four warps per TMEM lane
+// quadrant, each taking a quarter of the window rows q (straight-line code per
+// 32-column chunk when the group size g is a compile-time case).  The head
+// maxima of G_h[q][t] stay in shared memory; when the KV heads are split over
+// several CTAs each group writes its maxima to a partial buffer and the heads
+// kernel combines the groups into I.  The raw rows go to the slot arrays;
+// pooling happens in the heads kernel.
+#include <cudaTypedefs.h>
+
 #include "kvec_internal.cuh"
+#include "sm100_ptx.cuh"
 
 namespace kvec {
 
 namespace {
 
-constexpr int kBlockT = 32;                 // candidate tokens per CTA
-constexpr int kGroups = kBlockT / 8;        // 8-token groups per CTA
-constexpr int kMaxRowsPerThread = 16;       // row loads a thread keeps in flight
-constexpr int kMaxWindowThreads = 512;
+constexpr int kWinThreads = 576;                      // warp 0 TMA, warp 1 MMA, warps 2..17 epilogue
+constexpr int kEpiThreads = 512;
+constexpr int kEpiWarps = kEpiThreads / 32;
+constexpr int kMaxSmemWin = 232448;                   // opt-in shared memory per CTA on sm_103
+constexpr int kWinCuParam = 64;                       // sequences whose offsets travel in the kernel parameters
+constexpr int kKTileBytes = kTileT * kHeadDim * 2;    // 32 KB: two 64-column swizzled halves
+constexpr int kRsRows = 288;                          // row-statistics buffer: R <= 256 plus a chunk's overrun
 
-struct WinShape {
-    int HP;       // head lanes per group
-    int TPQ;      // threads per row subset: kGroups * HP rounded up to whole warps
-    int QS;       // window-row subsets
-    int threads;  // TPQ * QS
+struct WinArgs {
+    Geometry G;
+    Scratch sc;
+    Slot sl;
+    const int* cu;                  // device cu_seqlens
+    int cuv[kWinCuParam + 1];       // the same offsets (when batch <= kWinCuParam)
+    int Npad;                       // query rows padded to a multiple of 16 (MMA N)
+    int kst;                        // operand stages
+    int nacc;                       // TMEM accumulators (2, or 1 when 2 do not fit)
+    uint32_t tmem_cols;
 };
 
-// Every warp lies inside one row subset, so all its lanes run the same q loop
-// (the head-max shuffles need the whole warp).  A thread loads its rows in
-// batches of kMaxRowsPerThread, all loads of a batch in flight together.
-__host__ __device__ inline WinShape win_shape(int Hkv, int w, int g) {
-    WinShape s{};
-    s.HP = 1;
-    while (s.HP < Hkv) s.HP <<= 1;
-    s.TPQ = (kGroups * s.HP + 31) & ~31;
-    const int qper = kMaxRowsPerThread / g > 0 ? kMaxRowsPerThread / g : 1;   // window rows per subset
-    s.QS = (w + qper - 1) / qper;
-    if (s.QS * s.TPQ > kMaxWindowThreads) s.QS = kMaxWindowThreads / s.TPQ > 0 ? kMaxWindowThreads / s.TPQ : 1;
-    s.threads = s.TPQ * s.QS;
-    return s;
+struct __align__(8) WinBars {
+    uint64_t full[2], empty[2], acc_full[2], acc_empty[2];
+    uint64_t mma_done;
+    uint32_t tmem_base;
+    volatile int abort_flag;
+    volatile int epi_fail;     // set by an epilogue warp whose accumulator wait gave up
+};
+
+__host__ __device__ inline size_t stage_bytes(int Npad) { return (size_t)kKTileBytes + 2 * (size_t)Npad * 128; }
+
+__host__ __device__ inline size_t win_smem_bytes(int Npad, int O, int kst) {
+    return 1024 + (size_t)kst * stage_bytes(Npad) + kWinHeadsPerCta * kRsRows * sizeof(float2) +
+           (size_t)O * kTileT * sizeof(float) + kWinHeadsPerCta * 4 * kTileT * sizeof(float2) + sizeof(WinBars);
 }
 
-__device__ __forceinline__ void unpack8(const uint4& raw, float* f) {
-    const __half2* h = reinterpret_cast<const __half2*>(&raw);
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const float2 x = __half22float2(h[i]);
-        f[2 * i] = x.x;
-        f[2 * i + 1] = x.y;
-    }
+__device__ __forceinline__ void win_abort(WinBars* bars, int* err) {
+    bars->abort_flag = 1;
+    atomicExch(err, 3);
 }
 
-template <int HP>
-__global__ void __launch_bounds__(kMaxWindowThreads) window_kernel(Geometry G, LayerIO io, Scratch sc, Slot sl) {
-    extern __shared__ float wsm[];
-    const WinShape ws = win_shape(G.Hkv, G.w, G.g);
-    int s, blk, base;
-    if (!locate_item(G.batch, blockIdx.x,
-                     [&](int b) {
-                         const int Lc = io.cu[b + 1] - io.cu[b] - G.w;
-                         return Lc > 0 ? (Lc + kBlockT - 1) / kBlockT : 0;
-                     },
-                     s, blk, base))
-        return;
-    const int L = io.cu[s + 1] - io.cu[s];
-    const int Lc = L - G.w;
-    int tbase = 0;
-    for (int b = 0; b < s; ++b) tbase += tiles_of(io.cu[b + 1] - io.cu[b]);
-    const int R = G.R, Hkv = G.Hkv;
-    const int t0 = blk * kBlockT;
-    const int jt = t0 / kTileT, toff0 = t0 - jt * kTileT;
-    const int tid = threadIdx.x;
-    const int qper = (G.w + ws.QS - 1) / ws.QS;
-
-    float* cfac = wsm;                                          // [Hkv][R]
-    float* part = cfac + Hkv * R;                               // [QS][kBlockT][Hkv][3]
-
-    {
-        // Row factors of this tile, four loads in flight per thread.
-        const int n = Hkv * R;
-        for (int i0 = tid; i0 < n; i0 += 4 * blockDim.x) {
-            float2 ts[4], rs[4];
+// One head's window rows [q_lo, q_hi) of this thread's token: adds the rows'
+// group sums G_h[q] to po (q >= w-O) and poe (q >= w-O') and folds them into
+// the head maxima.  GG > 0 is the group size g known at compile time: each
+// 32-column chunk holds 32 / GG whole groups and runs as straight-line code.
+template <int GG>
+__device__ __forceinline__ void head_rows(uint32_t taddr, const float2* __restrict__ rsb, int g, int q_lo, int q_hi,
+                                          float sl2, int qO, int qOe, float* maxg_col, bool first, float& po,
+                                          float& poe) {
+    if constexpr (GG > 0) {
+        constexpr int QPC = 32 / GG, CW = QPC * GG;
+        for (int qb = q_lo; qb < q_hi; qb += QPC) {
+            const int c0 = qb * GG;
+            float v[32];
+            ptx::tmem_ld32(taddr + (uint32_t)c0, v);
+            ptx::tmem_wait_ld();
+            float pr[CW];
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int i = i0 + u * blockDim.x;
-                if (i < n) {
-                    const int hh = i / R, r = i - hh * R;
-                    ts[u] = sc.tstat[((size_t)(tbase + jt) * Hkv + hh) * R + r];
-                    rs[u] = sc.rowstat[((size_t)s * Hkv + hh) * R + r];
-                }
+            for (int i = 0; i < CW; ++i) {
+                const float2 mz = rsb[c0 + i];
+                pr[i] = ptx::ex2(fmaf(v[i], sl2, -mz.x)) * mz.y;
             }
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int i = i0 + u * blockDim.x;
-                if (i < n) cfac[i] = exp2f(ts[u].x - rs[u].x - kEScaleLog2) / rs[u].y;
-            }
-        }
-    }
-    __syncthreads();
-
-    // Thread role: row subset (whole warps), then group, then head lane (adjacent lanes).
-    const int qs = tid / ws.TPQ;
-    const int local = tid - qs * ws.TPQ;
-    const int hh = local % HP;
-    const int grp = local / HP;
-    const int t8 = t0 + grp * 8;
-    const bool act = grp < kGroups && hh < Hkv && t8 < Lc;
-    const __half* ebase = sc.ebuf + ((size_t)(tbase + jt) * Hkv + (act ? hh : 0)) * R * kTileT + toff0 + grp * 8;
-    const float* cf = cfac + (act ? hh : 0) * R;
-    const int q_lo = min(qs * qper, G.w), q_hi = min(q_lo + qper, G.w);
-    const int r_end = q_hi * G.g;
-
-    float accO[8], accOe[8], accI[8], gsum[8];
+            for (int k = 0; k < QPC; ++k) {
+                float gs = 0.f;
 #pragma unroll
-    for (int x = 0; x < 8; ++x) accO[x] = accOe[x] = accI[x] = gsum[x] = 0.f;
-    int q = q_lo, jq = 0;
-    for (int r0 = q_lo * G.g; r0 < r_end; r0 += kMaxRowsPerThread) {
-        const int nrows = min(kMaxRowsPerThread, r_end - r0);
-        uint4 raw[kMaxRowsPerThread];
-#pragma unroll
-        for (int k = 0; k < kMaxRowsPerThread; ++k) {
-            raw[k] = make_uint4(0, 0, 0, 0);
-            if (act && k < nrows) raw[k] = __ldcg(reinterpret_cast<const uint4*>(ebase + (size_t)(r0 + k) * kTileT));
-        }
-#pragma unroll
-        for (int k = 0; k < kMaxRowsPerThread; ++k) {
-            if (k >= nrows) break;
-            float f[8];
-            unpack8(raw[k], f);
-            const float c = cf[r0 + k];
-#pragma unroll
-            for (int x = 0; x < 8; ++x) gsum[x] = fmaf(c, f[x], gsum[x]);
-            if (++jq == G.g) {
-                if (q >= G.w - G.Oe) {
-#pragma unroll
-                    for (int x = 0; x < 8; ++x) accOe[x] += gsum[x];
-                }
-                if (q >= G.w - G.O) {
-#pragma unroll
-                    for (int x = 0; x < 8; ++x) {
-                        float m = gsum[x];
-#pragma unroll
-                        for (int off = 1; off < HP; off <<= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
-                        accO[x] += gsum[x];
-                        accI[x] += m;
+                for (int j = 0; j < GG; ++j) gs += pr[k * GG + j];
+                const int q = qb + k;
+                if (q < q_hi) {
+                    if (q >= qOe) poe += gs;
+                    if (q >= qO) {
+                        po += gs;
+                        float* mg = maxg_col + (q - qO) * kTileT;
+                        *mg = first ? gs : fmaxf(*mg, gs);
                     }
                 }
+            }
+        }
+    } else {
+        float gs = 0.f;
+        int q = q_lo, jq = 0;
+        const int c_end = q_hi * g;
+        for (int c0 = q_lo * g; c0 < c_end; c0 += 32) {
+            float v[32];
+            ptx::tmem_ld32(taddr + (uint32_t)c0, v);
+            ptx::tmem_wait_ld();
+            const int n = min(32, c_end - c0);
 #pragma unroll
-                for (int x = 0; x < 8; ++x) gsum[x] = 0.f;
-                jq = 0;
-                ++q;
+            for (int i = 0; i < 32; ++i) {
+                if (i >= n) break;
+                const float2 mz = rsb[c0 + i];
+                gs += ptx::ex2(fmaf(v[i], sl2, -mz.x)) * mz.y;
+                if (++jq == g) {
+                    if (q >= qOe) poe += gs;
+                    if (q >= qO) {
+                        po += gs;
+                        float* mg = maxg_col + (q - qO) * kTileT;
+                        *mg = first ? gs : fmaxf(*mg, gs);
+                    }
+                    gs = 0.f;
+                    jq = 0;
+                    ++q;
+                }
             }
         }
     }
-    if (grp < kGroups && hh < Hkv) {
-#pragma unroll
-        for (int x = 0; x < 8; ++x) {
-            float* pp = part + (((size_t)qs * kBlockT + grp * 8 + x) * Hkv + hh) * 3;
-            pp[0] = accO[x];
-            pp[1] = accOe[x];
-            pp[2] = accI[x];
+}
+
+template <int GG>
+__global__ void __launch_bounds__(kWinThreads, 1)
+    window_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap qmap,
+                  const __grid_constant__ WinArgs A) {
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const Geometry& G = A.G;
+    const int Npad = A.Npad, R = G.R;
+    const size_t sbytes = stage_bytes(Npad);
+    float2* rs = reinterpret_cast<float2*>(smem + A.kst * sbytes);      // [HG][kRsRows] (m_r, 1 / Z_r)
+    float* maxg = reinterpret_cast<float*>(rs + kWinHeadsPerCta * kRsRows);   // [O][128] max over heads of G_h[q][t]
+    float2* xfer = reinterpret_cast<float2*>(maxg + G.O * kTileT);      // [HG][4][128] quarters' (P_O, P_O') sums
+    WinBars* bars = reinterpret_cast<WinBars*>(xfer + kWinHeadsPerCta * 4 * kTileT);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    // Work item -> (sequence, candidate tile, head group); sequence s owns
+    // ceil(Lc / 128) * NG consecutive CTAs.
+    const bool cu_param = G.batch <= kWinCuParam;
+    auto cu = [&](int b) { return cu_param ? A.cuv[b] : __ldg(&A.cu[b]); };
+    int s = -1, jt = 0, ng = 0, tg = 0;
+    {
+        int base = 0, tbase = 0;
+        for (int b = 0; b < G.batch; ++b) {
+            const int Lc = cu(b + 1) - cu(b) - G.w;
+            const int nt = Lc > 0 ? (Lc + kTileT - 1) / kTileT : 0;
+            if ((int)blockIdx.x < base + nt * G.NG) {
+                const int local = (int)blockIdx.x - base;
+                s = b;
+                jt = local / G.NG;
+                ng = local - jt * G.NG;
+                tg = tbase + jt;
+                break;
+            }
+            base += nt * G.NG;
+            tbase += nt;
         }
     }
+    if (s < 0) return;   // the whole CTA, before any barrier or TMEM use
+    const int L = cu(s + 1) - cu(s), Lc = L - G.w;
+    const int h0 = ng * G.HG;
+    const int nh = min(G.HG, G.Hkv - h0);
+    const int NB = A.nacc;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < 2; ++i) {
+            ptx::mbar_init(&bars->full[i], 1);
+            ptx::mbar_init(&bars->empty[i], 1);
+            ptx::mbar_init(&bars->acc_full[i], 1);
+            ptx::mbar_init(&bars->acc_empty[i], kEpiThreads / 32);   // one arrival per epilogue warp
+        }
+        ptx::mbar_init(&bars->mma_done, 1);
+        bars->abort_flag = 0;
+        bars->epi_fail = 0;
+        ptx::fence_barrier_init();
+    }
+    if (warp == 1) {
+        ptx::tmem_alloc(&bars->tmem_base, A.tmem_cols);
+        ptx::tmem_relinquish();
+    }
+    if (warp == 0 && lane == 0) {
+        ptx::prefetch_tensormap(&kmap);
+        ptx::prefetch_tensormap(&qmap);
+    }
+    ptx::tc_fence_before();
     __syncthreads();
+    ptx::tc_fence_after();
+    const uint32_t tmem = bars->tmem_base;
 
-    // Sum the row subsets and write the raw rows (positions of one head are consecutive).
-    const float invO = 1.f / G.O, invOe = 1.f / G.Oe;
-    for (int i = tid; i < kBlockT * Hkv; i += blockDim.x) {
-        const int h2 = i / kBlockT, x = i - h2 * kBlockT;
-        const int t = t0 + x;
-        if (t >= Lc) continue;
-        float o = 0.f, oe = 0.f, im = 0.f;
-        for (int qq = 0; qq < ws.QS; ++qq) {
-            const float* pp = part + (((size_t)qq * kBlockT + x) * Hkv + h2) * 3;
-            o += pp[0];
-            oe += pp[1];
-            im += pp[2];
+    if (warp == 0) {
+        // ------------------------------------------------------------ TMA producer
+        if (lane == 0) {
+            const uint64_t policy = ptx::policy_evict_first();   // the K tiles' last use
+            const int row0 = cu(s) + jt * kTileT;
+            int fills[2] = {0, 0};
+            for (int hh = 0; hh < nh && !bars->abort_flag; ++hh) {
+                const int st = hh % A.kst, u = hh / A.kst;
+                if (u > 0 && !ptx::mbar_wait(&bars->empty[st], (u - 1) & 1)) {
+                    win_abort(bars, A.sc.err);
+                    break;
+                }
+                uint8_t* sk = smem + st * sbytes;
+                uint8_t* sq = sk + kKTileBytes;
+                const int h = h0 + hh;
+                ptx::mbar_arrive_expect_tx(&bars->full[st], (uint32_t)kKTileBytes + 2u * (uint32_t)R * 128u);
+                ptx::tma_load_3d(sk, &kmap, &bars->full[st], 0, h, row0, policy);
+                ptx::tma_load_3d(sk + kKTileBytes / 2, &kmap, &bars->full[st], 64, h, row0, policy);
+                ptx::tma_load_4d(sq, &qmap, &bars->full[st], 0, h * G.g, 0, s);
+                ptx::tma_load_4d(sq + Npad * 128, &qmap, &bars->full[st], 64, h * G.g, 0, s);
+                ++fills[st];
+            }
+            // Drain: every issued copy lands before the CTA may exit.
+            for (int st = 0; st < A.kst; ++st)
+                if (fills[st] > 0) ptx::mbar_wait(&bars->full[st], (fills[st] - 1) & 1, 50000000ull);
         }
-        sl.rawO[((size_t)s * Hkv + h2) * G.ML + t] = o * invO;
-        sl.rawOe[((size_t)s * Hkv + h2) * G.ML + t] = oe * invOe;
-        if (h2 == 0) sl.rawI[(size_t)s * G.ML + t] = im * invO;
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            const uint32_t idesc = ptx::idesc_bf16_f32(128, Npad);
+            for (int hh = 0; hh < nh && !bars->abort_flag; ++hh) {
+                const int st = hh % A.kst, u = hh / A.kst;
+                const int b = hh % NB, ub = hh / NB;
+                if (!ptx::mbar_wait(&bars->full[st], u & 1) ||
+                    (ub > 0 && !ptx::mbar_wait(&bars->acc_empty[b], (ub - 1) & 1))) {
+                    win_abort(bars, A.sc.err);
+                    break;
+                }
+                ptx::tc_fence_after();
+                const uint32_t sk = ptx::smem_u32(smem + st * sbytes), sq = sk + kKTileBytes;
+                const uint32_t d = tmem + (uint32_t)(b * Npad);
+#pragma unroll
+                for (int kk = 0; kk < 8; ++kk) {
+                    const int half = kk >> 2, kin = kk & 3;
+                    const uint64_t ad = ptx::smem_desc_k_sw128(sk + half * (kKTileBytes / 2) + kin * 32);
+                    const uint64_t bd = ptx::smem_desc_k_sw128(sq + half * Npad * 128 + kin * 32);
+                    ptx::mma_bf16(d, ad, bd, idesc, kk > 0 ? 1u : 0u);
+                }
+                ptx::mma_commit(&bars->empty[st]);
+                ptx::mma_commit(&bars->acc_full[b]);
+            }
+            ptx::mma_commit(&bars->mma_done);
+        }
+    } else {
+        // ------------------------------------------------------------ epilogue
+        const int e = threadIdx.x - 64;                   // 0 .. kEpiThreads - 1
+        const int qt = (warp - 2) >> 2;                   // quarter of the window rows
+        const int quad = warp & 3;                        // TMEM lanes 32*quad .. +31
+        const int tokl = quad * 32 + lane;
+        const int t = jt * kTileT + tokl;
+        const bool valid = t < Lc;
+        const int q_lo = (qt * G.w) >> 2, q_hi = ((qt + 1) * G.w) >> 2;
+        const int qO = G.w - G.O, qOe = G.w - G.Oe;
+        const float invO = 1.f / (float)G.O, invOe = 1.f / (float)G.Oe;
+        // Row statistics of every head of the group: (m_r, 1 / Z_r).
+        for (int i = e; i < nh * R; i += kEpiThreads) {
+            const int hh = i / R, r = i - hh * R;
+            const float2 ms = __ldcg(&A.sc.rowstat[((size_t)s * G.Hkv + h0 + hh) * R + r]);
+            rs[hh * kRsRows + r] = make_float2(ms.x, 1.f / ms.y);
+        }
+        ptx::named_bar_sync(1, kEpiThreads);
+        // The warps run through the heads independently: each waits for the
+        // accumulator itself and leaves its partial sums in xfer.
+        for (int hh = 0; hh < nh; ++hh) {
+            const int b = hh % NB, ub = hh / NB;
+            int got = 1;
+            if (lane == 0) got = !bars->abort_flag && ptx::mbar_wait(&bars->acc_full[b], ub & 1);
+            got = __shfl_sync(0xffffffffu, got, 0);
+            if (!got) {
+                if (lane == 0) {
+                    bars->epi_fail = 1;
+                    win_abort(bars, A.sc.err);
+                }
+                break;
+            }
+            ptx::tc_fence_after();
+            const uint32_t taddr = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(b * Npad);
+            float po = 0.f, poe = 0.f;
+            head_rows<GG>(taddr, rs + hh * kRsRows, G.g, q_lo, q_hi, G.sl2, qO, qOe, maxg + tokl, hh == 0, po, poe);
+            ptx::tc_fence_before();
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(&bars->acc_empty[b]);
+            xfer[(hh * 4 + qt) * kTileT + tokl] = make_float2(po, poe);
+        }
+        // Every epilogue warp arrives here, failed or not; epi_fail is only written
+        // before this barrier, so the branch below is uniform.
+        ptx::named_bar_sync(1, kEpiThreads);
+        const bool aborted = bars->epi_fail != 0;
+        if (!aborted) {
+            // P_O and P_O' of every head of the group: the four quarters' sums.
+            for (int i = e; i < nh * kTileT; i += kEpiThreads) {
+                const int hh = i >> 7, tk = i & (kTileT - 1);
+                const int tt = jt * kTileT + tk;
+                if (tt < Lc) {
+                    float so = 0.f, soe = 0.f;
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) {
+                        const float2 x = xfer[(hh * 4 + k) * kTileT + tk];
+                        so += x.x;
+                        soe += x.y;
+                    }
+                    const size_t row = (size_t)s * G.Hkv + h0 + hh;
+                    A.sl.rawO[row * G.ML + tt] = so * invO;
+                    A.sl.rawOe[row * G.ML + tt] = soe * invOe;
+                }
+            }
+        }
+        if (!aborted) {
+            // I[t] = (1/O) sum over q >= w - O of the maxima over every KV head.  With
+            // the heads in one CTA it is complete here; otherwise each group leaves its
+            // maxima and the heads kernel takes the maximum over the groups.
+            const int n_el = G.O * kTileT;
+            if (G.NG > 1) {
+                float* wp = A.sl.wpart + ((size_t)tg * G.NG + ng) * n_el;
+                for (int i = e; i < n_el; i += kEpiThreads) wp[i] = maxg[i];
+            } else if (e < kTileT && jt * kTileT + e < Lc) {
+                float ip = 0.f;
+                for (int qi = 0; qi < G.O; ++qi) ip += maxg[qi * kTileT + e];
+                A.sl.rawI[(size_t)s * G.ML + jt * kTileT + e] = ip * invO;
+            }
+        }
     }
+
+    // ---------------------------------------------------------------- teardown
+    if (warp == 1 && lane == 0) ptx::mbar_wait(&bars->mma_done, 0, 50000000ull);
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    if (warp == 1) ptx::tmem_dealloc(tmem, A.tmem_cols);
 }
 
-template <int HP>
-void launch_hp(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st) {
-    const WinShape ws = win_shape(g.Hkv, g.w, g.g);
-    window_kernel<HP><<<g.total_chunks, ws.threads, window_smem_bytes(g), st>>>(g, io, sc, sl);
-}
+int npad_of(int R) { return (R + 15) & ~15; }
 
-template <int HP>
-cudaError_t configure_hp(size_t bytes) {
-    return cudaFuncSetAttribute(window_kernel<HP>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
-}
+int kst_for(int Npad, int O) { return win_smem_bytes(Npad, O, 2) <= (size_t)kMaxSmemWin ? 2 : 1; }
 
 }  // namespace
 
-int window_blocks(int Lc) { return Lc > 0 ? (Lc + kBlockT - 1) / kBlockT : 0; }
-
-int window_threads(const Geometry& g) { return win_shape(g.Hkv, g.w, g.g).threads; }
-
 size_t window_smem_bytes(const Geometry& g) {
-    const WinShape ws = win_shape(g.Hkv, g.w, g.g);
-    return sizeof(float) * ((size_t)g.Hkv * g.R + (size_t)ws.QS * kBlockT * g.Hkv * 3);
+    const int Npad = npad_of(g.R);
+    return win_smem_bytes(Npad, g.O, kst_for(Npad, g.O));
 }
 
 cudaError_t configure_window(const Geometry& g) {
-    // Per-function attributes shared by every handle: the largest geometry kvec_create accepts.
+    // Per-function attribute shared by every handle: the largest supported geometry.
     size_t need = 0;
-    for (int h = 1; h <= 32; ++h)
-        for (int gg = 1; gg <= 256; ++gg) {
-            Geometry t = g;
-            t.Hkv = h;
-            t.g = gg;
-            t.w = 256 / gg;
-            t.R = t.g * t.w;
-            const size_t b = window_smem_bytes(t);
-            if (b > need) need = b;
-        }
-    cudaError_t e = configure_hp<1>(need);
-    if (e == cudaSuccess) e = configure_hp<2>(need);
-    if (e == cudaSuccess) e = configure_hp<4>(need);
-    if (e == cudaSuccess) e = configure_hp<8>(need);
-    if (e == cudaSuccess) e = configure_hp<16>(need);
-    if (e == cudaSuccess) e = configure_hp<32>(need);
+    for (int R = 16; R <= 256; R += 16) {
+        const size_t b = win_smem_bytes(R, kMaxObsWindow, kst_for(R, kMaxObsWindow));
+        if (b > need) need = b;
+    }
+    (void)g;
+    cudaError_t e = cudaSuccess;
+    for (auto fn : {window_kernel<0>, window_kernel<1>, window_kernel<2>, window_kernel<4>, window_kernel<7>,
+                    window_kernel<8>})
+        if (e == cudaSuccess) e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)need);
     return e;
 }
 
-void launch_window(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st) {
-    if (g.total_chunks == 0) return;
-    const WinShape ws = win_shape(g.Hkv, g.w, g.g);
-    switch (ws.HP) {
-        case 1: launch_hp<1>(g, io, sc, sl, st); break;
-        case 2: launch_hp<2>(g, io, sc, sl, st); break;
-        case 4: launch_hp<4>(g, io, sc, sl, st); break;
-        case 8: launch_hp<8>(g, io, sc, sl, st); break;
-        case 16: launch_hp<16>(g, io, sc, sl, st); break;
-        default: launch_hp<32>(g, io, sc, sl, st); break;
+cudaError_t launch_window(const ScorePlan& sp, const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl,
+                          cudaStream_t st) {
+    if (g.win_tiles == 0) return cudaSuccess;
+    WinArgs a{};
+    a.G = g;
+    a.sc = sc;
+    a.sl = sl;
+    a.cu = io.cu;
+    for (int b = 0; b <= g.batch && b <= kWinCuParam; ++b) a.cuv[b] = g.cu_host ? g.cu_host[b] : 0;
+    a.Npad = npad_of(g.R);
+    a.kst = kst_for(a.Npad, g.O);
+    a.nacc = 2 * a.Npad + 32 <= 512 ? 2 : 1;
+    uint32_t need = a.nacc == 2 ? (uint32_t)(2 * a.Npad + 32) : 512u, cols = 32;
+    while (cols < need) cols <<= 1;
+    a.tmem_cols = cols;
+    const size_t smem = win_smem_bytes(a.Npad, g.O, a.kst);
+    const int grid = g.win_tiles * g.NG;
+    switch (g.g) {
+        case 1: window_kernel<1><<<grid, kWinThreads, smem, st>>>(sp.kmap, sp.qmap, a); break;
+        case 2: window_kernel<2><<<grid, kWinThreads, smem, st>>>(sp.kmap, sp.qmap, a); break;
+        case 4: window_kernel<4><<<grid, kWinThreads, smem, st>>>(sp.kmap, sp.qmap, a); break;
+        case 7: window_kernel<7><<<grid, kWinThreads, smem, st>>>(sp.kmap, sp.qmap, a); break;
+        case 8: window_kernel<8><<<grid, kWinThreads, smem, st>>>(sp.kmap, sp.qmap, a); break;
+        default: window_kernel<0><<<grid, kWinThreads, smem, st>>>(sp.kmap, sp.qmap, a); break;
     }
+    return cudaGetLastError();
 }
 
 }  // namespace kvec

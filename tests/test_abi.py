@@ -87,3 +87,17 @@ def test_calls_on_null_handle_are_rejected(lib):
 def test_status_strings(lib):
     for code in range(6):
         assert kvec.kvec_status_string(code)
+
+
+def test_noalloc_refuses_oversize_calls_before_cuda(lib):
+    # The scratch check comes before any CUDA call, so it runs without a GPU and the
+    # (never dereferenced) pointers can be placeholders.
+    batch, L = 16, 131072
+    p = kvec.make_params(num_q_heads=32, num_kv_heads=8, max_batch=batch, max_seqlen=L)
+    cu = (ctypes.c_int32 * (batch + 1))(*[b * L for b in range(batch + 1)])
+    fake = 256
+    with pytest.raises(kvec.KvecError) as e:
+        kvec.kvec_select_layer_noalloc(p, batch, ctypes.addressof(cu), ctypes.addressof(cu), fake, fake, fake, fake,
+                                       512, fake, fake, fake, None)
+    assert e.value.status == kvec.KVEC_ERR_INVALID_ARG
+    assert "scratch" in str(e.value)

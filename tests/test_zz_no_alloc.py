@@ -61,13 +61,20 @@ def test_noalloc_matches_handle_entry_point_on_two_calls_in_a_row():
 
 
 def test_noalloc_rejects_calls_beyond_its_scratch():
+    # The buffers below are 16-byte dummies, so the call must be refused before
+    # anything is launched.  The geometry is chosen so that the per-position
+    # score rows alone (seven fp32 / uint32 rows per KV head and position) are far
+    # beyond the 32 MiB array, whatever else the scratch holds.
     wl = synth.WORKLOADS["llama8b_l32768_b128"]
-    params = kvec.params_from_workload(wl)
-    cu = torch.tensor(wl.cu_seqlens, dtype=torch.int32)
+    batch, L = 16, 131072
+    params = kvec.params_from_workload(wl, max_batch=batch, max_seqlen=L)
+    lower_bound = batch * params.num_kv_heads * L * 4 * 7
+    assert lower_bound > 8 * 32 * 2**20, "the geometry no longer exceeds the scratch by a safe margin"
+    cu = torch.arange(0, (batch + 1) * L, L, dtype=torch.int32)
     dummy = torch.zeros(16, dtype=torch.uint8, device="cuda")
     p = dummy.data_ptr()
     with pytest.raises(kvec.KvecError) as e:
-        kvec.kvec_select_layer_noalloc(params, 1, cu.data_ptr(), cu.cuda().data_ptr(), p, p, p, p, wl.budget,
+        kvec.kvec_select_layer_noalloc(params, batch, cu.data_ptr(), cu.cuda().data_ptr(), p, p, p, p, wl.budget,
                                        p, p, p, torch.cuda.current_stream().cuda_stream)
     assert e.value.status == kvec.KVEC_ERR_INVALID_ARG
     assert "scratch" in str(e.value)

@@ -222,7 +222,7 @@ Geometry make_geometry(const kvec_handle* h, int batch, int budget, int tiles, i
 // One layer, every kernel on one stream with one slot (used without a handle).
 kvec_status run_layer_sequential(kvec_handle* h, const Geometry& G, const LayerIO& io, cudaStream_t st) {
     ScorePlan plan;
-    cudaError_t se = plan_score(G, io, h->sc, h->num_sms, &plan);
+    cudaError_t se = plan_score(G, io, h->sc, h->num_sms, nullptr, &plan);
     if (se != cudaSuccess) return cuda_fail(se, "score kernel tensor maps");
     se = launch_score(plan, st);
     if (se != cudaSuccess) return cuda_fail(se, "score kernel launch");
@@ -258,7 +258,7 @@ kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* io
         const LayerIO& io = ios[l];
         if (l >= 2) KV_CHECK(cudaStreamWaitEvent(h->s_score, h->ev_win[l - 2], 0));
         ScorePlan plan;
-        cudaError_t se = plan_score(G, io, sc, h->num_sms, &plan);
+        cudaError_t se = plan_score(G, io, sc, h->num_sms, l + 1 < n ? ios[l + 1].k : nullptr, &plan);
         if (se != cudaSuccess) return cuda_fail(se, "score kernel tensor maps");
         timed_launch(h, 0, h->s_score, [&] { se = launch_score(plan, h->s_score); });
         if (se != cudaSuccess) return cuda_fail(se, "score kernel launch");
@@ -678,10 +678,10 @@ kvec_status kvec_select_layer_noalloc(const kvec_params* params, int batch, cons
     cudaError_t e = cudaGetDevice(&prev);
     if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
     tmp.device = prev;
-    Geometry G = make_geometry(&tmp, batch, budget, tiles, chunks, cu_seqlens_host[batch]);
-    G.cu_host = cu_seqlens_host;
     e = cudaDeviceGetAttribute(&tmp.num_sms, cudaDevAttrMultiProcessorCount, prev);
     if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
+    Geometry G = make_geometry(&tmp, batch, budget, tiles, chunks, cu_seqlens_host[batch]);
+    G.cu_host = cu_seqlens_host;
     void* base = nullptr;
     s = noalloc_setup(prev, &base, G);
     if (s != KVEC_OK) return s;

@@ -103,7 +103,9 @@ struct ScorePlan {
     int grid, threads;
     size_t smem;
 };
-cudaError_t plan_score(const Geometry& g, const LayerIO& io, const Scratch& sc, int num_sms, ScorePlan* plan);
+// next_k: the next layer's K (same shape), prefetched into L2 by this launch; may be null.
+cudaError_t plan_score(const Geometry& g, const LayerIO& io, const Scratch& sc, int num_sms, const void* next_k,
+                       ScorePlan* plan);
 cudaError_t launch_score(const ScorePlan& plan, cudaStream_t st);
 cudaError_t launch_window(const ScorePlan& sp, const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl,
                           cudaStream_t st);

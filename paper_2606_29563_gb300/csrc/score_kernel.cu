@@ -71,8 +71,8 @@ struct ScoreArgs {
     Geometry G;
     const int* cu;                 // device cu_seqlens
     int cuv[kMaxCuParam + 1];      // the same offsets (when batch <= kMaxCuParam)
-    const uint8_t* kbytes;         // the layer's K, for the L2 prefetch
-    long long kbytes_total;
+    const uint8_t* next_k;         // the next layer's K (L2 prefetch), or null
+    long long kbytes_total;        // bytes of one layer's K
     Scratch sc;
     int W;        // total work items
     int MB;       // 128-row M-blocks per KV head (1 or 2)
@@ -121,7 +121,11 @@ __global__ void __launch_bounds__(576, 1)
     const int Gc = gridDim.x;
     const int i0 = range_start(blockIdx.x, A.W, Gc), i1 = range_start(blockIdx.x + 1, A.W, Gc);
 
-    if (threadIdx.x == 0) {
+    if (warp == 0 && lane == 0) {
+        ptx::prefetch_tensormap(&kmap);
+        ptx::prefetch_tensormap(&qmap);
+    }
+    if (threadIdx.x == 32) {
         for (int s = 0; s < A.kst; ++s) {
             ptx::mbar_init(&bars->k_full[s], 1);
             ptx::mbar_init(&bars->k_empty[s], 1);
@@ -140,10 +144,6 @@ __global__ void __launch_bounds__(576, 1)
         ptx::tmem_alloc(&bars->tmem_base, kTmemCols);
         ptx::tmem_relinquish();
     }
-    if (warp == 0 && lane == 0) {
-        ptx::prefetch_tensormap(&kmap);
-        ptx::prefetch_tensormap(&qmap);
-    }
     ptx::tc_fence_before();
     __syncthreads();
     ptx::tc_fence_after();
@@ -152,18 +152,26 @@ __global__ void __launch_bounds__(576, 1)
     if (warp == 0) {
         // ------------------------------------------------------------ TMA producer
         if (lane == 0) {
-            // Stream this CTA's contiguous slice of the layer's K into L2 first: DRAM then
-            // sees sequential reads, and the strided per-head tiles below hit in L2.
-            {
+            // Ask L2 for every K tile of this CTA's items up front (beyond the ring's
+            // first loads), so DRAM sees the whole range at once.
+            for (int i = i0 + A.kst; i < i1; ++i) {
+                const ItemPos p = decode_item(cuview, G.batch, G.Hkv, i);
+                const int row = cu(p.s) + p.j * kTileT;
+                ptx::prefetch_tile_3d(&kmap, 0, p.h, row);
+                ptx::prefetch_tile_3d(&kmap, 64, p.h, row);
+            }
+            const uint64_t policy = ptx::policy_evict_normal();   // the window kernel reads K again
+            // Once this layer's first tiles are requested, stream this CTA's slice of
+            // the next layer's K into L2: that layer's score pass then reads from L2.
+            auto prefetch_next = [&]() {
                 const long long per = ((A.kbytes_total / Gc) + 15) & ~15LL;
                 long long lo = per * blockIdx.x, hi = lo + per;
                 if (hi > A.kbytes_total) hi = A.kbytes_total;
                 for (long long o = lo; o < hi; o += 32768) {
                     const long long n = hi - o < 32768 ? hi - o : 32768;
-                    ptx::prefetch_l2_bulk(A.kbytes + o, (uint32_t)(n & ~15LL));
+                    ptx::prefetch_l2_bulk(A.next_k + o, (uint32_t)(n & ~15LL));
                 }
-            }
-            const uint64_t policy = ptx::policy_evict_normal();   // the window kernel reads K again
+            };
             int prev_sh = -1, qloads = 0;
             int fills[kKStages] = {0, 0, 0, 0};
             for (int i = i0, it = 0; i < i1 && !bars->abort_flag; ++i, ++it) {
@@ -191,7 +199,9 @@ __global__ void __launch_bounds__(576, 1)
                 ptx::tma_load_3d(dst, &kmap, &bars->k_full[st], 0, p.h, row, policy);
                 ptx::tma_load_3d(dst + kKHalfBytes, &kmap, &bars->k_full[st], 64, p.h, row, policy);
                 ++fills[st];
+                if (it + 1 == A.kst && A.next_k) prefetch_next();
             }
+            if (i1 - i0 < A.kst && A.next_k) prefetch_next();
             // Drain: every issued copy lands before the CTA may exit.
             for (int st = 0; st < A.kst; ++st)
                 if (fills[st] > 0) ptx::mbar_wait(&bars->k_full[st], (fills[st] - 1) & 1, 50000000ull);
@@ -450,7 +460,8 @@ cudaError_t configure_score(const Geometry& g) {
     return cudaFuncSetAttribute(score_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)need);
 }
 
-cudaError_t plan_score(const Geometry& g, const LayerIO& io, const Scratch& sc, int num_sms, ScorePlan* plan) {
+cudaError_t plan_score(const Geometry& g, const LayerIO& io, const Scratch& sc, int num_sms, const void* next_k,
+                       ScorePlan* plan) {
     PFN_cuTensorMapEncodeTiled_v12000 enc = encode_fn();
     if (!enc) return cudaErrorNotSupported;
     CUtensorMap& kmap = plan->kmap;
@@ -482,7 +493,7 @@ cudaError_t plan_score(const Geometry& g, const LayerIO& io, const Scratch& sc, 
     a.G = g;
     a.cu = io.cu;
     for (int b = 0; b <= g.batch && b <= kMaxCuParam; ++b) a.cuv[b] = g.cu_host ? g.cu_host[b] : 0;
-    a.kbytes = reinterpret_cast<const uint8_t*>(io.k);
+    a.next_k = reinterpret_cast<const uint8_t*>(next_k);
     a.kbytes_total = (long long)g.total_tokens * g.Hkv * kHeadDim * 2;
     a.sc = sc;
     a.W = g.total_tiles * g.Hkv;

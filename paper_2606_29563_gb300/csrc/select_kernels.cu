@@ -22,7 +22,7 @@ __host__ __device__ inline bool keys_in_smem(int ML) { return ML <= kSmemKeys; }
 __host__ __device__ inline int key_stride(const Geometry& g) { return keys_in_smem(g.ML) ? (g.words | 1) : g.words; }
 __device__ __forceinline__ int key_index(int t, int kw) { return (t & 31) * kw + (t >> 5); }
 
-constexpr int kIChunk = 2048;                  // positions of raw I combined per pass in the heads kernel
+constexpr int kPoolSmemBytes = 96 * 1024;     // raw-I chunk of the heads pooling kernel
 constexpr int kTopkWarps = 8;                  // warps that run the radix select
 constexpr int kTopkThreads = 32 * kTopkWarps;
 constexpr int kTopkSeg = 1024;                 // positions per warp segment (32 per lane)
@@ -432,24 +432,37 @@ __device__ __forceinline__ uint32_t range_bits(int word, int lo, int hi) {
 }
 
 // Max-pool (width 2*halo+1, stride 1, neighbours outside [0, Lc) ignored) of
-// the four positions [t4, t4+4) of a row: the raw values [t4-8, t4+12) arrive
-// as five float4 loads issued together.
+// the four positions [t4, t4+4) of a row given as the sum of `parts` partial
+// rows `stride` floats apart: the raw values [t4-8, t4+12) of every part
+// arrive as five float4 loads issued together.
 struct Pooled4 {
     float v[4];
 };
 
-__device__ __forceinline__ Pooled4 pool4(const float* __restrict__ raw, int t4, int Lc, int halo) {
+__device__ __forceinline__ Pooled4 pool4(const float* __restrict__ raw, size_t stride, int parts, int t4, int Lc,
+                                         int halo) {
     float x[20];
 #pragma unroll
-    for (int b = 0; b < 5; ++b) {
-        const int p = t4 - 8 + 4 * b;
-        float4 f = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
-        if (p >= 0 && p < Lc) f = __ldcg(reinterpret_cast<const float4*>(raw + p));
-        x[4 * b] = p < Lc ? f.x : -INFINITY;
-        x[4 * b + 1] = p + 1 < Lc ? f.y : -INFINITY;
-        x[4 * b + 2] = p + 2 < Lc ? f.z : -INFINITY;
-        x[4 * b + 3] = p + 3 < Lc ? f.w : -INFINITY;
+    for (int i = 0; i < 20; ++i) x[i] = 0.f;
+    for (int pt = 0; pt < parts; ++pt) {
+        const float* r = raw + pt * stride;
+        float4 f[5];
+#pragma unroll
+        for (int b = 0; b < 5; ++b) {
+            const int p = t4 - 8 + 4 * b;
+            f[b] = (p >= 0 && p < Lc) ? __ldcg(reinterpret_cast<const float4*>(r + p)) : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+#pragma unroll
+        for (int b = 0; b < 5; ++b) {
+            x[4 * b] += f[b].x;
+            x[4 * b + 1] += f[b].y;
+            x[4 * b + 2] += f[b].z;
+            x[4 * b + 3] += f[b].w;
+        }
     }
+#pragma unroll
+    for (int i = 0; i < 20; ++i)
+        if (t4 - 8 + i < 0 || t4 - 8 + i >= Lc) x[i] = -INFINITY;
     Pooled4 out;
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
@@ -509,7 +522,7 @@ __device__ Moments block_moments(Moments v, float3* red) {
 // in fp32).
 __global__ void __launch_bounds__(kSelectThreads) heads_pool_kernel(Geometry G, LayerIO io, Scratch sc, Slot sl) {
     __shared__ float3 red[32];
-    __shared__ float ibuf[kIChunk + 2 * (kMaxPool / 2)];
+    extern __shared__ float mbuf[];   // raw I of a chunk, per window row (several head groups only)
     const int h = blockIdx.x, s = blockIdx.y;
     const int tid = threadIdx.x, NT = blockDim.x;
     const int L = io.cu[s + 1] - io.cu[s];
@@ -522,8 +535,8 @@ __global__ void __launch_bounds__(kSelectThreads) heads_pool_kernel(Geometry G, 
     const float* rO = sl.rawO + row * G.ML;
     const float* rOe = sl.rawOe + row * G.ML;
     for (int t4 = 4 * tid; t4 < Lc; t4 += 4 * NT) {
-        const Pooled4 a = pool4(rO, t4, Lc, halo);
-        const Pooled4 b = pool4(rOe, t4, Lc, halo);
+        const Pooled4 a = pool4(rO, 0, 1, t4, Lc, halo);
+        const Pooled4 b = pool4(rOe, 0, 1, t4, Lc, halo);
         *reinterpret_cast<float4*>(sl.PO + row * G.ML + t4) = make_float4(a.v[0], a.v[1], a.v[2], a.v[3]);
         *reinterpret_cast<float4*>(sl.POe + row * G.ML + t4) = make_float4(b.v[0], b.v[1], b.v[2], b.v[3]);
 #pragma unroll
@@ -537,13 +550,14 @@ __global__ void __launch_bounds__(kSelectThreads) heads_pool_kernel(Geometry G, 
         if (G.NG == 1) {
             const float* rI = sl.rawI + (size_t)s * G.ML;
             for (int t4 = a0 + 4 * tid; t4 < b0; t4 += 4 * NT) {
-                const Pooled4 c = pool4(rI, t4, Lc, halo);
+                const Pooled4 c = pool4(rI, 0, 1, t4, Lc, halo);
                 *reinterpret_cast<float4*>(sl.I + (size_t)s * G.ML + t4) = make_float4(c.v[0], c.v[1], c.v[2], c.v[3]);
             }
         } else {
-            // The window kernel left, per head group, the maxima over its KV heads of
-            // G_h[q][t]: raw I is the sum over q of the maxima over the groups, built
-            // chunk by chunk (with the pool halo) in shared memory, then pooled.
+            // The window kernel left, per group of KV heads, the maxima over the
+            // group of G_h[q][t] (q >= w - O): raw I is (1/O) times the sum over q of
+            // the maxima over the groups.  Built in shared memory chunk by chunk (with
+            // the pool halo), each (q, t) element loaded by its own thread, then pooled.
             int tbase = 0;
             for (int b = 0; b < s; ++b) {
                 const int lb = io.cu[b + 1] - io.cu[b] - G.w;
@@ -551,25 +565,47 @@ __global__ void __launch_bounds__(kSelectThreads) heads_pool_kernel(Geometry G, 
             }
             const float invO = 1.f / (float)G.O;
             const size_t n_el = (size_t)G.O * kTileT;
-            for (int c = a0; c < b0; c += kIChunk) {
-                const int ce = min(c + kIChunk, b0);
-                const int lo = max(c - halo, 0), hi = min(ce + halo, Lc);
-                for (int t = lo + tid; t < hi; t += NT) {
-                    const float* wt = sl.wpart + (size_t)(tbase + (t >> 7)) * G.NG * n_el + (t & (kTileT - 1));
-                    float sum = 0.f;
-                    for (int qi = 0; qi < G.O; ++qi) {
-                        float m = __ldcg(wt + (size_t)qi * kTileT);
-                        for (int gg = 1; gg < G.NG; ++gg) m = fmaxf(m, __ldcg(wt + ((size_t)gg * G.O + qi) * kTileT));
-                        sum += m;
+            const int chunk = ((kPoolSmemBytes / 4) / G.O - 2 * halo) & ~3;
+            for (int c = a0; c < b0; c += chunk) {
+                const int ce = min(c + chunk, b0);
+                const int lo = max(c - halo, 0), hi = min(ce + halo, Lc), span = hi - lo;
+                const int n = G.O * span;   // mbuf[q][span]: element index q * span + (t - lo)
+                for (int base = tid; base < n; base += 8 * NT) {
+                    float m[8];
+#pragma unroll
+                    for (int u = 0; u < 8; ++u) {
+                        const int idx = base + u * NT;
+                        const int q = idx / span, t = lo + idx - q * span;
+                        m[u] = idx < n ? __ldcg(sl.wpart + (size_t)(tbase + (t >> 7)) * G.NG * n_el + q * kTileT + (t & 127))
+                                       : 0.f;
                     }
-                    ibuf[t - lo] = sum * invO;
+                    for (int gg = 1; gg < G.NG; ++gg) {
+#pragma unroll
+                        for (int u = 0; u < 8; ++u) {
+                            const int idx = base + u * NT;
+                            const int q = idx / span, t = lo + idx - q * span;
+                            if (idx < n)
+                                m[u] = fmaxf(m[u], __ldcg(sl.wpart + ((size_t)(tbase + (t >> 7)) * G.NG + gg) * n_el +
+                                                           q * kTileT + (t & 127)));
+                        }
+                    }
+#pragma unroll
+                    for (int u = 0; u < 8; ++u)
+                        if (base + u * NT < n) mbuf[base + u * NT] = m[u];
+                }
+                __syncthreads();
+                // Sum over q in place: column tt of row 0 becomes raw I (each thread owns its columns).
+                for (int tt = tid; tt < span; tt += NT) {
+                    float sum = 0.f;
+                    for (int q = 0; q < G.O; ++q) sum += mbuf[q * span + tt];
+                    mbuf[tt] = sum * invO;
                 }
                 __syncthreads();
                 for (int t = c + tid; t < ce; t += NT) {
-                    float m = ibuf[t - lo];
+                    float m = mbuf[t - lo];
                     for (int d = 1; d <= halo; ++d) {
-                        if (t - d >= 0) m = fmaxf(m, ibuf[t - d - lo]);
-                        if (t + d < Lc) m = fmaxf(m, ibuf[t + d - lo]);
+                        if (t - d >= 0) m = fmaxf(m, mbuf[t - d - lo]);
+                        if (t + d < Lc) m = fmaxf(m, mbuf[t + d - lo]);
                     }
                     sl.I[(size_t)s * G.ML + t] = m;
                 }
@@ -797,6 +833,8 @@ cudaError_t configure_select() {
     const int need = (int)(sizeof(uint32_t) * (kSmemKeys / 32 + 32 * ((kSmemKeys / 32) | 1)));
     cudaError_t e = cudaFuncSetAttribute(heads_topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, need);
     if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(heads_pool_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kPoolSmemBytes);
+    if (e == cudaSuccess)
         e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, need);
     return e;
 }
@@ -804,7 +842,8 @@ cudaError_t configure_select() {
 cudaError_t launch_heads(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st,
                          int priority) {
     const dim3 grid(g.Hkv, g.batch);
-    cudaError_t e = launch_prio(heads_pool_kernel, grid, dim3(kSelectThreads), 0, st, priority, false, g, io, sc, sl);
+    cudaError_t e = launch_prio(heads_pool_kernel, grid, dim3(kSelectThreads), g.NG > 1 ? (size_t)kPoolSmemBytes : 0, st,
+                                priority, false, g, io, sc, sl);
     if (e == cudaSuccess)
         e = launch_prio(heads_topk_kernel, grid, dim3(kSelectThreads), heads_smem_bytes(g), st, priority, false, g, io,
                         sc, sl);

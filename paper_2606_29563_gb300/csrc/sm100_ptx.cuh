@@ -91,6 +91,14 @@ __device__ __forceinline__ void prefetch_l2_bulk(const void* src, uint32_t bytes
                  : "memory");
 }
 
+// L2 prefetch of one box of a tiled tensor map (no shared memory, no barrier).
+__device__ __forceinline__ void prefetch_tile_3d(const CUtensorMap* map, int c0, int c1, int c2) {
+    asm volatile("cp.async.bulk.prefetch.tensor.3d.L2.global.tile [%0, {%1, %2, %3}];\n" ::"l"(
+                     reinterpret_cast<uint64_t>(map)),
+                 "r"(c0), "r"(c1), "r"(c2)
+                 : "memory");
+}
+
 __device__ __forceinline__ void prefetch_tensormap(const CUtensorMap* map) {
     asm volatile("prefetch.tensormap [%0];\n" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
 }

@@ -59,7 +59,7 @@ struct __align__(8) WinBars {
 __host__ __device__ inline size_t stage_bytes(int Npad) { return (size_t)kKTileBytes + 2 * (size_t)Npad * 128; }
 
 __host__ __device__ inline size_t win_smem_bytes(int Npad, int O, int kst) {
-    return 1024 + (size_t)kst * stage_bytes(Npad) + kWinHeadsPerCta * kRsRows * sizeof(float2) +
+    return 1024 + (size_t)kst * stage_bytes(Npad) + kWinHeadsPerCta * kRsRows * sizeof(float) +
            (size_t)O * kTileT * sizeof(float) + kWinHeadsPerCta * 4 * kTileT * sizeof(float2) + sizeof(WinBars);
 }
 
@@ -73,7 +73,7 @@ __device__ __forceinline__ void win_abort(WinBars* bars, int* err) {
 // the head maxima.  GG > 0 is the group size g known at compile time: each
 // 32-column chunk holds 32 / GG whole groups and runs as straight-line code.
 template <int GG>
-__device__ __forceinline__ void head_rows(uint32_t taddr, const float2* __restrict__ rsb, int g, int q_lo, int q_hi,
+__device__ __forceinline__ void head_rows(uint32_t taddr, const float* __restrict__ rsb, int g, int q_lo, int q_hi,
                                           float sl2, int qO, int qOe, float* maxg_col, bool first, float& po,
                                           float& poe) {
     if constexpr (GG > 0) {
@@ -86,8 +86,7 @@ __device__ __forceinline__ void head_rows(uint32_t taddr, const float2* __restri
             float pr[CW];
 #pragma unroll
             for (int i = 0; i < CW; ++i) {
-                const float2 mz = rsb[c0 + i];
-                pr[i] = ptx::ex2(fmaf(v[i], sl2, -mz.x)) * mz.y;
+                pr[i] = ptx::ex2(fmaf(v[i], sl2, -rsb[c0 + i]));
             }
 #pragma unroll
             for (int k = 0; k < QPC; ++k) {
@@ -117,8 +116,7 @@ __device__ __forceinline__ void head_rows(uint32_t taddr, const float2* __restri
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
                 if (i >= n) break;
-                const float2 mz = rsb[c0 + i];
-                gs += ptx::ex2(fmaf(v[i], sl2, -mz.x)) * mz.y;
+                gs += ptx::ex2(fmaf(v[i], sl2, -rsb[c0 + i]));
                 if (++jq == g) {
                     if (q >= qOe) poe += gs;
                     if (q >= qO) {
@@ -140,11 +138,15 @@ __global__ void __launch_bounds__(kWinThreads, 1)
     window_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap qmap,
                   const __grid_constant__ WinArgs A) {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
+    if (threadIdx.x == 0) {
+        ptx::prefetch_tensormap(&kmap);
+        ptx::prefetch_tensormap(&qmap);
+    }
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const Geometry& G = A.G;
     const int Npad = A.Npad, R = G.R;
     const size_t sbytes = stage_bytes(Npad);
-    float2* rs = reinterpret_cast<float2*>(smem + A.kst * sbytes);      // [HG][kRsRows] (m_r, 1 / Z_r)
+    float* rs = reinterpret_cast<float*>(smem + A.kst * sbytes);        // [HG][kRsRows] m_r + log2 Z_r
     float* maxg = reinterpret_cast<float*>(rs + kWinHeadsPerCta * kRsRows);   // [O][128] max over heads of G_h[q][t]
     float2* xfer = reinterpret_cast<float2*>(maxg + G.O * kTileT);      // [HG][4][128] quarters' (P_O, P_O') sums
     WinBars* bars = reinterpret_cast<WinBars*>(xfer + kWinHeadsPerCta * 4 * kTileT);
@@ -178,7 +180,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
     const int nh = min(G.HG, G.Hkv - h0);
     const int NB = A.nacc;
 
-    if (threadIdx.x == 0) {
+    if (threadIdx.x == 32) {
         for (int i = 0; i < 2; ++i) {
             ptx::mbar_init(&bars->full[i], 1);
             ptx::mbar_init(&bars->empty[i], 1);
@@ -193,10 +195,6 @@ __global__ void __launch_bounds__(kWinThreads, 1)
     if (warp == 1) {
         ptx::tmem_alloc(&bars->tmem_base, A.tmem_cols);
         ptx::tmem_relinquish();
-    }
-    if (warp == 0 && lane == 0) {
-        ptx::prefetch_tensormap(&kmap);
-        ptx::prefetch_tensormap(&qmap);
     }
     ptx::tc_fence_before();
     __syncthreads();
@@ -267,11 +265,11 @@ __global__ void __launch_bounds__(kWinThreads, 1)
         const int q_lo = (qt * G.w) >> 2, q_hi = ((qt + 1) * G.w) >> 2;
         const int qO = G.w - G.O, qOe = G.w - G.Oe;
         const float invO = 1.f / (float)G.O, invOe = 1.f / (float)G.Oe;
-        // Row statistics of every head of the group: (m_r, 1 / Z_r).
+        // Row statistics of every head of the group: A = 2^(s * sl2 - (m_r + log2 Z_r)).
         for (int i = e; i < nh * R; i += kEpiThreads) {
             const int hh = i / R, r = i - hh * R;
             const float2 ms = __ldcg(&A.sc.rowstat[((size_t)s * G.Hkv + h0 + hh) * R + r]);
-            rs[hh * kRsRows + r] = make_float2(ms.x, 1.f / ms.y);
+            rs[hh * kRsRows + r] = ms.x + __log2f(ms.y);
         }
         ptx::named_bar_sync(1, kEpiThreads);
         // The warps run through the heads independently: each waits for the

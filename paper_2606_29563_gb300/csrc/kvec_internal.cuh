@@ -14,7 +14,7 @@ constexpr int kTileT = 128;        // tokens per score / window tile (one MMA N 
 constexpr int kMaxPool = 15;       // largest pool kernel (halo 7)
 constexpr int kSelectThreads = 512;
 constexpr int kMaxObsWindow = 64;  // largest O: the window kernel keeps O x 128 head maxima in shared memory
-constexpr int kWinHeadsPerCta = 4; // KV heads one window CTA processes
+constexpr int kWinHeadsPerCta = 8; // KV heads one window CTA processes
 
 // Sizes and hyper-parameters shared by every kernel of one call.
 struct Geometry {

@@ -66,6 +66,7 @@ __device__ __forceinline__ int range_start(int b, int W, int G) {
 
 constexpr int kMaxCuParam = 64;          // sequences whose offsets travel in the kernel parameters
 constexpr int kScoreReserveSms = 8;      // SMs a score launch leaves to the other kernels
+constexpr int kScoreItemsPerCta = 8;     // fewest (sequence, head, tile) items a score CTA takes
 
 struct ScoreArgs {
     Geometry G;
@@ -152,26 +153,7 @@ __global__ void __launch_bounds__(576, 1)
     if (warp == 0) {
         // ------------------------------------------------------------ TMA producer
         if (lane == 0) {
-            // Ask L2 for every K tile of this CTA's items up front (beyond the ring's
-            // first loads), so DRAM sees the whole range at once.
-            for (int i = i0 + A.kst; i < i1; ++i) {
-                const ItemPos p = decode_item(cuview, G.batch, G.Hkv, i);
-                const int row = cu(p.s) + p.j * kTileT;
-                ptx::prefetch_tile_3d(&kmap, 0, p.h, row);
-                ptx::prefetch_tile_3d(&kmap, 64, p.h, row);
-            }
             const uint64_t policy = ptx::policy_evict_normal();   // the window kernel reads K again
-            // Once this layer's first tiles are requested, stream this CTA's slice of
-            // the next layer's K into L2: that layer's score pass then reads from L2.
-            auto prefetch_next = [&]() {
-                const long long per = ((A.kbytes_total / Gc) + 15) & ~15LL;
-                long long lo = per * blockIdx.x, hi = lo + per;
-                if (hi > A.kbytes_total) hi = A.kbytes_total;
-                for (long long o = lo; o < hi; o += 32768) {
-                    const long long n = hi - o < 32768 ? hi - o : 32768;
-                    ptx::prefetch_l2_bulk(A.next_k + o, (uint32_t)(n & ~15LL));
-                }
-            };
             int prev_sh = -1, qloads = 0;
             int fills[kKStages] = {0, 0, 0, 0};
             for (int i = i0, it = 0; i < i1 && !bars->abort_flag; ++i, ++it) {
@@ -199,9 +181,7 @@ __global__ void __launch_bounds__(576, 1)
                 ptx::tma_load_3d(dst, &kmap, &bars->k_full[st], 0, p.h, row, policy);
                 ptx::tma_load_3d(dst + kKHalfBytes, &kmap, &bars->k_full[st], 64, p.h, row, policy);
                 ++fills[st];
-                if (it + 1 == A.kst && A.next_k) prefetch_next();
             }
-            if (i1 - i0 < A.kst && A.next_k) prefetch_next();
             // Drain: every issued copy lands before the CTA may exit.
             for (int st = 0; st < A.kst; ++st)
                 if (fills[st] > 0) ptx::mbar_wait(&bars->k_full[st], (fills[st] - 1) & 1, 50000000ull);
@@ -500,11 +480,13 @@ cudaError_t plan_score(const Geometry& g, const LayerIO& io, const Scratch& sc, 
     a.MB = mblocks(g);
     a.Rpad = 128 * a.MB;
     a.kst = kstages_for(g);
-    // As few CTAs as give the same items per CTA on all but kScoreReserveSms SMs:
-    // the SMs left free run the window, heads and selection kernels of other
-    // layers, which cannot share an SM with a score CTA.
+    // At least kScoreItemsPerCta items per CTA (the CTA's set-up and merge are paid
+    // once and its K stream overlaps the epilogue), on at most all but
+    // kScoreReserveSms SMs: the rest run the window, heads and selection kernels of
+    // neighbouring layers, which cannot share an SM with a score CTA.
     const int usable = num_sms > 2 * kScoreReserveSms ? num_sms - kScoreReserveSms : num_sms;
-    const int per_cta = (a.W + usable - 1) / usable;
+    int per_cta = (a.W + usable - 1) / usable;
+    if (per_cta < kScoreItemsPerCta) per_cta = kScoreItemsPerCta;
     plan->grid = (a.W + per_cta - 1) / per_cta;
     plan->threads = 32 * (2 + 8 * a.MB);
     plan->smem = smem_bytes_for(g);

@@ -16,6 +16,9 @@ constexpr int kSmemKeys = 40960;   // positions whose keys fit in shared memory 
 
 __host__ __device__ inline bool keys_in_smem(int ML) { return ML <= kSmemKeys; }
 
+constexpr int kSmemScores = 16448;  // row stride up to which the select kernel caches P and I in shared memory
+__host__ __device__ inline bool scores_in_smem(int ML) { return ML <= kSmemScores; }
+
 // Key rows are stored transposed, key t at keys[(t & 31) * kw + (t >> 5)]: a lane
 // that owns the 32 positions of one bits word then reads them from consecutive
 // words of its warp's neighbours (an odd stride keeps the writers' banks apart).
@@ -613,6 +616,8 @@ __global__ void __launch_bounds__(kSelectThreads) heads_pool_kernel(Geometry G, 
             }
         }
     }
+    // The preserved-token kernel may be scheduled now; it waits for this grid before reading sigma.
+    asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
     mom = block_moments(mom, red);
     if (tid == 0) sl.sigma[row] = Lc >= 2 ? sqrtf(fmaxf(mom.m2, 0.f) / (float)(Lc - 1)) : 0.f;
 }
@@ -631,6 +636,9 @@ __global__ void __launch_bounds__(kSelectThreads) heads_topk_kernel(Geometry G, 
     const int Lc = L - G.w;
     const size_t row = (size_t)s * G.Hkv + h;
     for (int wd = tid; wd < G.words; wd += NT) bits[wd] = 0u;
+    // Programmatic dependent of the pooling kernel: its sigmas and pooled rows are
+    // read only after that grid has completed.
+    asm volatile("griddepcontrol.wait;\n" ::: "memory");
     if (tid < 32) {
         const float sigma = __ldcg(&sl.sigma[row]);
         const float so = tid < G.Hkv ? __ldcg(&sl.sigma[(size_t)s * G.Hkv + tid]) : INFINITY;
@@ -677,13 +685,30 @@ __global__ void __launch_bounds__(kSelectThreads) heads_topk_kernel(Geometry G, 
 __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, LayerIO io, Scratch sc, Slot sl) {
     __shared__ TopkShared sm;
     __shared__ int last_head;
-    extern __shared__ uint32_t bits[];
+    extern __shared__ __align__(16) uint32_t bits[];
     const int h = blockIdx.x, s = blockIdx.y;
     const int tid = threadIdx.x, NT = blockDim.x;
     const int L = io.cu[s + 1] - io.cu[s];
     const int Lc = L - G.w;
     const int wordsL = (L + 31) >> 5;
     for (int wd = tid; wd < G.words; wd += NT) bits[wd] = 0u;
+    const int kw = key_stride(G);
+    const bool cached = scores_in_smem(G.ML) && L > G.budget;
+    // 16-byte aligned (float4 stores): the bits and keys before it have any length.
+    const size_t sp_off = ((size_t)G.words + (keys_in_smem(G.ML) ? 32 * (size_t)kw : 0) + 3) & ~(size_t)3;
+    float* sP = reinterpret_cast<float*>(bits + sp_off);
+    float* sI = sP + G.ML;
+    const size_t row = (size_t)s * G.Hkv + h;
+    const int top = sl.htop[row];
+    const float* P = (top ? sl.POe : sl.PO) + row * G.ML;
+    const float* I = sl.I + (size_t)s * G.ML;
+    if (cached) {
+        // This layer's scores do not depend on the previous layer: stage them now.
+        for (int t4 = 4 * tid; t4 < Lc; t4 += 4 * NT) {
+            *reinterpret_cast<float4*>(sP + t4) = __ldcg(reinterpret_cast<const float4*>(P + t4));
+            *reinterpret_cast<float4*>(sI + t4) = __ldcg(reinterpret_cast<const float4*>(I + t4));
+        }
+    }
     // Launched as a programmatic dependent of the previous layer's selection:
     // everything above overlaps its tail; the coverage state is read only after
     // that grid has completed and its writes are visible.
@@ -697,31 +722,28 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
     }
     __syncthreads();
     if (L > G.budget) {
-        const size_t row = (size_t)s * G.Hkv + h;
-        const int top = sl.htop[row];
-        const float* P = (top ? sl.POe : sl.PO) + row * G.ML;
-        const float* I = sl.I + (size_t)s * G.ML;
         const uint32_t* pres = sl.pres + row * G.words;
         float* Pp = sl.Pprime + row * G.ML;
         uint32_t* keys = keys_in_smem(G.ML) ? bits + G.words : sc.keys_sel + row * G.ML;
-        const int kw = key_stride(G);
+        const float* Pr = cached ? sP : P;
+        const float* Ir = cached ? sI : I;
         const float denom = (float)(ell + 1u);
-        for (int b0 = 4 * tid; b0 < Lc; b0 += 8 * NT) {
-            float4 pv[2], iv[2];
-            uchar4 nv[2];
-            uint32_t pw[2];
+        for (int b0 = 4 * tid; b0 < Lc; b0 += 16 * NT) {
+            float4 pv[4], iv[4];
+            uchar4 nv[4];
+            uint32_t pw[4];
 #pragma unroll
-            for (int u = 0; u < 2; ++u) {
+            for (int u = 0; u < 4; ++u) {
                 const int t4 = b0 + 4 * u * NT;
                 if (t4 < Lc) {
-                    pv[u] = *reinterpret_cast<const float4*>(P + t4);
-                    iv[u] = *reinterpret_cast<const float4*>(I + t4);
+                    pv[u] = *reinterpret_cast<const float4*>(Pr + t4);
+                    iv[u] = *reinterpret_cast<const float4*>(Ir + t4);
                     nv[u] = *reinterpret_cast<const uchar4*>(ncount + t4);
                     pw[u] = pres[t4 >> 5];
                 }
             }
 #pragma unroll
-            for (int u = 0; u < 2; ++u) {
+            for (int u = 0; u < 4; ++u) {
                 const int t4 = b0 + 4 * u * NT;
                 if (t4 >= Lc) continue;
                 const float p4[4] = {pv[u].x, pv[u].y, pv[u].z, pv[u].w};
@@ -824,18 +846,25 @@ __global__ void __launch_bounds__(256) gather_kernel(Geometry G, LayerIO io) {
 }  // namespace
 
 size_t select_smem_bytes(const Geometry& g) {
+    const size_t head = ((size_t)g.words + (keys_in_smem(g.ML) ? 32 * (size_t)key_stride(g) : 0) + 3) & ~(size_t)3;
+    return sizeof(uint32_t) * (head + (scores_in_smem(g.ML) ? 2 * (size_t)g.ML : 0));
+}
+
+size_t heads_smem_bytes(const Geometry& g) {
     return sizeof(uint32_t) * ((size_t)g.words + (keys_in_smem(g.ML) ? 32 * (size_t)key_stride(g) : 0));
 }
 
-size_t heads_smem_bytes(const Geometry& g) { return select_smem_bytes(g); }
-
 cudaError_t configure_select() {
     const int need = (int)(sizeof(uint32_t) * (kSmemKeys / 32 + 32 * ((kSmemKeys / 32) | 1)));
+    // The select kernel also caches P and I rows up to kSmemScores positions.
+    const int need_sel_scores =
+        (int)(sizeof(uint32_t) * (kSmemScores / 32 + 32 * ((kSmemScores / 32) | 1) + 2 * kSmemScores + 64));
+    const int need_sel = need > need_sel_scores ? need : need_sel_scores;
     cudaError_t e = cudaFuncSetAttribute(heads_topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, need);
     if (e == cudaSuccess)
         e = cudaFuncSetAttribute(heads_pool_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kPoolSmemBytes);
     if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, need);
+        e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, need_sel);
     return e;
 }
 
@@ -845,8 +874,8 @@ cudaError_t launch_heads(const Geometry& g, const LayerIO& io, const Scratch& sc
     cudaError_t e = launch_prio(heads_pool_kernel, grid, dim3(kSelectThreads), g.NG > 1 ? (size_t)kPoolSmemBytes : 0, st,
                                 priority, false, g, io, sc, sl);
     if (e == cudaSuccess)
-        e = launch_prio(heads_topk_kernel, grid, dim3(kSelectThreads), heads_smem_bytes(g), st, priority, false, g, io,
-                        sc, sl);
+        e = launch_prio(heads_topk_kernel, grid, dim3(kSelectThreads), heads_smem_bytes(g), st, priority,
+                        /*programmatic=*/true, g, io, sc, sl);
     return e;
 }
 

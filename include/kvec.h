@@ -120,7 +120,10 @@ KVEC_API kvec_status kvec_select_layer(kvec_handle* h, int batch,
  * holds num_layers device pointers with the per-layer meaning above.  The
  * library overlaps the score work of later layers with the coverage-dependent
  * selection of earlier ones; the results are identical to the layer-by-layer
- * calls.  num_layers must not exceed max_layers. */
+ * calls.  num_layers must not exceed max_layers.  A sequence whose state would
+ * pass 255 layers (layers_done + num_layers > 255) keeps its state unchanged and
+ * gets no selection for any layer of the call; kvec_sync_status then returns
+ * KVEC_ERR_INVALID_ARG. */
 KVEC_API kvec_status kvec_select_layers(kvec_handle* h, int num_layers, int batch,
                                const int32_t* cu_seqlens_host, const int32_t* cu_seqlens_dev,
                                const void* const* q_obs, const void* const* k, const void* const* v,

@@ -216,23 +216,29 @@ Geometry make_geometry(const kvec_handle* h, int batch, int budget, int tiles, i
     G.state_stride = h->state_stride;
     G.state_n_off = h->n_off;
     G.state_union_off = h->union_off;
+    G.nlen = (int)round_up((size_t)p.max_seqlen, 16);
     return G;
 }
 
 // One layer, every kernel on one stream with one slot (used without a handle).
 kvec_status run_layer_sequential(kvec_handle* h, const Geometry& G, const LayerIO& io, cudaStream_t st) {
+    // The union ring starts empty (the select kernel reads entry 2 as the previous union).
+    cudaError_t me = cudaMemsetAsync(h->sc.ubits, 0, 3 * (size_t)G.batch * G.words * sizeof(uint32_t), st);
+    if (me != cudaSuccess) return cuda_fail(me, "cudaMemsetAsync(union ring)");
     ScorePlan plan;
-    cudaError_t se = plan_score(G, io, h->sc, h->num_sms, nullptr, &plan);
+    cudaError_t se = plan_score(G, io, h->sc, h->num_sms, &plan);
     if (se != cudaSuccess) return cuda_fail(se, "score kernel tensor maps");
-    se = launch_score(plan, st);
+    se = launch_score(plan, st, false);
     if (se != cudaSuccess) return cuda_fail(se, "score kernel launch");
-    se = launch_window(plan, G, io, h->sc, h->slots[0], st);
+    se = launch_window(plan, G, io, h->sc, h->slots[0], st, false);
     if (se != cudaSuccess) return cuda_fail(se, "window kernel launch");
     se = launch_heads(G, io, h->sc, h->slots[0], st, h->prio_hi);
     if (se != cudaSuccess) return cuda_fail(se, "heads kernel launch");
-    se = launch_select(G, io, h->sc, h->slots[0], st, h->prio_hi);
+    se = launch_select(G, io, h->sc, h->slots[0], st, h->prio_hi, 0, 1);
     if (se != cudaSuccess) return cuda_fail(se, "select kernel launch");
     launch_gather(G, io, st);
+    se = launch_finalize(G, io, h->sc, st, h->prio_hi, 1);
+    if (se != cudaSuccess) return cuda_fail(se, "finalize kernel launch");
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_fail(e, "kernel launch");
     return KVEC_OK;
@@ -252,20 +258,22 @@ kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* io
     KV_CHECK(cudaEventRecord(h->ev_fork, origin));
     for (cudaStream_t st : {h->s_score, h->s_win, h->s_heads, h->s_heads2, h->s_chain, h->s_gather})
         KV_CHECK(cudaStreamWaitEvent(st, h->ev_fork, 0));
+    // The layers' unions start empty (ring of three, see launch_select).
+    KV_CHECK(cudaMemsetAsync(h->sc.ubits, 0, 3 * (size_t)G.batch * G.words * sizeof(uint32_t), h->s_chain));
     for (int l = 0; l < n; ++l) {
         const Slot& sl = h->slots[l % kSlots];
         const Scratch& sc = h->score_buf[l & 1];
         const LayerIO& io = ios[l];
         if (l >= 2) KV_CHECK(cudaStreamWaitEvent(h->s_score, h->ev_win[l - 2], 0));
         ScorePlan plan;
-        cudaError_t se = plan_score(G, io, sc, h->num_sms, l + 1 < n ? ios[l + 1].k : nullptr, &plan);
+        cudaError_t se = plan_score(G, io, sc, h->num_sms, &plan);
         if (se != cudaSuccess) return cuda_fail(se, "score kernel tensor maps");
-        timed_launch(h, 0, h->s_score, [&] { se = launch_score(plan, h->s_score); });
+        timed_launch(h, 0, h->s_score, [&] { se = launch_score(plan, h->s_score, true); });
         if (se != cudaSuccess) return cuda_fail(se, "score kernel launch");
         KV_CHECK(cudaEventRecord(h->ev_score[l], h->s_score));
         KV_CHECK(cudaStreamWaitEvent(h->s_win, h->ev_score[l], 0));
         if (l >= kSlots) KV_CHECK(cudaStreamWaitEvent(h->s_win, h->ev_sel[l - kSlots], 0));
-        timed_launch(h, 1, h->s_win, [&] { se = launch_window(plan, G, io, sc, sl, h->s_win); });
+        timed_launch(h, 1, h->s_win, [&] { se = launch_window(plan, G, io, sc, sl, h->s_win, true); });
         if (se != cudaSuccess) return cuda_fail(se, "window kernel launch");
         KV_CHECK(cudaEventRecord(h->ev_win[l], h->s_win));
         cudaStream_t s_h = (l & 1) ? h->s_heads2 : h->s_heads;
@@ -274,11 +282,16 @@ kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* io
         if (se != cudaSuccess) return cuda_fail(se, "heads kernel launch");
         KV_CHECK(cudaEventRecord(h->ev_heads[l], s_h));
         KV_CHECK(cudaStreamWaitEvent(h->s_chain, h->ev_heads[l], 0));
-        timed_launch(h, 3, h->s_chain, [&] { se = launch_select(G, io, sc, sl, h->s_chain, h->prio_hi); });
+        timed_launch(h, 3, h->s_chain, [&] { se = launch_select(G, io, sc, sl, h->s_chain, h->prio_hi, l, n); });
         if (se != cudaSuccess) return cuda_fail(se, "select kernel launch");
         KV_CHECK(cudaEventRecord(h->ev_sel[l], h->s_chain));
         KV_CHECK(cudaStreamWaitEvent(h->s_gather, h->ev_sel[l], 0));
         timed_launch(h, 4, h->s_gather, [&] { launch_gather(G, io, h->s_gather); });
+    }
+    // The last layer's union goes into the state.
+    {
+        cudaError_t se = launch_finalize(G, ios[n - 1], h->score_buf[(n - 1) & 1], h->s_chain, h->prio_hi, n);
+        if (se != cudaSuccess) return cuda_fail(se, "finalize kernel launch");
     }
     KV_CHECK(cudaGetLastError());
     KV_CHECK(cudaEventRecord(h->ev_join[0], h->s_score));
@@ -286,7 +299,8 @@ kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* io
     KV_CHECK(cudaEventRecord(h->ev_join[2], h->s_heads));
     KV_CHECK(cudaEventRecord(h->ev_join[3], h->s_gather));
     KV_CHECK(cudaEventRecord(h->ev_join[4], h->s_heads2));
-    KV_CHECK(cudaStreamWaitEvent(origin, h->ev_sel[n - 1], 0));
+    KV_CHECK(cudaEventRecord(h->ev_fork, h->s_chain));   // reused: the end of the chain stream
+    KV_CHECK(cudaStreamWaitEvent(origin, h->ev_fork, 0));
     for (cudaEvent_t e : h->ev_join) KV_CHECK(cudaStreamWaitEvent(origin, e, 0));
     h->last_slot = (n - 1) % kSlots;
     h->last_parity = (n - 1) & 1;
@@ -369,15 +383,15 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
     std::vector<Part> parts = {
 
         {(void**)&h->sc.keys, MB * Hkv * ML * sizeof(uint32_t)},
-        {(void**)&h->sc.ubits, MB * W * sizeof(uint32_t)},
-        {(void**)&h->sc.ucount, MB * sizeof(unsigned)},
+        {(void**)&h->sc.ubits, 3 * MB * W * sizeof(uint32_t)},
+        {(void**)&h->sc.nbuf, MB * round_up((size_t)p.max_seqlen, 16)},
         {(void**)&h->sc.err, sizeof(int)},
         {(void**)&h->sc.keys_sel, MB * Hkv * ML * sizeof(uint32_t)},
     };
     for (int k = 0; k < 2; ++k) {
         Scratch& b = h->score_buf[k];
         std::vector<Part> sp = {
-            {(void**)&b.segpart, max_tiles * Hkv * 2 * R * sizeof(float2)},
+            {(void**)&b.segpart, max_tiles * Hkv * R * sizeof(float2)},
             {(void**)&b.shcount, MB * Hkv * sizeof(unsigned)},
             {(void**)&b.rowstat, MB * Hkv * R * sizeof(float2)},
         };
@@ -414,7 +428,7 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
         b.keys = h->sc.keys;
         b.keys_sel = h->sc.keys_sel;
         b.ubits = h->sc.ubits;
-        b.ucount = h->sc.ucount;
+        b.nbuf = h->sc.nbuf;
         b.err = h->sc.err;
     }
     Geometry G = make_geometry(h, 1, p.window, 1, 1, p.window);
@@ -423,8 +437,11 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
     if (e == cudaSuccess) e = configure_window(G);
     if (e == cudaSuccess) e = configure_select();
     if (e == cudaSuccess) e = cudaDeviceGetStreamPriorityRange(&h->prio_lo, &h->prio_hi);
-    for (cudaStream_t* st : {&h->s_score, &h->s_win, &h->s_gather, &h->s_cap})
+    for (cudaStream_t* st : {&h->s_score, &h->s_gather, &h->s_cap})
         if (e == cudaSuccess) e = cudaStreamCreateWithPriority(st, cudaStreamNonBlocking, h->prio_lo);
+    // A layer's window sums go ahead of the next layer's statistics when both wait for SMs.
+    if (e == cudaSuccess)
+        e = cudaStreamCreateWithPriority(&h->s_win, cudaStreamNonBlocking, h->prio_hi < h->prio_lo ? h->prio_lo - 1 : h->prio_lo);
     for (cudaStream_t* st : {&h->s_heads, &h->s_heads2, &h->s_chain})
         if (e == cudaSuccess) e = cudaStreamCreateWithPriority(st, cudaStreamNonBlocking, h->prio_hi);
     h->ev_score.assign(p.max_layers, nullptr);
@@ -643,11 +660,11 @@ kvec_status kvec_select_layer_noalloc(const kvec_params* params, int batch, cons
     const size_t HGv = Hkv < (size_t)kWinHeadsPerCta ? Hkv : (size_t)kWinHeadsPerCta;
     const size_t NGv = (Hkv + HGv - 1) / HGv;
     Part parts[] = {
-        {(void**)&tmp.sc.ucount, nb * sizeof(unsigned)},      // zeroed every call (first four parts)
-        {(void**)&tmp.sc.err, sizeof(int)},
-        {(void**)&tmp.sc.ubits, nb * W * sizeof(uint32_t)},
+        {(void**)&tmp.sc.err, sizeof(int)},                   // zeroed every call (first two parts)
         {(void**)&tmp.sc.shcount, nb * Hkv * sizeof(unsigned)},
-        {(void**)&tmp.sc.segpart, nt * Hkv * 2 * R * sizeof(float2)},
+        {(void**)&tmp.sc.ubits, 3 * nb * W * sizeof(uint32_t)},
+        {(void**)&tmp.sc.nbuf, nb * round_up((size_t)params->max_seqlen, 16)},
+        {(void**)&tmp.sc.segpart, nt * Hkv * R * sizeof(float2)},
         {(void**)&tmp.slots[0].wpart, nt * NGv * (size_t)params->obs_window * kTileT * sizeof(float)},
         {(void**)&tmp.sc.rowstat, nb * Hkv * R * sizeof(float2)},
         {(void**)&tmp.sc.keys, nb * Hkv * ML * sizeof(uint32_t)},
@@ -666,7 +683,7 @@ kvec_status kvec_select_layer_noalloc(const kvec_params* params, int batch, cons
     size_t need = 0, zero_bytes = 0;
     for (size_t i = 0; i < sizeof(parts) / sizeof(parts[0]); ++i) {
         need += round_up(parts[i].bytes, 256);
-        if (i == 3) zero_bytes = need;
+        if (i == 1) zero_bytes = need;
     }
     if (need > kNoallocScratchBytes)
         return fail(KVEC_ERR_INVALID_ARG,
@@ -691,7 +708,7 @@ kvec_status kvec_select_layer_noalloc(const kvec_params* params, int batch, cons
         off += round_up(pt.bytes, 256);
     }
     cudaStream_t st = (cudaStream_t)stream;
-    // The array keeps the previous call's contents: the counters and union bits must start at zero.
+    // The array keeps the previous call's contents: the error word and tile counters must start at zero.
     e = cudaMemsetAsync(base, 0, zero_bytes, st);
     if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync(scratch)");
     LayerIO io{};
@@ -735,7 +752,7 @@ kvec_status kvec_sync_status(kvec_handle* h) {
     if (e != cudaSuccess) return cuda_fail(e, "reading the device error word");
     if (err) {
         cudaMemset(h->sc.err, 0, sizeof(int));
-        if (err == 2) return fail(KVEC_ERR_INVALID_ARG, "a coverage state already counted 255 layers");
+        if (err == 2) return fail(KVEC_ERR_INVALID_ARG, "a call would have taken a coverage state past 255 layers (that state was left unchanged)");
         return fail(KVEC_ERR_DEVICE_TIMEOUT, "a bounded device wait gave up (code %d)", err);
     }
     return KVEC_OK;

@@ -32,6 +32,7 @@ struct Geometry {
     const int* cu_host;  // host copy of cu_seqlens (host-side planning only; not for device code)
     size_t state_stride;
     size_t state_n_off, state_union_off;
+    int nlen;          // bytes of one sequence's n_t array (round_up(max_seqlen, 16))
 };
 
 // Device workspace owned by the handle (one slot of per-layer score arrays).
@@ -50,13 +51,13 @@ struct Slot {
 };
 
 struct Scratch {
-    float2* segpart;      // [total_tiles * Hkv][2][R] per-CTA segment (max, sum) per column half, keyed by first item
+    float2* segpart;      // [total_tiles * Hkv][R] per-CTA segment (max, sum), keyed by the segment's first item
     unsigned* shcount;    // [max_batch][Hkv]       tiles finished per (sequence, KV head)
     float2* rowstat;      // [max_batch][Hkv][R]    (row max in log2 units, softmax denominator)
     uint32_t* keys;       // [max_batch][Hkv][ML]   radix-select keys of the heads kernel
     uint32_t* keys_sel;   // [max_batch][Hkv][ML]   radix-select keys of the select kernel
-    uint32_t* ubits;      // [max_batch][words]     union of this layer's selections
-    unsigned* ucount;     // [max_batch]            heads finished (last-CTA fold)
+    uint32_t* ubits;      // [3][max_batch][words]  union of a layer's selections, ring over layers
+    uint8_t* nbuf;        // [max_batch][nlen]      second copy of n_t (the coverage counts alternate)
     int* err;             // device error word
 };
 
@@ -100,15 +101,16 @@ __device__ __forceinline__ int tiles_of(int L) { return (L + kTileT - 1) / kTile
 struct ScorePlan {
     CUtensorMap kmap, qmap;
     alignas(16) unsigned char args[512];
-    int grid, threads;
+    int grid, threads, mb;   // mb: 128-row M-blocks per KV head
     size_t smem;
 };
-// next_k: the next layer's K (same shape), prefetched into L2 by this launch; may be null.
-cudaError_t plan_score(const Geometry& g, const LayerIO& io, const Scratch& sc, int num_sms, const void* next_k,
-                       ScorePlan* plan);
-cudaError_t launch_score(const ScorePlan& plan, cudaStream_t st);
+cudaError_t plan_score(const Geometry& g, const LayerIO& io, const Scratch& sc, int num_sms, ScorePlan* plan);
+// after_own_launch: the stream's previous kernel is the previous layer's launch
+// of the same kernel (the multi-stream layer pipeline); the launch may then
+// overlap it (programmatic stream serialization), as it reads none of its results.
+cudaError_t launch_score(const ScorePlan& plan, cudaStream_t st, bool after_own_launch);
 cudaError_t launch_window(const ScorePlan& sp, const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl,
-                          cudaStream_t st);
+                          cudaStream_t st, bool after_own_launch);
 // Launches kernel<<<grid, block, smem, st>>> with a scheduling priority (lower
 // numbers first; the range comes from cudaDeviceGetStreamPriorityRange) and,
 // with `programmatic`, as a programmatic dependent of the stream's previous
@@ -134,8 +136,14 @@ cudaError_t launch_prio(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t 
 
 cudaError_t launch_heads(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st,
                          int priority);
+// lcall: the layer's index within a call of ncall layers (0 for the first).
+// The coverage counts alternate between the state and sc.nbuf and each layer's
+// union goes to ring entry lcall % 3; launch_finalize folds the last union into
+// the state.
 cudaError_t launch_select(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st,
-                          int priority);
+                          int priority, int lcall, int ncall);
+cudaError_t launch_finalize(const Geometry& g, const LayerIO& io, const Scratch& sc, cudaStream_t st, int priority,
+                            int ncall);
 void launch_gather(const Geometry& g, const LayerIO& io, cudaStream_t st);
 
 size_t score_smem_bytes(const Geometry& g);

@@ -9,12 +9,13 @@
 //               a ring of 128-token K tiles, both 128-byte swizzled;
 //   warp 1      one thread issues tcgen05.mma (M = 128 query rows per M-block,
 //               N = 128 tokens, K = 128 = d) into TMEM accumulators;
-//   warps 2..   epilogue, one thread per (query row, half of the tile's
-//               columns): tcgen05.ld of 64 logits, their max and sum of
+//   warps 2..17 epilogue, one thread per (query row, column split of the
+//               tile): tcgen05.ld of its logits, their max and sum of
 //               2^(s - max), merged online into the thread's running
 //               (max, sum) of the CTA's contiguous segment of (s, h).
-// Each CTA writes one (max, sum) partial per segment, row and column half; the
-// last CTA to finish a (s, h) merges them into rowstat[s][h][r] = (m_r, Z_r).
+// At the end of a segment the column splits merge in shared memory and the CTA
+// writes one (max, sum) partial per row; the last CTA to finish a (s, h) merges
+// the partials into rowstat[s][h][r] = (m_r, Z_r).
 // The window kernel recomputes the logits with these statistics.
 #include <cudaTypedefs.h>
 
@@ -31,32 +32,46 @@ constexpr int kKStageBytes = kTileT * kHeadDim * 2;   // 32 KB: two 64-column sw
 constexpr int kKHalfBytes = kTileT * 128;             // 16 KB
 constexpr uint32_t kTmemCols = 512;
 
-struct ItemPos {
-    int s, h, j, gt, ibase, ntiles;  // ibase: first item of (s, h)
-};
+// Position of work item i: sequence s, KV head h, tile j.  Items are ordered
+// (s, h, j); sequence s owns ntiles(s) * Hkv consecutive items.  A CTA walks its
+// items in order, so the walker decodes once and then steps, reading the
+// sequence offsets (device memory) only when the sequence changes.
+struct ItemWalker {
+    const int* cu;
+    int batch, Hkv;
+    int s, h, j, ibase, ntiles;   // ibase: first item of (s, h)
+    int row0, L;                  // cu[s], L_s
 
-// Items are ordered (s, h, j); sequence s owns ntiles(s) * Hkv consecutive items.
-template <class Cu>
-__device__ __forceinline__ ItemPos decode_item(const Cu& cu, int batch, int Hkv, int i) {
-    ItemPos p{};
-    int ibase = 0, tbase = 0;
-    for (int b = 0; b < batch; ++b) {
-        const int nt = tiles_of(cu[b + 1] - cu[b]);
-        if (i < ibase + nt * Hkv) {
-            const int local = i - ibase;
-            p.s = b;
-            p.h = local / nt;
-            p.j = local - p.h * nt;
-            p.gt = tbase + p.j;
-            p.ibase = ibase + p.h * nt;
-            p.ntiles = nt;
-            return p;
-        }
-        ibase += nt * Hkv;
-        tbase += nt;
+    __device__ __forceinline__ void enter_sequence() {
+        row0 = __ldg(&cu[s]);
+        L = __ldg(&cu[s + 1]) - row0;
+        ntiles = tiles_of(L);
     }
-    return p;
-}
+    __device__ __forceinline__ void init(const int* cu_, int batch_, int Hkv_, int i) {
+        cu = cu_;
+        batch = batch_;
+        Hkv = Hkv_;
+        int base = 0;
+        for (s = 0; s < batch; ++s) {
+            enter_sequence();
+            if (i < base + ntiles * Hkv) break;
+            base += ntiles * Hkv;
+        }
+        const int local = i - base;
+        h = local / ntiles;
+        j = local - h * ntiles;
+        ibase = base + h * ntiles;
+    }
+    __device__ __forceinline__ bool last_of_head() const { return j + 1 == ntiles; }
+    __device__ __forceinline__ void next() {
+        if (++j < ntiles) return;
+        j = 0;
+        ibase += ntiles;
+        if (++h < Hkv) return;
+        h = 0;
+        if (++s < batch) enter_sequence();
+    }
+};
 
 // CTA b of G owns items [start(b), start(b+1)) with start(b) = b*q + min(b, r), W = q*G + r.
 __device__ __forceinline__ int range_start(int b, int W, int G) {
@@ -64,22 +79,20 @@ __device__ __forceinline__ int range_start(int b, int W, int G) {
     return b * q + min(b, r);
 }
 
-constexpr int kMaxCuParam = 64;          // sequences whose offsets travel in the kernel parameters
 constexpr int kScoreReserveSms = 8;      // SMs a score launch leaves to the other kernels
 constexpr int kScoreItemsPerCta = 8;     // fewest (sequence, head, tile) items a score CTA takes
 
 struct ScoreArgs {
     Geometry G;
     const int* cu;                 // device cu_seqlens
-    int cuv[kMaxCuParam + 1];      // the same offsets (when batch <= kMaxCuParam)
-    const uint8_t* next_k;         // the next layer's K (L2 prefetch), or null
-    long long kbytes_total;        // bytes of one layer's K
     Scratch sc;
     int W;        // total work items
-    int MB;       // 128-row M-blocks per KV head (1 or 2)
-    int Rpad;     // 128 * MB
     int kst;      // K ring depth
 };
+
+constexpr int kEpiWarps = 16;
+constexpr int kEpiThreads = 32 * kEpiWarps;
+constexpr int kScoreThreads = 64 + kEpiThreads;
 
 struct __align__(8) Barriers {
     uint64_t k_full[kKStages], k_empty[kKStages];
@@ -89,8 +102,7 @@ struct __align__(8) Barriers {
     uint32_t tmem_base;
     volatile int abort_flag;
     volatile int last_flag;
-    volatile int go;
-    float2 xfer[256];          // merged (max, sum) of the second column half, last CTA only
+    float2 xf[512];            // a segment's (max, sum) per column split and row, merged at its end
 };
 
 __device__ __forceinline__ void raise_abort(Barriers* bars, int* err) {
@@ -98,36 +110,41 @@ __device__ __forceinline__ void raise_abort(Barriers* bars, int* err) {
     atomicExch(err, 3);
 }
 
-__global__ void __launch_bounds__(576, 1)
+// MB: 128-row M-blocks per KV head (R <= 128 * MB).  The 16 epilogue warps cover
+// 4 lane quarters x MB M-blocks x CS = 4 / MB column splits of COLS = 32 * MB.
+template <int MB>
+__global__ void __launch_bounds__(kScoreThreads, 1)
     score_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap qmap,
                  const __grid_constant__ ScoreArgs A) {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     // 1024-byte alignment for the swizzled operand tiles.
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    const Geometry& G = A.G;
-    const int MB = A.MB, Rpad = A.Rpad, R = G.R;
+    // Scalars and pointers in registers: values read through a reference to the
+    // parameter block would be re-read after every asm statement that clobbers memory.
+    const Geometry G = A.G;
+    const Scratch sc = A.sc;
+    const int W = A.W, kst = A.kst;
+    const int* const cu_dev = A.cu;
+    constexpr int CS = 4 / MB, COLS = 32 * MB;
+    const int Rpad = 128 * MB, R = G.R;
     uint8_t* sQ = smem;                                   // 2 halves x Rpad rows x 128 B
-    uint8_t* sK = sQ + 2 * Rpad * 128;                    // A.kst x 32 KB
-    Barriers* bars = reinterpret_cast<Barriers*>(sK + A.kst * kKStageBytes);
+    uint8_t* sK = sQ + 2 * Rpad * 128;                    // kst x 32 KB
+    Barriers* bars = reinterpret_cast<Barriers*>(sK + kst * kKStageBytes);
 
-    const bool cu_param = G.batch <= kMaxCuParam;
-    auto cu = [&](int b) { return cu_param ? A.cuv[b] : A.cu[b]; };
-    struct CuView {
-        decltype(cu)& f;
-        __device__ int operator[](int b) const { return f(b); }
-    } cuview{cu};
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int nepi = 8 * MB * 32;                          // epilogue threads: 2 column halves x MB x 4 quads
-    const int NB = 4 / MB;                                 // TMEM accumulator buffers
+    constexpr int NB = 4 / MB;                             // TMEM accumulator buffers
     const int Gc = gridDim.x;
-    const int i0 = range_start(blockIdx.x, A.W, Gc), i1 = range_start(blockIdx.x + 1, A.W, Gc);
+    const int i0 = range_start(blockIdx.x, W, Gc), i1 = range_start(blockIdx.x + 1, W, Gc);
 
     if (warp == 0 && lane == 0) {
         ptx::prefetch_tensormap(&kmap);
         ptx::prefetch_tensormap(&qmap);
+        // The next launch on this stream (the next layer's statistics) reads
+        // nothing this grid writes: let it be scheduled as SMs free up.
+        asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
     }
     if (threadIdx.x == 32) {
-        for (int s = 0; s < A.kst; ++s) {
+        for (int s = 0; s < kst; ++s) {
             ptx::mbar_init(&bars->k_full[s], 1);
             ptx::mbar_init(&bars->k_empty[s], 1);
         }
@@ -135,7 +152,7 @@ __global__ void __launch_bounds__(576, 1)
         ptx::mbar_init(&bars->q_empty, 1);
         for (int b = 0; b < 4; ++b) {
             ptx::mbar_init(&bars->acc_full[b], 1);
-            ptx::mbar_init(&bars->acc_empty[b], 8 * MB);  // one arrival per epilogue warp
+            ptx::mbar_init(&bars->acc_empty[b], kEpiWarps);  // one arrival per epilogue warp
         }
         ptx::mbar_init(&bars->mma_done, 1);
         bars->abort_flag = 0;
@@ -154,14 +171,14 @@ __global__ void __launch_bounds__(576, 1)
         // ------------------------------------------------------------ TMA producer
         if (lane == 0) {
             const uint64_t policy = ptx::policy_evict_normal();   // the window kernel reads K again
-            int prev_sh = -1, qloads = 0;
-            int fills[kKStages] = {0, 0, 0, 0};
-            for (int i = i0, it = 0; i < i1 && !bars->abort_flag; ++i, ++it) {
-                const ItemPos p = decode_item(cuview, G.batch, G.Hkv, i);
+            int prev_sh = -1, qloads = 0, issued = 0;
+            ItemWalker p;
+            p.init(cu_dev, G.batch, G.Hkv, i0);
+            for (int i = i0, it = 0; i < i1 && !bars->abort_flag; ++i, ++it, p.next()) {
                 const int sh = p.s * G.Hkv + p.h;
                 if (sh != prev_sh) {
                     if (qloads > 0 && !ptx::mbar_wait(&bars->q_empty, (qloads - 1) & 1)) {
-                        raise_abort(bars, A.sc.err);
+                        raise_abort(bars, sc.err);
                         break;
                     }
                     ptx::mbar_arrive_expect_tx(&bars->q_full, 2u * R * 128u);
@@ -170,21 +187,24 @@ __global__ void __launch_bounds__(576, 1)
                     ++qloads;
                     prev_sh = sh;
                 }
-                const int st = it % A.kst, n = it / A.kst;
+                const int st = it % kst, n = it / kst;
                 if (n > 0 && !ptx::mbar_wait(&bars->k_empty[st], (n - 1) & 1)) {
-                    raise_abort(bars, A.sc.err);
+                    raise_abort(bars, sc.err);
                     break;
                 }
                 uint8_t* dst = sK + st * kKStageBytes;
-                const int row = cu(p.s) + p.j * kTileT;
+                const int row = p.row0 + p.j * kTileT;
                 ptx::mbar_arrive_expect_tx(&bars->k_full[st], (uint32_t)kKStageBytes);
                 ptx::tma_load_3d(dst, &kmap, &bars->k_full[st], 0, p.h, row, policy);
                 ptx::tma_load_3d(dst + kKHalfBytes, &kmap, &bars->k_full[st], 64, p.h, row, policy);
-                ++fills[st];
+                ++issued;
             }
-            // Drain: every issued copy lands before the CTA may exit.
-            for (int st = 0; st < A.kst; ++st)
-                if (fills[st] > 0) ptx::mbar_wait(&bars->k_full[st], (fills[st] - 1) & 1, 50000000ull);
+            // Drain: every issued copy lands before the CTA may exit (stage st was
+            // filled ceil((issued - st) / kst) times).
+            for (int st = 0; st < kst && st < issued; ++st) {
+                const int fills = (issued - st + kst - 1) / kst;
+                ptx::mbar_wait(&bars->k_full[st], (fills - 1) & 1, 50000000ull);
+            }
             if (qloads > 0) ptx::mbar_wait(&bars->q_full, (qloads - 1) & 1, 50000000ull);
         }
     } else if (warp == 1) {
@@ -193,22 +213,23 @@ __global__ void __launch_bounds__(576, 1)
             const uint32_t idesc = ptx::idesc_bf16_f32(128, kTileT);
             const uint32_t sQa = ptx::smem_u32(sQ), sKa = ptx::smem_u32(sK);
             int prev_sh = -1, qk = 0;
-            for (int i = i0, it = 0; i < i1 && !bars->abort_flag; ++i, ++it) {
-                const ItemPos p = decode_item(cuview, G.batch, G.Hkv, i);
+            ItemWalker p;
+            p.init(cu_dev, G.batch, G.Hkv, i0);
+            for (int i = i0, it = 0; i < i1 && !bars->abort_flag; ++i, ++it, p.next()) {
                 const int sh = p.s * G.Hkv + p.h;
                 if (sh != prev_sh) {
                     if (!ptx::mbar_wait(&bars->q_full, qk & 1)) {
-                        raise_abort(bars, A.sc.err);
+                        raise_abort(bars, sc.err);
                         break;
                     }
                     ++qk;
                     prev_sh = sh;
                 }
-                const int st = it % A.kst, n = it / A.kst;
+                const int st = it % kst, n = it / kst;
                 const int buf = it % NB, nb = it / NB;
                 if (!ptx::mbar_wait(&bars->k_full[st], n & 1) ||
                     (nb > 0 && !ptx::mbar_wait(&bars->acc_empty[buf], (nb - 1) & 1))) {
-                    raise_abort(bars, A.sc.err);
+                    raise_abort(bars, sc.err);
                     break;
                 }
                 ptx::tc_fence_after();
@@ -225,22 +246,21 @@ __global__ void __launch_bounds__(576, 1)
                 }
                 ptx::mma_commit(&bars->k_empty[st]);
                 ptx::mma_commit(&bars->acc_full[buf]);
-                bool q_done = i + 1 >= i1;
-                if (!q_done) {
-                    const ItemPos nx = decode_item(cuview, G.batch, G.Hkv, i + 1);
-                    q_done = nx.s * G.Hkv + nx.h != sh;
-                }
-                if (q_done) ptx::mma_commit(&bars->q_empty);
+                if (i + 1 >= i1 || p.last_of_head()) ptx::mma_commit(&bars->q_empty);
             }
             ptx::mma_commit(&bars->mma_done);
         }
-    } else if (warp < 2 + 8 * MB) {
+    } else {
         // ------------------------------------------------------------ epilogue
-        const int epi = threadIdx.x - 64;                   // 0 .. nepi-1
+        // Warp ew = warp - 2 reads TMEM lanes 32*(warp % 4) .. +31 (the lane
+        // quarter its warp id allows) of M-block m, columns [COLS*split, +COLS).
+        // Each warp waits for the accumulators itself; the warps meet only when a
+        // segment ends.
+        const int epi = threadIdx.x - 64;                   // 0 .. kEpiThreads-1
         const int ew = warp - 2;
-        const int m = (ew >> 2) % MB;                       // M-block of this warp
-        const int half = (ew >> 2) / MB;                    // column half: tokens [64*half, 64*half + 64)
-        const int quad = warp & 3;                          // TMEM lanes 32*quad .. +31
+        const int m = (ew >> 2) % MB;
+        const int split = (ew >> 2) / MB;
+        const int quad = warp & 3;
         const int row = m * 128 + quad * 32 + lane;
         const bool vrow = row < R;
         const int q = vrow ? row / G.g : 0;
@@ -249,23 +269,40 @@ __global__ void __launch_bounds__(576, 1)
         float seg_m = -INFINITY, seg_z = 0.f;
         int cur_sh = -1, seg_first = 0, seg_n = 0, seg_s = 0, seg_h = 0, seg_ibase = 0, seg_nt = 0;
 
+        auto merge = [](float& M, float& Z, float2 o) {
+            if (o.x == -INFINITY) return;
+            if (o.x > M) {
+                Z = Z * ptx::ex2(M - o.x) + o.y;
+                M = o.x;
+            } else {
+                Z += o.y * ptx::ex2(o.x - M);
+            }
+        };
+        // Every epilogue thread calls this at the same segment boundaries (aborted
+        // warps included), so the named barriers always complete.
         auto flush_segment = [&]() {
-            if (vrow) A.sc.segpart[((size_t)seg_first * 2 + half) * R + row] = make_float2(seg_m, seg_z);
-            ptx::named_bar_sync(1, nepi);
+            bars->xf[split * Rpad + row] = make_float2(seg_m, seg_z);
+            ptx::named_bar_sync(1, kEpiThreads);
+            if (split == 0) {
+                float M = seg_m, Z = seg_z;
+#pragma unroll
+                for (int c = 1; c < CS; ++c) merge(M, Z, bars->xf[c * Rpad + row]);
+                if (vrow) sc.segpart[(size_t)seg_first * R + row] = make_float2(M, Z);
+            }
+            ptx::named_bar_sync(1, kEpiThreads);
             if (issuer) {
                 // The barrier orders the CTA's writes before this thread's fence (cumulativity).
                 __threadfence();
-                const unsigned old = atomicAdd(&A.sc.shcount[seg_s * G.Hkv + seg_h], (unsigned)seg_n);
+                const unsigned old = atomicAdd(&sc.shcount[seg_s * G.Hkv + seg_h], (unsigned)seg_n);
                 __threadfence();
                 bars->last_flag = old + (unsigned)seg_n == (unsigned)seg_nt;
             }
-            ptx::named_bar_sync(1, nepi);
-            if (bars->last_flag) {
-                // Merge the partials of (s, h): each half its own column half, every
-                // segment start (the first item, then each CTA range start after it)
-                // loaded in independent batches; then the halves combine.
+            ptx::named_bar_sync(1, kEpiThreads);
+            if (bars->last_flag && split == 0) {
+                // Merge the partials of (s, h): the first item, then each CTA range
+                // start after it, loaded in independent batches.
                 float M = -INFINITY, Z = 0.f;
-                const int qW = A.W / Gc, rW = A.W % Gc;
+                const int qW = W / Gc, rW = W % Gc;
                 const int iend = seg_ibase + seg_nt;
                 auto cta_of = [&](int i) { return i < rW * (qW + 1) ? i / (qW + 1) : rW + (i - rW * (qW + 1)) / qW; };
                 int b = cta_of(seg_ibase) + 1;
@@ -276,42 +313,22 @@ __global__ void __launch_bounds__(576, 1)
                     for (int k = 0; k < 16; ++k) {
                         pz[k] = make_float2(-INFINITY, 0.f);
                         if (next < iend) {
-                            if (vrow) pz[k] = __ldcg(&A.sc.segpart[((size_t)next * 2 + half) * R + row]);
+                            if (vrow) pz[k] = __ldcg(&sc.segpart[(size_t)next * R + row]);
                             next = b * qW + min(b, rW);
                             ++b;
                         }
                     }
 #pragma unroll
-                    for (int k = 0; k < 16; ++k) {
-                        if (pz[k].x == -INFINITY) continue;
-                        if (pz[k].x > M) {
-                            Z = Z * ptx::ex2(M - pz[k].x) + pz[k].y;
-                            M = pz[k].x;
-                        } else {
-                            Z += pz[k].y * ptx::ex2(pz[k].x - M);
-                        }
-                    }
+                    for (int k = 0; k < 16; ++k) merge(M, Z, pz[k]);
                 }
-                if (half == 1) bars->xfer[row] = make_float2(M, Z);
-                ptx::named_bar_sync(1, nepi);
-                if (half == 0) {
-                    const float2 o = bars->xfer[row];
-                    if (o.x != -INFINITY) {
-                        if (o.x > M) {
-                            Z = Z * ptx::ex2(M - o.x) + o.y;
-                            M = o.x;
-                        } else {
-                            Z += o.y * ptx::ex2(o.x - M);
-                        }
-                    }
-                    if (vrow) A.sc.rowstat[((size_t)seg_s * G.Hkv + seg_h) * R + row] = make_float2(M, Z);
-                }
-                if (issuer) A.sc.shcount[seg_s * G.Hkv + seg_h] = 0u;
+                if (vrow) sc.rowstat[((size_t)seg_s * G.Hkv + seg_h) * R + row] = make_float2(M, Z);
+                if (issuer) sc.shcount[seg_s * G.Hkv + seg_h] = 0u;
             }
         };
 
-        for (int i = i0, it = 0; i < i1; ++i, ++it) {
-            const ItemPos p = decode_item(cuview, G.batch, G.Hkv, i);
+        ItemWalker p;
+        p.init(cu_dev, G.batch, G.Hkv, i0);
+        for (int i = i0, it = 0; i < i1; ++i, ++it, p.next()) {
             const int sh = p.s * G.Hkv + p.h;
             if (sh != cur_sh) {
                 if (cur_sh >= 0) flush_segment();
@@ -325,68 +342,57 @@ __global__ void __launch_bounds__(576, 1)
                 seg_ibase = p.ibase;
                 seg_nt = p.ntiles;
             }
+            ++seg_n;
+            if (aborted) continue;   // keep walking the items for the segment barriers
             const int buf = it % NB, nb = it / NB;
-            // One thread waits for the accumulator and publishes the outcome; every
-            // epilogue thread takes the same branch.
-            if (issuer) {
-                const bool ok = !bars->abort_flag && ptx::mbar_wait(&bars->acc_full[buf], nb & 1);
-                if (!ok) raise_abort(bars, A.sc.err);
-                bars->go = ok ? 1 : 0;
+            int ok = 1;
+            if (lane == 0) {
+                ok = !bars->abort_flag && ptx::mbar_wait(&bars->acc_full[buf], nb & 1);
+                if (!ok) raise_abort(bars, sc.err);
             }
-            ptx::named_bar_sync(1, nepi);
-            if (!bars->go) {
+            ok = __shfl_sync(0xffffffffu, ok, 0);
+            if (!ok) {
                 aborted = true;
-                break;
+                continue;
             }
             ptx::tc_fence_after();
             const uint32_t taddr = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(buf * 128 * MB + m * 128);
-            const int L = cu(p.s + 1) - cu(p.s);
+            const int L = p.L;
             const int t0 = p.j * kTileT;
             const int last = vrow ? min(L - 1, L - G.w + q) : -1;   // causal on the window part
             const int nvalid = max(0, min(kTileT, last - t0 + 1));
-            // This warp's 64 columns of the accumulator.
-            const int c0 = half * 64;
-            float v[64];
-            ptx::tmem_ld32(taddr + c0, v);
-            ptx::tmem_ld32(taddr + c0 + 32, v + 32);
+            const int c0 = split * COLS;
+            float v[COLS];
+#pragma unroll
+            for (int c = 0; c < COLS; c += 32) ptx::tmem_ld32(taddr + c0 + c, v + c);
             ptx::tmem_wait_ld();
             ptx::tc_fence_before();
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&bars->acc_empty[buf]);
             const int lim = nvalid - c0;
-            if (lim <= 0) {
-                ++seg_n;
-                continue;
-            }
+            if (lim <= 0) continue;
             float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-            if (lim >= 64) {
+            if (lim >= COLS) {
 #pragma unroll
-                for (int c = 0; c < 64; ++c) m4[c & 3] = fmaxf(m4[c & 3], v[c]);
+                for (int c = 0; c < COLS; ++c) m4[c & 3] = fmaxf(m4[c & 3], v[c]);
             } else {
 #pragma unroll
-                for (int c = 0; c < 64; ++c)
+                for (int c = 0; c < COLS; ++c)
                     if (c < lim) m4[c & 3] = fmaxf(m4[c & 3], v[c]);
             }
             const float mu = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * G.sl2;
             float z4[4] = {0.f, 0.f, 0.f, 0.f};
-            if (lim >= 64) {
+            if (lim >= COLS) {
 #pragma unroll
-                for (int c = 0; c < 64; ++c) z4[c & 3] += ptx::ex2(fmaf(v[c], G.sl2, -mu));
+                for (int c = 0; c < COLS; ++c) z4[c & 3] += ptx::ex2(fmaf(v[c], G.sl2, -mu));
             } else {
 #pragma unroll
-                for (int c = 0; c < 64; ++c)
+                for (int c = 0; c < COLS; ++c)
                     if (c < lim) z4[c & 3] += ptx::ex2(fmaf(v[c], G.sl2, -mu));
             }
-            const float z = (z4[0] + z4[1]) + (z4[2] + z4[3]);
-            if (mu > seg_m) {
-                seg_z = seg_z * ptx::ex2(seg_m - mu) + z;
-                seg_m = mu;
-            } else {
-                seg_z += z * ptx::ex2(mu - seg_m);
-            }
-            ++seg_n;
+            merge(seg_m, seg_z, make_float2(mu, (z4[0] + z4[1]) + (z4[2] + z4[3])));
         }
-        if (cur_sh >= 0 && !aborted) flush_segment();
+        if (cur_sh >= 0) flush_segment();
     }
 
     // ---------------------------------------------------------------- teardown
@@ -437,11 +443,12 @@ cudaError_t configure_score(const Geometry& g) {
         gr.R = R;
         if (smem_bytes_for(gr) > need) need = smem_bytes_for(gr);
     }
-    return cudaFuncSetAttribute(score_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)need);
+    cudaError_t e = cudaFuncSetAttribute(score_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)need);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(score_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)need);
+    return e;
 }
 
-cudaError_t plan_score(const Geometry& g, const LayerIO& io, const Scratch& sc, int num_sms, const void* next_k,
-                       ScorePlan* plan) {
+cudaError_t plan_score(const Geometry& g, const LayerIO& io, const Scratch& sc, int num_sms, ScorePlan* plan) {
     PFN_cuTensorMapEncodeTiled_v12000 enc = encode_fn();
     if (!enc) return cudaErrorNotSupported;
     CUtensorMap& kmap = plan->kmap;
@@ -472,13 +479,8 @@ cudaError_t plan_score(const Geometry& g, const LayerIO& io, const Scratch& sc, 
     a = ScoreArgs{};
     a.G = g;
     a.cu = io.cu;
-    for (int b = 0; b <= g.batch && b <= kMaxCuParam; ++b) a.cuv[b] = g.cu_host ? g.cu_host[b] : 0;
-    a.next_k = reinterpret_cast<const uint8_t*>(next_k);
-    a.kbytes_total = (long long)g.total_tokens * g.Hkv * kHeadDim * 2;
     a.sc = sc;
     a.W = g.total_tiles * g.Hkv;
-    a.MB = mblocks(g);
-    a.Rpad = 128 * a.MB;
     a.kst = kstages_for(g);
     // At least kScoreItemsPerCta items per CTA (the CTA's set-up and merge are paid
     // once and its K stream overlaps the epilogue), on at most all but
@@ -488,15 +490,29 @@ cudaError_t plan_score(const Geometry& g, const LayerIO& io, const Scratch& sc, 
     int per_cta = (a.W + usable - 1) / usable;
     if (per_cta < kScoreItemsPerCta) per_cta = kScoreItemsPerCta;
     plan->grid = (a.W + per_cta - 1) / per_cta;
-    plan->threads = 32 * (2 + 8 * a.MB);
+    plan->threads = kScoreThreads;
+    plan->mb = mblocks(g);
     plan->smem = smem_bytes_for(g);
     return cudaSuccess;
 }
 
-cudaError_t launch_score(const ScorePlan& plan, cudaStream_t st) {
-    score_kernel<<<plan.grid, plan.threads, plan.smem, st>>>(plan.kmap, plan.qmap,
-                                                              *reinterpret_cast<const ScoreArgs*>(plan.args));
-    return cudaGetLastError();
+cudaError_t launch_score(const ScorePlan& plan, cudaStream_t st, bool after_own_launch) {
+    const ScoreArgs& a = *reinterpret_cast<const ScoreArgs*>(plan.args);
+    // after_own_launch: the previous kernel on the stream is the previous
+    // layer's launch, whose results this grid does not read; the launch is then
+    // its programmatic dependent and never executes griddepcontrol.wait.
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(plan.grid);
+    cfg.blockDim = dim3(plan.threads);
+    cfg.dynamicSmemBytes = plan.smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = after_own_launch ? 1 : 0;
+    if (plan.mb == 2) return cudaLaunchKernelEx(&cfg, score_kernel<2>, plan.kmap, plan.qmap, a);
+    return cudaLaunchKernelEx(&cfg, score_kernel<1>, plan.kmap, plan.qmap, a);
 }
 
 }  // namespace kvec

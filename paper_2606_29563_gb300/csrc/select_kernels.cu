@@ -26,11 +26,14 @@ __host__ __device__ inline int key_stride(const Geometry& g) { return keys_in_sm
 __device__ __forceinline__ int key_index(int t, int kw) { return (t & 31) * kw + (t >> 5); }
 
 constexpr int kPoolSmemBytes = 96 * 1024;     // raw-I chunk of the heads pooling kernel
-constexpr int kTopkWarps = 8;                  // warps that run the radix select
+constexpr int kTopkWarps = 16;                 // warps that run the radix select
 constexpr int kTopkThreads = 32 * kTopkWarps;
-constexpr int kTopkSeg = 1024;                 // positions per warp segment (32 per lane)
+constexpr int kTopkKPL = 16;                   // positions per lane in a warp segment (half a bits word)
+constexpr int kTopkSeg = 32 * kTopkKPL;        // positions per warp segment
 constexpr int kTopkBarrier = 1;                // named barrier of the select warps
-constexpr int kTopkCap = 1792;                 // keys a compacted candidate list holds (7 per thread)
+constexpr int kTopkCap = 2048;                 // keys a compacted candidate list holds (4 per thread)
+static_assert(kTopkKPL == 16, "two lanes share a bits word");
+static_assert(kTopkCap % kTopkThreads == 0, "the compacted list is split evenly over the select threads");
 constexpr int kTopkFew = 32;                   // a threshold bucket this small is ranked directly
 
 struct TopkShared {
@@ -117,9 +120,9 @@ __device__ __forceinline__ int warp_digit_counts(const uint32_t* pair, int lane)
 // the caller guarantees k <= #eligible.
 //
 // MSB radix select run by kTopkWarps warps.  Warp w owns a contiguous run of
-// 1024-position segments; in a segment lane l owns the 32 positions of bits
-// word 32 s + l, which stay in registers when one segment covers the warp's
-// share.  A first reduction of OR and AND over the eligible keys fixes the bits
+// 512-position segments; in a segment lane l owns the 16 positions [16 l, 16 l
+// + 16) (half of a bits word), which stay in registers when one segment covers
+// the warp's share.  A first reduction of OR and AND over the eligible keys fixes the bits
 // they all share; each pass then resolves the next (up to) 4 bits that differ:
 // threads count digits in registers, warps add the counts with the hardware
 // warp reduction, and after one barrier every warp scans the 16 bucket totals
@@ -137,33 +140,28 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
         const int nseg = (n + kTopkSeg - 1) / kTopkSeg;
         const int spw = (nseg + kTopkWarps - 1) / kTopkWarps;   // segments per warp
         const int seg0 = min(warp * spw, nseg), seg1 = min(seg0 + spw, nseg);
-        auto fetch = [&](int sg, uint32_t* v) {
-            const int wd = sg * 32 + lane;
-#pragma unroll
-            for (int j = 0; j < 32; ++j) v[j] = (wd < nwords && wd * 32 + j < n) ? keys[j * kw + wd] : 0u;
+        // Key j of this lane's positions in segment sg (0 past the row).  With one
+        // segment per warp (kCached) a lane's keys stay in registers.
+        auto fetch_key = [&](int sg, int j) -> uint32_t {
+            const int t = sg * kTopkSeg + lane * kTopkKPL + j;
+            return t < n ? keys[key_index(t, kw)] : 0u;
         };
-        // With one segment per warp (kCached) a lane's 32 keys stay in registers.
-        uint32_t ureg[kCached ? 32 : 1];
-        if (kCached) fetch(seg0 < seg1 ? seg0 : nseg, ureg);
-        auto load_seg = [&](int sg, uint32_t* v) {
-            if (kCached) {
+        uint32_t ureg[kCached ? kTopkKPL : 1];
+        if (kCached) {
 #pragma unroll
-                for (int j = 0; j < 32; ++j) v[j] = ureg[kCached ? j : 0];
-            } else {
-                fetch(sg, v);
-            }
-        };
+            for (int j = 0; j < kTopkKPL; ++j) ureg[kCached ? j : 0] = fetch_key(seg0 < seg1 ? seg0 : nseg, j);
+        }
+        auto key_at = [&](int sg, int j) -> uint32_t { return kCached ? ureg[kCached ? j : 0] : fetch_key(sg, j); };
 
         // Bits shared by every eligible key.
         {
             uint32_t kor = 0u, kand = 0xffffffffu;
             for (int sg = seg0; sg < seg1; ++sg) {
-                uint32_t v[32];
-                load_seg(sg, v);
 #pragma unroll
-                for (int j = 0; j < 32; ++j) {
-                    kor |= v[j];
-                    kand &= v[j] != 0u ? v[j] : 0xffffffffu;
+                for (int j = 0; j < kTopkKPL; ++j) {
+                    const uint32_t v = key_at(sg, j);
+                    kor |= v;
+                    kand &= v != 0u ? v : 0xffffffffu;
                 }
             }
             kor = __reduce_or_sync(0xffffffffu, kor);
@@ -210,21 +208,20 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
             if (mlist < 0) {
                 uint32_t pair[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
                 for (int sg = seg0; sg < seg1; ++sg) {
-                    uint32_t v[32];
-                    load_seg(sg, v);
                     DigitBytes db;
 #pragma unroll
-                    for (int j0 = 0; j0 < 32; j0 += 15) {
+                    for (int j0 = 0; j0 < kTopkKPL; j0 += 15) {
                         unsigned long long nib = 0ull;
 #pragma unroll
-                        for (int j = j0; j < j0 + 15 && j < 32; ++j) nib += digit_nibble(v[j], mask, prefix, lo, wmask);
+                        for (int j = j0; j < j0 + 15 && j < kTopkKPL; ++j)
+                            nib += digit_nibble(key_at(sg, j), mask, prefix, lo, wmask);
                         db.add(nib);
                     }
                     db.to_pairs(pair);
                 }
                 mine = warp_digit_counts(pair, lane);
             } else {
-                // At most 7 list entries per thread: a warp's count of a digit fits a byte.
+                // At most 4 list entries per thread: a warp's count of a digit fits a byte.
                 unsigned long long nib = 0ull;
 #pragma unroll
                 for (int r = 0; r < kTopkCap / kTopkThreads; ++r) {
@@ -280,11 +277,12 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
                 int off = 0;
                 for (int x = 0; x < warp; ++x) off += sm.wcnt[buf][x][D];
                 for (int sg = seg0; sg < seg1; ++sg) {
-                    uint32_t v[32];
-                    load_seg(sg, v);
                     int mc = 0;
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) mc += (v[j] != 0u && (v[j] & mask) == prefix) ? 1 : 0;
+                    for (int j = 0; j < kTopkKPL; ++j) {
+                        const uint32_t v = key_at(sg, j);
+                        mc += (v != 0u && (v & mask) == prefix) ? 1 : 0;
+                    }
                     int incl = mc;
 #pragma unroll
                     for (int o = 1; o < 32; o <<= 1) {
@@ -292,12 +290,13 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
                         if (lane >= o) incl += y;
                     }
                     int at = off + incl - mc;
-                    const int pos0 = (sg * 32 + lane) * 32;
+                    const int pos0 = sg * kTopkSeg + lane * kTopkKPL;
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) {
-                        const bool m = v[j] != 0u && (v[j] & mask) == prefix;
+                    for (int j = 0; j < kTopkKPL; ++j) {
+                        const uint32_t v = key_at(sg, j);
+                        const bool m = v != 0u && (v & mask) == prefix;
                         if (m && at < kTopkCap) {
-                            sm.ckey[at] = v[j];
+                            sm.ckey[at] = v;
                             sm.cpos[at] = pos0 + j;
                         }
                         at += m ? 1 : 0;
@@ -326,15 +325,14 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
                 }
             } else {
                 for (int sg = seg0; sg < seg1; ++sg) {
-                    uint32_t v[32];
-                    load_seg(sg, v);
-                    const int pos0 = (sg * 32 + lane) * 32;
+                    const int pos0 = sg * kTopkSeg + lane * kTopkKPL;
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) {
-                        if (v[j] != 0u && (v[j] & mask) == prefix) {
+                    for (int j = 0; j < kTopkKPL; ++j) {
+                        const uint32_t v = key_at(sg, j);
+                        if (v != 0u && (v & mask) == prefix) {
                             const int slot = atomicAdd(&sm.fcount, 1);
                             if (slot < kTopkFew) {
-                                sm.fkey[slot] = v[j];
+                                sm.fkey[slot] = v;
                                 sm.fpos[slot] = pos0 + j;
                             }
                         }
@@ -347,10 +345,11 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
             // More equal keys straddle the threshold than kTopkFew: rank by position.
             int eqc = 0;
             for (int sg = seg0; sg < seg1; ++sg) {
-                uint32_t v[32];
-                load_seg(sg, v);
 #pragma unroll
-                for (int j = 0; j < 32; ++j) eqc += (v[j] != 0u && (v[j] & mask) == prefix) ? 1 : 0;
+                for (int j = 0; j < kTopkKPL; ++j) {
+                    const uint32_t v = key_at(sg, j);
+                    eqc += (v != 0u && (v & mask) == prefix) ? 1 : 0;
+                }
             }
             eqc = __reduce_add_sync(0xffffffffu, eqc);
             if (lane == 0) sm.weq[warp] = eqc;
@@ -362,20 +361,22 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
         // Mark the keys above the threshold prefix (all of the bucket when it is
         // taken whole; with ties, the equal keys at the kk lowest positions).
         for (int sg = seg0; sg < seg1; ++sg) {
-            uint32_t v[32];
-            load_seg(sg, v);
-            uint32_t word = 0u;
+            uint32_t half = 0u;   // this lane's 16 positions
             if (!ties) {
 #pragma unroll
-                for (int j = 0; j < 32; ++j) {
-                    const uint32_t um = v[j] & mask;
-                    const bool sel = v[j] != 0u && (um > prefix || (whole_bin && um == prefix));
-                    word |= (sel ? 1u : 0u) << j;
+                for (int j = 0; j < kTopkKPL; ++j) {
+                    const uint32_t v = key_at(sg, j);
+                    const uint32_t um = v & mask;
+                    const bool sel = v != 0u && (um > prefix || (whole_bin && um == prefix));
+                    half |= (sel ? 1u : 0u) << j;
                 }
             } else {
                 int ec = 0;
 #pragma unroll
-                for (int j = 0; j < 32; ++j) ec += (v[j] != 0u && (v[j] & mask) == prefix) ? 1 : 0;
+                for (int j = 0; j < kTopkKPL; ++j) {
+                    const uint32_t v = key_at(sg, j);
+                    ec += (v != 0u && (v & mask) == prefix) ? 1 : 0;
+                }
                 int incl = ec;
 #pragma unroll
                 for (int o = 1; o < 32; o <<= 1) {
@@ -384,17 +385,21 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
                 }
                 int rank = base + incl - ec;
 #pragma unroll
-                for (int j = 0; j < 32; ++j) {
-                    const uint32_t um = v[j] & mask;
-                    const bool eq = v[j] != 0u && um == prefix;
-                    const bool sel = (v[j] != 0u && um > prefix) || (eq && rank < kk);
+                for (int j = 0; j < kTopkKPL; ++j) {
+                    const uint32_t v = key_at(sg, j);
+                    const uint32_t um = v & mask;
+                    const bool eq = v != 0u && um == prefix;
+                    const bool sel = (v != 0u && um > prefix) || (eq && rank < kk);
                     rank += eq ? 1 : 0;
-                    word |= (sel ? 1u : 0u) << j;
+                    half |= (sel ? 1u : 0u) << j;
                 }
                 base += __shfl_sync(0xffffffffu, incl, 31);
             }
-            const int wd = sg * 32 + lane;
-            if (wd < nwords && word) bits[wd] |= word;
+            // Lanes 2m and 2m + 1 hold the low and high halves of the segment's word m.
+            const uint32_t high = __shfl_xor_sync(0xffffffffu, half, 1);
+            const int wd = sg * (kTopkSeg / 32) + (lane >> 1);
+            const uint32_t word = half | (high << 16);
+            if ((lane & 1) == 0 && wd < nwords && word) bits[wd] |= word;
         }
         if (few) {
             topk_bar();   // the sweep's plain stores are done before warp 0 adds bits
@@ -680,75 +685,113 @@ __global__ void __launch_bounds__(kSelectThreads) heads_topk_kernel(Geometry G, 
 
 // Section 4.2: P' = P + lambda * I * (1 - n_t / (l + 1)); the preserved tokens
 // stay, the rest of B - w goes to the largest P'; the last w tokens are kept.
-// Writes out_idx (ascending) and folds the union of all heads into n_t once the
-// last head of the sequence is done.  Grid (Hkv, batch).
-__global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, LayerIO io, Scratch sc, Slot sl) {
+// Writes out_idx (ascending) and ORs the head's kept tokens into the layer's
+// union.  Grid (Hkv, batch).
+//
+// Coverage counts: n_t before this layer = A[t] + U_prev[t], where A is the
+// count array of the previous layer (the state for lcall = 0) and U_prev the
+// previous layer's union.  Every CTA reads them for its keys and writes the sum
+// for its slice of positions to the other count array, which is the next
+// layer's A; the last union is folded into the state by finalize_kernel.  No
+// CTA waits for another, and the previous layer's selection (a programmatic
+// dependency) is the only one this kernel waits for.
+__global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, LayerIO io, Scratch sc, Slot sl, int lcall,
+                                                                 int ncall) {
     __shared__ TopkShared sm;
-    __shared__ int last_head;
     extern __shared__ __align__(16) uint32_t bits[];
     const int h = blockIdx.x, s = blockIdx.y;
     const int tid = threadIdx.x, NT = blockDim.x;
     const int L = io.cu[s + 1] - io.cu[s];
     const int Lc = L - G.w;
     const int wordsL = (L + 31) >> 5;
-    for (int wd = tid; wd < G.words; wd += NT) bits[wd] = 0u;
     const int kw = key_stride(G);
     const bool cached = scores_in_smem(G.ML) && L > G.budget;
-    // 16-byte aligned (float4 stores): the bits and keys before it have any length.
-    const size_t sp_off = ((size_t)G.words + (keys_in_smem(G.ML) ? 32 * (size_t)kw : 0) + 3) & ~(size_t)3;
+    // Shared memory: bits[words] | preserved bits[words] | keys | P row | I row
+    // (P and I 16-byte aligned for float4 stores; what precedes them has any length).
+    uint32_t* spres = bits + G.words;
+    const size_t sp_off = ((size_t)2 * G.words + (keys_in_smem(G.ML) ? 32 * (size_t)kw : 0) + 3) & ~(size_t)3;
     float* sP = reinterpret_cast<float*>(bits + sp_off);
     float* sI = sP + G.ML;
     const size_t row = (size_t)s * G.Hkv + h;
     const int top = sl.htop[row];
     const float* P = (top ? sl.POe : sl.PO) + row * G.ML;
     const float* I = sl.I + (size_t)s * G.ML;
+    const uint32_t* pres = sl.pres + row * G.words;
+    uint8_t* st = io.state + (size_t)s * G.state_stride;
+    // This layer's scores and preserved tokens do not depend on the previous
+    // layer: stage them now, overlapping the previous layer's selection.
+    for (int wd = tid; wd < G.words; wd += NT) {
+        bits[wd] = 0u;
+        spres[wd] = __ldcg(&pres[wd]);
+    }
     if (cached) {
-        // This layer's scores do not depend on the previous layer: stage them now.
         for (int t4 = 4 * tid; t4 < Lc; t4 += 4 * NT) {
             *reinterpret_cast<float4*>(sP + t4) = __ldcg(reinterpret_cast<const float4*>(P + t4));
             *reinterpret_cast<float4*>(sI + t4) = __ldcg(reinterpret_cast<const float4*>(I + t4));
         }
     }
+    // The state header changes only at the end of a call (finalize_kernel).
+    // From the second layer of a call on, the previous call's finalize has
+    // completed before this grid could start, so the header is read early.
+    uint32_t ell0 = lcall > 0 ? __ldcg(reinterpret_cast<const uint32_t*>(st)) : 0u;
+    __syncthreads();
     // Launched as a programmatic dependent of the previous layer's selection:
-    // everything above overlaps its tail; the coverage state is read only after
+    // everything above overlaps its tail; the coverage counts are read only after
     // that grid has completed and its writes are visible.
     asm volatile("griddepcontrol.wait;\n" ::: "memory");
-    uint8_t* st = io.state + (size_t)s * G.state_stride;
-    const uint32_t ell = reinterpret_cast<const uint32_t*>(st)[0];
-    uint8_t* ncount = st + G.state_n_off;
-    if (ell >= 255u) {  // n_t is 8-bit: a state that already saw 255 layers cannot count another
-        if (tid == 0) atomicExch(sc.err, 2);
+    if (lcall == 0) ell0 = __ldcg(reinterpret_cast<const uint32_t*>(st));
+    if (ell0 + (uint32_t)ncall > 255u) {  // n_t is 8-bit: no state may count more than 255 layers
+        if (tid == 0) atomicExch(sc.err, 2);  // every layer of the call refuses; the state stays as it was
         return;
     }
-    __syncthreads();
+    const uint32_t ell = ell0 + (uint32_t)lcall;
+    uint8_t* nstate = st + G.state_n_off;
+    uint8_t* nscr = sc.nbuf + (size_t)s * G.nlen;
+    const uint8_t* nA = (lcall & 1) ? nscr : nstate;          // counts before the previous layer's union
+    uint8_t* nB = (lcall & 1) ? nstate : nscr;                // counts before this layer's union
+    const size_t ustride = (size_t)G.batch * G.words;
+    const uint32_t* uprev = sc.ubits + (size_t)((lcall + 2) % 3) * ustride + (size_t)s * G.words;
+    uint32_t* ucur = sc.ubits + (size_t)(lcall % 3) * ustride + (size_t)s * G.words;
+    uint32_t* unext = sc.ubits + (size_t)((lcall + 1) % 3) * ustride + (size_t)s * G.words;
+    // This CTA's slice of positions (a multiple of 32 long) for the count arrays
+    // and of union words for clearing the next layer's union.
+    const int fper = (((L + G.Hkv - 1) / G.Hkv) + 31) & ~31;
+    const int f0 = min(h * fper, L), f1 = min(f0 + fper, L);
+    auto counts4 = [&](int t4, uchar4 a, uint32_t uw) {
+        const uint32_t b = uw >> (t4 & 31);
+        return make_uchar4((uint8_t)(a.x + (b & 1u)), (uint8_t)(a.y + ((b >> 1) & 1u)), (uint8_t)(a.z + ((b >> 2) & 1u)),
+                           (uint8_t)(a.w + ((b >> 3) & 1u)));
+    };
     if (L > G.budget) {
-        const uint32_t* pres = sl.pres + row * G.words;
         float* Pp = sl.Pprime + row * G.ML;
-        uint32_t* keys = keys_in_smem(G.ML) ? bits + G.words : sc.keys_sel + row * G.ML;
+        uint32_t* keys = keys_in_smem(G.ML) ? spres + G.words : sc.keys_sel + row * G.ML;
         const float* Pr = cached ? sP : P;
         const float* Ir = cached ? sI : I;
         const float denom = (float)(ell + 1u);
         for (int b0 = 4 * tid; b0 < Lc; b0 += 16 * NT) {
             float4 pv[4], iv[4];
             uchar4 nv[4];
-            uint32_t pw[4];
+            uint32_t pw[4], uw[4];
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
                 const int t4 = b0 + 4 * u * NT;
                 if (t4 < Lc) {
+                    nv[u] = *reinterpret_cast<const uchar4*>(nA + t4);
+                    uw[u] = __ldcg(&uprev[t4 >> 5]);
                     pv[u] = *reinterpret_cast<const float4*>(Pr + t4);
                     iv[u] = *reinterpret_cast<const float4*>(Ir + t4);
-                    nv[u] = *reinterpret_cast<const uchar4*>(ncount + t4);
-                    pw[u] = pres[t4 >> 5];
+                    pw[u] = spres[t4 >> 5];
                 }
             }
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
                 const int t4 = b0 + 4 * u * NT;
                 if (t4 >= Lc) continue;
+                const uchar4 c = counts4(t4, nv[u], uw[u]);
+                if (t4 >= f0 && t4 + 4 <= f1 && t4 + 4 <= Lc) *reinterpret_cast<uchar4*>(nB + t4) = c;
                 const float p4[4] = {pv[u].x, pv[u].y, pv[u].z, pv[u].w};
                 const float i4[4] = {iv[u].x, iv[u].y, iv[u].z, iv[u].w};
-                const uint8_t n4[4] = {nv[u].x, nv[u].y, nv[u].z, nv[u].w};
+                const uint8_t n4[4] = {c.x, c.y, c.z, c.w};
                 float out[4];
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
@@ -766,10 +809,29 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
         block_topk(keys, kw, Lc, G.k2, bits, sm);
         // The next layer's selection may be scheduled now (it waits for this grid).
         asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
-        for (int wd = tid; wd < wordsL; wd += NT) bits[wd] |= pres[wd] | range_bits(wd, Lc, L);
+        for (int wd = tid; wd < wordsL; wd += NT) bits[wd] |= spres[wd] | range_bits(wd, Lc, L);
     } else {
+        // Every token is kept; the slice's counts still move to the next array.
+        for (int t4 = f0 + 4 * tid; t4 < min(f1, Lc & ~3); t4 += 4 * NT) {
+            const uchar4 c = counts4(t4, *reinterpret_cast<const uchar4*>(nA + t4), __ldcg(&uprev[t4 >> 5]));
+            *reinterpret_cast<uchar4*>(nB + t4) = c;
+        }
         for (int wd = tid; wd < wordsL; wd += NT) bits[wd] = range_bits(wd, 0, L);
     }
+    // For the next layer only: the counts of this slice outside the candidates
+    // (the kept window; positions from L on keep what the array holds) and the
+    // slice's words of the next layer's union, cleared.
+    for (int t4 = max(f0, Lc & ~3) + 4 * tid; t4 < f1; t4 += 4 * NT) {
+        if (t4 + 4 <= Lc) continue;   // written with the candidates
+        const uchar4 c = counts4(t4, *reinterpret_cast<const uchar4*>(nA + t4), __ldcg(&uprev[t4 >> 5]));
+        if (t4 + 4 <= L) {
+            *reinterpret_cast<uchar4*>(nB + t4) = c;
+        } else {
+            const uint8_t c4[4] = {c.x, c.y, c.z, c.w};
+            for (int i = 0; t4 + i < L; ++i) nB[t4 + i] = c4[i];
+        }
+    }
+    for (int wd = (f0 >> 5) + tid; wd < ((f1 + 31) >> 5); wd += NT) unext[wd] = 0u;
     __syncthreads();
 
     // Ascending positions: each thread owns a contiguous run of words.
@@ -791,35 +853,41 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
     }
     for (int j = total + tid; j < G.budget; j += NT) oi[j] = -1;
 
-    // Union over heads, then the last head of the sequence updates n_t (Section 4.2).
-    uint32_t* ub = sc.ubits + (size_t)s * G.words;
+    // Union over heads (Section 4.2); nothing waits for it within this grid.
     for (int wd = tid; wd < wordsL; wd += NT)
-        if (bits[wd]) atomicOr(&ub[wd], bits[wd]);
-    __threadfence();
-    __syncthreads();
-    if (tid == 0) last_head = atomicAdd(&sc.ucount[s], 1u) == (unsigned)(G.Hkv - 1);
-    __syncthreads();
-    if (!last_head) return;
-    __threadfence();
+        if (bits[wd]) atomicOr(&ucur[wd], bits[wd]);
+}
+
+// After the last layer of a call: n_t of the state = the last count array plus
+// the last union, last_union = that union, layers_done and seqlen updated.
+// Grid (batch).
+__global__ void __launch_bounds__(kSelectThreads) finalize_kernel(Geometry G, LayerIO io, Scratch sc, int ncall) {
+    const int s = blockIdx.x, tid = threadIdx.x, NT = blockDim.x;
+    asm volatile("griddepcontrol.wait;\n" ::: "memory");
+    const int L = io.cu[s + 1] - io.cu[s];
+    uint8_t* st = io.state + (size_t)s * G.state_stride;
+    const uint32_t ell0 = reinterpret_cast<const uint32_t*>(st)[0];
+    if (ell0 + (uint32_t)ncall > 255u) return;   // the select kernels reported it and wrote nothing
+    const int l = ncall - 1;
+    uint8_t* nstate = st + G.state_n_off;
+    const uint8_t* nlast = (l & 1) ? nstate : sc.nbuf + (size_t)s * G.nlen;   // written by the last layer
+    const uint32_t* ulast = sc.ubits + (size_t)(l % 3) * G.batch * G.words + (size_t)s * G.words;
     for (int t4 = 4 * tid; t4 < L; t4 += 4 * NT) {
-        const uint32_t wv = __ldcg(&ub[t4 >> 5]) >> (t4 & 31);
-        uchar4 n4 = *reinterpret_cast<uchar4*>(ncount + t4);
-        n4.x = (uint8_t)(n4.x + (wv & 1u));
-        if (t4 + 1 < L) n4.y = (uint8_t)(n4.y + ((wv >> 1) & 1u));
-        if (t4 + 2 < L) n4.z = (uint8_t)(n4.z + ((wv >> 2) & 1u));
-        if (t4 + 3 < L) n4.w = (uint8_t)(n4.w + ((wv >> 3) & 1u));
-        *reinterpret_cast<uchar4*>(ncount + t4) = n4;
+        const uchar4 a = *reinterpret_cast<const uchar4*>(nlast + t4);
+        const uint32_t b = __ldcg(&ulast[t4 >> 5]) >> (t4 & 31);
+        const uint8_t c4[4] = {(uint8_t)(a.x + (b & 1u)), (uint8_t)(a.y + ((b >> 1) & 1u)),
+                               (uint8_t)(a.z + ((b >> 2) & 1u)), (uint8_t)(a.w + ((b >> 3) & 1u))};
+        if (t4 + 4 <= L) {
+            *reinterpret_cast<uchar4*>(nstate + t4) = make_uchar4(c4[0], c4[1], c4[2], c4[3]);
+        } else {
+            for (int i = 0; t4 + i < L; ++i) nstate[t4 + i] = c4[i];
+        }
     }
-    __syncthreads();
     uint32_t* last_union = reinterpret_cast<uint32_t*>(st + G.state_union_off);
-    for (int wd = tid; wd < G.words; wd += NT) {
-        last_union[wd] = __ldcg(&ub[wd]);
-        ub[wd] = 0u;
-    }
+    for (int wd = tid; wd < G.words; wd += NT) last_union[wd] = __ldcg(&ulast[wd]);
     if (tid == 0) {
-        reinterpret_cast<uint32_t*>(st)[0] = ell + 1u;
+        reinterpret_cast<uint32_t*>(st)[0] = ell0 + (uint32_t)ncall;
         reinterpret_cast<uint32_t*>(st)[1] = (uint32_t)L;
-        sc.ucount[s] = 0u;
     }
 }
 
@@ -846,7 +914,7 @@ __global__ void __launch_bounds__(256) gather_kernel(Geometry G, LayerIO io) {
 }  // namespace
 
 size_t select_smem_bytes(const Geometry& g) {
-    const size_t head = ((size_t)g.words + (keys_in_smem(g.ML) ? 32 * (size_t)key_stride(g) : 0) + 3) & ~(size_t)3;
+    const size_t head = ((size_t)2 * g.words + (keys_in_smem(g.ML) ? 32 * (size_t)key_stride(g) : 0) + 3) & ~(size_t)3;
     return sizeof(uint32_t) * (head + (scores_in_smem(g.ML) ? 2 * (size_t)g.ML : 0));
 }
 
@@ -856,10 +924,12 @@ size_t heads_smem_bytes(const Geometry& g) {
 
 cudaError_t configure_select() {
     const int need = (int)(sizeof(uint32_t) * (kSmemKeys / 32 + 32 * ((kSmemKeys / 32) | 1)));
-    // The select kernel also caches P and I rows up to kSmemScores positions.
+    // The select kernel also keeps the preserved bits and caches P and I rows
+    // up to kSmemScores positions.
+    const int need_sel_keys = need + (int)(sizeof(uint32_t) * (kSmemKeys / 32 + 4));
     const int need_sel_scores =
-        (int)(sizeof(uint32_t) * (kSmemScores / 32 + 32 * ((kSmemScores / 32) | 1) + 2 * kSmemScores + 64));
-    const int need_sel = need > need_sel_scores ? need : need_sel_scores;
+        (int)(sizeof(uint32_t) * (2 * (kSmemScores / 32) + 32 * ((kSmemScores / 32) | 1) + 2 * kSmemScores + 64));
+    const int need_sel = need_sel_keys > need_sel_scores ? need_sel_keys : need_sel_scores;
     cudaError_t e = cudaFuncSetAttribute(heads_topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, need);
     if (e == cudaSuccess)
         e = cudaFuncSetAttribute(heads_pool_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kPoolSmemBytes);
@@ -880,9 +950,15 @@ cudaError_t launch_heads(const Geometry& g, const LayerIO& io, const Scratch& sc
 }
 
 cudaError_t launch_select(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st,
-                          int priority) {
+                          int priority, int lcall, int ncall) {
     return launch_prio(select_kernel, dim3(g.Hkv, g.batch), dim3(kSelectThreads), select_smem_bytes(g), st, priority,
-                       /*programmatic=*/true, g, io, sc, sl);
+                       /*programmatic=*/true, g, io, sc, sl, lcall, ncall);
+}
+
+cudaError_t launch_finalize(const Geometry& g, const LayerIO& io, const Scratch& sc, cudaStream_t st, int priority,
+                            int ncall) {
+    return launch_prio(finalize_kernel, dim3(g.batch), dim3(kSelectThreads), 0, st, priority, /*programmatic=*/true, g,
+                       io, sc, ncall);
 }
 
 void launch_gather(const Geometry& g, const LayerIO& io, cudaStream_t st) {

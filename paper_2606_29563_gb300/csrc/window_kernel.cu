@@ -32,7 +32,6 @@ constexpr int kWinThreads = 576;                      // warp 0 TMA, warp 1 MMA,
 constexpr int kEpiThreads = 512;
 constexpr int kEpiWarps = kEpiThreads / 32;
 constexpr int kMaxSmemWin = 232448;                   // opt-in shared memory per CTA on sm_103
-constexpr int kWinCuParam = 64;                       // sequences whose offsets travel in the kernel parameters
 constexpr int kKTileBytes = kTileT * kHeadDim * 2;    // 32 KB: two 64-column swizzled halves
 constexpr int kRsRows = 288;                          // row-statistics buffer: R <= 256 plus a chunk's overrun
 
@@ -41,7 +40,6 @@ struct WinArgs {
     Scratch sc;
     Slot sl;
     const int* cu;                  // device cu_seqlens
-    int cuv[kWinCuParam + 1];       // the same offsets (when batch <= kWinCuParam)
     int Npad;                       // query rows padded to a multiple of 16 (MMA N)
     int kst;                        // operand stages
     int nacc;                       // TMEM accumulators (2, or 1 when 2 do not fit)
@@ -141,12 +139,22 @@ __global__ void __launch_bounds__(kWinThreads, 1)
     if (threadIdx.x == 0) {
         ptx::prefetch_tensormap(&kmap);
         ptx::prefetch_tensormap(&qmap);
+        // The next launch on this stream (the next layer's window sums) reads
+        // nothing this grid writes: let it be scheduled as SMs free up.
+        asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
     }
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    const Geometry& G = A.G;
+    // Scalars and pointers in registers: values read through a reference to the
+    // parameter block would be re-read after every asm statement that clobbers memory.
+    const Geometry G = A.G;
+    const Scratch sc = A.sc;
+    const Slot sl = A.sl;
+    const int* const cu_dev = A.cu;
+    const int kst = A.kst, nacc = A.nacc;
+    const uint32_t tmem_cols = A.tmem_cols;
     const int Npad = A.Npad, R = G.R;
     const size_t sbytes = stage_bytes(Npad);
-    float* rs = reinterpret_cast<float*>(smem + A.kst * sbytes);        // [HG][kRsRows] m_r + log2 Z_r
+    float* rs = reinterpret_cast<float*>(smem + kst * sbytes);        // [HG][kRsRows] m_r + log2 Z_r
     float* maxg = reinterpret_cast<float*>(rs + kWinHeadsPerCta * kRsRows);   // [O][128] max over heads of G_h[q][t]
     float2* xfer = reinterpret_cast<float2*>(maxg + G.O * kTileT);      // [HG][4][128] quarters' (P_O, P_O') sums
     WinBars* bars = reinterpret_cast<WinBars*>(xfer + kWinHeadsPerCta * 4 * kTileT);
@@ -154,8 +162,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
 
     // Work item -> (sequence, candidate tile, head group); sequence s owns
     // ceil(Lc / 128) * NG consecutive CTAs.
-    const bool cu_param = G.batch <= kWinCuParam;
-    auto cu = [&](int b) { return cu_param ? A.cuv[b] : __ldg(&A.cu[b]); };
+    auto cu = [&](int b) { return __ldg(&cu_dev[b]); };
     int s = -1, jt = 0, ng = 0, tg = 0;
     {
         int base = 0, tbase = 0;
@@ -178,7 +185,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
     const int L = cu(s + 1) - cu(s), Lc = L - G.w;
     const int h0 = ng * G.HG;
     const int nh = min(G.HG, G.Hkv - h0);
-    const int NB = A.nacc;
+    const int NB = nacc;
 
     if (threadIdx.x == 32) {
         for (int i = 0; i < 2; ++i) {
@@ -193,7 +200,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
         ptx::fence_barrier_init();
     }
     if (warp == 1) {
-        ptx::tmem_alloc(&bars->tmem_base, A.tmem_cols);
+        ptx::tmem_alloc(&bars->tmem_base, tmem_cols);
         ptx::tmem_relinquish();
     }
     ptx::tc_fence_before();
@@ -208,9 +215,9 @@ __global__ void __launch_bounds__(kWinThreads, 1)
             const int row0 = cu(s) + jt * kTileT;
             int fills[2] = {0, 0};
             for (int hh = 0; hh < nh && !bars->abort_flag; ++hh) {
-                const int st = hh % A.kst, u = hh / A.kst;
+                const int st = hh % kst, u = hh / kst;
                 if (u > 0 && !ptx::mbar_wait(&bars->empty[st], (u - 1) & 1)) {
-                    win_abort(bars, A.sc.err);
+                    win_abort(bars, sc.err);
                     break;
                 }
                 uint8_t* sk = smem + st * sbytes;
@@ -224,7 +231,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
                 ++fills[st];
             }
             // Drain: every issued copy lands before the CTA may exit.
-            for (int st = 0; st < A.kst; ++st)
+            for (int st = 0; st < kst; ++st)
                 if (fills[st] > 0) ptx::mbar_wait(&bars->full[st], (fills[st] - 1) & 1, 50000000ull);
         }
     } else if (warp == 1) {
@@ -232,11 +239,11 @@ __global__ void __launch_bounds__(kWinThreads, 1)
         if (lane == 0) {
             const uint32_t idesc = ptx::idesc_bf16_f32(128, Npad);
             for (int hh = 0; hh < nh && !bars->abort_flag; ++hh) {
-                const int st = hh % A.kst, u = hh / A.kst;
+                const int st = hh % kst, u = hh / kst;
                 const int b = hh % NB, ub = hh / NB;
                 if (!ptx::mbar_wait(&bars->full[st], u & 1) ||
                     (ub > 0 && !ptx::mbar_wait(&bars->acc_empty[b], (ub - 1) & 1))) {
-                    win_abort(bars, A.sc.err);
+                    win_abort(bars, sc.err);
                     break;
                 }
                 ptx::tc_fence_after();
@@ -268,7 +275,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
         // Row statistics of every head of the group: A = 2^(s * sl2 - (m_r + log2 Z_r)).
         for (int i = e; i < nh * R; i += kEpiThreads) {
             const int hh = i / R, r = i - hh * R;
-            const float2 ms = __ldcg(&A.sc.rowstat[((size_t)s * G.Hkv + h0 + hh) * R + r]);
+            const float2 ms = __ldcg(&sc.rowstat[((size_t)s * G.Hkv + h0 + hh) * R + r]);
             rs[hh * kRsRows + r] = ms.x + __log2f(ms.y);
         }
         ptx::named_bar_sync(1, kEpiThreads);
@@ -282,7 +289,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
             if (!got) {
                 if (lane == 0) {
                     bars->epi_fail = 1;
-                    win_abort(bars, A.sc.err);
+                    win_abort(bars, sc.err);
                 }
                 break;
             }
@@ -313,8 +320,8 @@ __global__ void __launch_bounds__(kWinThreads, 1)
                         soe += x.y;
                     }
                     const size_t row = (size_t)s * G.Hkv + h0 + hh;
-                    A.sl.rawO[row * G.ML + tt] = so * invO;
-                    A.sl.rawOe[row * G.ML + tt] = soe * invOe;
+                    sl.rawO[row * G.ML + tt] = so * invO;
+                    sl.rawOe[row * G.ML + tt] = soe * invOe;
                 }
             }
         }
@@ -324,12 +331,12 @@ __global__ void __launch_bounds__(kWinThreads, 1)
             // maxima and the heads kernel takes the maximum over the groups.
             const int n_el = G.O * kTileT;
             if (G.NG > 1) {
-                float* wp = A.sl.wpart + ((size_t)tg * G.NG + ng) * n_el;
+                float* wp = sl.wpart + ((size_t)tg * G.NG + ng) * n_el;
                 for (int i = e; i < n_el; i += kEpiThreads) wp[i] = maxg[i];
             } else if (e < kTileT && jt * kTileT + e < Lc) {
                 float ip = 0.f;
                 for (int qi = 0; qi < G.O; ++qi) ip += maxg[qi * kTileT + e];
-                A.sl.rawI[(size_t)s * G.ML + jt * kTileT + e] = ip * invO;
+                sl.rawI[(size_t)s * G.ML + jt * kTileT + e] = ip * invO;
             }
         }
     }
@@ -339,7 +346,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
     ptx::tc_fence_before();
     __syncthreads();
     ptx::tc_fence_after();
-    if (warp == 1) ptx::tmem_dealloc(tmem, A.tmem_cols);
+    if (warp == 1) ptx::tmem_dealloc(tmem, tmem_cols);
 }
 
 int npad_of(int R) { return (R + 15) & ~15; }
@@ -369,14 +376,13 @@ cudaError_t configure_window(const Geometry& g) {
 }
 
 cudaError_t launch_window(const ScorePlan& sp, const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl,
-                          cudaStream_t st) {
+                          cudaStream_t st, bool after_own_launch) {
     if (g.win_tiles == 0) return cudaSuccess;
     WinArgs a{};
     a.G = g;
     a.sc = sc;
     a.sl = sl;
     a.cu = io.cu;
-    for (int b = 0; b <= g.batch && b <= kWinCuParam; ++b) a.cuv[b] = g.cu_host ? g.cu_host[b] : 0;
     a.Npad = npad_of(g.R);
     a.kst = kst_for(a.Npad, g.O);
     a.nacc = 2 * a.Npad + 32 <= 512 ? 2 : 1;
@@ -385,15 +391,27 @@ cudaError_t launch_window(const ScorePlan& sp, const Geometry& g, const LayerIO&
     a.tmem_cols = cols;
     const size_t smem = win_smem_bytes(a.Npad, g.O, a.kst);
     const int grid = g.win_tiles * g.NG;
+    // after_own_launch: the previous kernel on the stream is the previous
+    // layer's launch, whose results this grid does not read; the launch is then
+    // its programmatic dependent and never executes griddepcontrol.wait.
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(kWinThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = after_own_launch ? 1 : 0;
     switch (g.g) {
-        case 1: window_kernel<1><<<grid, kWinThreads, smem, st>>>(sp.kmap, sp.qmap, a); break;
-        case 2: window_kernel<2><<<grid, kWinThreads, smem, st>>>(sp.kmap, sp.qmap, a); break;
-        case 4: window_kernel<4><<<grid, kWinThreads, smem, st>>>(sp.kmap, sp.qmap, a); break;
-        case 7: window_kernel<7><<<grid, kWinThreads, smem, st>>>(sp.kmap, sp.qmap, a); break;
-        case 8: window_kernel<8><<<grid, kWinThreads, smem, st>>>(sp.kmap, sp.qmap, a); break;
-        default: window_kernel<0><<<grid, kWinThreads, smem, st>>>(sp.kmap, sp.qmap, a); break;
+        case 1: return cudaLaunchKernelEx(&cfg, window_kernel<1>, sp.kmap, sp.qmap, a);
+        case 2: return cudaLaunchKernelEx(&cfg, window_kernel<2>, sp.kmap, sp.qmap, a);
+        case 4: return cudaLaunchKernelEx(&cfg, window_kernel<4>, sp.kmap, sp.qmap, a);
+        case 7: return cudaLaunchKernelEx(&cfg, window_kernel<7>, sp.kmap, sp.qmap, a);
+        case 8: return cudaLaunchKernelEx(&cfg, window_kernel<8>, sp.kmap, sp.qmap, a);
+        default: return cudaLaunchKernelEx(&cfg, window_kernel<0>, sp.kmap, sp.qmap, a);
     }
-    return cudaGetLastError();
 }
 
 }  // namespace kvec

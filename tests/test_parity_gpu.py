@@ -122,6 +122,37 @@ def test_multi_layer_call_matches_layer_by_layer():
     sel.close()
 
 
+def test_layer_limit_refuses_the_whole_call_and_positions_past_L_stay_zero():
+    """n_t is 8-bit, so no state may count more than 255 layers (Section 4.2's
+    counters).  A call that would pass the limit reports it and leaves the state
+    as it was, whichever of its layers would have crossed it; a call that ends at
+    255 runs.  Positions from L on (here L = 301, not a multiple of 4, in a state
+    sized for 400) are never written."""
+    L, ML = 301, 400
+    wl = synth.small_workload(seqlens=(L,), layers=2)
+    layers = [{k: v.cuda() for k, v in x.items()} for x in synth.make_layers(wl, 2)]
+    cu = torch.tensor(wl.cu_seqlens, dtype=torch.int32)
+    sel = kvec.KvecSelector(kvec.params_from_workload(wl, max_seqlen=ML))
+    st = sel.new_state(1)
+    st[0, 0] = 254   # layers_done, little endian
+    before = st.clone()
+    outs = [sel.alloc_outputs(1, wl.budget) for _ in layers]
+    sel.select_layers(cu, cu.cuda(), [x["q_obs"] for x in layers], [x["k"] for x in layers],
+                      [x["v"] for x in layers], st, wl.budget, outs)
+    with pytest.raises(kvec.KvecError) as e:
+        kvec.kvec_sync_status(sel.handle)
+    assert e.value.status == kvec.KVEC_ERR_INVALID_ARG
+    assert torch.equal(st, before)
+    x = layers[0]
+    sel.select_layer(cu, cu.cuda(), x["q_obs"], x["k"], x["v"], st, wl.budget)
+    kvec.kvec_sync_status(sel.handle)
+    s = st.cpu()
+    assert s[0, 0].item() == 255 and s[0, 4:8].view(torch.int32).item() == L
+    n = s[0, 16:16 + ((ML + 15) // 16) * 16]
+    assert int(n[:L].sum()) > 0 and not n[L:].any()
+    sel.close()
+
+
 def test_call_validation_on_device():
     wl = synth.small_workload(seqlens=(300,))
     sel = kvec.KvecSelector(kvec.params_from_workload(wl))

@@ -69,7 +69,7 @@ struct kvec_handle {
     // layer, so consecutive layers' head passes overlap) | coverage select | gather.
     cudaStream_t s_score = nullptr, s_win = nullptr, s_heads = nullptr, s_heads2 = nullptr, s_chain = nullptr,
                  s_gather = nullptr, s_cap = nullptr;
-    std::vector<cudaEvent_t> ev_score, ev_win, ev_heads, ev_sel;
+    std::vector<cudaEvent_t> ev_score, ev_win, ev_heads, ev_sel, ev_gather;
     cudaEvent_t ev_fork = nullptr, ev_join[5] = {nullptr, nullptr, nullptr, nullptr, nullptr};
     // Scheduling priorities: the heads and coverage-select kernels (the serial
     // chain of the pipeline) take SMs before the score, window and gather kernels.
@@ -222,9 +222,6 @@ Geometry make_geometry(const kvec_handle* h, int batch, int budget, int tiles, i
 
 // One layer, every kernel on one stream with one slot (used without a handle).
 kvec_status run_layer_sequential(kvec_handle* h, const Geometry& G, const LayerIO& io, cudaStream_t st) {
-    // The union ring starts empty (the select kernel reads entry 2 as the previous union).
-    cudaError_t me = cudaMemsetAsync(h->sc.ubits, 0, 3 * (size_t)G.batch * G.words * sizeof(uint32_t), st);
-    if (me != cudaSuccess) return cuda_fail(me, "cudaMemsetAsync(union ring)");
     ScorePlan plan;
     cudaError_t se = plan_score(G, io, h->sc, h->num_sms, &plan);
     if (se != cudaSuccess) return cuda_fail(se, "score kernel tensor maps");
@@ -234,10 +231,10 @@ kvec_status run_layer_sequential(kvec_handle* h, const Geometry& G, const LayerI
     if (se != cudaSuccess) return cuda_fail(se, "window kernel launch");
     se = launch_heads(G, io, h->sc, h->slots[0], st, h->prio_hi);
     if (se != cudaSuccess) return cuda_fail(se, "heads kernel launch");
-    se = launch_select(G, io, h->sc, h->slots[0], st, h->prio_hi, 0, 1);
+    se = launch_select(G, io, h->sc, h->slots[0], nullptr, st, h->prio_hi, 0, 1);
     if (se != cudaSuccess) return cuda_fail(se, "select kernel launch");
-    launch_gather(G, io, st);
-    se = launch_finalize(G, io, h->sc, st, h->prio_hi, 1);
+    launch_gather(G, io, h->slots[0], st);
+    se = launch_finalize(G, io, h->sc, h->slots[0], st, h->prio_hi, 1);
     if (se != cudaSuccess) return cuda_fail(se, "finalize kernel launch");
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_fail(e, "kernel launch");
@@ -258,8 +255,6 @@ kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* io
     KV_CHECK(cudaEventRecord(h->ev_fork, origin));
     for (cudaStream_t st : {h->s_score, h->s_win, h->s_heads, h->s_heads2, h->s_chain, h->s_gather})
         KV_CHECK(cudaStreamWaitEvent(st, h->ev_fork, 0));
-    // The layers' unions start empty (ring of three, see launch_select).
-    KV_CHECK(cudaMemsetAsync(h->sc.ubits, 0, 3 * (size_t)G.batch * G.words * sizeof(uint32_t), h->s_chain));
     for (int l = 0; l < n; ++l) {
         const Slot& sl = h->slots[l % kSlots];
         const Scratch& sc = h->score_buf[l & 1];
@@ -272,7 +267,14 @@ kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* io
         if (se != cudaSuccess) return cuda_fail(se, "score kernel launch");
         KV_CHECK(cudaEventRecord(h->ev_score[l], h->s_score));
         KV_CHECK(cudaStreamWaitEvent(h->s_win, h->ev_score[l], 0));
-        if (l >= kSlots) KV_CHECK(cudaStreamWaitEvent(h->s_win, h->ev_sel[l - kSlots], 0));
+        // Slot reuse: the window, heads and select of this layer rewrite the slot
+        // that layer l - kSlots used; its selection and gather (which reads the
+        // slot's kept bits) are done first.  The select stream itself then waits
+        // only for this layer's heads, so consecutive selections stay programmatic.
+        if (l >= kSlots) {
+            KV_CHECK(cudaStreamWaitEvent(h->s_win, h->ev_sel[l - kSlots], 0));
+            KV_CHECK(cudaStreamWaitEvent(h->s_win, h->ev_gather[l - kSlots], 0));
+        }
         timed_launch(h, 1, h->s_win, [&] { se = launch_window(plan, G, io, sc, sl, h->s_win, true); });
         if (se != cudaSuccess) return cuda_fail(se, "window kernel launch");
         KV_CHECK(cudaEventRecord(h->ev_win[l], h->s_win));
@@ -282,15 +284,18 @@ kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* io
         if (se != cudaSuccess) return cuda_fail(se, "heads kernel launch");
         KV_CHECK(cudaEventRecord(h->ev_heads[l], s_h));
         KV_CHECK(cudaStreamWaitEvent(h->s_chain, h->ev_heads[l], 0));
-        timed_launch(h, 3, h->s_chain, [&] { se = launch_select(G, io, sc, sl, h->s_chain, h->prio_hi, l, n); });
+        const Slot* prev = l > 0 ? &h->slots[(l - 1) % kSlots] : nullptr;
+        timed_launch(h, 3, h->s_chain, [&] { se = launch_select(G, io, sc, sl, prev, h->s_chain, h->prio_hi, l, n); });
         if (se != cudaSuccess) return cuda_fail(se, "select kernel launch");
         KV_CHECK(cudaEventRecord(h->ev_sel[l], h->s_chain));
         KV_CHECK(cudaStreamWaitEvent(h->s_gather, h->ev_sel[l], 0));
-        timed_launch(h, 4, h->s_gather, [&] { launch_gather(G, io, h->s_gather); });
+        timed_launch(h, 4, h->s_gather, [&] { launch_gather(G, io, sl, h->s_gather); });
+        KV_CHECK(cudaEventRecord(h->ev_gather[l], h->s_gather));
     }
     // The last layer's union goes into the state.
     {
-        cudaError_t se = launch_finalize(G, ios[n - 1], h->score_buf[(n - 1) & 1], h->s_chain, h->prio_hi, n);
+        cudaError_t se = launch_finalize(G, ios[n - 1], h->score_buf[(n - 1) & 1], h->slots[(n - 1) % kSlots], h->s_chain,
+                                         h->prio_hi, n);
         if (se != cudaSuccess) return cuda_fail(se, "finalize kernel launch");
     }
     KV_CHECK(cudaGetLastError());
@@ -328,7 +333,7 @@ void release_handle(kvec_handle* h) {
     if (h->gexec) cudaGraphExecDestroy(h->gexec);
     for (cudaStream_t st : {h->s_score, h->s_win, h->s_heads, h->s_heads2, h->s_chain, h->s_gather, h->s_cap})
         if (st) cudaStreamDestroy(st);
-    for (auto* v : {&h->ev_score, &h->ev_win, &h->ev_heads, &h->ev_sel})
+    for (auto* v : {&h->ev_score, &h->ev_win, &h->ev_heads, &h->ev_sel, &h->ev_gather})
         for (cudaEvent_t ev : *v)
             if (ev) cudaEventDestroy(ev);
     if (h->ev_fork) cudaEventDestroy(h->ev_fork);
@@ -383,7 +388,6 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
     std::vector<Part> parts = {
 
         {(void**)&h->sc.keys, MB * Hkv * ML * sizeof(uint32_t)},
-        {(void**)&h->sc.ubits, 3 * MB * W * sizeof(uint32_t)},
         {(void**)&h->sc.nbuf, MB * round_up((size_t)p.max_seqlen, 16)},
         {(void**)&h->sc.err, sizeof(int)},
         {(void**)&h->sc.keys_sel, MB * Hkv * ML * sizeof(uint32_t)},
@@ -405,6 +409,7 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
             {(void**)&sl.POe, MB * Hkv * ML * sizeof(float)},   {(void**)&sl.I, MB * ML * sizeof(float)},
             {(void**)&sl.sigma, MB * Hkv * sizeof(float)},      {(void**)&sl.htop, MB * Hkv * sizeof(int)},
             {(void**)&sl.pres, MB * Hkv * W * sizeof(uint32_t)}, {(void**)&sl.Pprime, MB * Hkv * ML * sizeof(float)},
+            {(void**)&sl.sel, MB * Hkv * W * sizeof(uint32_t)},
             {(void**)&sl.wpart, max_tiles * NGmax * p.obs_window * kTileT * sizeof(float)},
         };
         parts.insert(parts.end(), sp.begin(), sp.end());
@@ -427,7 +432,6 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
     for (Scratch& b : h->score_buf) {
         b.keys = h->sc.keys;
         b.keys_sel = h->sc.keys_sel;
-        b.ubits = h->sc.ubits;
         b.nbuf = h->sc.nbuf;
         b.err = h->sc.err;
     }
@@ -448,7 +452,8 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
     h->ev_win.assign(p.max_layers, nullptr);
     h->ev_heads.assign(p.max_layers, nullptr);
     h->ev_sel.assign(p.max_layers, nullptr);
-    for (auto* v : {&h->ev_score, &h->ev_win, &h->ev_heads, &h->ev_sel})
+    h->ev_gather.assign(p.max_layers, nullptr);
+    for (auto* v : {&h->ev_score, &h->ev_win, &h->ev_heads, &h->ev_sel, &h->ev_gather})
         for (auto& ev : *v)
             if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
     if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming);
@@ -662,7 +667,6 @@ kvec_status kvec_select_layer_noalloc(const kvec_params* params, int batch, cons
     Part parts[] = {
         {(void**)&tmp.sc.err, sizeof(int)},                   // zeroed every call (first two parts)
         {(void**)&tmp.sc.shcount, nb * Hkv * sizeof(unsigned)},
-        {(void**)&tmp.sc.ubits, 3 * nb * W * sizeof(uint32_t)},
         {(void**)&tmp.sc.nbuf, nb * round_up((size_t)params->max_seqlen, 16)},
         {(void**)&tmp.sc.segpart, nt * Hkv * R * sizeof(float2)},
         {(void**)&tmp.slots[0].wpart, nt * NGv * (size_t)params->obs_window * kTileT * sizeof(float)},
@@ -679,6 +683,7 @@ kvec_status kvec_select_layer_noalloc(const kvec_params* params, int batch, cons
         {(void**)&tmp.slots[0].htop, nb * Hkv * sizeof(int)},
         {(void**)&tmp.slots[0].pres, nb * Hkv * W * sizeof(uint32_t)},
         {(void**)&tmp.slots[0].Pprime, nb * Hkv * ML * sizeof(float)},
+        {(void**)&tmp.slots[0].sel, nb * Hkv * W * sizeof(uint32_t)},
     };
     size_t need = 0, zero_bytes = 0;
     for (size_t i = 0; i < sizeof(parts) / sizeof(parts[0]); ++i) {

@@ -48,6 +48,7 @@ struct Slot {
     uint32_t* pres;       // [max_batch][Hkv][words]
     float* Pprime;        // [max_batch][Hkv][ML]
     float* wpart;         // [win_tiles][NG][O][kTileT] per-group head maxima of G_h[q][t] (NG > 1)
+    uint32_t* sel;        // [max_batch][Hkv][words]  kept positions of the layer, one bit each
 };
 
 struct Scratch {
@@ -56,7 +57,6 @@ struct Scratch {
     float2* rowstat;      // [max_batch][Hkv][R]    (row max in log2 units, softmax denominator)
     uint32_t* keys;       // [max_batch][Hkv][ML]   radix-select keys of the heads kernel
     uint32_t* keys_sel;   // [max_batch][Hkv][ML]   radix-select keys of the select kernel
-    uint32_t* ubits;      // [3][max_batch][words]  union of a layer's selections, ring over layers
     uint8_t* nbuf;        // [max_batch][nlen]      second copy of n_t (the coverage counts alternate)
     int* err;             // device error word
 };
@@ -136,15 +136,17 @@ cudaError_t launch_prio(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t 
 
 cudaError_t launch_heads(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st,
                          int priority);
-// lcall: the layer's index within a call of ncall layers (0 for the first).
-// The coverage counts alternate between the state and sc.nbuf and each layer's
-// union goes to ring entry lcall % 3; launch_finalize folds the last union into
-// the state.
-cudaError_t launch_select(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st,
-                          int priority, int lcall, int ncall);
-cudaError_t launch_finalize(const Geometry& g, const LayerIO& io, const Scratch& sc, cudaStream_t st, int priority,
-                            int ncall);
-void launch_gather(const Geometry& g, const LayerIO& io, cudaStream_t st);
+// lcall: the layer's index within a call of ncall layers (0 for the first);
+// prev: the previous layer's slot (null for lcall = 0), whose kept-position
+// bits give that layer's union.  The coverage counts alternate between the
+// state and sc.nbuf; launch_finalize folds the last layer's union (from its
+// slot) into the state.
+cudaError_t launch_select(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, const Slot* prev,
+                          cudaStream_t st, int priority, int lcall, int ncall);
+cudaError_t launch_finalize(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& last, cudaStream_t st,
+                            int priority, int ncall);
+// out_idx from the slot's kept-position bits, then the K/V rows.
+void launch_gather(const Geometry& g, const LayerIO& io, const Slot& sl, cudaStream_t st);
 
 size_t score_smem_bytes(const Geometry& g);
 size_t window_smem_bytes(const Geometry& g);

@@ -685,18 +685,20 @@ __global__ void __launch_bounds__(kSelectThreads) heads_topk_kernel(Geometry G, 
 
 // Section 4.2: P' = P + lambda * I * (1 - n_t / (l + 1)); the preserved tokens
 // stay, the rest of B - w goes to the largest P'; the last w tokens are kept.
-// Writes out_idx (ascending) and ORs the head's kept tokens into the layer's
-// union.  Grid (Hkv, batch).
+// Writes the head's kept positions as bits (sl.sel); gather_kernel turns them
+// into out_idx.  Grid (Hkv, batch).
 //
 // Coverage counts: n_t before this layer = A[t] + U_prev[t], where A is the
 // count array of the previous layer (the state for lcall = 0) and U_prev the
-// previous layer's union.  Every CTA reads them for its keys and writes the sum
-// for its slice of positions to the other count array, which is the next
-// layer's A; the last union is folded into the state by finalize_kernel.  No
-// CTA waits for another, and the previous layer's selection (a programmatic
-// dependency) is the only one this kernel waits for.
-__global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, LayerIO io, Scratch sc, Slot sl, int lcall,
-                                                                 int ncall) {
+// previous layer's union, the OR of its heads' kept bits (prev_sel; none for
+// lcall = 0).  Every CTA reads them for its keys and writes the sum for its
+// slice of positions to the other count array, which is the next layer's A;
+// finalize_kernel folds the last union into the state.  No CTA waits for
+// another, and the previous layer's selection (a programmatic dependency) is
+// the only one this kernel waits for: everything after that wait is the serial
+// part of a multi-layer call.
+__global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, LayerIO io, Scratch sc, Slot sl,
+                                                                 const uint32_t* prev_sel, int lcall, int ncall) {
     __shared__ TopkShared sm;
     extern __shared__ __align__(16) uint32_t bits[];
     const int h = blockIdx.x, s = blockIdx.y;
@@ -706,10 +708,11 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
     const int wordsL = (L + 31) >> 5;
     const int kw = key_stride(G);
     const bool cached = scores_in_smem(G.ML) && L > G.budget;
-    // Shared memory: bits[words] | preserved bits[words] | keys | P row | I row
-    // (P and I 16-byte aligned for float4 stores; what precedes them has any length).
+    // Shared memory: bits[words] | preserved bits[words] | union[words] | keys |
+    // P row | I row (P and I 16-byte aligned for float4 stores).
     uint32_t* spres = bits + G.words;
-    const size_t sp_off = ((size_t)2 * G.words + (keys_in_smem(G.ML) ? 32 * (size_t)kw : 0) + 3) & ~(size_t)3;
+    uint32_t* suni = spres + G.words;
+    const size_t sp_off = ((size_t)3 * G.words + (keys_in_smem(G.ML) ? 32 * (size_t)kw : 0) + 3) & ~(size_t)3;
     float* sP = reinterpret_cast<float*>(bits + sp_off);
     float* sI = sP + G.ML;
     const size_t row = (size_t)s * G.Hkv + h;
@@ -734,6 +737,14 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
     // From the second layer of a call on, the previous call's finalize has
     // completed before this grid could start, so the header is read early.
     uint32_t ell0 = lcall > 0 ? __ldcg(reinterpret_cast<const uint32_t*>(st)) : 0u;
+    uint8_t* nstate = st + G.state_n_off;
+    uint8_t* nscr = sc.nbuf + (size_t)s * G.nlen;
+    const uint8_t* nA = (lcall & 1) ? nscr : nstate;          // counts before the previous layer's union
+    uint8_t* nB = (lcall & 1) ? nstate : nscr;                // counts before this layer's union
+    // This CTA's slice of positions (a multiple of 32 long) for the next count array.
+    const int fper = (((L + G.Hkv - 1) / G.Hkv) + 31) & ~31;
+    const int f0 = min(h * fper, L), f1 = min(f0 + fper, L);
+    const bool select = L > G.budget;
     __syncthreads();
     // Launched as a programmatic dependent of the previous layer's selection:
     // everything above overlaps its tail; the coverage counts are read only after
@@ -745,39 +756,50 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
         return;
     }
     const uint32_t ell = ell0 + (uint32_t)lcall;
-    uint8_t* nstate = st + G.state_n_off;
-    uint8_t* nscr = sc.nbuf + (size_t)s * G.nlen;
-    const uint8_t* nA = (lcall & 1) ? nscr : nstate;          // counts before the previous layer's union
-    uint8_t* nB = (lcall & 1) ? nstate : nscr;                // counts before this layer's union
-    const size_t ustride = (size_t)G.batch * G.words;
-    const uint32_t* uprev = sc.ubits + (size_t)((lcall + 2) % 3) * ustride + (size_t)s * G.words;
-    uint32_t* ucur = sc.ubits + (size_t)(lcall % 3) * ustride + (size_t)s * G.words;
-    uint32_t* unext = sc.ubits + (size_t)((lcall + 1) % 3) * ustride + (size_t)s * G.words;
-    // This CTA's slice of positions (a multiple of 32 long) for the count arrays
-    // and of union words for clearing the next layer's union.
-    const int fper = (((L + G.Hkv - 1) / G.Hkv) + 31) & ~31;
-    const int f0 = min(h * fper, L), f1 = min(f0 + fper, L);
-    auto counts4 = [&](int t4, uchar4 a, uint32_t uw) {
-        const uint32_t b = uw >> (t4 & 31);
+    // One round of loads: this thread's first group of counts and the previous
+    // layer's union words (the OR over its heads' kept bits).
+    const int g0 = 4 * tid;
+    uchar4 nv0[4];
+    if (select) {
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int t4 = g0 + 4 * u * NT;
+            if (t4 < Lc) nv0[u] = *reinterpret_cast<const uchar4*>(nA + t4);
+        }
+    }
+    const uint32_t* prow = prev_sel ? prev_sel + (size_t)s * G.Hkv * G.words : nullptr;
+    for (int wd = tid; wd < wordsL; wd += NT) {
+        uint32_t u = 0u;
+        if (prow) {
+#pragma unroll 8
+            for (int hh = 0; hh < G.Hkv; ++hh) u |= __ldcg(&prow[(size_t)hh * G.words + wd]);
+        }
+        suni[wd] = u;
+    }
+    __syncthreads();
+    auto counts4 = [&](int t4, uchar4 a) {
+        const uint32_t b = suni[t4 >> 5] >> (t4 & 31);
         return make_uchar4((uint8_t)(a.x + (b & 1u)), (uint8_t)(a.y + ((b >> 1) & 1u)), (uint8_t)(a.z + ((b >> 2) & 1u)),
                            (uint8_t)(a.w + ((b >> 3) & 1u)));
     };
-    if (L > G.budget) {
-        float* Pp = sl.Pprime + row * G.ML;
-        uint32_t* keys = keys_in_smem(G.ML) ? spres + G.words : sc.keys_sel + row * G.ML;
+    if (select) {
+        // P' of the last layer of a call is kept for inspection (kvec_debug_scores).
+        float* Pp = lcall + 1 == ncall ? sl.Pprime + row * G.ML : nullptr;
+        uint32_t* keys = keys_in_smem(G.ML) ? suni + G.words : sc.keys_sel + row * G.ML;
         const float* Pr = cached ? sP : P;
         const float* Ir = cached ? sI : I;
-        const float denom = (float)(ell + 1u);
-        for (int b0 = 4 * tid; b0 < Lc; b0 += 16 * NT) {
+        // coverage = n_t / (l + 1) as n_t times the rounded reciprocal: a divide
+        // per position costs more than the rest of the key.
+        const float inv_l1 = __frcp_rn((float)(ell + 1u));
+        for (int b0 = g0; b0 < Lc; b0 += 16 * NT) {
             float4 pv[4], iv[4];
             uchar4 nv[4];
-            uint32_t pw[4], uw[4];
+            uint32_t pw[4];
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
                 const int t4 = b0 + 4 * u * NT;
                 if (t4 < Lc) {
-                    nv[u] = *reinterpret_cast<const uchar4*>(nA + t4);
-                    uw[u] = __ldcg(&uprev[t4 >> 5]);
+                    nv[u] = b0 == g0 ? nv0[u] : *reinterpret_cast<const uchar4*>(nA + t4);
                     pv[u] = *reinterpret_cast<const float4*>(Pr + t4);
                     iv[u] = *reinterpret_cast<const float4*>(Ir + t4);
                     pw[u] = spres[t4 >> 5];
@@ -787,7 +809,7 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
             for (int u = 0; u < 4; ++u) {
                 const int t4 = b0 + 4 * u * NT;
                 if (t4 >= Lc) continue;
-                const uchar4 c = counts4(t4, nv[u], uw[u]);
+                const uchar4 c = counts4(t4, nv[u]);
                 if (t4 >= f0 && t4 + 4 <= f1 && t4 + 4 <= Lc) *reinterpret_cast<uchar4*>(nB + t4) = c;
                 const float p4[4] = {pv[u].x, pv[u].y, pv[u].z, pv[u].w};
                 const float i4[4] = {iv[u].x, iv[u].y, iv[u].z, iv[u].w};
@@ -796,34 +818,35 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
                     const int t = t4 + i;
-                    const float coverage = (float)n4[i] / denom;
+                    const float coverage = (float)n4[i] * inv_l1;
                     const float pp = p4[i] + G.lambda * (i4[i] * (1.f - coverage));
                     out[i] = pp;
                     const bool kept = (pw[u] >> (t & 31)) & 1u;
                     if (t < Lc) keys[key_index(t, kw)] = kept ? 0u : float_order_key(pp);
                 }
-                *reinterpret_cast<float4*>(Pp + t4) = make_float4(out[0], out[1], out[2], out[3]);
+                if (Pp) *reinterpret_cast<float4*>(Pp + t4) = make_float4(out[0], out[1], out[2], out[3]);
             }
         }
         __syncthreads();
-        block_topk(keys, kw, Lc, G.k2, bits, sm);
-        // The next layer's selection may be scheduled now (it waits for this grid).
+        // The next layer's selection may be scheduled now: its staging overlaps
+        // this top-k, then it waits for this grid.
         asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
+        block_topk(keys, kw, Lc, G.k2, bits, sm);
         for (int wd = tid; wd < wordsL; wd += NT) bits[wd] |= spres[wd] | range_bits(wd, Lc, L);
     } else {
         // Every token is kept; the slice's counts still move to the next array.
-        for (int t4 = f0 + 4 * tid; t4 < min(f1, Lc & ~3); t4 += 4 * NT) {
-            const uchar4 c = counts4(t4, *reinterpret_cast<const uchar4*>(nA + t4), __ldcg(&uprev[t4 >> 5]));
-            *reinterpret_cast<uchar4*>(nB + t4) = c;
-        }
+        for (int t4 = f0 + 4 * tid; t4 < min(f1, Lc & ~3); t4 += 4 * NT)
+            *reinterpret_cast<uchar4*>(nB + t4) = counts4(t4, *reinterpret_cast<const uchar4*>(nA + t4));
         for (int wd = tid; wd < wordsL; wd += NT) bits[wd] = range_bits(wd, 0, L);
     }
+    // The head's kept positions, for the gather and the next layer.
+    uint32_t* out_bits = sl.sel + row * G.words;
+    for (int wd = tid; wd < wordsL; wd += NT) out_bits[wd] = bits[wd];
     // For the next layer only: the counts of this slice outside the candidates
-    // (the kept window; positions from L on keep what the array holds) and the
-    // slice's words of the next layer's union, cleared.
+    // (the kept window; positions from L on keep what the array holds).
     for (int t4 = max(f0, Lc & ~3) + 4 * tid; t4 < f1; t4 += 4 * NT) {
         if (t4 + 4 <= Lc) continue;   // written with the candidates
-        const uchar4 c = counts4(t4, *reinterpret_cast<const uchar4*>(nA + t4), __ldcg(&uprev[t4 >> 5]));
+        const uchar4 c = counts4(t4, *reinterpret_cast<const uchar4*>(nA + t4));
         if (t4 + 4 <= L) {
             *reinterpret_cast<uchar4*>(nB + t4) = c;
         } else {
@@ -831,50 +854,35 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
             for (int i = 0; t4 + i < L; ++i) nB[t4 + i] = c4[i];
         }
     }
-    for (int wd = (f0 >> 5) + tid; wd < ((f1 + 31) >> 5); wd += NT) unext[wd] = 0u;
-    __syncthreads();
-
-    // Ascending positions: each thread owns a contiguous run of words.
-    int32_t* oi = io.out_idx + ((size_t)s * G.Hkv + h) * G.budget;
-    const int wpt = (wordsL + NT - 1) / NT;
-    const int w_lo = min(tid * wpt, wordsL), w_hi = min(w_lo + wpt, wordsL);
-    int mine = 0;
-    for (int wd = w_lo; wd < w_hi; ++wd) mine += __popc(bits[wd]);
-    int total;
-    int pos = block_exclusive_sum(mine, sm.wsum, total);
-    for (int wd = w_lo; wd < w_hi; ++wd) {
-        uint32_t b = bits[wd];
-        while (b) {
-            const int bit = __ffs(b) - 1;
-            b &= b - 1u;
-            if (pos < G.budget) oi[pos] = wd * 32 + bit;
-            ++pos;
-        }
-    }
-    for (int j = total + tid; j < G.budget; j += NT) oi[j] = -1;
-
-    // Union over heads (Section 4.2); nothing waits for it within this grid.
-    for (int wd = tid; wd < wordsL; wd += NT)
-        if (bits[wd]) atomicOr(&ucur[wd], bits[wd]);
 }
 
 // After the last layer of a call: n_t of the state = the last count array plus
-// the last union, last_union = that union, layers_done and seqlen updated.
-// Grid (batch).
-__global__ void __launch_bounds__(kSelectThreads) finalize_kernel(Geometry G, LayerIO io, Scratch sc, int ncall) {
+// the last union (the OR of the last layer's kept bits over heads), last_union
+// = that union, layers_done and seqlen updated.  Grid (batch).
+__global__ void __launch_bounds__(kSelectThreads) finalize_kernel(Geometry G, LayerIO io, Scratch sc, Slot last,
+                                                                   int ncall) {
     const int s = blockIdx.x, tid = threadIdx.x, NT = blockDim.x;
     asm volatile("griddepcontrol.wait;\n" ::: "memory");
     const int L = io.cu[s + 1] - io.cu[s];
+    const int wordsL = (L + 31) >> 5;
     uint8_t* st = io.state + (size_t)s * G.state_stride;
     const uint32_t ell0 = reinterpret_cast<const uint32_t*>(st)[0];
     if (ell0 + (uint32_t)ncall > 255u) return;   // the select kernels reported it and wrote nothing
     const int l = ncall - 1;
     uint8_t* nstate = st + G.state_n_off;
     const uint8_t* nlast = (l & 1) ? nstate : sc.nbuf + (size_t)s * G.nlen;   // written by the last layer
-    const uint32_t* ulast = sc.ubits + (size_t)(l % 3) * G.batch * G.words + (size_t)s * G.words;
+    const uint32_t* srow = last.sel + (size_t)s * G.Hkv * G.words;
+    uint32_t* last_union = reinterpret_cast<uint32_t*>(st + G.state_union_off);
+    for (int wd = tid; wd < G.words; wd += NT) {
+        uint32_t u = 0u;
+        if (wd < wordsL)
+            for (int hh = 0; hh < G.Hkv; ++hh) u |= __ldcg(&srow[(size_t)hh * G.words + wd]);
+        last_union[wd] = u;
+    }
+    __syncthreads();   // the union words are read back below by other threads
     for (int t4 = 4 * tid; t4 < L; t4 += 4 * NT) {
         const uchar4 a = *reinterpret_cast<const uchar4*>(nlast + t4);
-        const uint32_t b = __ldcg(&ulast[t4 >> 5]) >> (t4 & 31);
+        const uint32_t b = last_union[t4 >> 5] >> (t4 & 31);
         const uint8_t c4[4] = {(uint8_t)(a.x + (b & 1u)), (uint8_t)(a.y + ((b >> 1) & 1u)),
                                (uint8_t)(a.z + ((b >> 2) & 1u)), (uint8_t)(a.w + ((b >> 3) & 1u))};
         if (t4 + 4 <= L) {
@@ -883,24 +891,53 @@ __global__ void __launch_bounds__(kSelectThreads) finalize_kernel(Geometry G, La
             for (int i = 0; t4 + i < L; ++i) nstate[t4 + i] = c4[i];
         }
     }
-    uint32_t* last_union = reinterpret_cast<uint32_t*>(st + G.state_union_off);
-    for (int wd = tid; wd < G.words; wd += NT) last_union[wd] = __ldcg(&ulast[wd]);
     if (tid == 0) {
         reinterpret_cast<uint32_t*>(st)[0] = ell0 + (uint32_t)ncall;
         reinterpret_cast<uint32_t*>(st)[1] = (uint32_t)L;
     }
 }
 
-// out_k[s,h,j,:] = K[cu[s] + idx[s,h,j], h, :] (zeros for idx = -1); the same for V.
-// Grid (ceil(B/16), Hkv, batch), 256 threads: a half-warp moves one 256-byte row.
-__global__ void __launch_bounds__(256) gather_kernel(Geometry G, LayerIO io) {
+// out_idx[s,h,j] = position of the j-th kept bit of (s, h) (-1 past the last);
+// out_k[s,h,j,:] = K[cu[s] + idx, h, :] (zeros for idx = -1); the same for V.
+// Grid (ceil(B/16), Hkv, batch), 256 threads: the block finds its 16 ranks from
+// a prefix count over the row's bits words, then a half-warp moves one 256-byte row.
+__global__ void __launch_bounds__(256) gather_kernel(Geometry G, LayerIO io, Slot sl) {
+    __shared__ int wsum[32];
+    __shared__ int spos[16];
     const int s = blockIdx.z, h = blockIdx.y;
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int row = blockIdx.x * 16 + warp * 2 + (lane >> 4), sub = lane & 15;
-    if (row >= G.budget) return;
-    const size_t orow = ((size_t)s * G.Hkv + h) * G.budget + row;
-    const int idx = io.out_idx[orow];
+    const int tid = threadIdx.x, NT = blockDim.x;
+    const int lane = tid & 31, warp = tid >> 5;
     const int L = io.cu[s + 1] - io.cu[s];
+    const int wordsL = (L + 31) >> 5;
+    const size_t srow = (size_t)s * G.Hkv + h;
+    const uint32_t* sel = sl.sel + srow * G.words;
+    const int r0 = blockIdx.x * 16;
+    if (tid < 16) spos[tid] = -1;
+    // Contiguous runs of words per thread, ranked by an exclusive prefix sum.
+    const int wpt = (wordsL + NT - 1) / NT;
+    const int w_lo = min(tid * wpt, wordsL), w_hi = min(w_lo + wpt, wordsL);
+    int mine = 0;
+    for (int wd = w_lo; wd < w_hi; ++wd) mine += __popc(__ldcg(&sel[wd]));
+    int total;
+    int rank = block_exclusive_sum(mine, wsum, total);   // its barriers also order spos's initialisation
+    if (rank < r0 + 16 && rank + mine > r0) {
+        for (int wd = w_lo; wd < w_hi && rank < r0 + 16; ++wd) {
+            uint32_t b = __ldcg(&sel[wd]);
+            while (b && rank < r0 + 16) {
+                const int bit = __ffs(b) - 1;
+                b &= b - 1u;
+                if (rank >= r0) spos[rank - r0] = wd * 32 + bit;
+                ++rank;
+            }
+        }
+    }
+    __syncthreads();
+    const int rloc = warp * 2 + (lane >> 4), sub = lane & 15;
+    const int j = r0 + rloc;
+    if (j >= G.budget) return;
+    const size_t orow = srow * G.budget + j;
+    const int idx = spos[rloc];
+    if (sub == 0) io.out_idx[orow] = idx;
     uint4 kv = make_uint4(0, 0, 0, 0), vv = make_uint4(0, 0, 0, 0);
     if (idx >= 0 && idx < L) {
         const size_t src = (((size_t)io.cu[s] + idx) * G.Hkv + h) * kHeadDim + sub * 8;
@@ -914,7 +951,7 @@ __global__ void __launch_bounds__(256) gather_kernel(Geometry G, LayerIO io) {
 }  // namespace
 
 size_t select_smem_bytes(const Geometry& g) {
-    const size_t head = ((size_t)2 * g.words + (keys_in_smem(g.ML) ? 32 * (size_t)key_stride(g) : 0) + 3) & ~(size_t)3;
+    const size_t head = ((size_t)3 * g.words + (keys_in_smem(g.ML) ? 32 * (size_t)key_stride(g) : 0) + 3) & ~(size_t)3;
     return sizeof(uint32_t) * (head + (scores_in_smem(g.ML) ? 2 * (size_t)g.ML : 0));
 }
 
@@ -926,9 +963,9 @@ cudaError_t configure_select() {
     const int need = (int)(sizeof(uint32_t) * (kSmemKeys / 32 + 32 * ((kSmemKeys / 32) | 1)));
     // The select kernel also keeps the preserved bits and caches P and I rows
     // up to kSmemScores positions.
-    const int need_sel_keys = need + (int)(sizeof(uint32_t) * (kSmemKeys / 32 + 4));
+    const int need_sel_keys = need + (int)(sizeof(uint32_t) * (2 * (kSmemKeys / 32) + 4));
     const int need_sel_scores =
-        (int)(sizeof(uint32_t) * (2 * (kSmemScores / 32) + 32 * ((kSmemScores / 32) | 1) + 2 * kSmemScores + 64));
+        (int)(sizeof(uint32_t) * (3 * (kSmemScores / 32) + 32 * ((kSmemScores / 32) | 1) + 2 * kSmemScores + 64));
     const int need_sel = need_sel_keys > need_sel_scores ? need_sel_keys : need_sel_scores;
     cudaError_t e = cudaFuncSetAttribute(heads_topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, need);
     if (e == cudaSuccess)
@@ -949,20 +986,21 @@ cudaError_t launch_heads(const Geometry& g, const LayerIO& io, const Scratch& sc
     return e;
 }
 
-cudaError_t launch_select(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st,
-                          int priority, int lcall, int ncall) {
+cudaError_t launch_select(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, const Slot* prev,
+                          cudaStream_t st, int priority, int lcall, int ncall) {
+    const uint32_t* prev_sel = prev ? prev->sel : nullptr;
     return launch_prio(select_kernel, dim3(g.Hkv, g.batch), dim3(kSelectThreads), select_smem_bytes(g), st, priority,
-                       /*programmatic=*/true, g, io, sc, sl, lcall, ncall);
+                       /*programmatic=*/true, g, io, sc, sl, prev_sel, lcall, ncall);
 }
 
-cudaError_t launch_finalize(const Geometry& g, const LayerIO& io, const Scratch& sc, cudaStream_t st, int priority,
-                            int ncall) {
+cudaError_t launch_finalize(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& last, cudaStream_t st,
+                            int priority, int ncall) {
     return launch_prio(finalize_kernel, dim3(g.batch), dim3(kSelectThreads), 0, st, priority, /*programmatic=*/true, g,
-                       io, sc, ncall);
+                       io, sc, last, ncall);
 }
 
-void launch_gather(const Geometry& g, const LayerIO& io, cudaStream_t st) {
-    gather_kernel<<<dim3((g.budget + 15) / 16, g.Hkv, g.batch), 256, 0, st>>>(g, io);
+void launch_gather(const Geometry& g, const LayerIO& io, const Slot& sl, cudaStream_t st) {
+    gather_kernel<<<dim3((g.budget + 15) / 16, g.Hkv, g.batch), 256, 0, st>>>(g, io, sl);
 }
 
 }  // namespace kvec

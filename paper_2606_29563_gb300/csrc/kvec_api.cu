@@ -47,7 +47,7 @@ struct TimedLaunch {
 
 }  // namespace
 
-constexpr int kSlots = 4;   // per-layer score arrays in flight between the score and select stages
+constexpr int kSlots = 8;   // per-layer score arrays in flight between the score and select stages
 
 struct kvec_handle {
     kvec_params p;

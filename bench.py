@@ -164,7 +164,7 @@ def committed_traffic(kernel: str, workload: str):
         return None
 
 
-LAUNCHES_PER_LAYER = 6
+LAUNCHES_PER_LAYER = 7   # score, row statistics, window, heads pooling, heads top-K, select, gather
 
 
 def workload_bytes(wl):
@@ -312,8 +312,9 @@ def run_ours(args, wl):
     # End to end through the public API: pinned host inputs copied in, indices and state copied out.
     e2e = run_e2e(args, wl, sel, layers, outs, state, cu_host, cu_dev, dev, stream) if args.e2e else None
 
-    # Per layer: score, window, heads pooling, heads top-K, select, gather.
-    gpu_launches = args.steps * L_layers * LAUNCHES_PER_LAYER
+    # Per layer: score, row statistics, window, heads pooling, heads top-K, select,
+    # gather; per call one finalize launch (the last layer's union into the state).
+    gpu_launches = args.steps * (L_layers * LAUNCHES_PER_LAYER + 1)
     sel.close()
     result = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,

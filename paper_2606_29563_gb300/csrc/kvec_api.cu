@@ -227,6 +227,8 @@ kvec_status run_layer_sequential(kvec_handle* h, const Geometry& G, const LayerI
     if (se != cudaSuccess) return cuda_fail(se, "score kernel tensor maps");
     se = launch_score(plan, st, false);
     if (se != cudaSuccess) return cuda_fail(se, "score kernel launch");
+    se = launch_rowstat(plan, G, io, h->sc, st);
+    if (se != cudaSuccess) return cuda_fail(se, "row statistics launch");
     se = launch_window(plan, G, io, h->sc, h->slots[0], st, false);
     if (se != cudaSuccess) return cuda_fail(se, "window kernel launch");
     se = launch_heads(G, io, h->sc, h->slots[0], st, h->prio_hi);
@@ -263,7 +265,10 @@ kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* io
         ScorePlan plan;
         cudaError_t se = plan_score(G, io, sc, h->num_sms, &plan);
         if (se != cudaSuccess) return cuda_fail(se, "score kernel tensor maps");
-        timed_launch(h, 0, h->s_score, [&] { se = launch_score(plan, h->s_score, true); });
+        timed_launch(h, 0, h->s_score, [&] {
+            se = launch_score(plan, h->s_score, true);
+            if (se == cudaSuccess) se = launch_rowstat(plan, G, io, sc, h->s_score);
+        });
         if (se != cudaSuccess) return cuda_fail(se, "score kernel launch");
         KV_CHECK(cudaEventRecord(h->ev_score[l], h->s_score));
         KV_CHECK(cudaStreamWaitEvent(h->s_win, h->ev_score[l], 0));
@@ -396,7 +401,6 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
         Scratch& b = h->score_buf[k];
         std::vector<Part> sp = {
             {(void**)&b.segpart, max_tiles * Hkv * R * sizeof(float2)},
-            {(void**)&b.shcount, MB * Hkv * sizeof(unsigned)},
             {(void**)&b.rowstat, MB * Hkv * R * sizeof(float2)},
         };
         parts.insert(parts.end(), sp.begin(), sp.end());
@@ -665,8 +669,7 @@ kvec_status kvec_select_layer_noalloc(const kvec_params* params, int batch, cons
     const size_t HGv = Hkv < (size_t)kWinHeadsPerCta ? Hkv : (size_t)kWinHeadsPerCta;
     const size_t NGv = (Hkv + HGv - 1) / HGv;
     Part parts[] = {
-        {(void**)&tmp.sc.err, sizeof(int)},                   // zeroed every call (first two parts)
-        {(void**)&tmp.sc.shcount, nb * Hkv * sizeof(unsigned)},
+        {(void**)&tmp.sc.err, sizeof(int)},                   // zeroed every call (the first part)
         {(void**)&tmp.sc.nbuf, nb * round_up((size_t)params->max_seqlen, 16)},
         {(void**)&tmp.sc.segpart, nt * Hkv * R * sizeof(float2)},
         {(void**)&tmp.slots[0].wpart, nt * NGv * (size_t)params->obs_window * kTileT * sizeof(float)},
@@ -688,7 +691,7 @@ kvec_status kvec_select_layer_noalloc(const kvec_params* params, int batch, cons
     size_t need = 0, zero_bytes = 0;
     for (size_t i = 0; i < sizeof(parts) / sizeof(parts[0]); ++i) {
         need += round_up(parts[i].bytes, 256);
-        if (i == 1) zero_bytes = need;
+        if (i == 0) zero_bytes = need;
     }
     if (need > kNoallocScratchBytes)
         return fail(KVEC_ERR_INVALID_ARG,
@@ -713,7 +716,7 @@ kvec_status kvec_select_layer_noalloc(const kvec_params* params, int batch, cons
         off += round_up(pt.bytes, 256);
     }
     cudaStream_t st = (cudaStream_t)stream;
-    // The array keeps the previous call's contents: the error word and tile counters must start at zero.
+    // The array keeps the previous call's contents: the error word must start at zero.
     e = cudaMemsetAsync(base, 0, zero_bytes, st);
     if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync(scratch)");
     LayerIO io{};

@@ -53,8 +53,7 @@ struct Slot {
 
 struct Scratch {
     float2* segpart;      // [total_tiles * Hkv][R] per-CTA segment (max, sum), keyed by the segment's first item
-    unsigned* shcount;    // [max_batch][Hkv]       tiles finished per (sequence, KV head)
-    float2* rowstat;      // [max_batch][Hkv][R]    (row max in log2 units, softmax denominator)
+    float2* rowstat;      // [max_batch][Hkv][R]    (row max in log2 units, softmax denominator), for inspection
     uint32_t* keys;       // [max_batch][Hkv][ML]   radix-select keys of the heads kernel
     uint32_t* keys_sel;   // [max_batch][Hkv][ML]   radix-select keys of the select kernel
     uint8_t* nbuf;        // [max_batch][nlen]      second copy of n_t (the coverage counts alternate)
@@ -109,6 +108,9 @@ cudaError_t plan_score(const Geometry& g, const LayerIO& io, const Scratch& sc, 
 // of the same kernel (the multi-stream layer pipeline); the launch may then
 // overlap it (programmatic stream serialization), as it reads none of its results.
 cudaError_t launch_score(const ScorePlan& plan, cudaStream_t st, bool after_own_launch);
+// (m_r, Z_r) from the score launch's partials; launched right after it on the same stream.
+cudaError_t launch_rowstat(const ScorePlan& plan, const Geometry& g, const LayerIO& io, const Scratch& sc,
+                           cudaStream_t st);
 cudaError_t launch_window(const ScorePlan& sp, const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl,
                           cudaStream_t st, bool after_own_launch);
 // Launches kernel<<<grid, block, smem, st>>> with a scheduling priority (lower

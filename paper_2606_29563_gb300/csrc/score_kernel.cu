@@ -14,8 +14,8 @@
 //               2^(s - max), merged online into the thread's running
 //               (max, sum) of the CTA's contiguous segment of (s, h).
 // At the end of a segment the column splits merge in shared memory and the CTA
-// writes one (max, sum) partial per row; the last CTA to finish a (s, h) merges
-// the partials into rowstat[s][h][r] = (m_r, Z_r).
+// writes one (max, sum) partial per row, keyed by the segment's first item;
+// rowstat_kernel then merges the partials of a (s, h) into (m_r, Z_r).
 // The window kernel recomputes the logits with these statistics.
 #include <cudaTypedefs.h>
 
@@ -101,7 +101,6 @@ struct __align__(8) Barriers {
     uint64_t mma_done;
     uint32_t tmem_base;
     volatile int abort_flag;
-    volatile int last_flag;
     float2 xf[512];            // a segment's (max, sum) per column split and row, merged at its end
 };
 
@@ -256,7 +255,6 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         // quarter its warp id allows) of M-block m, columns [COLS*split, +COLS).
         // Each warp waits for the accumulators itself; the warps meet only when a
         // segment ends.
-        const int epi = threadIdx.x - 64;                   // 0 .. kEpiThreads-1
         const int ew = warp - 2;
         const int m = (ew >> 2) % MB;
         const int split = (ew >> 2) / MB;
@@ -264,10 +262,9 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         const int row = m * 128 + quad * 32 + lane;
         const bool vrow = row < R;
         const int q = vrow ? row / G.g : 0;
-        const bool issuer = epi == 0;
         bool aborted = false;
         float seg_m = -INFINITY, seg_z = 0.f;
-        int cur_sh = -1, seg_first = 0, seg_n = 0, seg_s = 0, seg_h = 0, seg_ibase = 0, seg_nt = 0;
+        int cur_sh = -1, seg_first = 0;
 
         auto merge = [](float& M, float& Z, float2 o) {
             if (o.x == -INFINITY) return;
@@ -279,7 +276,9 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
             }
         };
         // Every epilogue thread calls this at the same segment boundaries (aborted
-        // warps included), so the named barriers always complete.
+        // warps included), so the named barriers always complete.  The column
+        // splits merge here; rowstat_kernel merges the CTAs' partials of a
+        // (sequence, head) into (m_r, Z_r).
         auto flush_segment = [&]() {
             bars->xf[split * Rpad + row] = make_float2(seg_m, seg_z);
             ptx::named_bar_sync(1, kEpiThreads);
@@ -289,41 +288,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                 for (int c = 1; c < CS; ++c) merge(M, Z, bars->xf[c * Rpad + row]);
                 if (vrow) sc.segpart[(size_t)seg_first * R + row] = make_float2(M, Z);
             }
-            ptx::named_bar_sync(1, kEpiThreads);
-            if (issuer) {
-                // The barrier orders the CTA's writes before this thread's fence (cumulativity).
-                __threadfence();
-                const unsigned old = atomicAdd(&sc.shcount[seg_s * G.Hkv + seg_h], (unsigned)seg_n);
-                __threadfence();
-                bars->last_flag = old + (unsigned)seg_n == (unsigned)seg_nt;
-            }
-            ptx::named_bar_sync(1, kEpiThreads);
-            if (bars->last_flag && split == 0) {
-                // Merge the partials of (s, h): the first item, then each CTA range
-                // start after it, loaded in independent batches.
-                float M = -INFINITY, Z = 0.f;
-                const int qW = W / Gc, rW = W % Gc;
-                const int iend = seg_ibase + seg_nt;
-                auto cta_of = [&](int i) { return i < rW * (qW + 1) ? i / (qW + 1) : rW + (i - rW * (qW + 1)) / qW; };
-                int b = cta_of(seg_ibase) + 1;
-                int next = seg_ibase;
-                while (next < iend) {
-                    float2 pz[16];
-#pragma unroll
-                    for (int k = 0; k < 16; ++k) {
-                        pz[k] = make_float2(-INFINITY, 0.f);
-                        if (next < iend) {
-                            if (vrow) pz[k] = __ldcg(&sc.segpart[(size_t)next * R + row]);
-                            next = b * qW + min(b, rW);
-                            ++b;
-                        }
-                    }
-#pragma unroll
-                    for (int k = 0; k < 16; ++k) merge(M, Z, pz[k]);
-                }
-                if (vrow) sc.rowstat[((size_t)seg_s * G.Hkv + seg_h) * R + row] = make_float2(M, Z);
-                if (issuer) sc.shcount[seg_s * G.Hkv + seg_h] = 0u;
-            }
+            ptx::named_bar_sync(1, kEpiThreads);   // xf is free for the next segment
         };
 
         ItemWalker p;
@@ -336,13 +301,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                 seg_m = -INFINITY;
                 seg_z = 0.f;
                 seg_first = i;
-                seg_n = 0;
-                seg_s = p.s;
-                seg_h = p.h;
-                seg_ibase = p.ibase;
-                seg_nt = p.ntiles;
             }
-            ++seg_n;
             if (aborted) continue;   // keep walking the items for the segment barriers
             const int buf = it % NB, nb = it / NB;
             int ok = 1;
@@ -401,6 +360,52 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     __syncthreads();
     ptx::tc_fence_after();
     if (warp == 1) ptx::tmem_dealloc(tmem, kTmemCols);
+}
+
+// (m_r, Z_r) of every row of (s, h) from the score CTAs' segment partials: one
+// at the head's first item, then one at every score CTA's first item inside
+// the head's range of items.  Grid (Hkv, batch), one thread per row.
+__global__ void __launch_bounds__(256) rowstat_kernel(Geometry G, Scratch sc, const int* __restrict__ cu, int W,
+                                                      int Gc) {
+    // A programmatic dependent of the score launch: its partials are read only
+    // after that grid has completed.
+    if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
+    asm volatile("griddepcontrol.wait;\n" ::: "memory");
+    const int h = blockIdx.x, s = blockIdx.y, r = threadIdx.x;
+    if (r >= G.R) return;
+    int ib = 0;
+    for (int b = 0; b < s; ++b) ib += tiles_of(__ldg(&cu[b + 1]) - __ldg(&cu[b])) * G.Hkv;
+    const int nt = tiles_of(__ldg(&cu[s + 1]) - __ldg(&cu[s]));
+    ib += h * nt;
+    const int iend = ib + nt;
+    const int qW = W / Gc, rW = W % Gc;
+    const int cta = ib < rW * (qW + 1) ? ib / (qW + 1) : rW + (ib - rW * (qW + 1)) / qW;
+    float M = -INFINITY, Z = 0.f;
+    int next = ib, b = cta + 1;
+    while (next < iend) {
+        float2 pz[16];
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+            pz[k] = make_float2(-INFINITY, 0.f);
+            if (next < iend) {
+                pz[k] = __ldcg(&sc.segpart[(size_t)next * G.R + r]);
+                next = b * qW + min(b, rW);
+                ++b;
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+            const float2 o = pz[k];
+            if (o.x == -INFINITY) continue;
+            if (o.x > M) {
+                Z = Z * ptx::ex2(M - o.x) + o.y;
+                M = o.x;
+            } else {
+                Z += o.y * ptx::ex2(o.x - M);
+            }
+        }
+    }
+    sc.rowstat[((size_t)s * G.Hkv + h) * G.R + r] = make_float2(M, Z);
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
@@ -494,6 +499,21 @@ cudaError_t plan_score(const Geometry& g, const LayerIO& io, const Scratch& sc, 
     plan->mb = mblocks(g);
     plan->smem = smem_bytes_for(g);
     return cudaSuccess;
+}
+
+cudaError_t launch_rowstat(const ScorePlan& plan, const Geometry& g, const LayerIO& io, const Scratch& sc,
+                           cudaStream_t st) {
+    const ScoreArgs& a = *reinterpret_cast<const ScoreArgs*>(plan.args);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(g.Hkv, g.batch);
+    cfg.blockDim = dim3(256);
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, rowstat_kernel, g, sc, io.cu, a.W, plan.grid);
 }
 
 cudaError_t launch_score(const ScorePlan& plan, cudaStream_t st, bool after_own_launch) {

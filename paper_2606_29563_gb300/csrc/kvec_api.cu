@@ -48,6 +48,7 @@ struct TimedLaunch {
 }  // namespace
 
 constexpr int kSlots = 8;   // per-layer score arrays in flight between the score and select stages
+constexpr int kScoreBufs = 2;   // score-statistics buffers in flight between the score and window stages
 
 struct kvec_handle {
     kvec_params p;
@@ -58,7 +59,7 @@ struct kvec_handle {
     void* ws = nullptr;
     size_t ws_bytes = 0;
     Scratch sc{};
-    Scratch score_buf[2]{};   // e-buffer, tile/segment/row statistics, counters: one per layer parity
+    Scratch score_buf[kScoreBufs]{};   // segment partials and row statistics, one per layer in flight
     Slot slots[kSlots]{};
     int last_slot = 0, last_parity = 0;
     int last_batch = 0;
@@ -259,9 +260,9 @@ kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* io
         KV_CHECK(cudaStreamWaitEvent(st, h->ev_fork, 0));
     for (int l = 0; l < n; ++l) {
         const Slot& sl = h->slots[l % kSlots];
-        const Scratch& sc = h->score_buf[l & 1];
+        const Scratch& sc = h->score_buf[l % kScoreBufs];
         const LayerIO& io = ios[l];
-        if (l >= 2) KV_CHECK(cudaStreamWaitEvent(h->s_score, h->ev_win[l - 2], 0));
+        if (l >= kScoreBufs) KV_CHECK(cudaStreamWaitEvent(h->s_score, h->ev_win[l - kScoreBufs], 0));
         ScorePlan plan;
         cudaError_t se = plan_score(G, io, sc, h->num_sms, &plan);
         if (se != cudaSuccess) return cuda_fail(se, "score kernel tensor maps");
@@ -299,7 +300,7 @@ kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* io
     }
     // The last layer's union goes into the state.
     {
-        cudaError_t se = launch_finalize(G, ios[n - 1], h->score_buf[(n - 1) & 1], h->slots[(n - 1) % kSlots], h->s_chain,
+        cudaError_t se = launch_finalize(G, ios[n - 1], h->score_buf[(n - 1) % kScoreBufs], h->slots[(n - 1) % kSlots], h->s_chain,
                                          h->prio_hi, n);
         if (se != cudaSuccess) return cuda_fail(se, "finalize kernel launch");
     }
@@ -313,7 +314,7 @@ kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* io
     KV_CHECK(cudaStreamWaitEvent(origin, h->ev_fork, 0));
     for (cudaEvent_t e : h->ev_join) KV_CHECK(cudaStreamWaitEvent(origin, e, 0));
     h->last_slot = (n - 1) % kSlots;
-    h->last_parity = (n - 1) & 1;
+    h->last_parity = (n - 1) % kScoreBufs;
     return KVEC_OK;
 }
 
@@ -397,7 +398,7 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
         {(void**)&h->sc.err, sizeof(int)},
         {(void**)&h->sc.keys_sel, MB * Hkv * ML * sizeof(uint32_t)},
     };
-    for (int k = 0; k < 2; ++k) {
+    for (int k = 0; k < kScoreBufs; ++k) {
         Scratch& b = h->score_buf[k];
         std::vector<Part> sp = {
             {(void**)&b.segpart, max_tiles * Hkv * R * sizeof(float2)},
@@ -555,7 +556,7 @@ kvec_status kvec_select_layers(kvec_handle* h, int num_layers, int batch, const 
         if (h->gexec && key == h->gkey) {
             KV_CHECK(cudaGraphLaunch(h->gexec, st));
             h->last_slot = (num_layers - 1) % kSlots;
-            h->last_parity = (num_layers - 1) & 1;
+            h->last_parity = (num_layers - 1) % kScoreBufs;
             h->last_batch = batch;
             return KVEC_OK;
         }

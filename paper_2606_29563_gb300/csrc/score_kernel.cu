@@ -330,6 +330,25 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
             if (lane == 0) ptx::mbar_arrive(&bars->acc_empty[buf]);
             const int lim = nvalid - c0;
             if (lim <= 0) continue;
+            if (lim >= COLS && seg_m != -INFINITY) {
+                // Relative to the segment's running reference seg_m: 2^(s - seg_m) sums
+                // the same mass as the online max/rescale, without a max pass.  A tile
+                // far above the reference (sum not below 2^64) takes the exact path.
+                float z4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+                for (int c = 0; c < COLS; ++c) z4[c & 3] += ptx::ex2(fmaf(v[c], G.sl2, -seg_m));
+                const float z = (z4[0] + z4[1]) + (z4[2] + z4[3]);
+                if (z < 0x1p64f) {
+                    seg_z += z;
+                    if (seg_z >= 0x1p40f) {
+                        // Keep the sum bounded: move a power of two into the reference.
+                        const int k = ilogbf(seg_z);
+                        seg_m += (float)k;
+                        seg_z = ldexpf(seg_z, -k);
+                    }
+                    continue;
+                }
+            }
             float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
             if (lim >= COLS) {
 #pragma unroll

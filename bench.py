@@ -16,6 +16,7 @@ from __future__ import annotations
 import argparse
 import hashlib
 import json
+import math
 import os
 import statistics
 import subprocess
@@ -222,6 +223,26 @@ def oracle_baseline(wl, budget_s: float = 12.0, max_layers: int = 8, cap_s: floa
                       f"(fp64 C oracle, OpenMP), {layers} layers in {spent:.1f} s of CPU work"}
 
 
+def window_lse_torch(wl, x, dev):
+    """Log-sum-exp of every window query row over the keys it sees, [batch][w][H_q]
+    fp32: what a caller's prefill attention hands to kvec_select_layers_lse.
+    Input preparation for the lse variant (torch, outside the timed region)."""
+    import torch
+    w, Hq, Hkv, d = wl.window, wl.num_q_heads, wl.num_kv_heads, wl.head_dim
+    g, scale = Hq // Hkv, 1.0 / math.sqrt(d)
+    out = torch.empty(wl.batch, w, Hq, dtype=torch.float32, device=dev)
+    cu = wl.cu_seqlens
+    for s in range(wl.batch):
+        L = cu[s + 1] - cu[s]
+        q = x["q_obs"][s].float()                                        # [w, Hq, d]
+        k = x["k"][cu[s]:cu[s + 1]].float().repeat_interleave(g, dim=1)  # [L, Hq, d]
+        logits = torch.einsum("qhd,thd->hqt", q, k) * scale              # [Hq, w, L]
+        hidden = torch.arange(L, device=dev)[None, :] > (L - w + torch.arange(w, device=dev))[:, None]
+        logits.masked_fill_(hidden[None], float("-inf"))
+        out[s] = torch.logsumexp(logits, dim=2).transpose(0, 1)
+    return out
+
+
 # ----------------------------------------------------------------------------- our arm
 
 def run_ours(args, wl):
@@ -309,6 +330,33 @@ def run_ours(args, wl):
     dom = max(per_kernel, key=lambda k: ktimes[k]["share"] or 0.0)
     path_gbs = by["layer_total"] * L_layers / (ms_per_step / 1e3) / 1e9
 
+    # The same step with the window rows' log-sum-exp supplied by the caller
+    # (kvec_select_layers_lse, no statistics pass over K); the lse inputs are
+    # prepared outside the timed region.
+    lse_variant = None
+    if args.lse_variant:
+        lses = [window_lse_torch(wl_rank, x, dev) for x in layers]
+
+        def step_lse():
+            kvec.kvec_reset(sel.handle, state.data_ptr(), wl.batch, stream.cuda_stream)
+            sel.select_layers(cu_host, cu_dev, qs, ks, vs, state, wl.budget, outs, stream, lses=lses)
+
+        for _ in range(max(args.warmup, 3)):
+            step_lse()
+        n_lse = min(args.steps, 500)
+        torch.cuda.synchronize()
+        start.record(stream)
+        for _ in range(n_lse):
+            step_lse()
+        stop.record(stream)
+        torch.cuda.synchronize()
+        kvec.kvec_sync_status(sel.handle)
+        ms_lse = max_over_ranks(start.elapsed_time(stop), dev) / n_lse
+        lse_variant = {"metric": METRIC, "value": world * evicted_per_step / (ms_lse / 1e3), "unit": "tokens/s",
+                       "ms_per_step": ms_lse, "steps": n_lse,
+                       "api": "kvec_select_layers_lse: window-row log-sum-exp from the caller's prefill attention",
+                       "path_roofline_frac": by["layer_total"] * L_layers / (ms_lse / 1e3) / 1e9 / peak}
+
     # End to end through the public API: pinned host inputs copied in, indices and state copied out.
     e2e = run_e2e(args, wl, sel, layers, outs, state, cu_host, cu_dev, dev, stream) if args.e2e else None
 
@@ -334,6 +382,7 @@ def run_ours(args, wl):
         "kernels": ktimes,
         "clocks": {k: v for k, v in clocks.summary(t_host0, t_host1).items()},
         "gpu_launches": gpu_launches,
+        "lse_variant": lse_variant,
         "e2e": e2e,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -428,6 +477,8 @@ def main(argv=None):
     ap.add_argument("--layers", type=int, default=None, help="run only the first N layers (not a bench line)")
     ap.add_argument("--no-e2e", dest="e2e", action="store_false")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-lse-variant", dest="lse_variant", action="store_false",
+                    help="skip timing the kvec_select_layers_lse variant")
     args = ap.parse_args(argv)
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3

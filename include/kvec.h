@@ -131,6 +131,33 @@ KVEC_API kvec_status kvec_select_layers(kvec_handle* h, int num_layers, int batc
                                int32_t* const* out_idx, void* const* out_k, void* const* out_v,
                                kvec_stream_t stream);
 
+/* kvec_select_layers with the window rows' softmax denominators supplied by the
+ * caller, who has them from the prefill attention it just ran (the step right
+ * before eviction, Section 5.1: selection happens in the prefill of each layer).
+ * The library then skips its own statistics pass over K (score kernel) and
+ * forms the attention A of Eq. 1 as exp(scale * <q, k> - lse) directly.
+ *   lse  array of num_layers device pointers, each fp32 [batch][w][H_q]:
+ *        lse[s][q][hq] = ln( sum over every key t the row sees (the prefix and
+ *        the causal part of the window, t <= L_s - w + q) of
+ *        exp(scale * <q_obs[s][q][hq], k_t>) ), with the same scale as
+ *        params.softmax_scale (1/sqrt(d) when that is <= 0).  4-byte aligned.
+ * Everything else as kvec_select_layers.  The library cannot check that lse
+ * matches q_obs and K; a wrong lse gives a wrong selection. */
+KVEC_API kvec_status kvec_select_layers_lse(kvec_handle* h, int num_layers, int batch,
+                               const int32_t* cu_seqlens_host, const int32_t* cu_seqlens_dev,
+                               const void* const* q_obs, const void* const* k, const void* const* v,
+                               const float* const* lse, void* coverage_state, int budget,
+                               int32_t* const* out_idx, void* const* out_k, void* const* out_v,
+                               kvec_stream_t stream);
+
+/* One layer of kvec_select_layers_lse. */
+KVEC_API kvec_status kvec_select_layer_lse(kvec_handle* h, int batch,
+                              const int32_t* cu_seqlens_host, const int32_t* cu_seqlens_dev,
+                              const void* q_obs, const void* k, const void* v, const float* lse,
+                              void* coverage_state, int budget,
+                              int32_t* out_idx, void* out_k, void* out_v,
+                              kvec_stream_t stream);
+
 /* kvec_select_layer for callers that cannot allocate device memory: the
  * library then needs no handle and calls no cudaMalloc, cudaFree or other
  * allocating routine.  It serves hosts whose device memory belongs to someone

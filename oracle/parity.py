@@ -30,9 +30,32 @@ def gpu_debug_numpy(sel: kvec.KvecSelector, batch: int, max_seqlen: int) -> Dict
             "Pprime": d["Pprime"][:batch], "row_stats": d["row_stats"][:batch]}
 
 
+def window_lse(wl: synth.Workload, x: Dict[str, torch.Tensor]) -> np.ndarray:
+    """fp64 log-sum-exp of every window query row over the keys it sees (the
+    prefix and the causal part of the window), [batch][w][H_q]: the input of
+    kvec_select_layer_lse, as the caller's prefill attention would give it."""
+    w, Hq, Hkv, d = wl.window, wl.num_q_heads, wl.num_kv_heads, wl.head_dim
+    g = Hq // Hkv
+    scale = 1.0 / math.sqrt(d)
+    q = x["q_obs"].float().cpu().numpy().astype(np.float64)
+    k = x["k"].float().cpu().numpy().astype(np.float64)
+    out = np.empty((wl.batch, w, Hq))
+    cu = wl.cu_seqlens
+    for s in range(wl.batch):
+        L = cu[s + 1] - cu[s]
+        visible = np.arange(L)[None, :] <= (L - w + np.arange(w))[:, None]   # [w][L]
+        for h in range(Hkv):
+            logits = scale * np.einsum("qjd,td->qjt", q[s, :, h * g:(h + 1) * g, :], k[cu[s]:cu[s + 1], h, :])
+            logits = np.where(visible[:, None, :], logits, -np.inf)
+            m = logits.max(axis=2, keepdims=True)
+            out[s, :, h * g:(h + 1) * g] = (m + np.log(np.exp(logits - m).sum(axis=2, keepdims=True)))[..., 0]
+    return out
+
+
 def run_parity(wl: synth.Workload, layers: Optional[int] = None, device: str = "cuda", budget: Optional[int] = None,
-               tol: float = compare.TOL, verbose: bool = False) -> List[str]:
-    """Returns every mismatch over `layers` layers of `wl` (empty list = parity)."""
+               tol: float = compare.TOL, verbose: bool = False, with_lse: bool = False) -> List[str]:
+    """Returns every mismatch over `layers` layers of `wl` (empty list = parity).
+    with_lse: the GPU layers take the window rows' log-sum-exp (window_lse) as input."""
     layers = layers or wl.layers
     budget = budget or wl.budget
     ML = wl.max_seqlen
@@ -48,8 +71,11 @@ def run_parity(wl: synth.Workload, layers: Optional[int] = None, device: str = "
     dev_inputs = [{k: v.to(device) for k, v in x.items()} for x in inputs]
     for l in range(layers):
         before = state.cpu().numpy().copy()
+        lse = None
+        if with_lse:
+            lse = torch.from_numpy(window_lse(wl, inputs[l]).astype(np.float32)).to(device)
         out_idx, out_k, out_v = sel.select_layer(cu_host, cu_dev, dev_inputs[l]["q_obs"], dev_inputs[l]["k"],
-                                                 dev_inputs[l]["v"], state, budget)
+                                                 dev_inputs[l]["v"], state, budget, lse=lse)
         torch.cuda.synchronize()
         kvec.kvec_sync_status(sel.handle)
         gdbg = gpu_debug_numpy(sel, wl.batch, ML)

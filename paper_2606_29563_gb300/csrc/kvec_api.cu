@@ -267,8 +267,12 @@ kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* io
         cudaError_t se = plan_score(G, io, sc, h->num_sms, &plan);
         if (se != cudaSuccess) return cuda_fail(se, "score kernel tensor maps");
         timed_launch(h, 0, h->s_score, [&] {
-            se = launch_score(plan, h->s_score, true);
-            if (se == cudaSuccess) se = launch_rowstat(plan, G, io, sc, h->s_score);
+            if (io.lse) {
+                se = launch_rowstat_lse(G, io, sc, h->s_score);
+            } else {
+                se = launch_score(plan, h->s_score, true);
+                if (se == cudaSuccess) se = launch_rowstat(plan, G, io, sc, h->s_score);
+            }
         });
         if (se != cudaSuccess) return cuda_fail(se, "score kernel launch");
         KV_CHECK(cudaEventRecord(h->ev_score[l], h->s_score));
@@ -325,7 +329,8 @@ std::vector<uint64_t> graph_key(int n, int batch, int budget, const int32_t* cu_
     for (int l = 0; l < n; ++l) {
         const LayerIO& io = ios[l];
         for (const void* ptr : {(const void*)io.q, (const void*)io.k, (const void*)io.v, (const void*)io.state,
-                                (const void*)io.out_idx, (const void*)io.out_k, (const void*)io.out_v})
+                                (const void*)io.out_idx, (const void*)io.out_k, (const void*)io.out_v,
+                                (const void*)io.lse})
             k.push_back((uint64_t)(uintptr_t)ptr);
     }
     return k;
@@ -512,10 +517,15 @@ kvec_status kvec_select_layer(kvec_handle* h, int batch, const int32_t* cu_seqle
                               oks, ovs, stream);
 }
 
-kvec_status kvec_select_layers(kvec_handle* h, int num_layers, int batch, const int32_t* cu_seqlens_host,
+}  // extern "C"
+
+namespace {
+
+kvec_status select_layers_impl(kvec_handle* h, int num_layers, int batch, const int32_t* cu_seqlens_host,
                                const int32_t* cu_seqlens_dev, const void* const* q_obs, const void* const* k,
-                               const void* const* v, void* coverage_state, int budget, int32_t* const* out_idx,
-                               void* const* out_k, void* const* out_v, kvec_stream_t stream) {
+                               const void* const* v, const float* const* lse, void* coverage_state, int budget,
+                               int32_t* const* out_idx, void* const* out_k, void* const* out_v,
+                               kvec_stream_t stream) {
     int tiles = 0, chunks = 0;
     kvec_status s = validate_call(h, batch, cu_seqlens_host, cu_seqlens_dev, budget, &tiles, &chunks);
     if (s != KVEC_OK) return s;
@@ -530,6 +540,8 @@ kvec_status kvec_select_layers(kvec_handle* h, int num_layers, int batch, const 
         if (!aligned16(q_obs[l]) || !aligned16(k[l]) || !aligned16(v[l]) || !aligned16(out_k[l]) ||
             !aligned16(out_v[l]) || (reinterpret_cast<uintptr_t>(out_idx[l]) & 3u))
             return fail(KVEC_ERR_INVALID_ARG, "layer %d: device pointers must be 16-byte aligned", l);
+        if (lse && (!lse[l] || (reinterpret_cast<uintptr_t>(lse[l]) & 3u)))
+            return fail(KVEC_ERR_INVALID_ARG, "layer %d: lse must be a non-NULL, 4-byte aligned device pointer", l);
     }
     int prev = 0;
     s = set_device(h, &prev);
@@ -549,6 +561,7 @@ kvec_status kvec_select_layers(kvec_handle* h, int num_layers, int batch, const 
         io.out_idx = out_idx[l];
         io.out_k = static_cast<__nv_bfloat16*>(out_k[l]);
         io.out_v = static_cast<__nv_bfloat16*>(out_v[l]);
+        io.lse = lse ? lse[l] : nullptr;
     }
     if (!h->profiling && num_layers >= 2) {
         // A call repeated with the same arguments replays a captured graph of the pipeline.
@@ -587,6 +600,43 @@ kvec_status kvec_select_layers(kvec_handle* h, int num_layers, int batch, const 
     if (s != KVEC_OK) return s;
     h->last_batch = batch;
     return KVEC_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+kvec_status kvec_select_layers(kvec_handle* h, int num_layers, int batch, const int32_t* cu_seqlens_host,
+                               const int32_t* cu_seqlens_dev, const void* const* q_obs, const void* const* k,
+                               const void* const* v, void* coverage_state, int budget, int32_t* const* out_idx,
+                               void* const* out_k, void* const* out_v, kvec_stream_t stream) {
+    return select_layers_impl(h, num_layers, batch, cu_seqlens_host, cu_seqlens_dev, q_obs, k, v, nullptr,
+                              coverage_state, budget, out_idx, out_k, out_v, stream);
+}
+
+kvec_status kvec_select_layers_lse(kvec_handle* h, int num_layers, int batch, const int32_t* cu_seqlens_host,
+                                   const int32_t* cu_seqlens_dev, const void* const* q_obs, const void* const* k,
+                                   const void* const* v, const float* const* lse, void* coverage_state, int budget,
+                                   int32_t* const* out_idx, void* const* out_k, void* const* out_v,
+                                   kvec_stream_t stream) {
+    if (!lse) return fail(KVEC_ERR_INVALID_ARG, "NULL pointer argument");
+    return select_layers_impl(h, num_layers, batch, cu_seqlens_host, cu_seqlens_dev, q_obs, k, v, lse,
+                              coverage_state, budget, out_idx, out_k, out_v, stream);
+}
+
+kvec_status kvec_select_layer_lse(kvec_handle* h, int batch, const int32_t* cu_seqlens_host,
+                                  const int32_t* cu_seqlens_dev, const void* q_obs, const void* k, const void* v,
+                                  const float* lse, void* coverage_state, int budget, int32_t* out_idx, void* out_k,
+                                  void* out_v, kvec_stream_t stream) {
+    const void* qs[1] = {q_obs};
+    const void* ks[1] = {k};
+    const void* vs[1] = {v};
+    const float* ls[1] = {lse};
+    int32_t* ois[1] = {out_idx};
+    void* oks[1] = {out_k};
+    void* ovs[1] = {out_v};
+    return kvec_select_layers_lse(h, 1, batch, cu_seqlens_host, cu_seqlens_dev, qs, ks, vs, ls, coverage_state,
+                                  budget, ois, oks, ovs, stream);
 }
 
 // ---------------------------------------------------------------------------

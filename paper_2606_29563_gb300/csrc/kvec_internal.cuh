@@ -69,6 +69,7 @@ struct LayerIO {
     int32_t* out_idx;
     __nv_bfloat16* out_k;
     __nv_bfloat16* out_v;
+    const float* lse;         // [batch][w][Hq] natural-log softmax denominators of the window rows, or null
 };
 
 // ---------------------------------------------------------------- helpers
@@ -111,6 +112,9 @@ cudaError_t launch_score(const ScorePlan& plan, cudaStream_t st, bool after_own_
 // (m_r, Z_r) from the score launch's partials; launched right after it on the same stream.
 cudaError_t launch_rowstat(const ScorePlan& plan, const Geometry& g, const LayerIO& io, const Scratch& sc,
                            cudaStream_t st);
+// (m_r, Z_r) = (lse * log2(e), 1) from the caller's log-sum-exp (io.lse), in place
+// of the score and row-statistics launches.
+cudaError_t launch_rowstat_lse(const Geometry& g, const LayerIO& io, const Scratch& sc, cudaStream_t st);
 cudaError_t launch_window(const ScorePlan& sp, const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl,
                           cudaStream_t st, bool after_own_launch);
 // Launches kernel<<<grid, block, smem, st>>> with a scheduling priority (lower

@@ -427,6 +427,17 @@ __global__ void __launch_bounds__(256) rowstat_kernel(Geometry G, Scratch sc, co
     sc.rowstat[((size_t)s * G.Hkv + h) * G.R + r] = make_float2(M, Z);
 }
 
+// Row statistics from the caller's log-sum-exp of each window query row (the
+// denominator its prefill attention already computed): row r = q * g + j of KV
+// head h is query head h * g + j at window position q.  Grid (Hkv, batch).
+__global__ void __launch_bounds__(256) rowstat_lse_kernel(Geometry G, Scratch sc, const float* __restrict__ lse) {
+    const int h = blockIdx.x, s = blockIdx.y, r = threadIdx.x;
+    if (r >= G.R) return;
+    const int q = r / G.g, j = r - q * G.g;
+    const float v = __ldg(&lse[((size_t)s * G.w + q) * G.Hq + h * G.g + j]);
+    sc.rowstat[((size_t)s * G.Hkv + h) * G.R + r] = make_float2(v * 1.4426950408889634f, 1.f);
+}
+
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
     if (!fn) {
@@ -533,6 +544,11 @@ cudaError_t launch_rowstat(const ScorePlan& plan, const Geometry& g, const Layer
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     return cudaLaunchKernelEx(&cfg, rowstat_kernel, g, sc, io.cu, a.W, plan.grid);
+}
+
+cudaError_t launch_rowstat_lse(const Geometry& g, const LayerIO& io, const Scratch& sc, cudaStream_t st) {
+    rowstat_lse_kernel<<<dim3(g.Hkv, g.batch), 256, 0, st>>>(g, sc, io.lse);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_score(const ScorePlan& plan, cudaStream_t st, bool after_own_launch) {

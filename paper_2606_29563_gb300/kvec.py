@@ -27,7 +27,8 @@ KERNEL_NAMES = ("score", "window", "heads", "select", "gather")
 
 EXPORTED = ("kvec_create", "kvec_destroy", "kvec_state_bytes", "kvec_reset", "kvec_select_layer",
             "kvec_select_layers", "kvec_debug_scores", "kvec_sync_status", "kvec_set_profiling",
-            "kvec_kernel_time", "kvec_status_string", "kvec_last_error", "kvec_select_layer_noalloc")
+            "kvec_kernel_time", "kvec_status_string", "kvec_last_error", "kvec_select_layer_noalloc",
+            "kvec_select_layer_lse", "kvec_select_layers_lse")
 
 
 class KvecUnavailable(ImportError):
@@ -91,6 +92,8 @@ def load() -> ctypes.CDLL:
             "kvec_last_error": ([], ctypes.c_char_p),
             "kvec_select_layer_noalloc": ([ctypes.POINTER(kvec_params), i, _vp, _vp, _vp, _vp, _vp, _vp, i, _vp,
                                            _vp, _vp, _vp], st),
+            "kvec_select_layer_lse": ([_vp, i, _vp, _vp, _vp, _vp, _vp, _vp, _vp, i, _vp, _vp, _vp, _vp], st),
+            "kvec_select_layers_lse": ([_vp, i, i, _vp, _vp, _pp, _pp, _pp, _pp, _vp, i, _pp, _pp, _pp, _vp], st),
         }
         for name, (args, res) in sig.items():
             fn = getattr(lib, name)
@@ -140,6 +143,23 @@ def kvec_select_layers(handle: int, batch: int, cu_host_ptr: int, cu_dev_ptr: in
     n = len(q_obs)
     _check(load().kvec_select_layers(handle, n, int(batch), cu_host_ptr, cu_dev_ptr, _arr(q_obs), _arr(k), _arr(v),
                                      state, int(budget), _arr(out_idx), _arr(out_k), _arr(out_v), stream))
+
+
+def kvec_select_layer_lse(handle: int, batch: int, cu_host_ptr: int, cu_dev_ptr: int, q_obs: int, k: int, v: int,
+                          lse: int, state: int, budget: int, out_idx: int, out_k: int, out_v: int,
+                          stream: int = 0) -> None:
+    _check(load().kvec_select_layer_lse(handle, int(batch), cu_host_ptr, cu_dev_ptr, q_obs, k, v, lse, state,
+                                        int(budget), out_idx, out_k, out_v, stream))
+
+
+def kvec_select_layers_lse(handle: int, batch: int, cu_host_ptr: int, cu_dev_ptr: int, q_obs: Sequence[int],
+                           k: Sequence[int], v: Sequence[int], lse: Sequence[int], state: int, budget: int,
+                           out_idx: Sequence[int], out_k: Sequence[int], out_v: Sequence[int],
+                           stream: int = 0) -> None:
+    n = len(q_obs)
+    _check(load().kvec_select_layers_lse(handle, n, int(batch), cu_host_ptr, cu_dev_ptr, _arr(q_obs), _arr(k),
+                                         _arr(v), _arr(lse), state, int(budget), _arr(out_idx), _arr(out_k),
+                                         _arr(out_v), stream))
 
 
 def kvec_select_layer_noalloc(params: kvec_params, batch: int, cu_host_ptr: int, cu_dev_ptr: int, q_obs: int,
@@ -234,25 +254,37 @@ class KvecSelector:
                 t.empty((batch, p.num_kv_heads, budget, p.head_dim), dtype=t.bfloat16, device=device),
                 t.empty((batch, p.num_kv_heads, budget, p.head_dim), dtype=t.bfloat16, device=device))
 
-    def select_layer(self, cu_host, cu_dev, q_obs, k, v, state, budget: int, outs=None, stream=None):
+    def select_layer(self, cu_host, cu_dev, q_obs, k, v, state, budget: int, outs=None, stream=None, lse=None):
+        """lse: optional fp32 [batch][w][H_q] window-row log-sum-exp (kvec_select_layer_lse)."""
         t = self._torch
         batch = cu_host.numel() - 1
         if outs is None:
             outs = self.alloc_outputs(batch, budget, q_obs.device)
         s = stream if stream is not None else t.cuda.current_stream(q_obs.device)
-        kvec_select_layer(self.handle, batch, cu_host.data_ptr(), cu_dev.data_ptr(), q_obs.data_ptr(),
-                          k.data_ptr(), v.data_ptr(), state.data_ptr(), budget, outs[0].data_ptr(),
-                          outs[1].data_ptr(), outs[2].data_ptr(), s.cuda_stream)
+        if lse is None:
+            kvec_select_layer(self.handle, batch, cu_host.data_ptr(), cu_dev.data_ptr(), q_obs.data_ptr(),
+                              k.data_ptr(), v.data_ptr(), state.data_ptr(), budget, outs[0].data_ptr(),
+                              outs[1].data_ptr(), outs[2].data_ptr(), s.cuda_stream)
+        else:
+            kvec_select_layer_lse(self.handle, batch, cu_host.data_ptr(), cu_dev.data_ptr(), q_obs.data_ptr(),
+                                  k.data_ptr(), v.data_ptr(), lse.data_ptr(), state.data_ptr(), budget,
+                                  outs[0].data_ptr(), outs[1].data_ptr(), outs[2].data_ptr(), s.cuda_stream)
         return outs
 
-    def select_layers(self, cu_host, cu_dev, qs, ks, vs, state, budget: int, outs, stream=None):
+    def select_layers(self, cu_host, cu_dev, qs, ks, vs, state, budget: int, outs, stream=None, lses=None):
+        """lses: optional per-layer fp32 [batch][w][H_q] window-row log-sum-exp (kvec_select_layers_lse)."""
         t = self._torch
         batch = cu_host.numel() - 1
         s = stream if stream is not None else t.cuda.current_stream(qs[0].device)
-        kvec_select_layers(self.handle, batch, cu_host.data_ptr(), cu_dev.data_ptr(), [x.data_ptr() for x in qs],
-                           [x.data_ptr() for x in ks], [x.data_ptr() for x in vs], state.data_ptr(), budget,
-                           [o[0].data_ptr() for o in outs], [o[1].data_ptr() for o in outs],
-                           [o[2].data_ptr() for o in outs], s.cuda_stream)
+        common = ([x.data_ptr() for x in qs], [x.data_ptr() for x in ks], [x.data_ptr() for x in vs])
+        tail = ([o[0].data_ptr() for o in outs], [o[1].data_ptr() for o in outs], [o[2].data_ptr() for o in outs],
+                s.cuda_stream)
+        if lses is None:
+            kvec_select_layers(self.handle, batch, cu_host.data_ptr(), cu_dev.data_ptr(), *common, state.data_ptr(),
+                               budget, *tail)
+        else:
+            kvec_select_layers_lse(self.handle, batch, cu_host.data_ptr(), cu_dev.data_ptr(), *common,
+                                   [x.data_ptr() for x in lses], state.data_ptr(), budget, *tail)
         return outs
 
     def debug(self, device="cuda"):

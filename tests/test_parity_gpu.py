@@ -122,6 +122,47 @@ def test_multi_layer_call_matches_layer_by_layer():
     sel.close()
 
 
+# ---- window-row log-sum-exp supplied by the caller (no statistics pass) ----
+
+@pytest.mark.parametrize("kw", [dict(seqlens=(700,), layers=2),
+                                dict(seqlens=(40, 900, 64, 1531), budget=64, layers=2),
+                                dict(seqlens=(523,), num_q_heads=28, num_kv_heads=4, layers=2)])
+def test_lse_input_matches_the_oracle(kw):
+    _assert_parity(synth.small_workload(**kw), with_lse=True)
+
+
+def test_lse_input_llama8b_l8192_b512_first_layers():
+    _assert_parity(synth.WORKLOADS["llama8b_l8192_b512"], layers=2, with_lse=True)
+
+
+def test_lse_multi_layer_call_matches_layer_by_layer():
+    wl = synth.small_workload(seqlens=(1100, 700), layers=3, budget=96)
+    cpu_layers = synth.make_layers(wl, 3)
+    layers = [{k: v.cuda() for k, v in x.items()} for x in cpu_layers]
+    lses = [torch.from_numpy(parity.window_lse(wl, x).astype(np.float32)).cuda() for x in cpu_layers]
+    cu = torch.tensor(wl.cu_seqlens, dtype=torch.int32)
+    sel = kvec.KvecSelector(kvec.params_from_workload(wl))
+    st1 = sel.new_state(wl.batch)
+    one = [sel.select_layer(cu, cu.cuda(), x["q_obs"], x["k"], x["v"], st1, wl.budget, lse=e)
+           for x, e in zip(layers, lses)]
+    st2 = sel.new_state(wl.batch)
+    many = [sel.alloc_outputs(wl.batch, wl.budget) for _ in layers]
+    sel.select_layers(cu, cu.cuda(), [x["q_obs"] for x in layers], [x["k"] for x in layers],
+                      [x["v"] for x in layers], st2, wl.budget, many, lses=lses)
+    torch.cuda.synchronize()
+    for a, b in zip(one, many):
+        for x, y in zip(a, b):
+            assert torch.equal(x, y)
+    assert torch.equal(st1, st2)
+    with pytest.raises(kvec.KvecError) as e:   # a misaligned lse pointer is refused before any launch
+        kvec.kvec_select_layer_lse(sel.handle, wl.batch, cu.data_ptr(), cu.cuda().data_ptr(),
+                                   layers[0]["q_obs"].data_ptr(), layers[0]["k"].data_ptr(),
+                                   layers[0]["v"].data_ptr(), lses[0].data_ptr() + 2, st2.data_ptr(), wl.budget,
+                                   *[t.data_ptr() for t in many[0]], torch.cuda.current_stream().cuda_stream)
+    assert e.value.status == kvec.KVEC_ERR_INVALID_ARG
+    sel.close()
+
+
 def test_layer_limit_refuses_the_whole_call_and_positions_past_L_stay_zero():
     """n_t is 8-bit, so no state may count more than 255 layers (Section 4.2's
     counters).  A call that would pass the limit reports it and leaves the state

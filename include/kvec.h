@@ -188,6 +188,30 @@ KVEC_API kvec_status kvec_select_layer_noalloc(const kvec_params* params, int ba
                                       int32_t* out_idx, void* out_k, void* out_v,
                                       kvec_stream_t stream);
 
+/* One decoding step of attention over the compacted cache that the selection
+ * produced.  Section 4.1: once each KV head has kept its B tokens, their keys
+ * and values are the cache that the subsequent decoding steps read; Section
+ * 5.3 (Computational Complexity) times decoding over that cache.  For every
+ * sequence s and query head hq (KV head h = hq / (H_q/H_kv)):
+ *   out[s][hq] = sum_{j < n_s} p_j * v_cache[s][h][j],
+ *   p_j = softmax_j( scale * <q[s][hq], k_cache[s][h][j]> ),
+ * with n_s = lens[s] clamped to [0, cap]; n_s = 0 gives a zero row.  scale is
+ * params.softmax_scale (1/sqrt(d) when that is <= 0).
+ *   q        device bf16 [batch][H_q][d]: the step's query rows.
+ *   k_cache, v_cache  device bf16 [batch][H_kv][cap][d]: for instance out_k and
+ *            out_v of kvec_select_layer (cap = B, lens[s] = min(L_s, B): the kept
+ *            rows come first), or that cache with decoded tokens appended.
+ *   lens     device int32 [batch].
+ *   out      device fp32 [batch][H_q][d].
+ * 1 <= batch <= max_batch, 1 <= cap <= 2^20, H_q/H_kv <= 8 (else UNSUPPORTED);
+ * q, k_cache, v_cache 16-byte aligned, lens 4-byte and out 8-byte aligned.
+ * Asynchronous on `stream`; the handle's decode workspace is reused by every
+ * call, so calls on different streams must not overlap. */
+KVEC_API kvec_status kvec_decode_attention(kvec_handle* h, int batch, const void* q,
+                                           const void* k_cache, const void* v_cache,
+                                           const int32_t* lens, int cap, float* out,
+                                           kvec_stream_t stream);
+
 /* Device views of the last processed layer's intermediates (valid until the
  * next call on the handle; read after synchronising the stream).  Row strides
  * use ML = max_seqlen + 4 rounded up to a multiple of 32 (reported in max_seqlen).

@@ -75,6 +75,9 @@ struct kvec_handle {
     // Scheduling priorities: the heads and coverage-select kernels (the serial
     // chain of the pipeline) take SMs before the score, window and gather kernels.
     int prio_hi = 0, prio_lo = 0;
+    // Split partials of kvec_decode_attention.
+    float* dec_part = nullptr;
+    float2* dec_ml = nullptr;
     // CUDA graph of the last repeated multi-layer call.
     cudaGraphExec_t gexec = nullptr;
     std::vector<uint64_t> gkey, pending_key;
@@ -185,6 +188,8 @@ kvec_status validate_call(kvec_handle* h, int batch, const int32_t* cu_host, con
 }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+constexpr int kDecodeMaxCap = 1 << 20;   // cached rows per (sequence, KV head) a decode call may pass
 
 Geometry make_geometry(const kvec_handle* h, int batch, int budget, int tiles, int chunks, int total_tokens) {
     const kvec_params& p = h->p;
@@ -402,6 +407,8 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
         {(void**)&h->sc.nbuf, MB * round_up((size_t)p.max_seqlen, 16)},
         {(void**)&h->sc.err, sizeof(int)},
         {(void**)&h->sc.keys_sel, MB * Hkv * ML * sizeof(uint32_t)},
+        {(void**)&h->dec_part, MB * (size_t)p.num_q_heads * kDecMaxSplits * kHeadDim * sizeof(float)},
+        {(void**)&h->dec_ml, MB * (size_t)p.num_q_heads * kDecMaxSplits * sizeof(float2)},
     };
     for (int k = 0; k < kScoreBufs; ++k) {
         Scratch& b = h->score_buf[k];
@@ -780,6 +787,40 @@ kvec_status kvec_select_layer_noalloc(const kvec_params* params, int batch, cons
     io.out_k = static_cast<__nv_bfloat16*>(out_k);
     io.out_v = static_cast<__nv_bfloat16*>(out_v);
     return run_layer_sequential(&tmp, G, io, st);
+}
+
+kvec_status kvec_decode_attention(kvec_handle* h, int batch, const void* q, const void* k_cache,
+                                  const void* v_cache, const int32_t* lens, int cap, float* out,
+                                  kvec_stream_t stream) {
+    if (!h) return fail(KVEC_ERR_INVALID_ARG, "handle is NULL");
+    const kvec_params& p = h->p;
+    if (batch < 1 || batch > p.max_batch)
+        return fail(KVEC_ERR_INVALID_ARG, "batch %d outside [1, max_batch = %d]", batch, p.max_batch);
+    if (cap < 1 || cap > kDecodeMaxCap)
+        return fail(KVEC_ERR_INVALID_ARG, "cap %d outside [1, %d]", cap, kDecodeMaxCap);
+    if (h->g > 8)
+        return fail(KVEC_ERR_UNSUPPORTED, "decode attention supports up to 8 query heads per KV head (g = %d)", h->g);
+    if (!q || !k_cache || !v_cache || !lens || !out) return fail(KVEC_ERR_INVALID_ARG, "a device pointer is NULL");
+    if (!aligned16(q) || !aligned16(k_cache) || !aligned16(v_cache))
+        return fail(KVEC_ERR_INVALID_ARG, "q, k_cache and v_cache must be 16-byte aligned");
+    if (reinterpret_cast<uintptr_t>(lens) % 4 || reinterpret_cast<uintptr_t>(out) % 8)
+        return fail(KVEC_ERR_INVALID_ARG, "lens must be 4-byte and out 8-byte aligned");
+    DecodeIO io{};
+    io.q = static_cast<const __nv_bfloat16*>(q);
+    io.k = static_cast<const __nv_bfloat16*>(k_cache);
+    io.v = static_cast<const __nv_bfloat16*>(v_cache);
+    io.lens = lens;
+    io.part = h->dec_part;
+    io.ml = h->dec_ml;
+    io.out = out;
+    io.batch = batch;
+    io.Hq = p.num_q_heads;
+    io.Hkv = p.num_kv_heads;
+    io.cap = cap;
+    io.scale = p.softmax_scale > 0.f ? p.softmax_scale : (float)(1.0 / sqrt((double)p.head_dim));
+    cudaError_t e = launch_decode(io, reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "decode attention launch");
+    return KVEC_OK;
 }
 
 kvec_status kvec_debug_scores(kvec_handle* h, kvec_debug_view* out) {

@@ -28,7 +28,7 @@ KERNEL_NAMES = ("score", "window", "heads", "select", "gather")
 EXPORTED = ("kvec_create", "kvec_destroy", "kvec_state_bytes", "kvec_reset", "kvec_select_layer",
             "kvec_select_layers", "kvec_debug_scores", "kvec_sync_status", "kvec_set_profiling",
             "kvec_kernel_time", "kvec_status_string", "kvec_last_error", "kvec_select_layer_noalloc",
-            "kvec_select_layer_lse", "kvec_select_layers_lse")
+            "kvec_select_layer_lse", "kvec_select_layers_lse", "kvec_decode_attention")
 
 
 class KvecUnavailable(ImportError):
@@ -94,6 +94,7 @@ def load() -> ctypes.CDLL:
                                            _vp, _vp, _vp], st),
             "kvec_select_layer_lse": ([_vp, i, _vp, _vp, _vp, _vp, _vp, _vp, _vp, i, _vp, _vp, _vp, _vp], st),
             "kvec_select_layers_lse": ([_vp, i, i, _vp, _vp, _pp, _pp, _pp, _pp, _vp, i, _pp, _pp, _pp, _vp], st),
+            "kvec_decode_attention": ([_vp, i, _vp, _vp, _vp, _vp, i, _vp, _vp], st),
         }
         for name, (args, res) in sig.items():
             fn = getattr(lib, name)
@@ -168,6 +169,11 @@ def kvec_select_layer_noalloc(params: kvec_params, batch: int, cu_host_ptr: int,
     """kvec_select_layer without a handle; scratch comes from the library's static device array."""
     _check(load().kvec_select_layer_noalloc(ctypes.byref(params), int(batch), cu_host_ptr, cu_dev_ptr, q_obs, k, v,
                                             state, int(budget), out_idx, out_k, out_v, stream))
+
+
+def kvec_decode_attention(handle: int, batch: int, q: int, k_cache: int, v_cache: int, lens: int, cap: int,
+                          out: int, stream: int = 0) -> None:
+    _check(load().kvec_decode_attention(handle, int(batch), q, k_cache, v_cache, lens, int(cap), out, stream))
 
 
 def kvec_debug_scores(handle: int) -> kvec_debug_view:
@@ -286,6 +292,20 @@ class KvecSelector:
             kvec_select_layers_lse(self.handle, batch, cu_host.data_ptr(), cu_dev.data_ptr(), *common,
                                    [x.data_ptr() for x in lses], state.data_ptr(), budget, *tail)
         return outs
+
+    def decode_attention(self, q, k_cache, v_cache, lens, out=None, stream=None):
+        """One decoding step over a compacted cache (kvec_decode_attention).
+
+        q bf16 [batch][H_q][d]; k_cache, v_cache bf16 [batch][H_kv][cap][d];
+        lens int32 [batch] on the device.  Returns fp32 [batch][H_q][d]."""
+        t = self._torch
+        batch, cap = q.shape[0], k_cache.shape[2]
+        if out is None:
+            out = t.empty((batch, q.shape[1], q.shape[2]), dtype=t.float32, device=q.device)
+        s = stream if stream is not None else t.cuda.current_stream(q.device)
+        kvec_decode_attention(self.handle, batch, q.data_ptr(), k_cache.data_ptr(), v_cache.data_ptr(),
+                              lens.data_ptr(), cap, out.data_ptr(), s.cuda_stream)
+        return out
 
     def debug(self, device="cuda"):
         """Copies of the last layer's intermediates (see kvec_debug_view)."""

@@ -357,6 +357,8 @@ def run_ours(args, wl):
                        "api": "kvec_select_layers_lse: window-row log-sum-exp from the caller's prefill attention",
                        "path_roofline_frac": by["layer_total"] * L_layers / (ms_lse / 1e3) / 1e9 / peak}
 
+    decode = run_decode(args, wl, sel, layers, outs, dev, peak) if args.decode else None
+
     # End to end through the public API: pinned host inputs copied in, indices and state copied out.
     e2e = run_e2e(args, wl, sel, layers, outs, state, cu_host, cu_dev, dev, stream) if args.e2e else None
 
@@ -383,11 +385,77 @@ def run_ours(args, wl):
         "clocks": {k: v for k, v in clocks.summary(t_host0, t_host1).items()},
         "gpu_launches": gpu_launches,
         "lse_variant": lse_variant,
+        "decode": decode,
         "e2e": e2e,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         result["cpu_baseline"] = oracle_baseline(wl)
     return rank, result
+
+
+def run_decode(args, wl, sel, layers, outs, dev, peak):
+    """One decoding step (one generated token: every layer) over the compacted
+    caches that the selection just wrote, kvec_decode_attention per layer with
+    lens = min(L_s, B).  The layer loop is captured in a CUDA graph so that the
+    device time is measured, not the host's launch rate.  Roofline bytes per
+    call: the kept K and V rows read, the query rows read, the fp32 output
+    written."""
+    import numpy as np
+    import torch
+    from paper_2606_29563_gb300 import kvec
+
+    lens = [min(L, wl.budget) for L in wl.seqlens]
+    lens_d = torch.tensor(lens, dtype=torch.int32, device=dev)
+    dq = [x["q_obs"][:, -1].contiguous() for x in layers]
+    dout = [torch.empty((wl.batch, wl.num_q_heads, wl.head_dim), dtype=torch.float32, device=dev) for _ in layers]
+
+    def dstep(st):
+        for l in range(len(layers)):
+            kvec.kvec_decode_attention(sel.handle, wl.batch, dq[l].data_ptr(), outs[l][1].data_ptr(),
+                                       outs[l][2].data_ptr(), lens_d.data_ptr(), wl.budget, dout[l].data_ptr(),
+                                       st.cuda_stream)
+
+    side = torch.cuda.Stream(dev)
+    side.wait_stream(torch.cuda.current_stream(dev))
+    with torch.cuda.stream(side):
+        for _ in range(3):
+            dstep(side)
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        dstep(torch.cuda.current_stream(dev))
+    for _ in range(3):
+        graph.replay()
+    torch.cuda.synchronize()
+    n = max(20, min(args.steps, 2000))
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    cur = torch.cuda.current_stream(dev)
+    a.record(cur)
+    for _ in range(n):
+        graph.replay()
+    b.record(cur)
+    torch.cuda.synchronize()
+    ms_token = a.elapsed_time(b) / n
+    us_call = ms_token * 1e3 / len(layers)
+    bytes_call = (sum(lens) * wl.num_kv_heads * wl.head_dim * 2 * 2 + wl.batch * wl.num_q_heads * wl.head_dim * (2 + 4)
+                  + 4 * wl.batch)
+    gbs = bytes_call / (us_call / 1e6) / 1e9
+    res_cpu = None
+    if not args.no_cpu_baseline:
+        # CPU baseline leg: the fp64 oracle on the same call (layer 0), host cores.
+        from oracle.decode import decode_attention as oracle_decode
+        f64 = lambda t: t.float().cpu().numpy().astype(np.float64)
+        q0, k0, v0 = f64(dq[0]), f64(outs[0][1]), f64(outs[0][2])
+        t0 = time.perf_counter()
+        oracle_decode(q0, k0, v0, lens, 1.0 / np.sqrt(wl.head_dim))
+        cpu_ms = (time.perf_counter() - t0) * 1e3
+        res_cpu = {"value": 1e3 / (cpu_ms * len(layers)), "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+                   "sample": "one layer call of the step (fp64 NumPy; its BLAS may use up to all host threads), scaled to all layers"}
+    return {"api": "kvec_decode_attention, one call per layer (one generated token), CUDA graph",
+            "ms_per_token": ms_token, "us_per_layer_call": us_call, "tokens_per_s": 1e3 / ms_token,
+            "gpu_launches_per_token": len(layers), "bytes_per_call": bytes_call,
+            "roofline": {"bound": "hbm", "achieved": gbs, "peak": peak, "unit": "GB/s", "frac": gbs / peak},
+            "cache_rows_per_head": lens, "cpu_baseline": res_cpu}
 
 
 def run_e2e(args, wl, sel, layers, outs, state, cu_host, cu_dev, dev, stream):
@@ -477,6 +545,8 @@ def main(argv=None):
     ap.add_argument("--layers", type=int, default=None, help="run only the first N layers (not a bench line)")
     ap.add_argument("--no-e2e", dest="e2e", action="store_false")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-decode", dest="decode", action="store_false",
+                    help="skip the decode-attention measurement over the compacted caches")
     ap.add_argument("--no-lse-variant", dest="lse_variant", action="store_false",
                     help="skip timing the kvec_select_layers_lse variant")
     args = ap.parse_args(argv)

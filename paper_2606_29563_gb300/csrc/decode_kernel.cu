@@ -7,19 +7,26 @@
 //
 // The work is a few MB of K/V rows per call, read once: HBM- and latency-bound,
 // no dense contraction worth the tensor cores (g <= 8 query rows per KV head).
-// Split-K over the cache: CTA (split, h, s) streams its range of cached rows
-// through shared memory in 64-row tiles and keeps an online (max, sum, output)
-// for the g query heads of KV head h; a second kernel merges the splits.
+// Split-K over the cache inside one thread-block cluster per (s, h): each of
+// the kDecSplits CTAs streams its range of cached rows through shared memory in
+// 64-row tiles and keeps an online (max, sum, output) per query head; after a
+// cluster barrier, CTA r merges query head r from every CTA's shared memory
+// (distributed shared memory), so one launch does the whole step.
 #include "kvec_internal.cuh"
 #include "sm100_ptx.cuh"
+
+#include <cooperative_groups.h>
 
 namespace kvec {
 
 namespace {
 
+namespace cg = cooperative_groups;
+
 constexpr int kDecTile = 64;                     // cached rows per shared-memory tile
 constexpr int kDecThreads = 256;
 constexpr int kDecMaxG = 8;                      // query heads per KV head
+constexpr int kDecSplits = 8;                    // CTAs per (sequence, KV head): one cluster
 constexpr int kKRowHalves = kHeadDim + 8;        // K row stride in bf16 (16-byte pad: no bank conflicts)
 
 struct DecArgs {
@@ -27,21 +34,19 @@ struct DecArgs {
     const __nv_bfloat16* k;      // [batch][Hkv][cap][d]
     const __nv_bfloat16* v;
     const int* lens;             // [batch]
-    float* part;                 // [batch][Hq][nsplit][d]  unnormalised split outputs
-    float2* ml;                  // [batch][Hq][nsplit]     split (max in log2 units, sum)
     float* out;                  // [batch][Hq][d]
-    int Hq, Hkv, g, cap, nsplit, chunk;
+    int Hq, Hkv, g, cap, chunk;
     float sl2;                   // softmax scale * log2(e)
 };
 
-__global__ void __launch_bounds__(kDecThreads) decode_partial_kernel(const __grid_constant__ DecArgs A) {
-    __shared__ __align__(16) float qs[kDecMaxG][kHeadDim];
+__global__ void __launch_bounds__(kDecThreads) decode_kernel(const __grid_constant__ DecArgs A) {
+    __shared__ __align__(16) float qs[kDecMaxG][kHeadDim];   // the group's queries; later this CTA's outputs
     __shared__ __align__(16) __nv_bfloat16 ks[kDecTile][kKRowHalves];
     __shared__ __align__(16) __nv_bfloat16 vs[kDecTile][kHeadDim];
     __shared__ float ps[kDecMaxG][kDecTile];
     __shared__ float m_run[kDecMaxG], l_run[kDecMaxG], corr[kDecMaxG];
-    if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
-    const int sp = blockIdx.x, h = blockIdx.y, s = blockIdx.z;
+    cg::cluster_group cluster = cg::this_cluster();
+    const int sp = (int)cluster.block_rank(), h = blockIdx.y, s = blockIdx.z;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int g = A.g, cap = A.cap;
     const int n = min(max(__ldg(&A.lens[s]), 0), cap);
@@ -145,46 +150,40 @@ __global__ void __launch_bounds__(kDecThreads) decode_partial_kernel(const __gri
             }
         }
     }
+    // This CTA's unnormalised outputs replace the queries in shared memory; its
+    // (max, sum) per query head stay in m_run / l_run.
     __syncthreads();
 #pragma unroll
     for (int k = 0; k < 2; ++k) {
         const int idx = tid + k * kDecThreads;
         const int j = idx >> 6, dp = idx & 63;
-        if (j < g) {
-            const size_t row = ((size_t)s * A.Hq + h * g + j) * A.nsplit + sp;
-            *reinterpret_cast<float2*>(A.part + row * kHeadDim + 2 * dp) = make_float2(acc[k][0], acc[k][1]);
-        }
+        if (j < g) *reinterpret_cast<float2*>(&qs[j][2 * dp]) = make_float2(acc[k][0], acc[k][1]);
     }
-    if (tid < g) A.ml[((size_t)s * A.Hq + h * g + tid) * A.nsplit + sp] = make_float2(m_run[tid], l_run[tid]);
-}
-
-// out = sum_s 2^(m_s - M) o_s / sum_s 2^(m_s - M) l_s over the splits; zeros
-// for an empty cache.  Grid (Hq, batch), one thread per output column.
-__global__ void __launch_bounds__(kHeadDim) decode_combine_kernel(const __grid_constant__ DecArgs A) {
-    asm volatile("griddepcontrol.wait;\n" ::: "memory");
-    const int hq = blockIdx.x, s = blockIdx.y, c = threadIdx.x;
-    const size_t row = ((size_t)s * A.Hq + hq) * A.nsplit;
-    float M = -INFINITY;
-    for (int sp = 0; sp < A.nsplit; ++sp) M = fmaxf(M, __ldcg(&A.ml[row + sp]).x);
-    float L = 0.f, O = 0.f;
-    if (M != -INFINITY) {
-        for (int sp = 0; sp < A.nsplit; ++sp) {
-            const float2 ml = __ldcg(&A.ml[row + sp]);
-            if (ml.x == -INFINITY) continue;
-            const float w = ptx::ex2(ml.x - M);
-            L = fmaf(w, ml.y, L);
-            O = fmaf(w, __ldcg(&A.part[(row + sp) * kHeadDim + c]), O);
+    cluster.sync();
+    // CTA r merges query head r over the cluster:
+    // out = sum_c 2^(m_c - M) o_c / sum_c 2^(m_c - M) l_c, zeros for an empty cache.
+    if (sp < g && tid < kHeadDim) {
+        const int j = sp;
+        float M = -INFINITY;
+#pragma unroll
+        for (int c = 0; c < kDecSplits; ++c) M = fmaxf(M, *cluster.map_shared_rank(&m_run[j], c));
+        float L = 0.f, O = 0.f;
+        if (M != -INFINITY) {
+#pragma unroll
+            for (int c = 0; c < kDecSplits; ++c) {
+                const float m = *cluster.map_shared_rank(&m_run[j], c);
+                if (m == -INFINITY) continue;
+                const float w = ptx::ex2(m - M);
+                L = fmaf(w, *cluster.map_shared_rank(&l_run[j], c), L);
+                O = fmaf(w, *cluster.map_shared_rank(&qs[j][tid], c), O);
+            }
         }
+        A.out[((size_t)s * A.Hq + h * g + j) * kHeadDim + tid] = L > 0.f ? O / L : 0.f;
     }
-    A.out[((size_t)s * A.Hq + hq) * kHeadDim + c] = L > 0.f ? O / L : 0.f;
+    cluster.sync();   // no CTA leaves while another still reads its shared memory
 }
 
 }  // namespace
-
-int decode_splits(int cap) {
-    int ns = (cap + kDecTile - 1) / kDecTile;
-    return ns < 1 ? 1 : (ns > kDecMaxSplits ? kDecMaxSplits : ns);
-}
 
 cudaError_t launch_decode(const DecodeIO& io, cudaStream_t st) {
     DecArgs a{};
@@ -192,30 +191,26 @@ cudaError_t launch_decode(const DecodeIO& io, cudaStream_t st) {
     a.k = io.k;
     a.v = io.v;
     a.lens = io.lens;
-    a.part = io.part;
-    a.ml = io.ml;
     a.out = io.out;
     a.Hq = io.Hq;
     a.Hkv = io.Hkv;
     a.g = io.Hq / io.Hkv;
     a.cap = io.cap;
-    a.nsplit = decode_splits(io.cap);
-    const int per = (io.cap + a.nsplit - 1) / a.nsplit;
+    const int per = (io.cap + kDecSplits - 1) / kDecSplits;
     a.chunk = (per + kDecTile - 1) / kDecTile * kDecTile;
     a.sl2 = io.scale * 1.4426950408889634f;
-    decode_partial_kernel<<<dim3(a.nsplit, io.Hkv, io.batch), kDecThreads, 0, st>>>(a);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(io.Hq, io.batch);
-    cfg.blockDim = dim3(kHeadDim);
+    cfg.gridDim = dim3(kDecSplits, io.Hkv, io.batch);
+    cfg.blockDim = dim3(kDecThreads);
     cfg.stream = st;
     cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = kDecSplits;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, decode_combine_kernel, a);
+    return cudaLaunchKernelEx(&cfg, decode_kernel, a);
 }
 
 }  // namespace kvec

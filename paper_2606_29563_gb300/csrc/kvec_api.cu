@@ -75,9 +75,6 @@ struct kvec_handle {
     // Scheduling priorities: the heads and coverage-select kernels (the serial
     // chain of the pipeline) take SMs before the score, window and gather kernels.
     int prio_hi = 0, prio_lo = 0;
-    // Split partials of kvec_decode_attention.
-    float* dec_part = nullptr;
-    float2* dec_ml = nullptr;
     // CUDA graph of the last repeated multi-layer call.
     cudaGraphExec_t gexec = nullptr;
     std::vector<uint64_t> gkey, pending_key;
@@ -407,8 +404,6 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
         {(void**)&h->sc.nbuf, MB * round_up((size_t)p.max_seqlen, 16)},
         {(void**)&h->sc.err, sizeof(int)},
         {(void**)&h->sc.keys_sel, MB * Hkv * ML * sizeof(uint32_t)},
-        {(void**)&h->dec_part, MB * (size_t)p.num_q_heads * kDecMaxSplits * kHeadDim * sizeof(float)},
-        {(void**)&h->dec_ml, MB * (size_t)p.num_q_heads * kDecMaxSplits * sizeof(float2)},
     };
     for (int k = 0; k < kScoreBufs; ++k) {
         Scratch& b = h->score_buf[k];
@@ -810,8 +805,6 @@ kvec_status kvec_decode_attention(kvec_handle* h, int batch, const void* q, cons
     io.k = static_cast<const __nv_bfloat16*>(k_cache);
     io.v = static_cast<const __nv_bfloat16*>(v_cache);
     io.lens = lens;
-    io.part = h->dec_part;
-    io.ml = h->dec_ml;
     io.out = out;
     io.batch = batch;
     io.Hq = p.num_q_heads;

@@ -73,14 +73,11 @@ struct LayerIO {
 };
 
 // One decoding step over a compacted cache (decode_kernel.cu).
-constexpr int kDecMaxSplits = 64;   // most cache splits per (sequence, KV head)
 struct DecodeIO {
     const __nv_bfloat16* q;   // [batch][Hq][d]
     const __nv_bfloat16* k;   // [batch][Hkv][cap][d]
     const __nv_bfloat16* v;
     const int* lens;          // [batch] valid cached rows, clamped to [0, cap]
-    float* part;              // [batch][Hq][kDecMaxSplits][d] split outputs (workspace)
-    float2* ml;               // [batch][Hq][kDecMaxSplits] split (max, sum) (workspace)
     float* out;               // [batch][Hq][d]
     int batch, Hq, Hkv, cap;
     float scale;              // softmax scale
@@ -166,7 +163,6 @@ cudaError_t launch_select(const Geometry& g, const LayerIO& io, const Scratch& s
 cudaError_t launch_finalize(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& last, cudaStream_t st,
                             int priority, int ncall);
 // out_idx from the slot's kept-position bits, then the K/V rows.
-int decode_splits(int cap);
 cudaError_t launch_decode(const DecodeIO& io, cudaStream_t st);
 void launch_gather(const Geometry& g, const LayerIO& io, const Slot& sl, cudaStream_t st);
 

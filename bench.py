@@ -37,6 +37,7 @@ KERNEL_SOURCES = {
     "heads": "paper_2606_29563_gb300/csrc/select_kernels.cu",
     "select": "paper_2606_29563_gb300/csrc/select_kernels.cu",
     "gather": "paper_2606_29563_gb300/csrc/select_kernels.cu",
+    "decode": "paper_2606_29563_gb300/csrc/decode_kernel.cu",
 }
 
 
@@ -454,7 +455,8 @@ def run_decode(args, wl, sel, layers, outs, dev, peak):
     return {"api": "kvec_decode_attention, one call per layer (one generated token), CUDA graph",
             "ms_per_token": ms_token, "us_per_layer_call": us_call, "tokens_per_s": 1e3 / ms_token,
             "gpu_launches_per_token": len(layers), "bytes_per_call": bytes_call,
-            "roofline": {"bound": "hbm", "achieved": gbs, "peak": peak, "unit": "GB/s", "frac": gbs / peak},
+            "roofline": {"bound": "hbm", "achieved": gbs, "peak": peak, "unit": "GB/s", "frac": gbs / peak,
+                         "traffic": committed_traffic("decode", wl.name)},
             "cache_rows_per_head": lens, "cpu_baseline": res_cpu}
 
 

@@ -44,6 +44,7 @@ class _Params(ctypes.Structure):
         ("window", ctypes.c_int), ("obs_window", ctypes.c_int), ("ext_window", ctypes.c_int),
         ("pool_kernel", ctypes.c_int), ("num_ext_heads", ctypes.c_int),
         ("lam", ctypes.c_double), ("beta", ctypes.c_double), ("softmax_scale", ctypes.c_double),
+        ("pool_mode", ctypes.c_int), ("head_criterion", ctypes.c_int),
     ]
 
 
@@ -91,20 +92,24 @@ class OracleParams:
     lam: float = 1.0
     beta: float = 0.25
     softmax_scale: float = 0.0
+    pool_mode: int = 0        # 0 max-pool, 1 average pool
+    head_criterion: int = 0   # 0 standard deviation, 1 entropy
 
     @classmethod
     def from_workload(cls, wl, **over) -> "OracleParams":
         kw = dict(num_q_heads=wl.num_q_heads, num_kv_heads=wl.num_kv_heads, head_dim=wl.head_dim,
                   window=wl.window, obs_window=wl.obs_window, ext_window=wl.ext_window,
                   pool_kernel=wl.pool_kernel, num_ext_heads=wl.num_ext_heads,
-                  lam=float(np.float32(wl.lam)), beta=float(np.float32(wl.beta)))
+                  lam=float(np.float32(wl.lam)), beta=float(np.float32(wl.beta)),
+                  pool_mode=getattr(wl, "pool_mode", 0), head_criterion=getattr(wl, "head_criterion", 0))
         kw.update(over)
         return cls(**kw)
 
     def _c(self) -> _Params:
         return _Params(self.num_q_heads, self.num_kv_heads, self.head_dim, self.window,
                        self.obs_window, self.ext_window, self.pool_kernel, self.num_ext_heads,
-                       float(self.lam), float(self.beta), float(self.softmax_scale))
+                       float(self.lam), float(self.beta), float(self.softmax_scale), int(self.pool_mode),
+                       int(self.head_criterion))
 
 
 def state_bytes(max_seqlen: int) -> int:

@@ -81,6 +81,20 @@ static void top_k(const double* key, const uint8_t* allowed, int n, int k, uint8
     free(r);
 }
 
+/* 1-D average pool, width `kernel`, stride 1, over x[0, n): the mean of the
+ * neighbours inside [0, n) (the pooling variant of the SnapKV lineage the paper
+ * builds on; the paper's own setting is the max-pool below). */
+static void avg_pool(const double* x, int n, int kernel, double* y) {
+    int r = kernel / 2;
+    for (int t = 0; t < n; ++t) {
+        int lo = t - r < 0 ? 0 : t - r;
+        int hi = t + r > n - 1 ? n - 1 : t + r;
+        double s = 0.0;
+        for (int j = lo; j <= hi; ++j) s += x[j];
+        y[t] = s / (hi - lo + 1);
+    }
+}
+
 /* 1-D max-pool, width `kernel`, stride 1, over x[0, n); neighbours outside [0, n) are ignored. */
 static void max_pool(const double* x, int n, int kernel, double* y) {
     int r = kernel / 2;
@@ -105,6 +119,8 @@ int kvo_select_layer(const kvo_params* p, int batch, const int32_t* cu_seqlens, 
     if (Hkv < 1 || Hq < Hkv || Hq % Hkv != 0 || d < 1 || w < 1) return -2;
     if (O < 1 || Oe < 1 || O > w || Oe > w) return -3;
     if (p->pool_kernel < 1 || p->pool_kernel % 2 == 0) return -4;
+    if (p->pool_mode != 0 && p->pool_mode != 1) return -4;
+    if (p->head_criterion != 0 && p->head_criterion != 1) return -5;
     if (p->num_ext_heads < 0 || p->num_ext_heads > Hkv) return -5;
     if (!(p->beta >= 0.0 && p->beta <= 1.0)) return -6;
     if (budget < w) return -7;
@@ -202,21 +218,36 @@ int kvo_select_layer(const kvo_params* p, int batch, const int32_t* cu_seqlens, 
         for (int t = 0; t < L; ++t) Iraw[t] /= O;
         free(Akv);
 
-        /* Step 4: max-pool every row over the candidates [0, Lc). */
+        /* Step 4: pool every row over the candidates [0, Lc) (max, or the average variant). */
+        void (*pool)(const double*, int, int, double*) = p->pool_mode == 1 ? avg_pool : max_pool;
         double* PpO = (double*)calloc((size_t)Hkv * (Lc > 0 ? Lc : 1), sizeof(double));
         double* PpOe = (double*)calloc((size_t)Hkv * (Lc > 0 ? Lc : 1), sizeof(double));
         double* Ip = (double*)calloc((size_t)(Lc > 0 ? Lc : 1), sizeof(double));
         for (int h = 0; h < Hkv && Lc > 0; ++h) {
-            max_pool(PO + (size_t)h * L, Lc, p->pool_kernel, PpO + (size_t)h * Lc);
-            max_pool(POe + (size_t)h * L, Lc, p->pool_kernel, PpOe + (size_t)h * Lc);
+            pool(PO + (size_t)h * L, Lc, p->pool_kernel, PpO + (size_t)h * Lc);
+            pool(POe + (size_t)h * L, Lc, p->pool_kernel, PpOe + (size_t)h * Lc);
         }
-        if (Lc > 0) max_pool(Iraw, Lc, p->pool_kernel, Ip);
+        if (Lc > 0) pool(Iraw, Lc, p->pool_kernel, Ip);
 
         /* Step 5 (Section 4.1): sigma_h = std(P_h) over candidates; the delta heads
          * with the lowest sigma take the extended-window scores. */
         double* sigma = (double*)calloc((size_t)Hkv, sizeof(double));
         int* htop = (int*)calloc((size_t)Hkv, sizeof(int));
-        for (int h = 0; h < Hkv; ++h) {
+        for (int h = 0; h < Hkv && p->head_criterion == 1; ++h) {
+            /* Entropy variant (Section 5.4, "Head Selection Criteria"): the least
+             * focused heads have the highest entropy of their pooled scores
+             * normalised over the candidates; the key is minus that entropy so the
+             * same lowest-first ranking applies.  0 with no mass. */
+            const double* x = PpO + (size_t)h * Lc;
+            double S = 0.0;
+            for (int t = 0; t < Lc; ++t) S += x[t];
+            double H = 0.0;
+            if (S > 0.0)
+                for (int t = 0; t < Lc; ++t)
+                    if (x[t] > 0.0) H -= (x[t] / S) * log(x[t] / S);
+            sigma[h] = -H;
+        }
+        for (int h = 0; h < Hkv && p->head_criterion == 0; ++h) {
             if (Lc < 2) { sigma[h] = 0.0; continue; }
             const double* x = PpO + (size_t)h * Lc;
             double mean = 0.0;

@@ -32,6 +32,9 @@ typedef struct {
     double lambda;       /* lambda (Section 4.2) */
     double beta;         /* beta: preserved fraction of the budget (Section 4.2) */
     double softmax_scale;/* <= 0 selects 1/sqrt(d) */
+    int pool_mode;       /* 0: max-pool (default); 1: average over the in-range neighbours */
+    int head_criterion;  /* 0: standard deviation (Section 4.1, default); 1: entropy
+                            (Section 5.4 ablation, "Head Selection Criteria") */
 } kvo_params;
 
 /* Optional debug outputs.  Any pointer may be NULL.  Sizes use the caller's
@@ -43,7 +46,8 @@ typedef struct {
     double* P_O;         /* [batch][H_kv][ML] max-pooled over candidates t < L - w */
     double* P_Oext;      /* [batch][H_kv][ML] */
     double* I;           /* [batch][ML] */
-    double* sigma;       /* [batch][H_kv] std of pooled P_O over candidates */
+    double* sigma;       /* [batch][H_kv] the heads' ranking key (lowest first): the std of
+                            pooled P_O over candidates, or minus its entropy */
     int32_t* htop;       /* [batch][H_kv] 1 if the head gets the extended window */
     double* P;           /* [batch][H_kv][ML] priority after the cross-head step */
     uint8_t* pres;       /* [batch][H_kv][ML] 1 for the preserved top-K tokens */

@@ -44,6 +44,8 @@ class Workload:
     obs_window: int = 16      # O
     ext_window: int = 32      # O'
     pool_kernel: int = 7
+    pool_mode: int = 0        # 0 max-pool, 1 average pool (variant)
+    head_criterion: int = 0   # 0 standard deviation, 1 entropy (variant)
     budget: int = 512         # B per KV head, window included
     num_ext_heads: int = 3    # delta
     lam: float = 1.0          # lambda

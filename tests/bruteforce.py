@@ -37,7 +37,8 @@ def _ranked(score: np.ndarray, positions: np.ndarray) -> np.ndarray:
 
 
 def select(q_full, k, *, num_kv_heads, window, obs_window, ext_window, pool_kernel,
-           num_ext_heads, lam, beta, budget, n_counts, layers_done, scale=None) -> Dict[str, np.ndarray]:
+           num_ext_heads, lam, beta, budget, n_counts, layers_done, scale=None, pool_mode=0,
+           head_criterion=0) -> Dict[str, np.ndarray]:
     """Algorithm 1 followed by per-head top-B for one sequence of length T = q_full.shape[0]."""
     T, Hq, d = q_full.shape
     Hkv = num_kv_heads
@@ -56,13 +57,24 @@ def select(q_full, k, *, num_kv_heads, window, obs_window, ext_window, pool_kern
     r = pool_kernel // 2
 
     def pool(x):
+        if pool_mode == 1:
+            return np.array([x[max(0, t - r):min(Lc, t + r + 1)].mean() for t in range(Lc)])
         return np.array([x[max(0, t - r):min(Lc, t + r + 1)].max() for t in range(Lc)])
 
     PO = np.stack([pool(P_O_raw[h]) for h in range(Hkv)]) if Lc > 0 else np.zeros((Hkv, 0))
     POe = np.stack([pool(P_Oe_raw[h]) for h in range(Hkv)]) if Lc > 0 else np.zeros((Hkv, 0))
     I = pool(I_raw) if Lc > 0 else np.zeros(0)
 
-    sigma = PO.std(axis=1, ddof=1) if Lc >= 2 else np.zeros(Hkv)
+    if head_criterion == 1:
+        # Minus the entropy of each head's pooled scores normalised to a distribution.
+        sigma = np.zeros(Hkv)
+        for h in range(Hkv):
+            tot = PO[h].sum()
+            if tot > 0:
+                pr = PO[h][PO[h] > 0] / tot
+                sigma[h] = float(np.sum(pr * np.log(pr)))
+    else:
+        sigma = PO.std(axis=1, ddof=1) if Lc >= 2 else np.zeros(Hkv)
     head_order = np.lexsort((np.arange(Hkv), sigma))
     htop = np.zeros(Hkv, bool)
     htop[head_order[:num_ext_heads]] = True

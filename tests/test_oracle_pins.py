@@ -309,3 +309,84 @@ def test_oracle_rejects_bad_parameters(bad):
     with pytest.raises(ValueError):
         oracle.select_layer(p, [0, 32], x["q_full"][24:].reshape(1, 8, 8, 8), x["k"], x["v"],
                             oracle.new_state(1, 32), 16)
+
+
+# ---- Paper variants: average pooling and the entropy head criterion (Section 5.4
+# "Head Selection Criteria"; the average pool of the SnapKV lineage).
+
+VARIANT_CASES = [c for c in TINY_CASES if c[0] in (2, 3, 5, 7)]
+
+
+@pytest.mark.parametrize("pool_mode,head_criterion", [(1, 0), (0, 1), (1, 1)])
+@pytest.mark.parametrize("case", VARIANT_CASES)
+def test_oracle_variants_match_bruteforce(case, pool_mode, head_criterion):
+    seed, T, Hq, Hkv, d, w, O, Oe, pool, delta, lam, beta, B = case
+    params = oracle.OracleParams(num_q_heads=Hq, num_kv_heads=Hkv, head_dim=d, window=w,
+                                 obs_window=O, ext_window=Oe, pool_kernel=pool,
+                                 num_ext_heads=delta, lam=lam, beta=beta, pool_mode=pool_mode,
+                                 head_criterion=head_criterion)
+    state = oracle.new_state(1, T)
+    n_bf = np.zeros(T, np.int64)
+    for layer in range(2):
+        x = synth.tiny_full_inputs(seed * 100 + layer, T, Hq, Hkv, d)
+        q_obs = x["q_full"][T - w:].reshape(1, w, Hq, d)
+        r = _run_oracle(params, q_obs, x["k"], x["v"], state, B)
+        bf = bf_select(_f64(x["q_full"]), _f64(x["k"]), num_kv_heads=Hkv, window=w, obs_window=O,
+                       ext_window=Oe, pool_kernel=pool, num_ext_heads=delta, lam=lam, beta=beta,
+                       budget=B, n_counts=n_bf, layers_done=layer, pool_mode=pool_mode,
+                       head_criterion=head_criterion)
+        Lc = T - w
+        np.testing.assert_allclose(r["P_O"][0, :, :Lc], bf["P_O"], rtol=1e-12, atol=1e-15)
+        np.testing.assert_allclose(r["P_Oext"][0, :, :Lc], bf["P_Oext"], rtol=1e-12, atol=1e-15)
+        np.testing.assert_allclose(r["I"][0, :Lc], bf["I"], rtol=1e-12, atol=1e-15)
+        np.testing.assert_allclose(r["sigma"][0], bf["sigma"], rtol=1e-9, atol=1e-15)
+        assert (r["htop"][0].astype(bool) == bf["htop"]).all()
+        np.testing.assert_allclose(r["Pprime"][0, :, :Lc], bf["Pprime"], rtol=1e-12, atol=1e-15)
+        assert (r["out_idx"][0] == bf["out_idx"]).all()
+        n_bf = bf["n"]
+
+
+def _tiny_layer(seed, T=48, Hq=8, Hkv=4, d=8, w=8):
+    x = synth.tiny_full_inputs(seed, T, Hq, Hkv, d)
+    return x["q_full"][T - w:].reshape(1, w, Hq, d), x["k"], x["v"]
+
+
+@pytest.mark.parametrize("delta", [0, 4])
+def test_head_criterion_is_moot_when_no_or_every_head_is_extended(delta):
+    q, k, v = _tiny_layer(11)
+    out = []
+    for crit in (0, 1):
+        p = oracle.OracleParams(num_q_heads=8, num_kv_heads=4, head_dim=8, window=8, obs_window=4, ext_window=8,
+                                pool_kernel=3, num_ext_heads=delta, head_criterion=crit)
+        out.append(_run_oracle(p, q, k, v, oracle.new_state(1, 48), 20)["out_idx"])
+    assert np.array_equal(out[0], out[1])
+
+
+def test_average_pool_of_width_one_is_the_identity():
+    q, k, v = _tiny_layer(12)
+    res = []
+    for mode in (0, 1):
+        p = oracle.OracleParams(num_q_heads=8, num_kv_heads=4, head_dim=8, window=8, obs_window=4, ext_window=8,
+                                pool_kernel=1, num_ext_heads=2, pool_mode=mode)
+        res.append(_run_oracle(p, q, k, v, oracle.new_state(1, 48), 20))
+    for name in ("P_O", "P_Oext", "I"):
+        assert np.array_equal(res[0][name], res[1][name])
+    assert np.array_equal(res[0]["out_idx"], res[1]["out_idx"])
+
+
+def test_uniform_keys_closed_forms_for_the_variants():
+    """K = 0: the candidates' raw scores are one constant per row, so the average
+    pool returns it unchanged and every head's normalised distribution is uniform:
+    entropy ln(Lc), key -ln(Lc)."""
+    T, Hq, Hkv, d, w, O, Oe, B = 64, 4, 2, 8, 8, 4, 8, 24
+    g = Hq // Hkv
+    x = synth.tiny_full_inputs(3, T, Hq, Hkv, d)
+    q_obs = x["q_full"][T - w:].reshape(1, w, Hq, d)
+    k = torch.zeros(T, Hkv, d, dtype=torch.bfloat16)
+    p = oracle.OracleParams(num_q_heads=Hq, num_kv_heads=Hkv, head_dim=d, window=w, obs_window=O, ext_window=Oe,
+                            pool_kernel=5, num_ext_heads=1, pool_mode=1, head_criterion=1)
+    r = _run_oracle(p, q_obs, k, x["v"], oracle.new_state(1, T), B)
+    Lc = T - w
+    expect_PO = g / O * sum(1.0 / (T - w + q + 1) for q in range(w - O, w))
+    np.testing.assert_allclose(r["P_O"][0, :, :Lc], expect_PO, rtol=1e-13)
+    np.testing.assert_allclose(r["sigma"][0], -math.log(Lc), rtol=1e-13)

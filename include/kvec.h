@@ -71,6 +71,12 @@ typedef struct {
     int   max_batch;      /* largest batch a call may pass */
     int   max_seqlen;     /* largest prefix length L a call may pass (<= 131072) */
     int   max_layers;     /* layers one coverage state may see (<= 255; n_t is 8-bit) */
+    int   pool_mode;      /* 0: max-pool (the paper's setting, default); 1: average of the
+                             in-range neighbours (variant of the SnapKV lineage) */
+    int   head_criterion; /* 0: the delta heads with the lowest standard deviation of pooled
+                             P_O take O' (Section 4.1, default); 1: those with the highest
+                             entropy of pooled P_O normalised over the candidates (the
+                             Section 5.4 ablation "Head Selection Criteria") */
 } kvec_params;
 
 /* Creates a handle and allocates its device workspace on the current device.
@@ -220,7 +226,9 @@ typedef struct {
     const float*    P_O;        /* [max_batch][H_kv][ML]  Eq. 1 with O, max-pooled */
     const float*    P_Oext;     /* [max_batch][H_kv][ML]  Eq. 1 with O', max-pooled */
     const float*    I;          /* [max_batch][ML]        Section 4.2 importance, max-pooled */
-    const float*    sigma;      /* [max_batch][H_kv]      std of pooled P_O over candidates */
+    const float*    sigma;      /* [max_batch][H_kv]      the heads' ranking key (lowest first):
+                                   std of pooled P_O over candidates, or minus its
+                                   entropy when head_criterion = 1 */
     const int32_t*  htop;       /* [max_batch][H_kv]      1 if the head uses O' */
     const uint32_t* pres_bits;  /* [max_batch][H_kv][ceil(ML/32)] preserved top-K tokens */
     const float*    Pprime;     /* [max_batch][H_kv][ML]  P + lambda * focus */

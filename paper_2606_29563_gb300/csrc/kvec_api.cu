@@ -133,6 +133,9 @@ kvec_status validate_params(const kvec_params* p) {
                     g, p->window);
     if (p->pool_kernel < 1 || p->pool_kernel > kMaxPool || p->pool_kernel % 2 == 0)
         return fail(KVEC_ERR_INVALID_ARG, "pool_kernel must be odd and in [1, %d]", kMaxPool);
+    if (p->pool_mode != 0 && p->pool_mode != 1) return fail(KVEC_ERR_INVALID_ARG, "pool_mode must be 0 or 1");
+    if (p->head_criterion != 0 && p->head_criterion != 1)
+        return fail(KVEC_ERR_INVALID_ARG, "head_criterion must be 0 or 1");
     if (p->num_ext_heads < 0 || p->num_ext_heads > p->num_kv_heads)
         return fail(KVEC_ERR_INVALID_ARG, "num_ext_heads must be in [0, num_kv_heads]");
     if (!(p->beta >= 0.f && p->beta <= 1.f)) return fail(KVEC_ERR_INVALID_ARG, "beta must be in [0, 1]");
@@ -198,6 +201,8 @@ Geometry make_geometry(const kvec_handle* h, int batch, int budget, int tiles, i
     G.O = p.obs_window;
     G.Oe = p.ext_window;
     G.pool = p.pool_kernel;
+    G.pool_avg = p.pool_mode;
+    G.head_entropy = p.head_criterion;
     G.delta = p.num_ext_heads;
     G.R = h->R;
     G.lambda = p.lambda;

@@ -19,6 +19,8 @@ constexpr int kWinHeadsPerCta = 8; // KV heads one window CTA processes
 // Sizes and hyper-parameters shared by every kernel of one call.
 struct Geometry {
     int Hq, Hkv, g, w, O, Oe, pool, delta;
+    int pool_avg;      // 1: average pool instead of max-pool
+    int head_entropy;  // 1: rank heads by minus the entropy of pooled P_O instead of its std
     int R;             // rows per KV head = g * w, ordered r = q * g + j
     float lambda;
     float sl2;         // softmax scale * log2(e)

@@ -448,7 +448,7 @@ struct Pooled4 {
 };
 
 __device__ __forceinline__ Pooled4 pool4(const float* __restrict__ raw, size_t stride, int parts, int t4, int Lc,
-                                         int halo) {
+                                         int halo, bool avg) {
     float x[20];
 #pragma unroll
     for (int i = 0; i < 20; ++i) x[i] = 0.f;
@@ -468,10 +468,30 @@ __device__ __forceinline__ Pooled4 pool4(const float* __restrict__ raw, size_t s
             x[4 * b + 3] += f[b].w;
         }
     }
+    Pooled4 out;
+    if (avg) {
+        // Average variant: the mean of the in-range neighbours.
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            float sum = x[8 + i], cnt = 1.f;
+#pragma unroll
+            for (int d = 1; d <= kMaxPool / 2; ++d) {
+                if (d <= halo && t4 + i - d >= 0) {
+                    sum += x[8 + i - d];
+                    cnt += 1.f;
+                }
+                if (d <= halo && t4 + i + d < Lc) {
+                    sum += x[8 + i + d];
+                    cnt += 1.f;
+                }
+            }
+            out.v[i] = sum / cnt;
+        }
+        return out;
+    }
 #pragma unroll
     for (int i = 0; i < 20; ++i)
         if (t4 - 8 + i < 0 || t4 - 8 + i >= Lc) x[i] = -INFINITY;
-    Pooled4 out;
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
         float m = x[8 + i];
@@ -508,6 +528,30 @@ struct Moments {
     }
 };
 
+// Sums of a and b over the block (the result is valid in thread 0).
+__device__ float2 block_sum2(float a, float b, float3* red) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    for (int off = 16; off; off >>= 1) {
+        a += __shfl_xor_sync(0xffffffffu, a, off);
+        b += __shfl_xor_sync(0xffffffffu, b, off);
+    }
+    if (lane == 0) red[warp] = make_float3(a, b, 0.f);
+    __syncthreads();
+    float2 r = make_float2(0.f, 0.f);
+    if (warp == 0) {
+        const float3 v = lane < nw ? red[lane] : make_float3(0.f, 0.f, 0.f);
+        a = v.x;
+        b = v.y;
+        for (int off = 16; off; off >>= 1) {
+            a += __shfl_xor_sync(0xffffffffu, a, off);
+            b += __shfl_xor_sync(0xffffffffu, b, off);
+        }
+        r = make_float2(a, b);
+    }
+    __syncthreads();
+    return r;
+}
+
 __device__ Moments block_moments(Moments v, float3* red) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
     for (int off = 16; off; off >>= 1)
@@ -525,9 +569,11 @@ __device__ Moments block_moments(Moments v, float3* red) {
 }
 
 // Section 4.1, first half.  One CTA per (KV head, sequence): pool the head's
-// P_O and P_O' rows and a slice of I (max-pool, inherited from SnapKV) and
-// sigma_h = sample std of pooled P_O over the candidates (Welford/Chan moments
-// in fp32).
+// P_O and P_O' rows and a slice of I (max-pool, inherited from SnapKV; or the
+// average variant) and the head's ranking key: sigma_h = sample std of pooled
+// P_O over the candidates (Welford/Chan moments in fp32), or, for the entropy
+// criterion of the Section 5.4 ablation, minus the entropy of pooled P_O
+// normalised over the candidates, sum(x ln x)/S - ln S with S = sum(x).
 __global__ void __launch_bounds__(kSelectThreads) heads_pool_kernel(Geometry G, LayerIO io, Scratch sc, Slot sl) {
     __shared__ float3 red[32];
     extern __shared__ float mbuf[];   // raw I of a chunk, per window row (several head groups only)
@@ -540,16 +586,25 @@ __global__ void __launch_bounds__(kSelectThreads) heads_pool_kernel(Geometry G, 
     // Pool P_O and P_O' of this head (four positions per thread per step) and
     // accumulate the moments of pooled P_O.
     Moments mom{0.f, 0.f, 0.f};
+    float es = 0.f, exl = 0.f;   // entropy criterion: sum x, sum x ln x
+    const bool avg = G.pool_avg != 0, entropy = G.head_entropy != 0;
     const float* rO = sl.rawO + row * G.ML;
     const float* rOe = sl.rawOe + row * G.ML;
     for (int t4 = 4 * tid; t4 < Lc; t4 += 4 * NT) {
-        const Pooled4 a = pool4(rO, 0, 1, t4, Lc, halo);
-        const Pooled4 b = pool4(rOe, 0, 1, t4, Lc, halo);
+        const Pooled4 a = pool4(rO, 0, 1, t4, Lc, halo, avg);
+        const Pooled4 b = pool4(rOe, 0, 1, t4, Lc, halo, avg);
         *reinterpret_cast<float4*>(sl.PO + row * G.ML + t4) = make_float4(a.v[0], a.v[1], a.v[2], a.v[3]);
         *reinterpret_cast<float4*>(sl.POe + row * G.ML + t4) = make_float4(b.v[0], b.v[1], b.v[2], b.v[3]);
 #pragma unroll
-        for (int i = 0; i < 4; ++i)
-            if (t4 + i < Lc) mom.add(a.v[i]);
+        for (int i = 0; i < 4; ++i) {
+            if (t4 + i >= Lc) continue;
+            if (entropy) {
+                es += a.v[i];
+                if (a.v[i] > 0.f) exl = fmaf(a.v[i], logf(a.v[i]), exl);
+            } else {
+                mom.add(a.v[i]);
+            }
+        }
     }
     // This CTA's slice of pooled I.
     {
@@ -558,7 +613,7 @@ __global__ void __launch_bounds__(kSelectThreads) heads_pool_kernel(Geometry G, 
         if (G.NG == 1) {
             const float* rI = sl.rawI + (size_t)s * G.ML;
             for (int t4 = a0 + 4 * tid; t4 < b0; t4 += 4 * NT) {
-                const Pooled4 c = pool4(rI, 0, 1, t4, Lc, halo);
+                const Pooled4 c = pool4(rI, 0, 1, t4, Lc, halo, avg);
                 *reinterpret_cast<float4*>(sl.I + (size_t)s * G.ML + t4) = make_float4(c.v[0], c.v[1], c.v[2], c.v[3]);
             }
         } else {
@@ -610,12 +665,18 @@ __global__ void __launch_bounds__(kSelectThreads) heads_pool_kernel(Geometry G, 
                 }
                 __syncthreads();
                 for (int t = c + tid; t < ce; t += NT) {
-                    float m = mbuf[t - lo];
+                    float m = mbuf[t - lo], cnt = 1.f;
                     for (int d = 1; d <= halo; ++d) {
-                        if (t - d >= 0) m = fmaxf(m, mbuf[t - d - lo]);
-                        if (t + d < Lc) m = fmaxf(m, mbuf[t + d - lo]);
+                        if (t - d >= 0) {
+                            m = avg ? m + mbuf[t - d - lo] : fmaxf(m, mbuf[t - d - lo]);
+                            cnt += 1.f;
+                        }
+                        if (t + d < Lc) {
+                            m = avg ? m + mbuf[t + d - lo] : fmaxf(m, mbuf[t + d - lo]);
+                            cnt += 1.f;
+                        }
                     }
-                    sl.I[(size_t)s * G.ML + t] = m;
+                    sl.I[(size_t)s * G.ML + t] = avg ? m / cnt : m;
                 }
                 __syncthreads();
             }
@@ -623,8 +684,13 @@ __global__ void __launch_bounds__(kSelectThreads) heads_pool_kernel(Geometry G, 
     }
     // The preserved-token kernel may be scheduled now; it waits for this grid before reading sigma.
     asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
-    mom = block_moments(mom, red);
-    if (tid == 0) sl.sigma[row] = Lc >= 2 ? sqrtf(fmaxf(mom.m2, 0.f) / (float)(Lc - 1)) : 0.f;
+    if (entropy) {
+        const float2 se = block_sum2(es, exl, red);
+        if (tid == 0) sl.sigma[row] = se.x > 0.f ? se.y / se.x - logf(se.x) : 0.f;
+    } else {
+        mom = block_moments(mom, red);
+        if (tid == 0) sl.sigma[row] = Lc >= 2 ? sqrtf(fmaxf(mom.m2, 0.f) / (float)(Lc - 1)) : 0.f;
+    }
 }
 
 // Section 4.1, second half, and the preserved tokens of Section 4.2.  One CTA

@@ -66,6 +66,27 @@ def test_hyperparameter_corners(over):
     _assert_parity(synth.small_workload(seqlens=(777,), layers=2, **over))
 
 
+@pytest.mark.parametrize("over", [dict(pool_mode=1), dict(head_criterion=1),
+                                  dict(pool_mode=1, head_criterion=1, num_ext_heads=2, pool_kernel=5),
+                                  dict(window=48, obs_window=32, ext_window=48)])
+def test_paper_variants(over):
+    # Average pooling, the entropy head criterion (Section 5.4 ablation) and the
+    # O = 32 / O' = 48 reading of the windows.
+    _assert_parity(synth.small_workload(seqlens=(900, 421), layers=2, **over))
+
+
+@pytest.mark.parametrize("over", [dict(pool_mode=1), dict(head_criterion=1, num_ext_heads=5)])
+def test_paper_variants_with_split_head_groups(over):
+    # 16 KV heads: the window kernel splits them over two CTAs per tile and the
+    # heads kernel combines the groups' maxima of I before pooling.
+    _assert_parity(synth.small_workload(seqlens=(700,), num_q_heads=16, num_kv_heads=16, layers=2, **over))
+
+
+def test_variants_llama8b_l8192_b512_first_layers():
+    wl = synth.WORKLOADS["llama8b_l8192_b512"].replace(layers=2, pool_mode=1, head_criterion=1)
+    _assert_parity(wl)
+
+
 def test_uniform_keys_tie_to_lowest_positions():
     """K = 0 makes every candidate score equal: selection must be the lowest positions (exact ties)."""
     wl = synth.small_workload(seqlens=(400,), budget=64, layers=1)

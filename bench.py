@@ -547,6 +547,8 @@ def main(argv=None):
     ap.add_argument("--layers", type=int, default=None, help="run only the first N layers (not a bench line)")
     ap.add_argument("--no-e2e", dest="e2e", action="store_false")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--coverage-sweep", action="store_true",
+                    help="print the token coverage of K-VEC and SnapKV at eviction rates 0.25-0.9 and exit")
     ap.add_argument("--no-decode", dest="decode", action="store_false",
                     help="skip the decode-attention measurement over the compacted caches")
     ap.add_argument("--no-lse-variant", dest="lse_variant", action="store_false",
@@ -560,6 +562,12 @@ def main(argv=None):
         wl = wl.replace(budget=args.budget, name=f"{wl.name.rsplit('_b', 1)[0]}_b{args.budget}")
     if args.layers:
         wl = wl.replace(layers=args.layers)
+    if args.coverage_sweep:
+        from paper_2606_29563_gb300 import build as kbuild
+        from paper_2606_29563_gb300 import coverage
+        kbuild.build()
+        print(json.dumps({"coverage_sweep": coverage.sweep(wl), "data": "synthetic"}), flush=True)
+        return 0
     rank, result = (run_reference if args.impl == "reference" else run_ours)(args, wl)
     if rank == 0 and result is not None:
         print(json.dumps(result), flush=True)

@@ -166,6 +166,7 @@ def committed_traffic(kernel: str, workload: str):
         return None
 
 
+E2E_CHUNK = 8            # layers per kvec_select_layers call in the end-to-end step
 LAUNCHES_PER_LAYER = 7   # score, row statistics, window, heads pooling, heads top-K, select, gather
 
 
@@ -461,22 +462,49 @@ def run_decode(args, wl, sel, layers, outs, dev, peak):
 
 
 def run_e2e(args, wl, sel, layers, outs, state, cu_host, cu_dev, dev, stream):
+    """End to end through the public API.  Every step copies the step's inputs
+    (q_obs, K, V of every layer) from pinned host memory and reads the kept
+    indices and the coverage state back.  The copies run on their own stream in
+    chunks of E2E_CHUNK layers; a chunk's selection (one kvec_select_layers call,
+    replayed from the handle's graph cache) starts once its inputs have landed,
+    so it overlaps the copy of the next chunks.  Two sets of device input
+    buffers alternate between steps, so the next step's copies do not wait for
+    this step's last chunk.  The host link (about 210 GB/s measured on this
+    machine for pinned copies, by copy engine or by SM loads alike) bounds the
+    step."""
     import torch
     from paper_2606_29563_gb300 import kvec
     host = [{k: v.cpu().pin_memory() for k, v in x.items()} for x in layers]
-    dev_in = [{k: torch.empty_like(v) for k, v in x.items()} for x in layers]
+    dev_sets = [[{k: torch.empty_like(v) for k, v in x.items()} for x in layers] for _ in range(2)]
     host_idx = [torch.empty(o[0].shape, dtype=o[0].dtype).pin_memory() for o in outs]
     host_state = torch.empty(state.shape, dtype=state.dtype).pin_memory()
     h2d = sum(t.numel() * t.element_size() for x in host for t in x.values())
     d2h = sum(t.numel() * t.element_size() for t in host_idx) + host_state.numel()
+    copy_stream = torch.cuda.Stream(dev)
+    chunks = [list(range(c, min(c + E2E_CHUNK, len(layers)))) for c in range(0, len(layers), E2E_CHUNK)]
+    landed = [[torch.cuda.Event() for _ in chunks] for _ in range(2)]
+    freed = [torch.cuda.Event() for _ in range(2)]
+    count = [0]
 
     def step():
-        for src, dst in zip(host, dev_in):
-            for k in src:
-                dst[k].copy_(src[k], non_blocking=True)
+        par = count[0] & 1
+        count[0] += 1
+        dev_in, land = dev_sets[par], landed[par]
+        # The selection of two steps ago must be done with this set of input buffers.
+        if count[0] > 2:
+            copy_stream.wait_event(freed[par])
+        with torch.cuda.stream(copy_stream):
+            for c, ls in enumerate(chunks):
+                for l in ls:
+                    for k in ("q_obs", "k", "v"):
+                        dev_in[l][k].copy_(host[l][k], non_blocking=True)
+                land[c].record(copy_stream)
         kvec.kvec_reset(sel.handle, state.data_ptr(), wl.batch, stream.cuda_stream)
-        sel.select_layers(cu_host, cu_dev, [x["q_obs"] for x in dev_in], [x["k"] for x in dev_in],
-                          [x["v"] for x in dev_in], state, wl.budget, outs, stream)
+        for c, ls in enumerate(chunks):
+            stream.wait_event(land[c])
+            sel.select_layers(cu_host, cu_dev, [dev_in[l]["q_obs"] for l in ls], [dev_in[l]["k"] for l in ls],
+                              [dev_in[l]["v"] for l in ls], state, wl.budget, [outs[l] for l in ls], stream)
+        freed[par].record(stream)
         for o, h in zip(outs, host_idx):
             h.copy_(o[0], non_blocking=True)
         host_state.copy_(state, non_blocking=True)
@@ -486,8 +514,9 @@ def run_e2e(args, wl, sel, layers, outs, state, cu_host, cu_dev, dev, stream):
     torch.cuda.synchronize()
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     barrier()
-    start.record(stream)
-    n = max(1, args.steps)
+    # The first copies run on the copy stream: the timed region opens there.
+    start.record(copy_stream)
+    n = max(1, min(args.steps, 200))
     for _ in range(n):
         step()
     stop.record(stream)
@@ -495,8 +524,10 @@ def run_e2e(args, wl, sel, layers, outs, state, cu_host, cu_dev, dev, stream):
     ms = max_over_ranks(start.elapsed_time(stop), dev)
     _, world, _ = dist_env()
     value = world * wl.evicted_per_layer() * wl.layers * n / (ms / 1e3)
-    return {"value": value, "unit": "tokens/s", "ms_per_step": ms / n, "h2d_bytes_per_step": h2d,
-            "d2h_bytes_per_step": d2h}
+    return {"value": value, "unit": "tokens/s", "ms_per_step": ms / n, "steps": n, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h,
+            "api": f"kvec_select_layers per chunk of {E2E_CHUNK} layers on the compute stream; pinned copies of "
+                   "the next chunks on a copy stream"}
 
 
 # ----------------------------------------------------------------------------- reference arm (the oracle)

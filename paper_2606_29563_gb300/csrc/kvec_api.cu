@@ -49,6 +49,7 @@ struct TimedLaunch {
 
 constexpr int kSlots = 8;   // per-layer score arrays in flight between the score and select stages
 constexpr int kScoreBufs = 2;   // score-statistics buffers in flight between the score and window stages
+constexpr size_t kGraphCache = 16;  // captured multi-layer calls kept per handle
 
 struct kvec_handle {
     kvec_params p;
@@ -76,8 +77,14 @@ struct kvec_handle {
     // chain of the pipeline) take SMs before the score, window and gather kernels.
     int prio_hi = 0, prio_lo = 0;
     // CUDA graph of the last repeated multi-layer call.
-    cudaGraphExec_t gexec = nullptr;
-    std::vector<uint64_t> gkey, pending_key;
+    // Captured graphs of repeated multi-layer calls, most recent last (at most
+    // kGraphCache), and the keys of calls seen once (a second sighting captures).
+    struct CachedGraph {
+        std::vector<uint64_t> key;
+        cudaGraphExec_t exec;
+    };
+    std::vector<CachedGraph> graphs;
+    std::vector<std::vector<uint64_t>> seen_keys;
 };
 
 namespace {
@@ -235,7 +242,7 @@ kvec_status run_layer_sequential(kvec_handle* h, const Geometry& G, const LayerI
     if (se != cudaSuccess) return cuda_fail(se, "score kernel tensor maps");
     se = launch_score(plan, st, false);
     if (se != cudaSuccess) return cuda_fail(se, "score kernel launch");
-    se = launch_rowstat(plan, G, io, h->sc, st);
+    se = launch_rowstat(plan, G, io, h->sc, st, true);
     if (se != cudaSuccess) return cuda_fail(se, "row statistics launch");
     se = launch_window(plan, G, io, h->sc, h->slots[0], st, false);
     if (se != cudaSuccess) return cuda_fail(se, "window kernel launch");
@@ -269,29 +276,33 @@ kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* io
         const Slot& sl = h->slots[l % kSlots];
         const Scratch& sc = h->score_buf[l % kScoreBufs];
         const LayerIO& io = ios[l];
+        // Statistics buffer reuse: layer l - kScoreBufs's row statistics and window
+        // (window stream) are done with it.
         if (l >= kScoreBufs) KV_CHECK(cudaStreamWaitEvent(h->s_score, h->ev_win[l - kScoreBufs], 0));
         ScorePlan plan;
         cudaError_t se = plan_score(G, io, sc, h->num_sms, &plan);
         if (se != cudaSuccess) return cuda_fail(se, "score kernel tensor maps");
-        timed_launch(h, 0, h->s_score, [&] {
-            if (io.lse) {
-                se = launch_rowstat_lse(G, io, sc, h->s_score);
-            } else {
-                se = launch_score(plan, h->s_score, true);
-                if (se == cudaSuccess) se = launch_rowstat(plan, G, io, sc, h->s_score);
-            }
-        });
-        if (se != cudaSuccess) return cuda_fail(se, "score kernel launch");
+        // A launch is a programmatic dependent of its stream predecessor only when
+        // no event wait stands between them: in a captured graph a programmatic
+        // launch turns every incoming edge programmatic, those from another
+        // stream's event included, and the kernel could start before that
+        // stream's kernel has finished writing.  The score launch of layer 1 is
+        // the only one without a wait before it.
+        if (!io.lse) {
+            timed_launch(h, 0, h->s_score, [&] { se = launch_score(plan, h->s_score, l > 0 && l < kScoreBufs); });
+            if (se != cudaSuccess) return cuda_fail(se, "score kernel launch");
+        }
         KV_CHECK(cudaEventRecord(h->ev_score[l], h->s_score));
+        // Window stream: the row statistics (after the score grid and, for slot
+        // reuse, after layer l - kSlots's selection and gather), then the window
+        // sums as their programmatic dependent (it waits before reading them).
         KV_CHECK(cudaStreamWaitEvent(h->s_win, h->ev_score[l], 0));
-        // Slot reuse: the window, heads and select of this layer rewrite the slot
-        // that layer l - kSlots used; its selection and gather (which reads the
-        // slot's kept bits) are done first.  The select stream itself then waits
-        // only for this layer's heads, so consecutive selections stay programmatic.
         if (l >= kSlots) {
             KV_CHECK(cudaStreamWaitEvent(h->s_win, h->ev_sel[l - kSlots], 0));
             KV_CHECK(cudaStreamWaitEvent(h->s_win, h->ev_gather[l - kSlots], 0));
         }
+        se = io.lse ? launch_rowstat_lse(G, io, sc, h->s_win) : launch_rowstat(plan, G, io, sc, h->s_win, false);
+        if (se != cudaSuccess) return cuda_fail(se, "row statistics launch");
         timed_launch(h, 1, h->s_win, [&] { se = launch_window(plan, G, io, sc, sl, h->s_win, true); });
         if (se != cudaSuccess) return cuda_fail(se, "window kernel launch");
         KV_CHECK(cudaEventRecord(h->ev_win[l], h->s_win));
@@ -348,7 +359,8 @@ std::vector<uint64_t> graph_key(int n, int batch, int budget, const int32_t* cu_
 namespace {
 
 void release_handle(kvec_handle* h) {
-    if (h->gexec) cudaGraphExecDestroy(h->gexec);
+    for (auto& g : h->graphs) cudaGraphExecDestroy(g.exec);
+    h->graphs.clear();
     for (cudaStream_t st : {h->s_score, h->s_win, h->s_heads, h->s_heads2, h->s_chain, h->s_gather, h->s_cap})
         if (st) cudaStreamDestroy(st);
     for (auto* v : {&h->ev_score, &h->ev_win, &h->ev_heads, &h->ev_sel, &h->ev_gather})
@@ -573,14 +585,17 @@ kvec_status select_layers_impl(kvec_handle* h, int num_layers, int batch, const 
     if (!h->profiling && num_layers >= 2) {
         // A call repeated with the same arguments replays a captured graph of the pipeline.
         std::vector<uint64_t> key = graph_key(num_layers, batch, budget, cu_seqlens_host, cu_seqlens_dev, ios.data());
-        if (h->gexec && key == h->gkey) {
-            KV_CHECK(cudaGraphLaunch(h->gexec, st));
+        for (size_t i = 0; i < h->graphs.size(); ++i) {
+            if (h->graphs[i].key != key) continue;
+            KV_CHECK(cudaGraphLaunch(h->graphs[i].exec, st));
             h->last_slot = (num_layers - 1) % kSlots;
             h->last_parity = (num_layers - 1) % kScoreBufs;
             h->last_batch = batch;
             return KVEC_OK;
         }
-        if (key == h->pending_key) {
+        bool seen = false;
+        for (const auto& k : h->seen_keys) seen = seen || k == key;
+        if (seen) {
             cudaGraph_t graph = nullptr;
             KV_CHECK(cudaStreamBeginCapture(h->s_cap, cudaStreamCaptureModeThreadLocal));
             s = launch_pipeline(h, G, ios.data(), num_layers, h->s_cap);
@@ -594,14 +609,17 @@ kvec_status select_layers_impl(kvec_handle* h, int num_layers, int batch, const 
             ce = cudaGraphInstantiateWithFlags(&exec, graph, cudaGraphInstantiateFlagUseNodePriority);
             cudaGraphDestroy(graph);
             if (ce != cudaSuccess) return cuda_fail(ce, "cudaGraphInstantiate");
-            if (h->gexec) cudaGraphExecDestroy(h->gexec);
-            h->gexec = exec;
-            h->gkey = key;
-            KV_CHECK(cudaGraphLaunch(h->gexec, st));
+            if (h->graphs.size() == kGraphCache) {
+                cudaGraphExecDestroy(h->graphs.front().exec);
+                h->graphs.erase(h->graphs.begin());
+            }
+            h->graphs.push_back({key, exec});
+            KV_CHECK(cudaGraphLaunch(exec, st));
             h->last_batch = batch;
             return KVEC_OK;
         }
-        h->pending_key = key;
+        if (h->seen_keys.size() == kGraphCache) h->seen_keys.erase(h->seen_keys.begin());
+        h->seen_keys.push_back(key);
     }
     s = launch_pipeline(h, G, ios.data(), num_layers, st);
     if (s != KVEC_OK) return s;

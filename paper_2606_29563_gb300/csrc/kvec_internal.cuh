@@ -124,7 +124,8 @@ cudaError_t plan_score(const Geometry& g, const LayerIO& io, const Scratch& sc, 
 cudaError_t launch_score(const ScorePlan& plan, cudaStream_t st, bool after_own_launch);
 // (m_r, Z_r) from the score launch's partials; launched right after it on the same stream.
 cudaError_t launch_rowstat(const ScorePlan& plan, const Geometry& g, const LayerIO& io, const Scratch& sc,
-                           cudaStream_t st);
+                           cudaStream_t st,
+                           bool after_score);
 // (m_r, Z_r) = (lse * log2(e), 1) from the caller's log-sum-exp (io.lse), in place
 // of the score and row-statistics launches.
 cudaError_t launch_rowstat_lse(const Geometry& g, const LayerIO& io, const Scratch& sc, cudaStream_t st);

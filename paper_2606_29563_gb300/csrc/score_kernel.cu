@@ -386,8 +386,8 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
 // the head's range of items.  Grid (Hkv, batch), one thread per row.
 __global__ void __launch_bounds__(256) rowstat_kernel(Geometry G, Scratch sc, const int* __restrict__ cu, int W,
                                                       int Gc) {
-    // A programmatic dependent of the score launch: its partials are read only
-    // after that grid has completed.
+    // Possibly a programmatic dependent of the score launch: its partials are read
+    // only after that grid has completed.  The window launch that follows may start.
     if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
     asm volatile("griddepcontrol.wait;\n" ::: "memory");
     const int h = blockIdx.x, s = blockIdx.y, r = threadIdx.x;
@@ -431,6 +431,8 @@ __global__ void __launch_bounds__(256) rowstat_kernel(Geometry G, Scratch sc, co
 // denominator its prefill attention already computed): row r = q * g + j of KV
 // head h is query head h * g + j at window position q.  Grid (Hkv, batch).
 __global__ void __launch_bounds__(256) rowstat_lse_kernel(Geometry G, Scratch sc, const float* __restrict__ lse) {
+    // The window launch that follows may start; it waits for this grid before reading.
+    if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
     const int h = blockIdx.x, s = blockIdx.y, r = threadIdx.x;
     if (r >= G.R) return;
     const int q = r / G.g, j = r - q * G.g;
@@ -532,7 +534,7 @@ cudaError_t plan_score(const Geometry& g, const LayerIO& io, const Scratch& sc, 
 }
 
 cudaError_t launch_rowstat(const ScorePlan& plan, const Geometry& g, const LayerIO& io, const Scratch& sc,
-                           cudaStream_t st) {
+                           cudaStream_t st, bool after_score) {
     const ScoreArgs& a = *reinterpret_cast<const ScoreArgs*>(plan.args);
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(g.Hkv, g.batch);
@@ -542,7 +544,7 @@ cudaError_t launch_rowstat(const ScorePlan& plan, const Geometry& g, const Layer
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = after_score ? 1 : 0;   // a programmatic dependent of the score launch right before it
     return cudaLaunchKernelEx(&cfg, rowstat_kernel, g, sc, io.cu, a.W, plan.grid);
 }
 

@@ -139,9 +139,6 @@ __global__ void __launch_bounds__(kWinThreads, 1)
     if (threadIdx.x == 0) {
         ptx::prefetch_tensormap(&kmap);
         ptx::prefetch_tensormap(&qmap);
-        // The next launch on this stream (the next layer's window sums) reads
-        // nothing this grid writes: let it be scheduled as SMs free up.
-        asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
     }
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     // Scalars and pointers in registers: values read through a reference to the
@@ -273,6 +270,9 @@ __global__ void __launch_bounds__(kWinThreads, 1)
         const int qO = G.w - G.O, qOe = G.w - G.Oe;
         const float invO = 1.f / (float)G.O, invOe = 1.f / (float)G.Oe;
         // Row statistics of every head of the group: A = 2^(s * sl2 - (m_r + log2 Z_r)).
+        // They come from the launch this grid is a programmatic dependent of: wait
+        // for it here, after the set-up and the first operand loads.
+        asm volatile("griddepcontrol.wait;\n" ::: "memory");
         for (int i = e; i < nh * R; i += kEpiThreads) {
             const int hh = i / R, r = i - hh * R;
             const float2 ms = __ldcg(&sc.rowstat[((size_t)s * G.Hkv + h0 + hh) * R + r]);
@@ -391,9 +391,10 @@ cudaError_t launch_window(const ScorePlan& sp, const Geometry& g, const LayerIO&
     a.tmem_cols = cols;
     const size_t smem = win_smem_bytes(a.Npad, g.O, a.kst);
     const int grid = g.win_tiles * g.NG;
-    // after_own_launch: the previous kernel on the stream is the previous
-    // layer's launch, whose results this grid does not read; the launch is then
-    // its programmatic dependent and never executes griddepcontrol.wait.
+    // after_own_launch: the previous kernel on the stream is this layer's
+    // row-statistics launch and no event wait stands between them; the launch is
+    // then its programmatic dependent and waits (griddepcontrol.wait) right
+    // before reading the statistics.
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
     cfg.blockDim = dim3(kWinThreads);

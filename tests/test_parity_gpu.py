@@ -124,6 +124,31 @@ def test_deterministic_rerun():
             assert torch.equal(x, y)
 
 
+def test_graph_cache_alternating_calls_match_eager_results():
+    # Two chunks of layers with different buffers, called alternately over three
+    # steps: the first sighting of each runs eagerly, the second captures a
+    # graph, the third replays it.  Every step must give the same indices and state.
+    wl = synth.small_workload(seqlens=(900, 450), layers=4)
+    sel = kvec.KvecSelector(kvec.params_from_workload(wl))
+    cu = torch.tensor(wl.cu_seqlens, dtype=torch.int32).pin_memory()
+    cud = cu.cuda()
+    xs = [{k: v.cuda() for k, v in x.items()} for x in synth.make_layers(wl, 4)]
+    outs = [sel.alloc_outputs(wl.batch, wl.budget) for _ in range(4)]
+    st = sel.new_state(wl.batch)
+    stream = torch.cuda.current_stream()
+    steps = []
+    for _ in range(3):
+        kvec.kvec_reset(sel.handle, st.data_ptr(), wl.batch, stream.cuda_stream)
+        for ls in ([0, 1], [2, 3]):
+            sel.select_layers(cu, cud, [xs[l]["q_obs"] for l in ls], [xs[l]["k"] for l in ls],
+                              [xs[l]["v"] for l in ls], st, wl.budget, [outs[l] for l in ls], stream)
+        kvec.kvec_sync_status(sel.handle)
+        steps.append([o[0].cpu() for o in outs] + [o[1].cpu() for o in outs] + [st.cpu()])
+    for later in steps[1:]:
+        for x, y in zip(steps[0], later):
+            assert torch.equal(x, y)
+
+
 def test_multi_layer_call_matches_layer_by_layer():
     wl = synth.small_workload(seqlens=(1100, 700), layers=4, budget=96)
     layers = [{k: v.cuda() for k, v in x.items()} for x in synth.make_layers(wl, 4)]

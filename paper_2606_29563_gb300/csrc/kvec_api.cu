@@ -85,6 +85,11 @@ struct kvec_handle {
     };
     std::vector<CachedGraph> graphs;
     std::vector<std::vector<uint64_t>> seen_keys;
+    // While a call is captured: each programmatic launch's graph node and the
+    // node of the kernel before it on the same stream (null if none), whose edge
+    // alone may stay programmatic (restore_full_edges).
+    bool capturing = false;
+    std::vector<std::pair<cudaGraphNode_t, cudaGraphNode_t>> prog_nodes;
 };
 
 namespace {
@@ -242,13 +247,13 @@ kvec_status run_layer_sequential(kvec_handle* h, const Geometry& G, const LayerI
     if (se != cudaSuccess) return cuda_fail(se, "score kernel tensor maps");
     se = launch_score(plan, st, false);
     if (se != cudaSuccess) return cuda_fail(se, "score kernel launch");
-    se = launch_rowstat(plan, G, io, h->sc, st, true);
+    se = launch_rowstat(plan, G, io, h->sc, st, /*programmatic=*/true, /*after_score=*/true);
     if (se != cudaSuccess) return cuda_fail(se, "row statistics launch");
     se = launch_window(plan, G, io, h->sc, h->slots[0], st, false);
     if (se != cudaSuccess) return cuda_fail(se, "window kernel launch");
     se = launch_heads(G, io, h->sc, h->slots[0], st, h->prio_hi);
     if (se != cudaSuccess) return cuda_fail(se, "heads kernel launch");
-    se = launch_select(G, io, h->sc, h->slots[0], nullptr, st, h->prio_hi, 0, 1);
+    se = launch_select(G, io, h->sc, h->slots[0], nullptr, st, h->prio_hi, 0, 1, /*programmatic=*/false);
     if (se != cudaSuccess) return cuda_fail(se, "select kernel launch");
     launch_gather(G, io, h->slots[0], st);
     se = launch_finalize(G, io, h->sc, h->slots[0], st, h->prio_hi, 1);
@@ -256,6 +261,48 @@ kvec_status run_layer_sequential(kvec_handle* h, const Geometry& G, const LayerI
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_fail(e, "kernel launch");
     return KVEC_OK;
+}
+
+// The node a capturing stream added last (its only current dependency), or null
+// when the stream is not capturing.
+cudaGraphNode_t captured_tail(cudaStream_t st) {
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    const cudaGraphNode_t* deps = nullptr;
+    const cudaGraphEdgeData* ed = nullptr;
+    size_t nd = 0;
+    if (cudaStreamGetCaptureInfo(st, &cs, nullptr, nullptr, &deps, &ed, &nd) != cudaSuccess) return nullptr;
+    return (cs == cudaStreamCaptureStatusActive && nd == 1) ? deps[0] : nullptr;
+}
+
+// Stream capture gives a programmatic launch's every incoming edge the
+// programmatic type, the edges from other streams' event waits included, and
+// such an edge lets the kernel start (and read) before that producer has
+// finished.  Launched eagerly, only the edge from the same stream's previous
+// kernel is relaxed.  This puts the captured graph back in that form: every
+// other programmatic edge into a recorded node becomes a full dependency.
+cudaError_t restore_full_edges(cudaGraph_t graph, const std::vector<std::pair<cudaGraphNode_t, cudaGraphNode_t>>& nodes) {
+    for (const auto& nd : nodes) {
+        cudaGraphNode_t node = nd.first;
+        size_t n = 0;
+        cudaError_t e = cudaGraphNodeGetDependencies(node, nullptr, nullptr, &n);
+        if (e != cudaSuccess && e != cudaErrorLossyQuery) return e;
+        std::vector<cudaGraphNode_t> deps(n);
+        std::vector<cudaGraphEdgeData> ed(n);
+        if (n > 0) {
+            e = cudaGraphNodeGetDependencies(node, deps.data(), ed.data(), &n);
+            if (e != cudaSuccess) return e;
+        }
+        for (size_t i = 0; i < n; ++i) {
+            if (deps[i] == nd.second) continue;
+            if (ed[i].type == cudaGraphDependencyTypeDefault && ed[i].from_port == 0 && ed[i].to_port == 0) continue;
+            e = cudaGraphRemoveDependencies(graph, &deps[i], &node, &ed[i], 1);
+            if (e != cudaSuccess) return e;
+            cudaGraphEdgeData full = {};
+            e = cudaGraphAddDependencies(graph, &deps[i], &node, &full, 1);
+            if (e != cudaSuccess) return e;
+        }
+    }
+    return cudaSuccess;
 }
 
 #define KV_CHECK(call)                                        \
@@ -272,6 +319,7 @@ kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* io
     KV_CHECK(cudaEventRecord(h->ev_fork, origin));
     for (cudaStream_t st : {h->s_score, h->s_win, h->s_heads, h->s_heads2, h->s_chain, h->s_gather})
         KV_CHECK(cudaStreamWaitEvent(st, h->ev_fork, 0));
+    cudaGraphNode_t prev_score = nullptr, prev_window = nullptr, prev_select = nullptr;   // captured (h->capturing)
     for (int l = 0; l < n; ++l) {
         const Slot& sl = h->slots[l % kSlots];
         const Scratch& sc = h->score_buf[l % kScoreBufs];
@@ -282,15 +330,18 @@ kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* io
         ScorePlan plan;
         cudaError_t se = plan_score(G, io, sc, h->num_sms, &plan);
         if (se != cudaSuccess) return cuda_fail(se, "score kernel tensor maps");
-        // A launch is a programmatic dependent of its stream predecessor only when
-        // no event wait stands between them: in a captured graph a programmatic
-        // launch turns every incoming edge programmatic, those from another
-        // stream's event included, and the kernel could start before that
-        // stream's kernel has finished writing.  The score launch of layer 1 is
-        // the only one without a wait before it.
+        // The score grid of layer l > 0 is a programmatic dependent of layer
+        // l - 1's (it reads none of its results); the event wait above stays a
+        // full dependency (restore_full_edges when captured).
         if (!io.lse) {
-            timed_launch(h, 0, h->s_score, [&] { se = launch_score(plan, h->s_score, l > 0 && l < kScoreBufs); });
+            timed_launch(h, 0, h->s_score, [&] { se = launch_score(plan, h->s_score, l > 0); });
             if (se != cudaSuccess) return cuda_fail(se, "score kernel launch");
+            if (h->capturing) {
+                cudaGraphNode_t node = captured_tail(h->s_score);
+                if (!node) return fail(KVEC_ERR_CUDA, "score kernel: no captured node");
+                if (l > 0) h->prog_nodes.emplace_back(node, prev_score);
+                prev_score = node;
+            }
         }
         KV_CHECK(cudaEventRecord(h->ev_score[l], h->s_score));
         // Window stream: the row statistics (after the score grid and, for slot
@@ -301,10 +352,25 @@ kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* io
             KV_CHECK(cudaStreamWaitEvent(h->s_win, h->ev_sel[l - kSlots], 0));
             KV_CHECK(cudaStreamWaitEvent(h->s_win, h->ev_gather[l - kSlots], 0));
         }
-        se = io.lse ? launch_rowstat_lse(G, io, sc, h->s_win) : launch_rowstat(plan, G, io, sc, h->s_win, false);
+        // The row statistics are a programmatic dependent of the previous layer's
+        // window grid, which they do not wait for: they read only this layer's
+        // partials (full dependency above), and the statistics buffer they
+        // overwrite was last read by layer l - 2's window grid, which this
+        // layer's score grid waited for.  So consecutive window grids overlap.
+        se = io.lse ? launch_rowstat_lse(G, io, sc, h->s_win, l > 0)
+                    : launch_rowstat(plan, G, io, sc, h->s_win, l > 0, /*after_score=*/false);
         if (se != cudaSuccess) return cuda_fail(se, "row statistics launch");
+        if (h->capturing) {
+            cudaGraphNode_t node = captured_tail(h->s_win);
+            if (!node) return fail(KVEC_ERR_CUDA, "row statistics: no captured node");
+            if (l > 0) h->prog_nodes.emplace_back(node, prev_window);
+        }
         timed_launch(h, 1, h->s_win, [&] { se = launch_window(plan, G, io, sc, sl, h->s_win, true); });
         if (se != cudaSuccess) return cuda_fail(se, "window kernel launch");
+        if (h->capturing) {
+            prev_window = captured_tail(h->s_win);
+            if (!prev_window) return fail(KVEC_ERR_CUDA, "window kernel: no captured node");
+        }
         KV_CHECK(cudaEventRecord(h->ev_win[l], h->s_win));
         cudaStream_t s_h = (l & 1) ? h->s_heads2 : h->s_heads;
         KV_CHECK(cudaStreamWaitEvent(s_h, h->ev_win[l], 0));
@@ -313,8 +379,18 @@ kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* io
         KV_CHECK(cudaEventRecord(h->ev_heads[l], s_h));
         KV_CHECK(cudaStreamWaitEvent(h->s_chain, h->ev_heads[l], 0));
         const Slot* prev = l > 0 ? &h->slots[(l - 1) % kSlots] : nullptr;
-        timed_launch(h, 3, h->s_chain, [&] { se = launch_select(G, io, sc, sl, prev, h->s_chain, h->prio_hi, l, n); });
+        // The selection is a programmatic dependent of the previous layer's: it
+        // stages this layer's scores (behind the full dependency on the heads
+        // kernels) while that one drains.
+        timed_launch(h, 3, h->s_chain,
+                     [&] { se = launch_select(G, io, sc, sl, prev, h->s_chain, h->prio_hi, l, n, /*programmatic=*/true); });
         if (se != cudaSuccess) return cuda_fail(se, "select kernel launch");
+        if (h->capturing) {
+            cudaGraphNode_t node = captured_tail(h->s_chain);
+            if (!node) return fail(KVEC_ERR_CUDA, "select kernel: no captured node");
+            h->prog_nodes.emplace_back(node, prev_select);
+            prev_select = node;
+        }
         KV_CHECK(cudaEventRecord(h->ev_sel[l], h->s_chain));
         KV_CHECK(cudaStreamWaitEvent(h->s_gather, h->ev_sel[l], 0));
         timed_launch(h, 4, h->s_gather, [&] { launch_gather(G, io, sl, h->s_gather); });
@@ -598,8 +674,16 @@ kvec_status select_layers_impl(kvec_handle* h, int num_layers, int batch, const 
         if (seen) {
             cudaGraph_t graph = nullptr;
             KV_CHECK(cudaStreamBeginCapture(h->s_cap, cudaStreamCaptureModeThreadLocal));
+            h->capturing = true;
+            h->prog_nodes.clear();
             s = launch_pipeline(h, G, ios.data(), num_layers, h->s_cap);
+            h->capturing = false;
             cudaError_t ce = cudaStreamEndCapture(h->s_cap, &graph);
+            if (s == KVEC_OK && ce == cudaSuccess) {
+                ce = restore_full_edges(graph, h->prog_nodes);
+                if (ce != cudaSuccess) s = cuda_fail(ce, "graph edges of the captured pipeline");
+            }
+            h->prog_nodes.clear();
             if (s != KVEC_OK) {
                 if (graph) cudaGraphDestroy(graph);
                 return s;

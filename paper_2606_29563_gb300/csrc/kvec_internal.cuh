@@ -122,13 +122,18 @@ cudaError_t plan_score(const Geometry& g, const LayerIO& io, const Scratch& sc, 
 // of the same kernel (the multi-stream layer pipeline); the launch may then
 // overlap it (programmatic stream serialization), as it reads none of its results.
 cudaError_t launch_score(const ScorePlan& plan, cudaStream_t st, bool after_own_launch);
-// (m_r, Z_r) from the score launch's partials; launched right after it on the same stream.
+// (m_r, Z_r) from the score launch's partials.  programmatic: a programmatic
+// dependent of the stream's previous kernel.  after_score: that kernel is this
+// layer's score launch, waited for (griddepcontrol.wait) before the partials
+// are read; without it the partials must come through a full dependency and the
+// previous kernel (the layer pipeline's previous window grid) is not waited for.
 cudaError_t launch_rowstat(const ScorePlan& plan, const Geometry& g, const LayerIO& io, const Scratch& sc,
-                           cudaStream_t st,
-                           bool after_score);
+                           cudaStream_t st, bool programmatic, bool after_score);
 // (m_r, Z_r) = (lse * log2(e), 1) from the caller's log-sum-exp (io.lse), in place
-// of the score and row-statistics launches.
-cudaError_t launch_rowstat_lse(const Geometry& g, const LayerIO& io, const Scratch& sc, cudaStream_t st);
+// of the score and row-statistics launches.  programmatic: as for launch_rowstat
+// without after_score (it reads only the caller's input).
+cudaError_t launch_rowstat_lse(const Geometry& g, const LayerIO& io, const Scratch& sc, cudaStream_t st,
+                               bool programmatic);
 cudaError_t launch_window(const ScorePlan& sp, const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl,
                           cudaStream_t st, bool after_own_launch);
 // Launches kernel<<<grid, block, smem, st>>> with a scheduling priority (lower
@@ -160,9 +165,14 @@ cudaError_t launch_heads(const Geometry& g, const LayerIO& io, const Scratch& sc
 // prev: the previous layer's slot (null for lcall = 0), whose kept-position
 // bits give that layer's union.  The coverage counts alternate between the
 // state and sc.nbuf; launch_finalize folds the last layer's union (from its
-// slot) into the state.
+// slot) into the state.  programmatic: the stream's previous kernel is the
+// previous layer's selection (the layer pipeline's chain stream, whose only
+// other dependency is a full one on this layer's heads kernels); the grid then
+// stages this layer's scores while that one drains and waits
+// (griddepcontrol.wait) before reading the coverage counts.  Never set it when
+// the stream's previous kernel wrote this layer's scores.
 cudaError_t launch_select(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, const Slot* prev,
-                          cudaStream_t st, int priority, int lcall, int ncall);
+                          cudaStream_t st, int priority, int lcall, int ncall, bool programmatic);
 cudaError_t launch_finalize(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& last, cudaStream_t st,
                             int priority, int ncall);
 // out_idx from the slot's kept-position bits, then the K/V rows.

@@ -385,11 +385,14 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
 // at the head's first item, then one at every score CTA's first item inside
 // the head's range of items.  Grid (Hkv, batch), one thread per row.
 __global__ void __launch_bounds__(256) rowstat_kernel(Geometry G, Scratch sc, const int* __restrict__ cu, int W,
-                                                      int Gc) {
-    // Possibly a programmatic dependent of the score launch: its partials are read
-    // only after that grid has completed.  The window launch that follows may start.
+                                                      int Gc, int wait_prev) {
+    // The window launch that follows may start; it waits for this grid.
     if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
-    asm volatile("griddepcontrol.wait;\n" ::: "memory");
+    // wait_prev: a programmatic dependent of the score launch right before it on
+    // the stream, whose partials are read only after that grid has completed.
+    // Otherwise the partials come through a full dependency and the stream's
+    // previous kernel (if a programmatic predecessor at all) is not waited for.
+    if (wait_prev) asm volatile("griddepcontrol.wait;\n" ::: "memory");
     const int h = blockIdx.x, s = blockIdx.y, r = threadIdx.x;
     if (r >= G.R) return;
     int ib = 0;
@@ -534,7 +537,7 @@ cudaError_t plan_score(const Geometry& g, const LayerIO& io, const Scratch& sc, 
 }
 
 cudaError_t launch_rowstat(const ScorePlan& plan, const Geometry& g, const LayerIO& io, const Scratch& sc,
-                           cudaStream_t st, bool after_score) {
+                           cudaStream_t st, bool programmatic, bool after_score) {
     const ScoreArgs& a = *reinterpret_cast<const ScoreArgs*>(plan.args);
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(g.Hkv, g.batch);
@@ -544,13 +547,22 @@ cudaError_t launch_rowstat(const ScorePlan& plan, const Geometry& g, const Layer
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = after_score ? 1 : 0;   // a programmatic dependent of the score launch right before it
-    return cudaLaunchKernelEx(&cfg, rowstat_kernel, g, sc, io.cu, a.W, plan.grid);
+    cfg.numAttrs = programmatic ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, rowstat_kernel, g, sc, io.cu, a.W, plan.grid, after_score ? 1 : 0);
 }
 
-cudaError_t launch_rowstat_lse(const Geometry& g, const LayerIO& io, const Scratch& sc, cudaStream_t st) {
-    rowstat_lse_kernel<<<dim3(g.Hkv, g.batch), 256, 0, st>>>(g, sc, io.lse);
-    return cudaGetLastError();
+cudaError_t launch_rowstat_lse(const Geometry& g, const LayerIO& io, const Scratch& sc, cudaStream_t st,
+                               bool programmatic) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(g.Hkv, g.batch);
+    cfg.blockDim = dim3(256);
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = programmatic ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, rowstat_lse_kernel, g, sc, io.lse);
 }
 
 cudaError_t launch_score(const ScorePlan& plan, cudaStream_t st, bool after_own_launch) {

@@ -1053,12 +1053,10 @@ cudaError_t launch_heads(const Geometry& g, const LayerIO& io, const Scratch& sc
 }
 
 cudaError_t launch_select(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, const Slot* prev,
-                          cudaStream_t st, int priority, int lcall, int ncall) {
+                          cudaStream_t st, int priority, int lcall, int ncall, bool programmatic) {
     const uint32_t* prev_sel = prev ? prev->sel : nullptr;
-    // Not programmatic: the chain stream waits for this layer's heads kernels
-    // right before the launch (see launch_pipeline).
     return launch_prio(select_kernel, dim3(g.Hkv, g.batch), dim3(kSelectThreads), select_smem_bytes(g), st, priority,
-                       /*programmatic=*/false, g, io, sc, sl, prev_sel, lcall, ncall);
+                       programmatic, g, io, sc, sl, prev_sel, lcall, ncall);
 }
 
 cudaError_t launch_finalize(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& last, cudaStream_t st,

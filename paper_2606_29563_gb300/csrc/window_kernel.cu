@@ -139,6 +139,9 @@ __global__ void __launch_bounds__(kWinThreads, 1)
     if (threadIdx.x == 0) {
         ptx::prefetch_tensormap(&kmap);
         ptx::prefetch_tensormap(&qmap);
+        // The next launch on this stream (the next layer's row statistics) reads
+        // nothing this grid writes and does not wait for it: let it be scheduled.
+        asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
     }
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     // Scalars and pointers in registers: values read through a reference to the

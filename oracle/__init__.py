@@ -44,7 +44,7 @@ class _Params(ctypes.Structure):
         ("window", ctypes.c_int), ("obs_window", ctypes.c_int), ("ext_window", ctypes.c_int),
         ("pool_kernel", ctypes.c_int), ("num_ext_heads", ctypes.c_int),
         ("lam", ctypes.c_double), ("beta", ctypes.c_double), ("softmax_scale", ctypes.c_double),
-        ("pool_mode", ctypes.c_int), ("head_criterion", ctypes.c_int),
+        ("pool_mode", ctypes.c_int), ("head_criterion", ctypes.c_int), ("all_positions", ctypes.c_int),
     ]
 
 
@@ -94,6 +94,7 @@ class OracleParams:
     softmax_scale: float = 0.0
     pool_mode: int = 0        # 0 max-pool, 1 average pool
     head_criterion: int = 0   # 0 standard deviation, 1 entropy
+    all_positions: int = 0    # 0 keep the window tail, 1 every position is a candidate
 
     @classmethod
     def from_workload(cls, wl, **over) -> "OracleParams":
@@ -101,7 +102,8 @@ class OracleParams:
                   window=wl.window, obs_window=wl.obs_window, ext_window=wl.ext_window,
                   pool_kernel=wl.pool_kernel, num_ext_heads=wl.num_ext_heads,
                   lam=float(np.float32(wl.lam)), beta=float(np.float32(wl.beta)),
-                  pool_mode=getattr(wl, "pool_mode", 0), head_criterion=getattr(wl, "head_criterion", 0))
+                  pool_mode=getattr(wl, "pool_mode", 0), head_criterion=getattr(wl, "head_criterion", 0),
+                  all_positions=getattr(wl, "all_positions", 0))
         kw.update(over)
         return cls(**kw)
 
@@ -109,7 +111,7 @@ class OracleParams:
         return _Params(self.num_q_heads, self.num_kv_heads, self.head_dim, self.window,
                        self.obs_window, self.ext_window, self.pool_kernel, self.num_ext_heads,
                        float(self.lam), float(self.beta), float(self.softmax_scale), int(self.pool_mode),
-                       int(self.head_criterion))
+                       int(self.head_criterion), int(self.all_positions))
 
 
 def state_bytes(max_seqlen: int) -> int:

@@ -13,6 +13,9 @@
  *  - "Heads" are KV heads; A is summed over the query heads of a GQA group.
  *  - Candidates are t in [0, L-w); the last w tokens are always kept and
  *    count toward the budget B (observation-window retention of SnapKV).
+ *    With all_positions = 1 every t in [0, L) is a candidate (the window part
+ *    scored by its causal attention) and nothing is kept unconditionally:
+ *    the top-B over the T input tokens of Section 4.1, read literally.
  *  - Scores are max-pooled (odd width, stride 1, neighbours outside the
  *    candidate range ignored) before sigma, preservation and focus.
  *  - sigma is the sample standard deviation (n-1); 0 when fewer than 2
@@ -123,7 +126,10 @@ int kvo_select_layer(const kvo_params* p, int batch, const int32_t* cu_seqlens, 
     if (p->head_criterion != 0 && p->head_criterion != 1) return -5;
     if (p->num_ext_heads < 0 || p->num_ext_heads > Hkv) return -5;
     if (!(p->beta >= 0.0 && p->beta <= 1.0)) return -6;
-    if (budget < w) return -7;
+    if (p->all_positions != 0 && p->all_positions != 1) return -4;
+    /* wk: the tail kept unconditionally (the window, or nothing). */
+    const int wk = p->all_positions ? 0 : w;
+    if (budget < wk || budget < 1) return -7;
     for (int b = 0; b < batch; ++b) {
         int L = cu_seqlens[b + 1] - cu_seqlens[b];
         if (L < w || L > max_seqlen) return -8;
@@ -137,7 +143,7 @@ int kvo_select_layer(const kvo_params* p, int batch, const int32_t* cu_seqlens, 
 
     for (int b = 0; b < batch; ++b) {
         const int L = cu_seqlens[b + 1] - cu_seqlens[b];
-        const int Lc = L - w;                  /* candidates t in [0, Lc) */
+        const int Lc = L - wk;                 /* candidates t in [0, Lc) */
         const uint16_t* kb = k + (size_t)cu_seqlens[b] * Hkv * d;
         const uint16_t* vb = v + (size_t)cu_seqlens[b] * Hkv * d;
         uint8_t* st = state + (size_t)b * sbytes;
@@ -271,8 +277,8 @@ int kvo_select_layer(const kvo_params* p, int batch, const int32_t* cu_seqlens, 
         /* Steps 6-8 (Section 4.2): preserve top-K of P, add lambda*focus, fill the rest. */
         const int keep_all = L <= budget;
         int Kp = (int)floor(p->beta * (double)budget);
-        if (Kp > budget - w) Kp = budget - w;
-        const int k2 = budget - w - Kp;
+        if (Kp > budget - wk) Kp = budget - wk;
+        const int k2 = budget - wk - Kp;
         uint8_t* pres = (uint8_t*)calloc((size_t)Hkv * (Lc > 0 ? Lc : 1), 1);
         double* Pp = (double*)calloc((size_t)Hkv * (Lc > 0 ? Lc : 1), sizeof(double));
         uint8_t* keep = (uint8_t*)calloc((size_t)Hkv * L, 1);   /* S_h as a mask over [0, L) */
@@ -301,7 +307,7 @@ int kvo_select_layer(const kvo_params* p, int batch, const int32_t* cu_seqlens, 
                 double* lit = (double*)malloc(sizeof(double) * (size_t)Lc);
                 uint8_t* lsel = (uint8_t*)calloc((size_t)Lc, 1);
                 for (int t = 0; t < Lc; ++t) lit[t] = ph[t] ? 1.0 : pph[t];
-                top_k(lit, NULL, Lc, budget - w, lsel);
+                top_k(lit, NULL, Lc, budget - wk, lsel);
                 int differs = 0;
                 for (int t = 0; t < Lc; ++t) if (lsel[t] != kh[t]) differs = 1;
                 dbg->literal_override_differs += differs;

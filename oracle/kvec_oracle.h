@@ -35,6 +35,10 @@ typedef struct {
     int pool_mode;       /* 0: max-pool (default); 1: average over the in-range neighbours */
     int head_criterion;  /* 0: standard deviation (Section 4.1, default); 1: entropy
                             (Section 5.4 ablation, "Head Selection Criteria") */
+    int all_positions;   /* 0: the last w tokens are always kept and count toward B,
+                            candidates are [0, L-w) (default); 1: every position
+                            [0, L) is a candidate and each head keeps the top B of
+                            them (Section 4.1's top-B over the T input tokens) */
 } kvo_params;
 
 /* Optional debug outputs.  Any pointer may be NULL.  Sizes use the caller's

@@ -38,7 +38,7 @@ def _ranked(score: np.ndarray, positions: np.ndarray) -> np.ndarray:
 
 def select(q_full, k, *, num_kv_heads, window, obs_window, ext_window, pool_kernel,
            num_ext_heads, lam, beta, budget, n_counts, layers_done, scale=None, pool_mode=0,
-           head_criterion=0) -> Dict[str, np.ndarray]:
+           head_criterion=0, all_positions=0) -> Dict[str, np.ndarray]:
     """Algorithm 1 followed by per-head top-B for one sequence of length T = q_full.shape[0]."""
     T, Hq, d = q_full.shape
     Hkv = num_kv_heads
@@ -53,7 +53,10 @@ def select(q_full, k, *, num_kv_heads, window, obs_window, ext_window, pool_kern
     P_Oe_raw = Akv[:, T - Oe:, :].mean(axis=1)
     I_raw = Akv[:, T - O:, :].max(axis=0).mean(axis=0)
 
-    Lc = T - w
+    # Candidates: every position before the kept window tail, or every position
+    # when nothing is kept unconditionally (top-B over the T input tokens).
+    wk = 0 if all_positions else w
+    Lc = T - wk
     r = pool_kernel // 2
 
     def pool(x):
@@ -82,7 +85,7 @@ def select(q_full, k, *, num_kv_heads, window, obs_window, ext_window, pool_kern
 
     coverage = n_counts[:Lc].astype(np.float64) / (layers_done + 1)
     Pprime = P + lam * (I * (1.0 - coverage))[None, :]
-    Kp = min(int(math.floor(beta * budget)), budget - w)
+    Kp = min(int(math.floor(beta * budget)), budget - wk)
     cand = np.arange(Lc)
     keep = np.zeros((Hkv, T), bool)
     pres = np.zeros((Hkv, max(Lc, 0)), bool)
@@ -93,7 +96,7 @@ def select(q_full, k, *, num_kv_heads, window, obs_window, ext_window, pool_kern
             top = _ranked(P[h], cand)[:Kp]
             pres[h, top] = True
             rest = cand[~pres[h]]
-            fill = _ranked(Pprime[h], rest)[:budget - w - Kp]
+            fill = _ranked(Pprime[h], rest)[:budget - wk - Kp]
             keep[h, top] = True
             keep[h, fill] = True
             keep[h, Lc:] = True

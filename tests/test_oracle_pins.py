@@ -390,3 +390,76 @@ def test_uniform_keys_closed_forms_for_the_variants():
     expect_PO = g / O * sum(1.0 / (T - w + q + 1) for q in range(w - O, w))
     np.testing.assert_allclose(r["P_O"][0, :, :Lc], expect_PO, rtol=1e-13)
     np.testing.assert_allclose(r["sigma"][0], -math.log(Lc), rtol=1e-13)
+
+
+# Top-B over every position (all_positions = 1): Section 4.1 states the top-B of
+# the T input tokens; by default the last w tokens are kept as in SnapKV.
+
+@pytest.mark.parametrize("variant", [dict(), dict(pool_mode=1, head_criterion=1)])
+@pytest.mark.parametrize("case", TINY_CASES)
+def test_all_positions_matches_bruteforce_over_layers(case, variant):
+    seed, T, Hq, Hkv, d, w, O, Oe, pool, delta, lam, beta, B = case
+    params = oracle.OracleParams(num_q_heads=Hq, num_kv_heads=Hkv, head_dim=d, window=w,
+                                 obs_window=O, ext_window=Oe, pool_kernel=pool,
+                                 num_ext_heads=delta, lam=lam, beta=beta, all_positions=1, **variant)
+    state = oracle.new_state(1, T)
+    n_bf = np.zeros(T, np.int64)
+    for layer in range(3):
+        x = synth.tiny_full_inputs(seed * 100 + layer + 7, T, Hq, Hkv, d)
+        q_obs = x["q_full"][T - w:].reshape(1, w, Hq, d)
+        r = _run_oracle(params, q_obs, x["k"], x["v"], state, B)
+        bf = bf_select(_f64(x["q_full"]), _f64(x["k"]), num_kv_heads=Hkv, window=w, obs_window=O,
+                       ext_window=Oe, pool_kernel=pool, num_ext_heads=delta, lam=lam, beta=beta,
+                       budget=B, n_counts=n_bf, layers_done=layer, all_positions=1, **variant)
+        np.testing.assert_allclose(r["P_O"][0, :, :T], bf["P_O"], rtol=1e-12, atol=1e-15)
+        np.testing.assert_allclose(r["P_Oext"][0, :, :T], bf["P_Oext"], rtol=1e-12, atol=1e-15)
+        np.testing.assert_allclose(r["I"][0, :T], bf["I"], rtol=1e-12, atol=1e-15)
+        np.testing.assert_allclose(r["sigma"][0], bf["sigma"], rtol=1e-9, atol=1e-15)
+        assert (r["htop"][0].astype(bool) == bf["htop"]).all()
+        np.testing.assert_allclose(r["Pprime"][0, :, :T], bf["Pprime"], rtol=1e-12, atol=1e-15)
+        if T > B:
+            assert (r["pres"][0, :, :T].astype(bool) == bf["pres"]).all()
+        assert (r["out_idx"][0] == bf["out_idx"]).all()
+        n_bf = bf["n"]
+        assert (oracle.state_fields(state, T)["n"][0].astype(np.int64) == n_bf).all()
+
+
+def test_all_positions_uniform_keys_evict_the_window():
+    """K = 0: the prefix and the first window positions tie at the highest score and
+    the later window positions, seen by fewer window rows, score lower.  The top B
+    are then [0, B): nothing of the window stays.  At layer 1 the preserved part
+    stays and the fill moves past the covered tokens."""
+    T, Hq, Hkv, d, w, O, Oe, B = 64, 4, 2, 8, 8, 4, 8, 24
+    params = oracle.OracleParams(num_q_heads=Hq, num_kv_heads=Hkv, head_dim=d, window=w, obs_window=O,
+                                 ext_window=Oe, pool_kernel=3, num_ext_heads=1, lam=1.0, beta=0.25,
+                                 all_positions=1)
+    g = Hq // Hkv
+    x = synth.tiny_full_inputs(3, T, Hq, Hkv, d)
+    q_obs = x["q_full"][T - w:].reshape(1, w, Hq, d)
+    k = torch.zeros(T, Hkv, d, dtype=torch.bfloat16)
+    state = oracle.new_state(1, T)
+    r = _run_oracle(params, q_obs, k, x["v"], state, B)
+    # Raw Eq. 1 score of window position T - w + j: rows q >= max(j, w - O) see it.
+    for j in range(w):
+        expect = g / O * sum(1.0 / (T - w + q + 1) for q in range(max(j, w - O), w))
+        np.testing.assert_allclose(r["P_O_raw"][0, :, T - w + j], expect, rtol=1e-13)
+    Kp = int(math.floor(0.25 * B))
+    assert (r["out_idx"][0] == np.arange(B)).all()
+    r1 = _run_oracle(params, q_obs, k, x["v"], state, B)
+    layer1 = list(range(Kp)) + list(range(B, B + (B - Kp)))
+    assert (r1["out_idx"][0] == np.array(layer1)).all()
+    expect_n = np.zeros(T, np.int64)
+    for sel in (list(range(B)), layer1):
+        expect_n[sel] += 1
+    assert (oracle.state_fields(state, T)["n"][0] == expect_n).all()
+
+
+def test_all_positions_rejects_nothing_the_default_needs():
+    """A budget below the window is refused only when the window is kept."""
+    q, k, v = _tiny_layer(5, T=40, w=8)
+    base = dict(num_q_heads=8, num_kv_heads=4, head_dim=8, window=8, obs_window=4, ext_window=8, pool_kernel=3,
+                num_ext_heads=1)
+    with pytest.raises(ValueError):
+        _run_oracle(oracle.OracleParams(**base), q, k, v, oracle.new_state(1, 40), 6)
+    r = _run_oracle(oracle.OracleParams(all_positions=1, **base), q, k, v, oracle.new_state(1, 40), 6)
+    assert (np.diff(r["out_idx"][0], axis=-1) > 0).all() and r["out_idx"].shape[-1] == 6

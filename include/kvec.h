@@ -60,7 +60,8 @@ typedef struct {
     int   num_kv_heads;   /* H_kv KV heads; query head hq uses KV head hq / (H_q/H_kv) */
     int   head_dim;       /* d; these kernels support 128 */
     int   window;         /* w: observation query rows given per sequence; the last w
-                             tokens are always kept and count toward the budget */
+                             tokens are always kept and count toward the budget unless
+                             all_positions = 1 */
     int   obs_window;     /* O of Eq. 1 (paper: "e.g., 16"), 1 <= O <= min(w, 64) */
     int   ext_window;     /* O' of Section 4.1 (paper default 32), 1 <= O' <= w */
     int   pool_kernel;    /* odd width of the 1-D max-pool over candidate scores, 1..15 */
@@ -77,6 +78,12 @@ typedef struct {
                              P_O take O' (Section 4.1, default); 1: those with the highest
                              entropy of pooled P_O normalised over the candidates (the
                              Section 5.4 ablation "Head Selection Criteria") */
+    int   all_positions;  /* 0: the last w tokens are always kept and count toward the
+                             budget; the candidates are [0, L - w) (SnapKV's retained
+                             observation window, default).  1: every position [0, L) is a
+                             candidate, the window part scored by its causal attention, and
+                             each head keeps the top B of them (Section 4.1's top-B over
+                             the T input tokens); budget >= 1 instead of >= window */
 } kvec_params;
 
 /* Creates a handle and allocates its device workspace on the current device.

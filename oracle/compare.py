@@ -36,7 +36,10 @@ def _threshold_band(key: np.ndarray, cand: np.ndarray, k: int, tol: float):
 
 def check_layer(gpu: Dict[str, np.ndarray], orc: Dict[str, np.ndarray], seqlens, window: int, budget: int,
                 Kp: int, num_ext_heads: int, tol: float = TOL) -> List[str]:
-    """Returns a list of human-readable mismatches (empty when the layer passes)."""
+    """Returns a list of human-readable mismatches (empty when the layer passes).
+
+    window: the tail kept unconditionally (w, or 0 when every position is a
+    candidate); the candidates are [0, L - window)."""
     errs: List[str] = []
     H = orc["out_idx"].shape[1]
     for b, L in enumerate(seqlens):

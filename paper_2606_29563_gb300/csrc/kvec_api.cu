@@ -148,6 +148,8 @@ kvec_status validate_params(const kvec_params* p) {
     if (p->pool_mode != 0 && p->pool_mode != 1) return fail(KVEC_ERR_INVALID_ARG, "pool_mode must be 0 or 1");
     if (p->head_criterion != 0 && p->head_criterion != 1)
         return fail(KVEC_ERR_INVALID_ARG, "head_criterion must be 0 or 1");
+    if (p->all_positions != 0 && p->all_positions != 1)
+        return fail(KVEC_ERR_INVALID_ARG, "all_positions must be 0 or 1");
     if (p->num_ext_heads < 0 || p->num_ext_heads > p->num_kv_heads)
         return fail(KVEC_ERR_INVALID_ARG, "num_ext_heads must be in [0, num_kv_heads]");
     if (!(p->beta >= 0.f && p->beta <= 1.f)) return fail(KVEC_ERR_INVALID_ARG, "beta must be in [0, 1]");
@@ -184,7 +186,9 @@ kvec_status validate_call(kvec_handle* h, int batch, const int32_t* cu_host, con
         return fail(KVEC_ERR_INVALID_ARG, "batch %d outside [1, max_batch=%d]", batch, h->p.max_batch);
     if (!cu_host || !cu_dev) return fail(KVEC_ERR_INVALID_ARG, "cu_seqlens pointers must not be NULL");
     if (cu_host[0] != 0) return fail(KVEC_ERR_INVALID_ARG, "cu_seqlens[0] must be 0");
-    if (budget < h->p.window) return fail(KVEC_ERR_INVALID_ARG, "budget %d < window %d", budget, h->p.window);
+    const int wk = h->p.all_positions ? 0 : h->p.window;   // the tail kept unconditionally
+    if (budget < 1) return fail(KVEC_ERR_INVALID_ARG, "budget %d < 1", budget);
+    if (budget < wk) return fail(KVEC_ERR_INVALID_ARG, "budget %d < window %d", budget, wk);
     int tiles = 0, chunks = 0;
     for (int b = 0; b < batch; ++b) {
         const int L = cu_host[b + 1] - cu_host[b];
@@ -192,7 +196,7 @@ kvec_status validate_call(kvec_handle* h, int batch, const int32_t* cu_host, con
             return fail(KVEC_ERR_INVALID_ARG, "sequence %d has length %d outside [window=%d, max_seqlen=%d]", b, L,
                         h->p.window, h->p.max_seqlen);
         tiles += (L + kTileT - 1) / kTileT;
-        chunks += (L - h->p.window + kTileT - 1) / kTileT;   // candidate tiles of the window kernel
+        chunks += (L - wk + kTileT - 1) / kTileT;   // candidate tiles of the window kernel
     }
     *total_tiles = tiles;
     *total_win_tiles = chunks;
@@ -224,10 +228,11 @@ Geometry make_geometry(const kvec_handle* h, int batch, int budget, int tiles, i
     G.words = h->words;
     G.batch = batch;
     G.budget = budget;
+    G.wk = p.all_positions ? 0 : p.window;
     int Kp = (int)floor((double)p.beta * (double)budget);
-    if (Kp > budget - p.window) Kp = budget - p.window;
+    if (Kp > budget - G.wk) Kp = budget - G.wk;
     G.Kp = Kp;
-    G.k2 = budget - p.window - Kp;
+    G.k2 = budget - G.wk - Kp;
     G.total_tiles = tiles;
     G.win_tiles = chunks;
     G.HG = p.num_kv_heads < kWinHeadsPerCta ? p.num_kv_heads : kWinHeadsPerCta;

@@ -19,6 +19,7 @@ constexpr int kWinHeadsPerCta = 8; // KV heads one window CTA processes
 // Sizes and hyper-parameters shared by every kernel of one call.
 struct Geometry {
     int Hq, Hkv, g, w, O, Oe, pool, delta;
+    int wk;            // kept tail: w, or 0 when every position is a candidate; candidates [0, L - wk)
     int pool_avg;      // 1: average pool instead of max-pool
     int head_entropy;  // 1: rank heads by minus the entropy of pooled P_O instead of its std
     int R;             // rows per KV head = g * w, ordered r = q * g + j
@@ -28,7 +29,7 @@ struct Geometry {
     int words;         // ceil(ML / 32)
     int batch, budget, Kp, k2;
     int total_tiles;   // sum over sequences of ceil(L_s / kTileT)
-    int win_tiles;     // sum over sequences of ceil((L_s - w) / kTileT): candidate tiles
+    int win_tiles;     // sum over sequences of ceil((L_s - wk) / kTileT): candidate tiles
     int HG, NG;        // KV heads per window CTA, window CTAs per candidate tile
     int total_tokens;  // cu_seqlens[batch]
     const int* cu_host;  // host copy of cu_seqlens (host-side planning only; not for device code)

@@ -580,7 +580,7 @@ __global__ void __launch_bounds__(kSelectThreads) heads_pool_kernel(Geometry G, 
     const int h = blockIdx.x, s = blockIdx.y;
     const int tid = threadIdx.x, NT = blockDim.x;
     const int L = io.cu[s + 1] - io.cu[s];
-    const int Lc = L - G.w;
+    const int Lc = L - G.wk;
     const int halo = G.pool / 2;
     const size_t row = (size_t)s * G.Hkv + h;
     // Pool P_O and P_O' of this head (four positions per thread per step) and
@@ -623,7 +623,7 @@ __global__ void __launch_bounds__(kSelectThreads) heads_pool_kernel(Geometry G, 
             // the pool halo), each (q, t) element loaded by its own thread, then pooled.
             int tbase = 0;
             for (int b = 0; b < s; ++b) {
-                const int lb = io.cu[b + 1] - io.cu[b] - G.w;
+                const int lb = io.cu[b + 1] - io.cu[b] - G.wk;
                 tbase += lb > 0 ? (lb + kTileT - 1) / kTileT : 0;
             }
             const float invO = 1.f / (float)G.O;
@@ -704,7 +704,7 @@ __global__ void __launch_bounds__(kSelectThreads) heads_topk_kernel(Geometry G, 
     const int h = blockIdx.x, s = blockIdx.y;
     const int tid = threadIdx.x, NT = blockDim.x;
     const int L = io.cu[s + 1] - io.cu[s];
-    const int Lc = L - G.w;
+    const int Lc = L - G.wk;
     const size_t row = (size_t)s * G.Hkv + h;
     for (int wd = tid; wd < G.words; wd += NT) bits[wd] = 0u;
     // Programmatic dependent of the pooling kernel: its sigmas and pooled rows are
@@ -770,7 +770,7 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
     const int h = blockIdx.x, s = blockIdx.y;
     const int tid = threadIdx.x, NT = blockDim.x;
     const int L = io.cu[s + 1] - io.cu[s];
-    const int Lc = L - G.w;
+    const int Lc = L - G.wk;
     const int wordsL = (L + 31) >> 5;
     const int kw = key_stride(G);
     const bool cached = scores_in_smem(G.ML) && L > G.budget;

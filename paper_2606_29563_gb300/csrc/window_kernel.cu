@@ -2,7 +2,8 @@
 // the window queries' attention over the candidate tokens, recomputed on the
 // tensor cores with the softmax statistics (m_r, Z_r) of the score kernel.
 //
-// One CTA per (sequence s, 128-token tile of candidates, group of KV heads).
+// One CTA per (sequence s, 128-token tile of candidates, group of KV heads);
+// the candidates are [0, L - w), or [0, L) when every position competes.
 // For each KV head h of the group the CTA computes S^T = K_tile Q_h^T with
 // tcgen05.mma (M = 128 tokens, N = g*w query rows padded to 16, K = d) into
 // TMEM, so one epilogue thread owns one token and every query row of it:
@@ -68,12 +69,14 @@ __device__ __forceinline__ void win_abort(WinBars* bars, int* err) {
 
 // One head's window rows [q_lo, q_hi) of this thread's token: adds the rows'
 // group sums G_h[q] to po (q >= w-O) and poe (q >= w-O') and folds them into
-// the head maxima.  GG > 0 is the group size g known at compile time: each
-// 32-column chunk holds 32 / GG whole groups and runs as straight-line code.
+// the head maxima.  Rows q < qmin come before the token (it lies in the window
+// part, which only later rows see): their attention to it is 0.  GG > 0 is the
+// group size g known at compile time: each 32-column chunk holds 32 / GG whole
+// groups and runs as straight-line code.
 template <int GG>
 __device__ __forceinline__ void head_rows(uint32_t taddr, const float* __restrict__ rsb, int g, int q_lo, int q_hi,
-                                          float sl2, int qO, int qOe, float* maxg_col, bool first, float& po,
-                                          float& poe) {
+                                          int qmin, float sl2, int qO, int qOe, float* maxg_col, bool first,
+                                          float& po, float& poe) {
     if constexpr (GG > 0) {
         constexpr int QPC = 32 / GG, CW = QPC * GG;
         for (int qb = q_lo; qb < q_hi; qb += QPC) {
@@ -92,6 +95,7 @@ __device__ __forceinline__ void head_rows(uint32_t taddr, const float* __restric
 #pragma unroll
                 for (int j = 0; j < GG; ++j) gs += pr[k * GG + j];
                 const int q = qb + k;
+                gs = q >= qmin ? gs : 0.f;
                 if (q < q_hi) {
                     if (q >= qOe) poe += gs;
                     if (q >= qO) {
@@ -116,6 +120,7 @@ __device__ __forceinline__ void head_rows(uint32_t taddr, const float* __restric
                 if (i >= n) break;
                 gs += ptx::ex2(fmaf(v[i], sl2, -rsb[c0 + i]));
                 if (++jq == g) {
+                    gs = q >= qmin ? gs : 0.f;
                     if (q >= qOe) poe += gs;
                     if (q >= qO) {
                         po += gs;
@@ -167,7 +172,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
     {
         int base = 0, tbase = 0;
         for (int b = 0; b < G.batch; ++b) {
-            const int Lc = cu(b + 1) - cu(b) - G.w;
+            const int Lc = cu(b + 1) - cu(b) - G.wk;
             const int nt = Lc > 0 ? (Lc + kTileT - 1) / kTileT : 0;
             if ((int)blockIdx.x < base + nt * G.NG) {
                 const int local = (int)blockIdx.x - base;
@@ -182,7 +187,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
         }
     }
     if (s < 0) return;   // the whole CTA, before any barrier or TMEM use
-    const int L = cu(s + 1) - cu(s), Lc = L - G.w;
+    const int L = cu(s + 1) - cu(s), Lc = L - G.wk;
     const int h0 = ng * G.HG;
     const int nh = min(G.HG, G.Hkv - h0);
     const int NB = nacc;
@@ -268,7 +273,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
         const int quad = warp & 3;                        // TMEM lanes 32*quad .. +31
         const int tokl = quad * 32 + lane;
         const int t = jt * kTileT + tokl;
-        const bool valid = t < Lc;
+        const int qmin = t - (L - G.w);   // > 0 only for tokens in the window part
         const int q_lo = (qt * G.w) >> 2, q_hi = ((qt + 1) * G.w) >> 2;
         const int qO = G.w - G.O, qOe = G.w - G.Oe;
         const float invO = 1.f / (float)G.O, invOe = 1.f / (float)G.Oe;
@@ -299,7 +304,8 @@ __global__ void __launch_bounds__(kWinThreads, 1)
             ptx::tc_fence_after();
             const uint32_t taddr = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(b * Npad);
             float po = 0.f, poe = 0.f;
-            head_rows<GG>(taddr, rs + hh * kRsRows, G.g, q_lo, q_hi, G.sl2, qO, qOe, maxg + tokl, hh == 0, po, poe);
+            head_rows<GG>(taddr, rs + hh * kRsRows, G.g, q_lo, q_hi, qmin, G.sl2, qO, qOe, maxg + tokl, hh == 0, po,
+                          poe);
             ptx::tc_fence_before();
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&bars->acc_empty[b]);

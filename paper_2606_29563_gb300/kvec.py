@@ -48,7 +48,7 @@ class kvec_params(ctypes.Structure):
         ("pool_kernel", ctypes.c_int), ("num_ext_heads", ctypes.c_int),
         ("lam", ctypes.c_float), ("beta", ctypes.c_float), ("softmax_scale", ctypes.c_float),
         ("max_batch", ctypes.c_int), ("max_seqlen", ctypes.c_int), ("max_layers", ctypes.c_int),
-        ("pool_mode", ctypes.c_int), ("head_criterion", ctypes.c_int),
+        ("pool_mode", ctypes.c_int), ("head_criterion", ctypes.c_int), ("all_positions", ctypes.c_int),
     ]
 
 
@@ -204,10 +204,11 @@ def kvec_status_string(status: int) -> str:
 def make_params(num_q_heads: int, num_kv_heads: int, head_dim: int = 128, window: int = 32, obs_window: int = 16,
                 ext_window: int = 32, pool_kernel: int = 7, num_ext_heads: int = 3, lam: float = 1.0,
                 beta: float = 0.25, softmax_scale: float = 0.0, max_batch: int = 1, max_seqlen: int = 8192,
-                max_layers: int = 32, pool_mode: int = 0, head_criterion: int = 0) -> kvec_params:
+                max_layers: int = 32, pool_mode: int = 0, head_criterion: int = 0,
+                all_positions: int = 0) -> kvec_params:
     return kvec_params(num_q_heads, num_kv_heads, head_dim, window, obs_window, ext_window, pool_kernel,
                        num_ext_heads, lam, beta, softmax_scale, max_batch, max_seqlen, max_layers, pool_mode,
-                       head_criterion)
+                       head_criterion, all_positions)
 
 
 def params_from_workload(wl, max_batch: Optional[int] = None, max_seqlen: Optional[int] = None,
@@ -215,7 +216,8 @@ def params_from_workload(wl, max_batch: Optional[int] = None, max_seqlen: Option
     return make_params(wl.num_q_heads, wl.num_kv_heads, wl.head_dim, wl.window, wl.obs_window, wl.ext_window,
                        wl.pool_kernel, wl.num_ext_heads, wl.lam, wl.beta, 0.0,
                        max_batch or wl.batch, max_seqlen or wl.max_seqlen, max_layers or max(wl.layers, 1),
-                       getattr(wl, "pool_mode", 0), getattr(wl, "head_criterion", 0))
+                       getattr(wl, "pool_mode", 0), getattr(wl, "head_criterion", 0),
+                       getattr(wl, "all_positions", 0))
 
 
 class _DeviceArray:

@@ -46,6 +46,7 @@ class Workload:
     pool_kernel: int = 7
     pool_mode: int = 0        # 0 max-pool, 1 average pool (variant)
     head_criterion: int = 0   # 0 standard deviation, 1 entropy (variant)
+    all_positions: int = 0    # 0 keep the window tail, 1 every position is a candidate (variant)
     budget: int = 512         # B per KV head, window included
     num_ext_heads: int = 3    # delta
     lam: float = 1.0          # lambda

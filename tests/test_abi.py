@@ -59,6 +59,7 @@ BAD_PARAMS = [
     (dict(max_seqlen=200000), kvec.KVEC_ERR_INVALID_ARG),
     (dict(num_q_heads=72, num_kv_heads=8), kvec.KVEC_ERR_UNSUPPORTED),   # 9 x 32 rows > 256
     (dict(num_q_heads=264, num_kv_heads=33), kvec.KVEC_ERR_UNSUPPORTED),
+    (dict(all_positions=2), kvec.KVEC_ERR_INVALID_ARG),
 ]
 
 

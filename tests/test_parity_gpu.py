@@ -287,3 +287,49 @@ def test_llama8b_ragged8_b256_first_layers():
 @pytest.mark.parametrize("budget", synth.QWEN_BUDGETS)
 def test_qwen7b_l16384_budget_sweep(budget):
     _assert_parity(synth.WORKLOADS["qwen7b_l16384_b512"].replace(budget=budget), layers=2)
+
+
+# ---- top-B over every position (all_positions = 1, Section 4.1 read literally) ----
+
+@pytest.mark.parametrize("kw", [dict(seqlens=(900, 421), layers=2),
+                                dict(seqlens=(40, 1000, 64, 257), budget=64, layers=2),
+                                dict(seqlens=(777,), budget=20, layers=2),
+                                dict(seqlens=(523,), num_q_heads=28, num_kv_heads=4, layers=2),
+                                dict(seqlens=(700,), num_q_heads=16, num_kv_heads=16, layers=2),
+                                dict(seqlens=(640,), pool_mode=1, head_criterion=1, layers=2),
+                                dict(seqlens=(600,), window=48, obs_window=32, ext_window=48, layers=2)])
+def test_all_positions_matches_the_oracle(kw):
+    # Candidates [0, L): the window part scored with its causal attention (a
+    # token there is seen only by the later window rows), nothing kept by rule;
+    # a budget below the window, keep-all members, split head groups, the variants.
+    _assert_parity(synth.small_workload(all_positions=1, **kw))
+
+
+def test_all_positions_with_caller_lse():
+    _assert_parity(synth.small_workload(seqlens=(1100, 333), layers=2, all_positions=1), with_lse=True)
+
+
+def test_all_positions_llama8b_l8192_b512_first_layers():
+    _assert_parity(synth.WORKLOADS["llama8b_l8192_b512"].replace(all_positions=1), layers=2)
+
+
+def test_all_positions_multi_layer_call_matches_layer_by_layer():
+    wl = synth.small_workload(seqlens=(1100, 700), layers=3, budget=96, all_positions=1)
+    layers = [{k: v.cuda() for k, v in x.items()} for x in synth.make_layers(wl, 3)]
+    cu = torch.tensor(wl.cu_seqlens, dtype=torch.int32)
+    sel = kvec.KvecSelector(kvec.params_from_workload(wl))
+    st1 = sel.new_state(wl.batch)
+    one = [sel.select_layer(cu, cu.cuda(), x["q_obs"], x["k"], x["v"], st1, wl.budget) for x in layers]
+    st2 = sel.new_state(wl.batch)
+    many = [sel.alloc_outputs(wl.batch, wl.budget) for _ in layers]
+    stream = torch.cuda.current_stream().cuda_stream
+    for _ in range(3):   # the second call captures the pipeline, the third replays the graph
+        kvec.kvec_reset(sel.handle, st2.data_ptr(), wl.batch, stream)
+        sel.select_layers(cu, cu.cuda(), [x["q_obs"] for x in layers], [x["k"] for x in layers],
+                          [x["v"] for x in layers], st2, wl.budget, many)
+    torch.cuda.synchronize()
+    for a, b in zip(one, many):
+        for x, y in zip(a, b):
+            assert torch.equal(x, y)
+    assert torch.equal(st1, st2)
+    sel.close()

@@ -359,6 +359,35 @@ def run_ours(args, wl):
                        "api": "kvec_select_layers_lse: window-row log-sum-exp from the caller's prefill attention",
                        "path_roofline_frac": by["layer_total"] * L_layers / (ms_lse / 1e3) / 1e9 / peak}
 
+    # The same step with every position a candidate (kvec_params.all_positions = 1:
+    # Section 4.1's top-B over the T input tokens, no retained window), own handle.
+    all_positions_variant = None
+    if args.all_positions_variant:
+        sel_ap = kvec.KvecSelector(kvec.params_from_workload(wl.replace(all_positions=1)))
+        state_ap = sel_ap.new_state(wl.batch, dev)
+
+        def step_ap():
+            kvec.kvec_reset(sel_ap.handle, state_ap.data_ptr(), wl.batch, stream.cuda_stream)
+            sel_ap.select_layers(cu_host, cu_dev, qs, ks, vs, state_ap, wl.budget, outs, stream)
+
+        for _ in range(max(args.warmup, 3)):
+            step_ap()
+        n_ap = min(args.steps, 500)
+        torch.cuda.synchronize()
+        start.record(stream)
+        for _ in range(n_ap):
+            step_ap()
+        stop.record(stream)
+        torch.cuda.synchronize()
+        kvec.kvec_sync_status(sel_ap.handle)
+        sel_ap.close()
+        ms_ap = max_over_ranks(start.elapsed_time(stop), dev) / n_ap
+        all_positions_variant = {
+            "metric": METRIC, "value": world * evicted_per_step / (ms_ap / 1e3), "unit": "tokens/s",
+            "ms_per_step": ms_ap, "steps": n_ap,
+            "api": "kvec_select_layers with kvec_params.all_positions = 1: top-B over every position",
+            "path_roofline_frac": by["layer_total"] * L_layers / (ms_ap / 1e3) / 1e9 / peak}
+
     decode = run_decode(args, wl, sel, layers, outs, dev, peak) if args.decode else None
 
     # End to end through the public API: pinned host inputs copied in, indices and state copied out.
@@ -387,6 +416,7 @@ def run_ours(args, wl):
         "clocks": {k: v for k, v in clocks.summary(t_host0, t_host1).items()},
         "gpu_launches": gpu_launches,
         "lse_variant": lse_variant,
+        "all_positions_variant": all_positions_variant,
         "decode": decode,
         "e2e": e2e,
     }
@@ -584,6 +614,8 @@ def main(argv=None):
                     help="skip the decode-attention measurement over the compacted caches")
     ap.add_argument("--no-lse-variant", dest="lse_variant", action="store_false",
                     help="skip timing the kvec_select_layers_lse variant")
+    ap.add_argument("--no-all-positions-variant", dest="all_positions_variant", action="store_false",
+                    help="skip timing the top-B-over-every-position variant")
     args = ap.parse_args(argv)
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3

@@ -102,3 +102,28 @@ def test_noalloc_refuses_oversize_calls_before_cuda(lib):
                                        512, fake, fake, fake, None)
     assert e.value.status == kvec.KVEC_ERR_INVALID_ARG
     assert "scratch" in str(e.value)
+
+
+@pytest.mark.parametrize("struct", [kvec.kvec_params, kvec.kvec_debug_view])
+def test_binding_structs_match_the_header_layout(tmp_path, struct):
+    """Every field of the ctypes mirror sits at the offset (and the struct has the
+    size) that a C compiler gives the declaration in include/kvec.h."""
+    import shutil
+    import subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    name = struct.__name__
+    c_name = {"lam": "lambda"}   # fields the binding renames (Python keywords)
+    lines = [f'printf("size %zu\\n", sizeof({name}));']
+    lines += [f'printf("{f} %zu\\n", offsetof({name}, {c_name.get(f, f)}));' for f, _ in struct._fields_]
+    src = tmp_path / "layout.c"
+    src.write_text("#include <stddef.h>\n#include <stdio.h>\n#include \"kvec.h\"\nint main(void) {\n" +
+                   "\n".join(lines) + "\nreturn 0;\n}\n")
+    exe = tmp_path / "layout"
+    subprocess.run([cc, "-std=c99", "-I", os.path.join(ROOT, "include"), str(src), "-o", str(exe)], check=True)
+    out = dict(line.split() for line in subprocess.run([str(exe)], capture_output=True, text=True,
+                                                        check=True).stdout.splitlines())
+    assert int(out["size"]) == ctypes.sizeof(struct)
+    for f, _ in struct._fields_:
+        assert int(out[f]) == getattr(struct, f).offset, f

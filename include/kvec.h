@@ -116,7 +116,8 @@ KVEC_API kvec_status kvec_reset(kvec_handle* h, void* coverage_state, int batch,
  *          (post-RoPE, as the attention saw them).
  *   k, v   device bf16 [cu[batch]][H_kv][d]: the layer's prefix keys and values.
  *   coverage_state  device, batch states (kvec_state_bytes each); read and updated.
- *   budget B: tokens kept per KV head, the w window tokens included; B >= w.
+ *   budget B: tokens kept per KV head, the w window tokens included; B >= w
+ *          (with all_positions = 1 nothing is kept by rule and B >= 1).
  *   out_idx device int32 [batch][H_kv][B]: kept positions (0-based within the
  *          sequence), ascending; -1 after the last one when L_s < B.
  *   out_k, out_v device bf16 [batch][H_kv][B][d]: gathered rows, zero padded.

@@ -463,3 +463,16 @@ def test_all_positions_rejects_nothing_the_default_needs():
         _run_oracle(oracle.OracleParams(**base), q, k, v, oracle.new_state(1, 40), 6)
     r = _run_oracle(oracle.OracleParams(all_positions=1, **base), q, k, v, oracle.new_state(1, 40), 6)
     assert (np.diff(r["out_idx"][0], axis=-1) > 0).all() and r["out_idx"].shape[-1] == 6
+
+
+@pytest.mark.parametrize("beta", [0.0, 0.25, 1.0])
+def test_all_positions_without_coverage_is_plain_topB_of_every_position(beta):
+    """delta = 0 and lambda = 0: every head keeps the top B of pooled P_O over
+    [0, L), whatever beta, with no window kept by rule."""
+    wl = synth.small_workload(seqlens=(400,), num_ext_heads=0, lam=0.0, budget=72, all_positions=1, beta=beta)
+    p = oracle.OracleParams.from_workload(wl)
+    st = oracle.new_state(1, 400)
+    for x in _wl_layers(wl, 2):
+        r = oracle.select_layer(p, wl.cu_seqlens, x["q_obs"], x["k"], x["v"], st, wl.budget)
+        for h in range(wl.num_kv_heads):
+            assert (r["out_idx"][0, h] == _top_positions(r["P_O"][0, h, :400], wl.budget)).all()

@@ -29,7 +29,7 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 METRIC = "prefix tokens evicted/sec (all layers, device-timed) and % of HBM roofline"
-DEFAULT_WORKLOAD = "llama8b_l8192_b512"
+DEFAULT_WORKLOAD = "llama8b_ragged8_b256"   # the largest single-GPU configuration
 FALLBACK_HBM_GBS = 6800.0
 KERNEL_SOURCES = {
     "score": "paper_2606_29563_gb300/csrc/score_kernel.cu",
@@ -162,6 +162,22 @@ def committed_traffic(kernel: str, workload: str):
         if entry.get("source_sha256") != hashlib.sha256(src).hexdigest():
             return None
         return float(entry["bytes_per_launch"])
+    except (OSError, ValueError, KeyError, TypeError):
+        return None
+
+
+def committed_step_traffic(wl, layers: int):
+    """DRAM bytes (read + written) of one whole step from the committed ncu record of
+    every kernel of a layer (profiles/traffic.json, "step"), if no kernel source has
+    changed since the capture; else None."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            entry = json.load(f)["step"][wl.name]
+        for rel, sha in entry["sources_sha256"].items():
+            if hashlib.sha256(open(os.path.join(ROOT, rel), "rb").read()).hexdigest() != sha:
+                return None
+        return float(entry["bytes_per_layer"]) * layers
     except (OSError, ValueError, KeyError, TypeError):
         return None
 
@@ -304,33 +320,30 @@ def run_ours(args, wl):
     value = world * evicted_per_step * args.steps / (elapsed_ms / 1e3)
     ms_per_step = elapsed_ms / args.steps
 
-    # Per-kernel device time (CUDA events recorded by the library on the launching stream).
-    kvec.kvec_set_profiling(sel.handle, True)
-    for _ in range(min(args.steps, 50)):
-        step()
-    torch.cuda.synchronize()
-    ktimes = {}
-    for i, name in enumerate(kvec.KERNEL_NAMES):
-        ms, n = kvec.kvec_kernel_time(sel.handle, i)
-        ktimes[name] = {"ms_per_launch": ms / n if n else None, "launches": n,
-                        "share": None}
-    total_k = sum(v["ms_per_launch"] * v["launches"] for v in ktimes.values() if v["ms_per_launch"])
-    for v in ktimes.values():
-        if v["ms_per_launch"]:
-            v["share"] = v["ms_per_launch"] * v["launches"] / total_k
-    kvec.kvec_set_profiling(sel.handle, False)
     peak, peak_kind = measured_hbm_gbs()
     by = workload_bytes(wl)
-    per_kernel = {}
-    for name, v in ktimes.items():
-        if not v["ms_per_launch"]:
-            continue
-        a = by["per_kernel"][name] / (v["ms_per_launch"] / 1e3) / 1e9
-        per_kernel[name] = {"achieved": a, "frac": a / peak, "bytes_per_launch": by["per_kernel"][name],
-                            "traffic": committed_traffic(name, wl.name)}
-    # The dominant kernel: the largest share of the step's kernel time (CUDA events on the launching streams).
-    dom = max(per_kernel, key=lambda k: ktimes[k]["share"] or 0.0)
-    path_gbs = by["layer_total"] * L_layers / (ms_per_step / 1e3) / 1e9
+    bytes_step = by["layer_total"] * L_layers
+    path_gbs = bytes_step / (ms_per_step / 1e3) / 1e9
+
+    # Clock evidence: when the timed region was too short for the sampler (it
+    # polls every 50 ms), the same step keeps running for about a second right
+    # after it, and the clocks are read over that run instead.
+    clk = clocks.summary(t_host0, t_host1)
+    if args.clock_probe and (clk.get("samples", 0) < 3 or clk.get("window") != "timed region"):
+        clocks2 = ClockSampler(local).start()
+        time.sleep(0.2)
+        n_more = max(1, int(1000.0 / max(ms_per_step, 1e-3)))
+        t2 = time.perf_counter()
+        for _ in range(n_more):
+            step()
+        torch.cuda.synchronize()
+        t3 = time.perf_counter()
+        clocks2.stop()
+        clk2 = clocks2.summary(t2, t3)
+        if clk2.get("sm_mhz") is not None:
+            clk2["window"] = (f"{n_more} more steps of the same workload right after the timed region "
+                              f"({clk.get('samples', 0)} samples fell inside it)")
+            clk = clk2
 
     # The same step with the window rows' log-sum-exp supplied by the caller
     # (kvec_select_layers_lse, no statistics pass over K); the lse inputs are
@@ -397,6 +410,9 @@ def run_ours(args, wl):
     # gather; per call one finalize launch (the last layer's union into the state).
     gpu_launches = args.steps * (L_layers * LAUNCHES_PER_LAYER + 1)
     sel.close()
+    del layers, qs, ks, vs, outs, state
+    torch.cuda.empty_cache()
+    other = run_other_configs(args, wl, dev, peak) if args.other_configs and world == 1 else None
     result = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
@@ -406,23 +422,81 @@ def run_ours(args, wl):
                    "window": wl.window, "budget": wl.budget, "parallelism": f"replicas{world}",
                    "l2": f"inputs larger than L2 ({(by['k_read'] * 2 + by['q_read']) * L_layers / 1e9:.2f} GB per step)",
                    "precision": "bf16 inputs, fp32 accumulation and scores"},
-        "roofline": {"bound": "hbm", "kernel": dom, "achieved": per_kernel[dom]["achieved"], "peak": peak,
-                     "unit": "GB/s", "frac": per_kernel[dom]["frac"], "traffic": per_kernel[dom]["traffic"],
-                     "peak_source": peak_kind, "bytes_per_launch": per_kernel[dom]["bytes_per_launch"]},
-        "roofline_by_kernel": per_kernel,
-        "path_roofline": {"achieved": path_gbs, "peak": peak, "unit": "GB/s", "frac": path_gbs / peak,
-                          "bytes_per_step": by["layer_total"] * L_layers},
-        "kernels": ktimes,
-        "clocks": {k: v for k, v in clocks.summary(t_host0, t_host1).items()},
+        "roofline": {"bound": "hbm", "kernel": "whole eviction pass: every kernel of one kvec_select_layers call",
+                     "achieved": path_gbs, "peak": peak, "unit": "GB/s", "frac": path_gbs / peak,
+                     "traffic": committed_step_traffic(wl, L_layers), "peak_source": peak_kind,
+                     "bytes_per_step": bytes_step,
+                     "bytes": "algorithmic: K read once + q_obs + kept K/V rows read and written + out_idx",
+                     "strict_frac": (by["k_read"] + by["gather"] // 2) * L_layers / (ms_per_step / 1e3) / 1e9 / peak},
+        "clocks": clk,
         "gpu_launches": gpu_launches,
         "lse_variant": lse_variant,
         "all_positions_variant": all_positions_variant,
         "decode": decode,
         "e2e": e2e,
+        "other_configs": other,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         result["cpu_baseline"] = oracle_baseline(wl)
     return rank, result
+
+
+def run_other_configs(args, wl_main, dev, peak):
+    """The other workloads of the benchmark set, each timed like the main one (one
+    step = reset + one kvec_select_layers call over every layer; device time with
+    CUDA events on the launching stream, inputs resident in HBM, larger than L2).
+    The Qwen2.5-7B-shaped workload runs at every budget of its sweep."""
+    import torch
+    from paper_2606_29563_gb300 import kvec, synth
+    names = [n for n in synth.WORKLOADS if n != wl_main.name]
+    runs = []
+    for n in names:
+        base = synth.WORKLOADS[n]
+        if n.startswith("qwen7b"):
+            runs += [base.replace(budget=b, name=f"{n.rsplit('_b', 1)[0]}_b{b}") for b in synth.QWEN_BUDGETS]
+        else:
+            runs.append(base)
+    out = {}
+    stream = torch.cuda.current_stream(dev)
+    for wl in runs:
+        if wl.name == wl_main.name:
+            continue
+        structure = [synth.salient_structure(wl, b, wl.layers) for b in range(wl.batch)]
+        xs = [synth.make_layer(wl, l, dev, structure) for l in range(wl.layers)]
+        sel = kvec.KvecSelector(kvec.params_from_workload(wl))
+        cu_host = torch.tensor(wl.cu_seqlens, dtype=torch.int32).pin_memory()
+        cu_dev = cu_host.to(dev)
+        outs = [sel.alloc_outputs(wl.batch, wl.budget, dev) for _ in range(wl.layers)]
+        state = sel.new_state(wl.batch, dev)
+        qs, ks, vs = [x["q_obs"] for x in xs], [x["k"] for x in xs], [x["v"] for x in xs]
+
+        def step():
+            kvec.kvec_reset(sel.handle, state.data_ptr(), wl.batch, stream.cuda_stream)
+            sel.select_layers(cu_host, cu_dev, qs, ks, vs, state, wl.budget, outs, stream)
+
+        for _ in range(max(args.warmup, 3)):
+            step()
+        torch.cuda.synchronize()
+        n_steps = max(10, min(args.steps, 200))
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(n_steps):
+            step()
+        b.record(stream)
+        torch.cuda.synchronize()
+        kvec.kvec_sync_status(sel.handle)
+        ms = a.elapsed_time(b) / n_steps
+        by = workload_bytes(wl)
+        bytes_step = by["layer_total"] * wl.layers
+        evicted = wl.evicted_per_layer() * wl.layers
+        out[wl.name] = {"ms_per_step": ms, "steps": n_steps, "value": evicted / (ms / 1e3), "unit": "tokens/s",
+                        "layers": wl.layers, "batch": wl.batch, "budget": wl.budget,
+                        "evicted_per_step": evicted, "bytes_per_step": bytes_step,
+                        "path_roofline_frac": bytes_step / (ms / 1e3) / 1e9 / peak}
+        sel.close()
+        del xs, qs, ks, vs, outs, state
+        torch.cuda.empty_cache()
+    return out
 
 
 def run_decode(args, wl, sel, layers, outs, dev, peak):
@@ -572,25 +646,38 @@ def run_reference(args, wl):
     p = oracle.OracleParams.from_workload(wl)
     structure = [synth.salient_structure(wl, b, 1) for b in range(wl.batch)]
     x = synth.make_layer(wl, 0, "cpu", structure)
-    # A bounded sample per step: the first layer of the workload, from a fresh state.
+    cu = wl.cu_seqlens
+    # A bounded sample per step: layer 0 of one sequence of the batch (the
+    # sequences in turn), from a fresh coverage state.
+    samples = []
+    for b in range(wl.batch):
+        wl_b = wl.replace(seqlens=(wl.seqlens[b],))
+        samples.append((wl_b, x["q_obs"][b:b + 1], x["k"][cu[b]:cu[b + 1]], x["v"][cu[b]:cu[b + 1]]))
+    count = [0]
+
     def step():
-        st = oracle.new_state(wl.batch, wl.max_seqlen)
-        oracle.select_layer(p, wl.cu_seqlens, x["q_obs"], x["k"], x["v"], st, wl.budget,
-                            max_seqlen=wl.max_seqlen, debug=False)
+        wl_b, q, k, v = samples[count[0] % len(samples)]
+        count[0] += 1
+        st = oracle.new_state(1, wl_b.max_seqlen)
+        oracle.select_layer(p, wl_b.cu_seqlens, q, k, v, st, wl.budget, max_seqlen=wl_b.max_seqlen, debug=False)
+        return wl_b.evicted_per_layer()
 
     for _ in range(args.warmup):
         step()
+    evicted = 0
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        step()
+        evicted += step()
     dt = time.perf_counter() - t0
-    value = wl.evicted_per_layer() * args.steps / dt
-    sample = f"layer 0 of {wl.name} per step (fp64 C oracle, OpenMP, {oracle.num_threads()} threads)"
+    value = evicted / dt
+    sample = (f"layer 0 of one sequence of {wl.name} per step (the {wl.batch} sequences in turn), fp64 C oracle, "
+              f"OpenMP, {oracle.num_threads()} threads")
     return rank, {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3 / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": wl.name, "layers_per_step": 1, "batch": wl.batch, "budget": wl.budget},
+        "config": {"workload": wl.name, "layers_per_step": 1, "sequences_per_step": 1, "batch": wl.batch,
+                   "budget": wl.budget},
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": oracle.num_threads(), "kind": "oracle",
                          "sample": sample},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -616,6 +703,10 @@ def main(argv=None):
                     help="skip timing the kvec_select_layers_lse variant")
     ap.add_argument("--no-all-positions-variant", dest="all_positions_variant", action="store_false",
                     help="skip timing the top-B-over-every-position variant")
+    ap.add_argument("--no-clock-probe", dest="clock_probe", action="store_false",
+                    help="do not extend a short timed region by a second of steps to read the clocks")
+    ap.add_argument("--no-other-configs", dest="other_configs", action="store_false",
+                    help="skip timing the other workloads of the benchmark set")
     args = ap.parse_args(argv)
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3

@@ -183,24 +183,38 @@ KVEC_API kvec_status kvec_select_layer_lse(kvec_handle* h, int batch,
  *   limits (max_batch, max_seqlen; max_seqlen also fixes the state layout)
  *   given in *params instead of a handle.
  *   Scratch: one 32 MiB static device array inside the library, held by every
- *   GPU that loads the library until the process exits.  A call whose
- *   geometry needs more (roughly: batch * H_kv * (L * g * w * 2 + 16 * L)
- *   bytes; one 8192-token Llama-3.1-8B-shaped sequence needs about 18 MiB) is
+ *   GPU that loads the library until the process exits.  A call needs about
+ *   (28 * H_kv + 9) * ML bytes per sequence (ML = max_seqlen + 4 rounded up to
+ *   a multiple of 32) plus (8 * H_kv * g * w + 512 * O * ceil(H_kv / 8)) bytes
+ *   per 128-token tile of its sequences; one 8192-token Llama-3.1-8B-shaped
+ *   sequence needs about 3 MiB.  A call that needs more than the array is
  *   rejected with KVEC_ERR_INVALID_ARG and a message giving both sizes.
- *   Every call shares that array and it keeps the last call's contents; the
- *   call clears what must start at zero.  Calls whose work overlaps on the
- *   GPU (different streams, or several host threads) race on it: serialise
- *   them.
- *   The first call on each device resolves the array's device address and
- *   sets kernel attributes (no allocation); make that first call before any
- *   stream capture.  The device-side 255-layer guard is not reported by this
- *   entry point: keep layers_done below 255 yourself. */
+ *   Every call shares that array and it keeps the last call's contents; each
+ *   part of it is written before it is read within a call.  Calls whose work
+ *   overlaps on the GPU (different streams, or several host threads) race on
+ *   it: serialise them.
+ *   The first call on each device resolves the array's device address, sets
+ *   kernel attributes and clears the array's error word, synchronously (no
+ *   allocation); make that first call before any stream capture.
+ *   Device-side errors (a bounded wait that gave up, or the refusal of a call
+ *   that would take a state past 255 layers, which leaves that state unchanged)
+ *   are recorded in the array's error word and reported by
+ *   kvec_noalloc_sync_status. */
 KVEC_API kvec_status kvec_select_layer_noalloc(const kvec_params* params, int batch,
                                       const int32_t* cu_seqlens_host, const int32_t* cu_seqlens_dev,
                                       const void* q_obs, const void* k, const void* v,
                                       void* coverage_state, int budget,
                                       int32_t* out_idx, void* out_k, void* out_v,
                                       kvec_stream_t stream);
+
+/* Device-side status of kvec_select_layer_noalloc on the current device:
+ * synchronises `stream`, then returns KVEC_ERR_DEVICE_TIMEOUT if a bounded
+ * wait of any call since the last check gave up, KVEC_ERR_INVALID_ARG if a
+ * call was refused because a state would have passed 255 layers (that state
+ * is unchanged), else KVEC_OK; the recorded error is cleared.  The outputs of
+ * a call that recorded an error are invalid.  Allocates nothing; KVEC_OK when
+ * no call has run on this device yet. */
+KVEC_API kvec_status kvec_noalloc_sync_status(kvec_stream_t stream);
 
 /* One decoding step of attention over the compacted cache that the selection
  * produced.  Section 4.1: once each KV head has kept its B tokens, their keys
@@ -229,7 +243,8 @@ KVEC_API kvec_status kvec_decode_attention(kvec_handle* h, int batch, const void
 /* Device views of the last processed layer's intermediates (valid until the
  * next call on the handle; read after synchronising the stream).  Row strides
  * use ML = max_seqlen + 4 rounded up to a multiple of 32 (reported in max_seqlen).
- * Only candidate positions t < L_s - w hold scores. */
+ * Only candidate positions hold scores: t < L_s - w by default, t < L_s with
+ * all_positions = 1.  Pprime is written only for sequences with L_s > budget. */
 typedef struct {
     const float*    P_O;        /* [max_batch][H_kv][ML]  Eq. 1 with O, max-pooled */
     const float*    P_Oext;     /* [max_batch][H_kv][ML]  Eq. 1 with O', max-pooled */
@@ -259,6 +274,16 @@ KVEC_API kvec_status kvec_sync_status(kvec_handle* h);
  * preserved tokens, 3 coverage-adjusted selection, 4 gather.  Synchronises. */
 KVEC_API kvec_status kvec_set_profiling(kvec_handle* h, int enable);
 KVEC_API kvec_status kvec_kernel_time(kvec_handle* h, int kernel, double* total_ms, int* launches);
+
+/* For tests of the error path only; never set in production.  fault = 1 makes
+ * every window kernel launched from then on withhold the signal of its first
+ * accumulator, so that the epilogue's bounded wait for it gives up after about
+ * 20 us: the kernel records KVEC_ERR_DEVICE_TIMEOUT in the error word (read by
+ * kvec_sync_status or kvec_noalloc_sync_status), drains its copies and returns,
+ * and that call's outputs are invalid.  fault = 0 (the default) switches it
+ * off.  Process-wide; while it is set, multi-layer calls are neither captured
+ * into nor replayed from the handle's graph cache. */
+KVEC_API void kvec_set_test_fault(int fault);
 
 KVEC_API const char* kvec_status_string(kvec_status s);
 KVEC_API const char* kvec_last_error(void);

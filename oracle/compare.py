@@ -1,7 +1,8 @@
 """Comparison of a GPU layer result with the oracle's (TEST INFRASTRUCTURE ONLY).
 
 Tolerances (bf16 inputs, fp32 accumulation on the GPU, fp64 in the oracle):
-* a score x passes if |x_gpu - x_orc| <= tol * (|x_orc| + mean over candidates of |x_orc|).
+* a score x (P_O, P_O', I and the coverage-adjusted P' of every candidate) passes
+  if |x_gpu - x_orc| <= tol * (|x_orc| + mean over candidates of |x_orc|).
   The mean term makes the bound meaningful for tiny scores: at L = 8192 the
   average score is ~1e-4, so a pure 2e-3 absolute bound would accept anything.
 * kept-index sets must be identical except for positions whose oracle key lies
@@ -53,6 +54,13 @@ def check_layer(gpu: Dict[str, np.ndarray], orc: Dict[str, np.ndarray], seqlens,
             e = rel_err(gpu["I"][b, :Lc], orc["I"][b, :Lc])
             if e.max() > tol:
                 errs.append(f"seq {b}: I rel err {e.max():.3g} at t={int(e.argmax())}")
+            # P' = P + lambda * I * (1 - n_t / (l + 1)) (Section 4.2), the key of the
+            # final fill; the GPU writes it only when the sequence is evicted (L > B).
+            if gpu.get("Pprime") is not None and L > budget:
+                for h in range(H):
+                    e = rel_err(gpu["Pprime"][b, h, :Lc], orc["Pprime"][b, h, :Lc])
+                    if e.max() > tol:
+                        errs.append(f"seq {b} head {h}: Pprime rel err {e.max():.3g} at t={int(e.argmax())}")
             e = np.abs(gpu["sigma"][b] - orc["sigma"][b]) / (np.abs(orc["sigma"][b]) + 1e-30)
             if e.max() > tol:
                 errs.append(f"seq {b}: sigma rel err {e.max():.3g}")

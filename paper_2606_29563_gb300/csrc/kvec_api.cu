@@ -5,6 +5,7 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <atomic>
 #include <mutex>
 #include <string>
 #include <vector>
@@ -40,12 +41,25 @@ size_t row_stride(int max_seqlen) { return round_up((size_t)max_seqlen + 4, 32);
 
 constexpr int kKernelKinds = 5;
 
+// Fault injected for tests of the error path (kvec_set_test_fault); 0 = none.
+std::atomic<int> g_test_fault{0};
+
+// Maps a device error word to a status (and the message of kvec_last_error).
+kvec_status device_error_status(int err) {
+    if (err == 2)
+        return fail(KVEC_ERR_INVALID_ARG,
+                    "a call would have taken a coverage state past 255 layers (that state was left unchanged)");
+    return fail(KVEC_ERR_DEVICE_TIMEOUT, "a bounded device wait gave up (code %d)", err);
+}
+
 struct TimedLaunch {
     int kind;
     cudaEvent_t start, stop;
 };
 
 }  // namespace
+
+int kvec::test_fault() { return g_test_fault.load(std::memory_order_relaxed); }
 
 constexpr int kSlots = 8;   // per-layer score arrays in flight between the score and select stages
 constexpr int kScoreBufs = 2;   // score-statistics buffers in flight between the score and window stages
@@ -663,7 +677,9 @@ kvec_status select_layers_impl(kvec_handle* h, int num_layers, int batch, const 
         io.out_v = static_cast<__nv_bfloat16*>(out_v[l]);
         io.lse = lse ? lse[l] : nullptr;
     }
-    if (!h->profiling && num_layers >= 2) {
+    // Graphs are neither captured nor replayed while a test fault is injected:
+    // a captured launch would keep the fault after it is switched off.
+    if (!h->profiling && num_layers >= 2 && test_fault() == 0) {
         // A call repeated with the same arguments replays a captured graph of the pipeline.
         std::vector<uint64_t> key = graph_key(num_layers, batch, budget, cu_seqlens_host, cu_seqlens_dev, ios.data());
         for (size_t i = 0; i < h->graphs.size(); ++i) {
@@ -788,6 +804,11 @@ kvec_status noalloc_setup(int dev, void** base, const Geometry& G) {
         if (e == cudaSuccess) e = configure_window(G);
         if (e == cudaSuccess) e = configure_select();
         if (e != cudaSuccess) return cuda_fail(e, "kernel attributes");
+        // The error word (the array's first bytes) starts at zero; calls leave it
+        // set until kvec_noalloc_sync_status reads and clears it.
+        e = cudaMemset(ptr, 0, sizeof(int));
+        if (e == cudaSuccess) e = cudaDeviceSynchronize();
+        if (e != cudaSuccess) return cuda_fail(e, "clearing the scratch error word");
         d.base = ptr;
         d.ready = true;
     }
@@ -834,7 +855,7 @@ kvec_status kvec_select_layer_noalloc(const kvec_params* params, int batch, cons
     const size_t HGv = Hkv < (size_t)kWinHeadsPerCta ? Hkv : (size_t)kWinHeadsPerCta;
     const size_t NGv = (Hkv + HGv - 1) / HGv;
     Part parts[] = {
-        {(void**)&tmp.sc.err, sizeof(int)},                   // zeroed every call (the first part)
+        {(void**)&tmp.sc.err, sizeof(int)},                   // error word, first: see noalloc_setup
         {(void**)&tmp.sc.nbuf, nb * round_up((size_t)params->max_seqlen, 16)},
         {(void**)&tmp.sc.segpart, nt * Hkv * R * sizeof(float2)},
         {(void**)&tmp.slots[0].wpart, nt * NGv * (size_t)params->obs_window * kTileT * sizeof(float)},
@@ -853,11 +874,8 @@ kvec_status kvec_select_layer_noalloc(const kvec_params* params, int batch, cons
         {(void**)&tmp.slots[0].Pprime, nb * Hkv * ML * sizeof(float)},
         {(void**)&tmp.slots[0].sel, nb * Hkv * W * sizeof(uint32_t)},
     };
-    size_t need = 0, zero_bytes = 0;
-    for (size_t i = 0; i < sizeof(parts) / sizeof(parts[0]); ++i) {
-        need += round_up(parts[i].bytes, 256);
-        if (i == 0) zero_bytes = need;
-    }
+    size_t need = 0;
+    for (size_t i = 0; i < sizeof(parts) / sizeof(parts[0]); ++i) need += round_up(parts[i].bytes, 256);
     if (need > kNoallocScratchBytes)
         return fail(KVEC_ERR_INVALID_ARG,
                     "this call needs %zu bytes of scratch; kvec_select_layer_noalloc has %zu (use kvec_create / "
@@ -881,9 +899,8 @@ kvec_status kvec_select_layer_noalloc(const kvec_params* params, int batch, cons
         off += round_up(pt.bytes, 256);
     }
     cudaStream_t st = (cudaStream_t)stream;
-    // The array keeps the previous call's contents: the error word must start at zero.
-    e = cudaMemsetAsync(base, 0, zero_bytes, st);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync(scratch)");
+    // The rest of the array keeps the previous call's contents: every part below
+    // the error word is written before it is read within the call.
     LayerIO io{};
     io.q = static_cast<const __nv_bfloat16*>(q_obs);
     io.k = static_cast<const __nv_bfloat16*>(k);
@@ -894,6 +911,30 @@ kvec_status kvec_select_layer_noalloc(const kvec_params* params, int batch, cons
     io.out_k = static_cast<__nv_bfloat16*>(out_k);
     io.out_v = static_cast<__nv_bfloat16*>(out_v);
     return run_layer_sequential(&tmp, G, io, st);
+}
+
+kvec_status kvec_noalloc_sync_status(kvec_stream_t stream) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    void* base = nullptr;
+    {
+        std::lock_guard<std::mutex> lock(g_noalloc_mutex);
+        if (dev >= 0 && dev < kMaxDevices && g_noalloc_dev[dev].ready) base = g_noalloc_dev[dev].base;
+    }
+    if (!base) return KVEC_OK;   // no call has run on this device
+    e = cudaStreamSynchronize((cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+    int err = 0;
+    e = cudaMemcpy(&err, base, sizeof(int), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(e, "reading the scratch error word");
+    if (err) {
+        e = cudaMemset(base, 0, sizeof(int));
+        if (e == cudaSuccess) e = cudaDeviceSynchronize();
+        if (e != cudaSuccess) return cuda_fail(e, "clearing the scratch error word");
+        return device_error_status(err);
+    }
+    return KVEC_OK;
 }
 
 kvec_status kvec_decode_attention(kvec_handle* h, int batch, const void* q, const void* k_cache,
@@ -957,11 +998,12 @@ kvec_status kvec_sync_status(kvec_handle* h) {
     if (e != cudaSuccess) return cuda_fail(e, "reading the device error word");
     if (err) {
         cudaMemset(h->sc.err, 0, sizeof(int));
-        if (err == 2) return fail(KVEC_ERR_INVALID_ARG, "a call would have taken a coverage state past 255 layers (that state was left unchanged)");
-        return fail(KVEC_ERR_DEVICE_TIMEOUT, "a bounded device wait gave up (code %d)", err);
+        return device_error_status(err);
     }
     return KVEC_OK;
 }
+
+void kvec_set_test_fault(int fault) { g_test_fault.store(fault == 1 ? 1 : 0, std::memory_order_relaxed); }
 
 kvec_status kvec_set_profiling(kvec_handle* h, int enable) {
     if (!h) return fail(KVEC_ERR_INVALID_ARG, "handle is NULL");

@@ -180,6 +180,9 @@ cudaError_t launch_finalize(const Geometry& g, const LayerIO& io, const Scratch&
 cudaError_t launch_decode(const DecodeIO& io, cudaStream_t st);
 void launch_gather(const Geometry& g, const LayerIO& io, const Slot& sl, cudaStream_t st);
 
+// Fault injected by kvec_set_test_fault (0: none), read when a kernel is launched.
+int test_fault();
+
 size_t score_smem_bytes(const Geometry& g);
 size_t window_smem_bytes(const Geometry& g);
 cudaError_t configure_score(const Geometry& g);

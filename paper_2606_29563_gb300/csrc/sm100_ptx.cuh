@@ -79,6 +79,22 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64
     }
 }
 
+// As mbar_wait, and also gives up (returns false) once *abort is set, i.e. once
+// another warp of the CTA has given up on a wait of its own.  Only for waits on
+// barriers that no asynchronous copy is about to complete: a wait for a TMA
+// load in flight must end with the load (mbar_wait), never with the abort.
+__device__ __forceinline__ bool mbar_wait_abortable(uint64_t* bar, uint32_t parity, const volatile int* abort,
+                                                    uint64_t limit_ns = 200000000ull) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const long long c0 = clock64();
+    const long long limit = (long long)(limit_ns * 3ull);
+    for (;;) {
+        if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
+        if (*abort) return false;
+        if (clock64() - c0 > limit) return false;
+    }
+}
+
 // ---------------------------------------------------------------- TMA
 
 __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, uint64_t* bar, int c0, int c1,

@@ -45,7 +45,12 @@ struct WinArgs {
     int kst;                        // operand stages
     int nacc;                       // TMEM accumulators (2, or 1 when 2 do not fit)
     uint32_t tmem_cols;
+    int fault;                      // test of the error path (kvec_set_test_fault): the first
+                                    // accumulator is never signalled and its wait gives up early
 };
+
+// Limit of the epilogue's wait for the withheld accumulator under the injected fault.
+constexpr uint64_t kFaultWaitNs = 20000;
 
 struct __align__(8) WinBars {
     uint64_t full[2], empty[2], acc_full[2], acc_empty[2];
@@ -155,7 +160,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
     const Scratch sc = A.sc;
     const Slot sl = A.sl;
     const int* const cu_dev = A.cu;
-    const int kst = A.kst, nacc = A.nacc;
+    const int kst = A.kst, nacc = A.nacc, fault = A.fault;
     const uint32_t tmem_cols = A.tmem_cols;
     const int Npad = A.Npad, R = G.R;
     const size_t sbytes = stage_bytes(Npad);
@@ -221,7 +226,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
             int fills[2] = {0, 0};
             for (int hh = 0; hh < nh && !bars->abort_flag; ++hh) {
                 const int st = hh % kst, u = hh / kst;
-                if (u > 0 && !ptx::mbar_wait(&bars->empty[st], (u - 1) & 1)) {
+                if (u > 0 && !ptx::mbar_wait_abortable(&bars->empty[st], (u - 1) & 1, &bars->abort_flag)) {
                     win_abort(bars, sc.err);
                     break;
                 }
@@ -247,7 +252,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
                 const int st = hh % kst, u = hh / kst;
                 const int b = hh % NB, ub = hh / NB;
                 if (!ptx::mbar_wait(&bars->full[st], u & 1) ||
-                    (ub > 0 && !ptx::mbar_wait(&bars->acc_empty[b], (ub - 1) & 1))) {
+                    (ub > 0 && !ptx::mbar_wait_abortable(&bars->acc_empty[b], (ub - 1) & 1, &bars->abort_flag))) {
                     win_abort(bars, sc.err);
                     break;
                 }
@@ -262,7 +267,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
                     ptx::mma_bf16(d, ad, bd, idesc, kk > 0 ? 1u : 0u);
                 }
                 ptx::mma_commit(&bars->empty[st]);
-                ptx::mma_commit(&bars->acc_full[b]);
+                if (!(fault && hh == 0)) ptx::mma_commit(&bars->acc_full[b]);
             }
             ptx::mma_commit(&bars->mma_done);
         }
@@ -292,7 +297,9 @@ __global__ void __launch_bounds__(kWinThreads, 1)
         for (int hh = 0; hh < nh; ++hh) {
             const int b = hh % NB, ub = hh / NB;
             int got = 1;
-            if (lane == 0) got = !bars->abort_flag && ptx::mbar_wait(&bars->acc_full[b], ub & 1);
+            if (lane == 0)
+                got = !bars->abort_flag &&
+                      ptx::mbar_wait(&bars->acc_full[b], ub & 1, fault && hh == 0 ? kFaultWaitNs : 200000000ull);
             got = __shfl_sync(0xffffffffu, got, 0);
             if (!got) {
                 if (lane == 0) {
@@ -395,6 +402,7 @@ cudaError_t launch_window(const ScorePlan& sp, const Geometry& g, const LayerIO&
     a.Npad = npad_of(g.R);
     a.kst = kst_for(a.Npad, g.O);
     a.nacc = 2 * a.Npad + 32 <= 512 ? 2 : 1;
+    a.fault = test_fault() == 1 ? 1 : 0;
     uint32_t need = a.nacc == 2 ? (uint32_t)(2 * a.Npad + 32) : 512u, cols = 32;
     while (cols < need) cols <<= 1;
     a.tmem_cols = cols;

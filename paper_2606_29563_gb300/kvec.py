@@ -28,7 +28,8 @@ KERNEL_NAMES = ("score", "window", "heads", "select", "gather")
 EXPORTED = ("kvec_create", "kvec_destroy", "kvec_state_bytes", "kvec_reset", "kvec_select_layer",
             "kvec_select_layers", "kvec_debug_scores", "kvec_sync_status", "kvec_set_profiling",
             "kvec_kernel_time", "kvec_status_string", "kvec_last_error", "kvec_select_layer_noalloc",
-            "kvec_select_layer_lse", "kvec_select_layers_lse", "kvec_decode_attention")
+            "kvec_select_layer_lse", "kvec_select_layers_lse", "kvec_decode_attention",
+            "kvec_noalloc_sync_status", "kvec_set_test_fault")
 
 
 class KvecUnavailable(ImportError):
@@ -96,6 +97,8 @@ def load() -> ctypes.CDLL:
             "kvec_select_layer_lse": ([_vp, i, _vp, _vp, _vp, _vp, _vp, _vp, _vp, i, _vp, _vp, _vp, _vp], st),
             "kvec_select_layers_lse": ([_vp, i, i, _vp, _vp, _pp, _pp, _pp, _pp, _vp, i, _pp, _pp, _pp, _vp], st),
             "kvec_decode_attention": ([_vp, i, _vp, _vp, _vp, _vp, i, _vp, _vp], st),
+            "kvec_noalloc_sync_status": ([_vp], st),
+            "kvec_set_test_fault": ([i], None),
         }
         for name, (args, res) in sig.items():
             fn = getattr(lib, name)
@@ -170,6 +173,16 @@ def kvec_select_layer_noalloc(params: kvec_params, batch: int, cu_host_ptr: int,
     """kvec_select_layer without a handle; scratch comes from the library's static device array."""
     _check(load().kvec_select_layer_noalloc(ctypes.byref(params), int(batch), cu_host_ptr, cu_dev_ptr, q_obs, k, v,
                                             state, int(budget), out_idx, out_k, out_v, stream))
+
+
+def kvec_noalloc_sync_status(stream: int = 0) -> None:
+    """Raises KvecError for a device-side error recorded by kvec_select_layer_noalloc calls."""
+    _check(load().kvec_noalloc_sync_status(stream))
+
+
+def kvec_set_test_fault(fault: int) -> None:
+    """Test hook of the error path (1: window kernels give up on a withheld accumulator; 0: off)."""
+    load().kvec_set_test_fault(int(fault))
 
 
 def kvec_decode_attention(handle: int, batch: int, q: int, k_cache: int, v_cache: int, lens: int, cap: int,

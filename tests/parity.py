@@ -1,7 +1,7 @@
 """Teacher-forced parity run of the CUDA path against the oracle (TEST INFRASTRUCTURE ONLY).
 
 For every layer: run the GPU layer, copy the GPU's state from *before* that layer
-into the oracle, run the oracle on the same inputs, and compare (oracle.compare).
+into the oracle, run the oracle on the same inputs, and compare (oracle/compare.py).
 Errors therefore never compound across layers.
 """
 from __future__ import annotations
@@ -53,14 +53,17 @@ def window_lse(wl: synth.Workload, x: Dict[str, torch.Tensor]) -> np.ndarray:
 
 
 def run_parity(wl: synth.Workload, layers: Optional[int] = None, device: str = "cuda", budget: Optional[int] = None,
-               tol: float = compare.TOL, verbose: bool = False, with_lse: bool = False) -> List[str]:
+               tol: float = compare.TOL, verbose: bool = False, with_lse: bool = False,
+               sel: Optional[kvec.KvecSelector] = None) -> List[str]:
     """Returns every mismatch over `layers` layers of `wl` (empty list = parity).
-    with_lse: the GPU layers take the window rows' log-sum-exp (window_lse) as input."""
+    with_lse: the GPU layers take the window rows' log-sum-exp (window_lse) as input.
+    sel: an existing selector made for `wl` (kept open), instead of a new one."""
     layers = layers or wl.layers
     budget = budget or wl.budget
     ML = wl.max_seqlen
-    params = kvec.params_from_workload(wl, max_layers=max(layers, 1))
-    sel = kvec.KvecSelector(params)
+    own = sel is None
+    if own:
+        sel = kvec.KvecSelector(kvec.params_from_workload(wl, max_layers=max(layers, 1)))
     oparams = oracle.OracleParams.from_workload(wl)
     kept_tail = 0 if getattr(wl, "all_positions", 0) else wl.window
     Kp = min(int(math.floor(float(np.float32(wl.beta)) * budget)), budget - kept_tail)
@@ -96,5 +99,6 @@ def run_parity(wl: synth.Workload, layers: Optional[int] = None, device: str = "
         if verbose:
             same = np.mean(g["out_idx"] == r["out_idx"])
             print(f"layer {l}: {len(layer_errs)} mismatches, index agreement {same:.5f}")
-    sel.close()
+    if own:
+        sel.close()
     return errs

@@ -58,23 +58,65 @@ def test_noalloc_matches_handle_entry_point_on_two_calls_in_a_row():
         assert torch.equal(rk, gk)
         assert torch.equal(rv, gv)
     assert torch.equal(st_ref, st)
+    kvec.kvec_noalloc_sync_status(torch.cuda.current_stream().cuda_stream)   # no device-side error
 
 
-def test_noalloc_rejects_calls_beyond_its_scratch():
-    # The buffers below are 16-byte dummies, so the call must be refused before
-    # anything is launched.  The geometry is chosen so that the per-position
-    # score rows alone (seven fp32 / uint32 rows per KV head and position) are far
-    # beyond the 32 MiB array, whatever else the scratch holds.
-    wl = synth.WORKLOADS["llama8b_l32768_b128"]
-    batch, L = 16, 131072
-    params = kvec.params_from_workload(wl, max_batch=batch, max_seqlen=L)
-    lower_bound = batch * params.num_kv_heads * L * 4 * 7
-    assert lower_bound > 8 * 32 * 2**20, "the geometry no longer exceeds the scratch by a safe margin"
-    cu = torch.arange(0, (batch + 1) * L, L, dtype=torch.int32)
-    dummy = torch.zeros(16, dtype=torch.uint8, device="cuda")
-    p = dummy.data_ptr()
+# (A call whose geometry exceeds the scratch array is refused before any CUDA
+# call; tests/test_abi.py checks that without a GPU.)
+
+
+def test_noalloc_reports_the_layer_limit_refusal():
+    """n_t is 8-bit (Section 4.2's counters), so a state may count at most 255
+    layers.  A call on a state that already counts 255 is refused on the device,
+    leaves the state as it was, and kvec_noalloc_sync_status reports it."""
+    wl = synth.small_workload(seqlens=(301,), layers=1)
+    params = kvec.params_from_workload(wl)
+    x = {k: v.cuda() for k, v in synth.make_layer(wl, 0).items()}
+    cu = torch.tensor(wl.cu_seqlens, dtype=torch.int32)
+    stream = torch.cuda.current_stream().cuda_stream
+    st = torch.zeros((1, kvec.kvec_state_bytes(params.max_seqlen)), dtype=torch.uint8, device="cuda")
+    st[0, 0] = 255   # layers_done, little endian
+    before = st.clone()
+    _noalloc_layer(params, cu, x, st, wl.budget)
     with pytest.raises(kvec.KvecError) as e:
-        kvec.kvec_select_layer_noalloc(params, batch, cu.data_ptr(), cu.cuda().data_ptr(), p, p, p, p, wl.budget,
-                                       p, p, p, torch.cuda.current_stream().cuda_stream)
+        kvec.kvec_noalloc_sync_status(stream)
     assert e.value.status == kvec.KVEC_ERR_INVALID_ARG
-    assert "scratch" in str(e.value)
+    assert torch.equal(st, before)
+    kvec.kvec_noalloc_sync_status(stream)   # reported once, then cleared
+    st[0, 0] = 254
+    _noalloc_layer(params, cu, x, st, wl.budget)
+    kvec.kvec_noalloc_sync_status(stream)
+    assert st[0, 0].item() == 255
+
+
+def test_noalloc_reports_a_device_timeout_and_recovers():
+    """A bounded device wait that gives up (forced with the test fault of the
+    window kernel) is reported by kvec_noalloc_sync_status; the next call runs
+    normally and matches the handle entry point."""
+    wl = synth.small_workload(seqlens=(700, 333), layers=1, budget=96, num_ext_heads=1)
+    params = kvec.params_from_workload(wl)
+    x = {k: v.cuda() for k, v in synth.make_layer(wl, 0).items()}
+    cu = torch.tensor(wl.cu_seqlens, dtype=torch.int32)
+    stream = torch.cuda.current_stream().cuda_stream
+    st = torch.zeros((wl.batch, kvec.kvec_state_bytes(params.max_seqlen)), dtype=torch.uint8, device="cuda")
+    try:
+        kvec.kvec_set_test_fault(1)
+        _noalloc_layer(params, cu, x, st, wl.budget)
+        with pytest.raises(kvec.KvecError) as e:
+            kvec.kvec_noalloc_sync_status(stream)
+        assert e.value.status == kvec.KVEC_ERR_DEVICE_TIMEOUT
+    finally:
+        kvec.kvec_set_test_fault(0)
+    st.zero_()
+    got = _noalloc_layer(params, cu, x, st, wl.budget)
+    kvec.kvec_noalloc_sync_status(stream)
+    sel = kvec.KvecSelector(params)
+    st_ref = sel.new_state(wl.batch)
+    ref = sel.select_layer(cu, cu.cuda(), x["q_obs"], x["k"], x["v"], st_ref, wl.budget)
+    torch.cuda.synchronize()
+    for a, b in zip(ref, got):
+        assert torch.equal(a, b)
+    assert torch.equal(st_ref, st)
+    sel.close()
+
+

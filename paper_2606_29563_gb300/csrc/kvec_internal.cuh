@@ -117,6 +117,7 @@ struct ScorePlan {
     alignas(16) unsigned char args[512];
     int grid, threads, mb;   // mb: 128-row M-blocks per KV head
     size_t smem;
+    int num_sms;             // SMs of the device (persistent grids are sized from it)
 };
 cudaError_t plan_score(const Geometry& g, const LayerIO& io, const Scratch& sc, int num_sms, ScorePlan* plan);
 // after_own_launch: the stream's previous kernel is the previous layer's launch

@@ -533,6 +533,7 @@ cudaError_t plan_score(const Geometry& g, const LayerIO& io, const Scratch& sc, 
     plan->threads = kScoreThreads;
     plan->mb = mblocks(g);
     plan->smem = smem_bytes_for(g);
+    plan->num_sms = num_sms;
     return cudaSuccess;
 }
 

@@ -2,24 +2,30 @@
 // the window queries' attention over the candidate tokens, recomputed on the
 // tensor cores with the softmax statistics (m_r, Z_r) of the score kernel.
 //
-// One CTA per (sequence s, 128-token tile of candidates, group of KV heads);
-// the candidates are [0, L - w), or [0, L) when every position competes.
-// For each KV head h of the group the CTA computes S^T = K_tile Q_h^T with
-// tcgen05.mma (M = 128 tokens, N = g*w query rows padded to 16, K = d) into
-// TMEM, so one epilogue thread owns one token and every query row of it:
+// Work unit: (sequence s, 128-token tile of candidates, group of up to 8 KV
+// heads); the candidates are [0, L - w), or [0, L) when every position
+// competes.  An item is one KV head h of a unit: S^T = K_tile Q_h^T on
+// tcgen05.mma (M = 128 tokens, N = g*w query rows padded to 16, K = d) into a
+// TMEM accumulator, so one epilogue thread owns one token and every query row
+// of it:
 //   A[r][t]   = 2^(s_rt * scale * log2(e) - m_r) / Z_r   (softmax over all visible keys)
 //   G_h[q][t] = sum_j A[(q, j)][t]                       (GQA group sum, r = q * g + j)
 //   P_O[h,t]  = (1/O)  sum_{q >= w-O}  G_h[q][t]
 //   P_O'[h,t] = (1/O') sum_{q >= w-O'} G_h[q][t]
 //   I[t]      = (1/O)  sum_{q >= w-O}  max_h G_h[q][t]
-// Warp 0 streams K_h and Q_h with TMA, warp 1 issues the MMAs into one or two
-// TMEM accumulators, warps 2..17 are the epilogue: four warps per TMEM lane
-// quadrant, each taking a quarter of the window rows q (straight-line code per
-// 32-column chunk when the group size g is a compile-time case).  The head
-// maxima of G_h[q][t] stay in shared memory; when the KV heads are split over
-// several CTAs each group writes its maxima to a partial buffer and the heads
-// kernel combines the groups into I.  The raw rows go to the slot arrays;
-// pooling happens in the heads kernel.
+// The grid is persistent: a CTA walks units blockIdx.x, blockIdx.x + gridDim.x,
+// ... and the items of its units in order.  Warp 0 streams K_h and Q_h with
+// TMA into a ring of stages, warp 1 issues the MMAs into A accumulators (4 of
+// N <= 128 columns, or 2 of N <= 256), and the epilogue is A groups of four
+// warps (one per TMEM lane quadrant): group a takes the CTA's items a, a + A,
+// ..., each thread all the query rows of its token, so every group streams
+// through its own accumulator without waiting for the others.  The head maxima
+// of G_h[q][t] meet in shared memory through atomicMax on the float bits
+// (values are >= +0, so the integer order is the float order and the result
+// does not depend on the order of the updates); the last group to finish a
+// unit sums them into I (or, with several head groups per tile, writes them to
+// a partial buffer that the heads kernel combines).  The raw rows go to the
+// slot arrays; pooling happens in the heads kernel.
 #include <cudaTypedefs.h>
 
 #include "kvec_internal.cuh"
@@ -30,11 +36,10 @@ namespace kvec {
 namespace {
 
 constexpr int kWinThreads = 576;                      // warp 0 TMA, warp 1 MMA, warps 2..17 epilogue
-constexpr int kEpiThreads = 512;
-constexpr int kEpiWarps = kEpiThreads / 32;
 constexpr int kMaxSmemWin = 232448;                   // opt-in shared memory per CTA on sm_103
 constexpr int kKTileBytes = kTileT * kHeadDim * 2;    // 32 KB: two 64-column swizzled halves
-constexpr int kRsRows = 288;                          // row-statistics buffer: R <= 256 plus a chunk's overrun
+constexpr int kMaxStages = 3;                         // deepest operand ring
+constexpr int kWinReserveSms = 8;                     // SMs a window launch leaves to the other kernels
 
 struct WinArgs {
     Geometry G;
@@ -43,7 +48,8 @@ struct WinArgs {
     const int* cu;                  // device cu_seqlens
     int Npad;                       // query rows padded to a multiple of 16 (MMA N)
     int kst;                        // operand stages
-    int nacc;                       // TMEM accumulators (2, or 1 when 2 do not fit)
+    int nacc;                       // accumulators = epilogue groups (4, or 2 when N > 128)
+    int units;                      // (sequence, candidate tile, head group) units of the launch
     uint32_t tmem_cols;
     int fault;                      // test of the error path (kvec_set_test_fault): the first
                                     // accumulator is never signalled and its wait gives up early
@@ -53,18 +59,22 @@ struct WinArgs {
 constexpr uint64_t kFaultWaitNs = 20000;
 
 struct __align__(8) WinBars {
-    uint64_t full[2], empty[2], acc_full[2], acc_empty[2];
+    uint64_t full[kMaxStages], empty[kMaxStages], acc_full[4], acc_empty[4];
     uint64_t mma_done;
     uint32_t tmem_base;
     volatile int abort_flag;
-    volatile int epi_fail;     // set by an epilogue warp whose accumulator wait gave up
+    volatile int gok[4];        // per group: the outcome of its last accumulator wait
+    int done[2];                // per unit parity: groups finished with the unit
+    volatile int ready[2];      // per unit parity: the local unit index whose maxima may use the buffer
+    int last[4];                // per group: 1 if it finished a unit last
 };
 
 __host__ __device__ inline size_t stage_bytes(int Npad) { return (size_t)kKTileBytes + 2 * (size_t)Npad * 128; }
 
+// Shared memory: stages | head maxima [2][O][128] | row statistics [4 groups][2][256] | barriers.
 __host__ __device__ inline size_t win_smem_bytes(int Npad, int O, int kst) {
-    return 1024 + (size_t)kst * stage_bytes(Npad) + kWinHeadsPerCta * kRsRows * sizeof(float) +
-           (size_t)O * kTileT * sizeof(float) + kWinHeadsPerCta * 4 * kTileT * sizeof(float2) + sizeof(WinBars);
+    return 1024 + (size_t)kst * stage_bytes(Npad) + 2 * (size_t)O * kTileT * sizeof(float) +
+           4 * 2 * 256 * sizeof(float) + sizeof(WinBars);
 }
 
 __device__ __forceinline__ void win_abort(WinBars* bars, int* err) {
@@ -72,28 +82,54 @@ __device__ __forceinline__ void win_abort(WinBars* bars, int* err) {
     atomicExch(err, 3);
 }
 
-// One head's window rows [q_lo, q_hi) of this thread's token: adds the rows'
-// group sums G_h[q] to po (q >= w-O) and poe (q >= w-O') and folds them into
-// the head maxima.  Rows q < qmin come before the token (it lies in the window
-// part, which only later rows see): their attention to it is 0.  GG > 0 is the
-// group size g known at compile time: each 32-column chunk holds 32 / GG whole
+// Unit u -> sequence s, candidate tile jt within it, head group ng, global
+// candidate tile tg; sequence s owns ceil(Lc / 128) * NG consecutive units.
+struct WinUnit {
+    int s, jt, ng, tg, L, Lc, row0;
+};
+
+__device__ __forceinline__ bool decode_unit(const Geometry& G, const int* cu, int u, WinUnit& w) {
+    int base = 0, tbase = 0;
+    for (int b = 0; b < G.batch; ++b) {
+        const int c0 = __ldg(&cu[b]), c1 = __ldg(&cu[b + 1]);
+        const int Lc = c1 - c0 - G.wk;
+        const int nt = Lc > 0 ? (Lc + kTileT - 1) / kTileT : 0;
+        if (u < base + nt * G.NG) {
+            const int local = u - base;
+            w.s = b;
+            w.jt = local / G.NG;
+            w.ng = local - w.jt * G.NG;
+            w.tg = tbase + w.jt;
+            w.L = c1 - c0;
+            w.Lc = Lc;
+            w.row0 = c0 + w.jt * kTileT;
+            return true;
+        }
+        base += nt * G.NG;
+        tbase += nt;
+    }
+    return false;
+}
+
+// One head of this thread's token: the group sums G_h[q] of every window row q,
+// added to po (q >= w-O) and poe (q >= w-O') and folded into the head maxima
+// (q >= w-O).  Rows q < qmin come before the token (it lies in the window part,
+// which only later rows see): their attention to it is 0.  GG > 0 is the group
+// size g known at compile time: each 32-column chunk holds 32 / GG whole
 // groups and runs as straight-line code.
 template <int GG>
-__device__ __forceinline__ void head_rows(uint32_t taddr, const float* __restrict__ rsb, int g, int q_lo, int q_hi,
-                                          int qmin, float sl2, int qO, int qOe, float* maxg_col, bool first,
-                                          float& po, float& poe) {
+__device__ __forceinline__ void head_rows(uint32_t taddr, const float* __restrict__ rsb, int g, int w, int qmin,
+                                          float sl2, int qO, int qOe, int* maxg_col, float& po, float& poe) {
     if constexpr (GG > 0) {
         constexpr int QPC = 32 / GG, CW = QPC * GG;
-        for (int qb = q_lo; qb < q_hi; qb += QPC) {
+        for (int qb = 0; qb < w; qb += QPC) {
             const int c0 = qb * GG;
             float v[32];
             ptx::tmem_ld32(taddr + (uint32_t)c0, v);
             ptx::tmem_wait_ld();
             float pr[CW];
 #pragma unroll
-            for (int i = 0; i < CW; ++i) {
-                pr[i] = ptx::ex2(fmaf(v[i], sl2, -rsb[c0 + i]));
-            }
+            for (int i = 0; i < CW; ++i) pr[i] = ptx::ex2(fmaf(v[i], sl2, -rsb[c0 + i]));
 #pragma unroll
             for (int k = 0; k < QPC; ++k) {
                 float gs = 0.f;
@@ -101,21 +137,20 @@ __device__ __forceinline__ void head_rows(uint32_t taddr, const float* __restric
                 for (int j = 0; j < GG; ++j) gs += pr[k * GG + j];
                 const int q = qb + k;
                 gs = q >= qmin ? gs : 0.f;
-                if (q < q_hi) {
+                if (q < w) {
                     if (q >= qOe) poe += gs;
                     if (q >= qO) {
                         po += gs;
-                        float* mg = maxg_col + (q - qO) * kTileT;
-                        *mg = first ? gs : fmaxf(*mg, gs);
+                        atomicMax(maxg_col + (q - qO) * kTileT, __float_as_int(gs));
                     }
                 }
             }
         }
     } else {
         float gs = 0.f;
-        int q = q_lo, jq = 0;
-        const int c_end = q_hi * g;
-        for (int c0 = q_lo * g; c0 < c_end; c0 += 32) {
+        int q = 0, jq = 0;
+        const int c_end = w * g;
+        for (int c0 = 0; c0 < c_end; c0 += 32) {
             float v[32];
             ptx::tmem_ld32(taddr + (uint32_t)c0, v);
             ptx::tmem_wait_ld();
@@ -129,8 +164,7 @@ __device__ __forceinline__ void head_rows(uint32_t taddr, const float* __restric
                     if (q >= qOe) poe += gs;
                     if (q >= qO) {
                         po += gs;
-                        float* mg = maxg_col + (q - qO) * kTileT;
-                        *mg = first ? gs : fmaxf(*mg, gs);
+                        atomicMax(maxg_col + (q - qO) * kTileT, __float_as_int(gs));
                     }
                     gs = 0.f;
                     jq = 0;
@@ -160,55 +194,34 @@ __global__ void __launch_bounds__(kWinThreads, 1)
     const Scratch sc = A.sc;
     const Slot sl = A.sl;
     const int* const cu_dev = A.cu;
-    const int kst = A.kst, nacc = A.nacc, fault = A.fault;
+    const int kst = A.kst, NA = A.nacc, units = A.units, fault = A.fault;
     const uint32_t tmem_cols = A.tmem_cols;
     const int Npad = A.Npad, R = G.R;
     const size_t sbytes = stage_bytes(Npad);
-    float* rs = reinterpret_cast<float*>(smem + kst * sbytes);        // [HG][kRsRows] m_r + log2 Z_r
-    float* maxg = reinterpret_cast<float*>(rs + kWinHeadsPerCta * kRsRows);   // [O][128] max over heads of G_h[q][t]
-    float2* xfer = reinterpret_cast<float2*>(maxg + G.O * kTileT);      // [HG][4][128] quarters' (P_O, P_O') sums
-    WinBars* bars = reinterpret_cast<WinBars*>(xfer + kWinHeadsPerCta * 4 * kTileT);
+    int* maxg = reinterpret_cast<int*>(smem + kst * sbytes);             // [2][O][128] float bits
+    float* rsm = reinterpret_cast<float*>(maxg + 2 * G.O * kTileT);      // [4][2][256] m_r + log2 Z_r
+    WinBars* bars = reinterpret_cast<WinBars*>(rsm + 4 * 2 * 256);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-
-    // Work item -> (sequence, candidate tile, head group); sequence s owns
-    // ceil(Lc / 128) * NG consecutive CTAs.
-    auto cu = [&](int b) { return __ldg(&cu_dev[b]); };
-    int s = -1, jt = 0, ng = 0, tg = 0;
-    {
-        int base = 0, tbase = 0;
-        for (int b = 0; b < G.batch; ++b) {
-            const int Lc = cu(b + 1) - cu(b) - G.wk;
-            const int nt = Lc > 0 ? (Lc + kTileT - 1) / kTileT : 0;
-            if ((int)blockIdx.x < base + nt * G.NG) {
-                const int local = (int)blockIdx.x - base;
-                s = b;
-                jt = local / G.NG;
-                ng = local - jt * G.NG;
-                tg = tbase + jt;
-                break;
-            }
-            base += nt * G.NG;
-            tbase += nt;
-        }
-    }
-    if (s < 0) return;   // the whole CTA, before any barrier or TMEM use
-    const int L = cu(s + 1) - cu(s), Lc = L - G.wk;
-    const int h0 = ng * G.HG;
-    const int nh = min(G.HG, G.Hkv - h0);
-    const int NB = nacc;
+    const int u0 = blockIdx.x, ustep = gridDim.x;
 
     if (threadIdx.x == 32) {
-        for (int i = 0; i < 2; ++i) {
+        for (int i = 0; i < kst; ++i) {
             ptx::mbar_init(&bars->full[i], 1);
             ptx::mbar_init(&bars->empty[i], 1);
+        }
+        for (int i = 0; i < 4; ++i) {
             ptx::mbar_init(&bars->acc_full[i], 1);
-            ptx::mbar_init(&bars->acc_empty[i], kEpiThreads / 32);   // one arrival per epilogue warp
+            ptx::mbar_init(&bars->acc_empty[i], 4);   // one arrival per warp of the group
         }
         ptx::mbar_init(&bars->mma_done, 1);
         bars->abort_flag = 0;
-        bars->epi_fail = 0;
+        for (int i = 0; i < 2; ++i) {
+            bars->done[i] = 0;
+            bars->ready[i] = i;
+        }
         ptx::fence_barrier_init();
     }
+    for (int i = threadIdx.x; i < 2 * G.O * kTileT; i += blockDim.x) maxg[i] = 0;
     if (warp == 1) {
         ptx::tmem_alloc(&bars->tmem_base, tmem_cols);
         ptx::tmem_relinquish();
@@ -222,23 +235,31 @@ __global__ void __launch_bounds__(kWinThreads, 1)
         // ------------------------------------------------------------ TMA producer
         if (lane == 0) {
             const uint64_t policy = ptx::policy_evict_first();   // the K tiles' last use
-            const int row0 = cu(s) + jt * kTileT;
-            int fills[2] = {0, 0};
-            for (int hh = 0; hh < nh && !bars->abort_flag; ++hh) {
-                const int st = hh % kst, u = hh / kst;
-                if (u > 0 && !ptx::mbar_wait_abortable(&bars->empty[st], (u - 1) & 1, &bars->abort_flag)) {
-                    win_abort(bars, sc.err);
-                    break;
+            int it = 0;
+            int fills[kMaxStages] = {0, 0, 0};
+            for (int u = u0; u < units && !bars->abort_flag; u += ustep) {
+                WinUnit wu;
+                decode_unit(G, cu_dev, u, wu);
+                const int h0 = wu.ng * G.HG, nh = min(G.HG, G.Hkv - h0);
+                bool stop = false;
+                for (int hh = 0; hh < nh; ++hh, ++it) {
+                    const int st = it % kst, n = it / kst;
+                    if (n > 0 && !ptx::mbar_wait_abortable(&bars->empty[st], (n - 1) & 1, &bars->abort_flag)) {
+                        win_abort(bars, sc.err);
+                        stop = true;
+                        break;
+                    }
+                    uint8_t* sk = smem + st * sbytes;
+                    uint8_t* sq = sk + kKTileBytes;
+                    const int h = h0 + hh;
+                    ptx::mbar_arrive_expect_tx(&bars->full[st], (uint32_t)kKTileBytes + 2u * (uint32_t)R * 128u);
+                    ptx::tma_load_3d(sk, &kmap, &bars->full[st], 0, h, wu.row0, policy);
+                    ptx::tma_load_3d(sk + kKTileBytes / 2, &kmap, &bars->full[st], 64, h, wu.row0, policy);
+                    ptx::tma_load_4d(sq, &qmap, &bars->full[st], 0, h * G.g, 0, wu.s);
+                    ptx::tma_load_4d(sq + Npad * 128, &qmap, &bars->full[st], 64, h * G.g, 0, wu.s);
+                    ++fills[st];
                 }
-                uint8_t* sk = smem + st * sbytes;
-                uint8_t* sq = sk + kKTileBytes;
-                const int h = h0 + hh;
-                ptx::mbar_arrive_expect_tx(&bars->full[st], (uint32_t)kKTileBytes + 2u * (uint32_t)R * 128u);
-                ptx::tma_load_3d(sk, &kmap, &bars->full[st], 0, h, row0, policy);
-                ptx::tma_load_3d(sk + kKTileBytes / 2, &kmap, &bars->full[st], 64, h, row0, policy);
-                ptx::tma_load_4d(sq, &qmap, &bars->full[st], 0, h * G.g, 0, s);
-                ptx::tma_load_4d(sq + Npad * 128, &qmap, &bars->full[st], 64, h * G.g, 0, s);
-                ++fills[st];
+                if (stop) break;
             }
             // Drain: every issued copy lands before the CTA may exit.
             for (int st = 0; st < kst; ++st)
@@ -248,111 +269,157 @@ __global__ void __launch_bounds__(kWinThreads, 1)
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
             const uint32_t idesc = ptx::idesc_bf16_f32(128, Npad);
-            for (int hh = 0; hh < nh && !bars->abort_flag; ++hh) {
-                const int st = hh % kst, u = hh / kst;
-                const int b = hh % NB, ub = hh / NB;
-                if (!ptx::mbar_wait(&bars->full[st], u & 1) ||
-                    (ub > 0 && !ptx::mbar_wait_abortable(&bars->acc_empty[b], (ub - 1) & 1, &bars->abort_flag))) {
-                    win_abort(bars, sc.err);
-                    break;
-                }
-                ptx::tc_fence_after();
-                const uint32_t sk = ptx::smem_u32(smem + st * sbytes), sq = sk + kKTileBytes;
-                const uint32_t d = tmem + (uint32_t)(b * Npad);
+            int it = 0;
+            bool stop = false;
+            for (int u = u0; u < units && !stop; u += ustep) {
+                WinUnit wu;
+                decode_unit(G, cu_dev, u, wu);
+                const int nh = min(G.HG, G.Hkv - wu.ng * G.HG);
+                for (int hh = 0; hh < nh; ++hh, ++it) {
+                    const int st = it % kst, n = it / kst;
+                    const int b = it % NA, ub = it / NA;
+                    // Giving up on a stage in flight is safe: the producer drains its own loads.
+                    if (bars->abort_flag || !ptx::mbar_wait_abortable(&bars->full[st], n & 1, &bars->abort_flag) ||
+                        (ub > 0 && !ptx::mbar_wait_abortable(&bars->acc_empty[b], (ub - 1) & 1, &bars->abort_flag))) {
+                        win_abort(bars, sc.err);
+                        stop = true;
+                        break;
+                    }
+                    ptx::tc_fence_after();
+                    const uint32_t sk = ptx::smem_u32(smem + st * sbytes), sq = sk + kKTileBytes;
+                    const uint32_t d = tmem + (uint32_t)(b * Npad);
 #pragma unroll
-                for (int kk = 0; kk < 8; ++kk) {
-                    const int half = kk >> 2, kin = kk & 3;
-                    const uint64_t ad = ptx::smem_desc_k_sw128(sk + half * (kKTileBytes / 2) + kin * 32);
-                    const uint64_t bd = ptx::smem_desc_k_sw128(sq + half * Npad * 128 + kin * 32);
-                    ptx::mma_bf16(d, ad, bd, idesc, kk > 0 ? 1u : 0u);
+                    for (int kk = 0; kk < 8; ++kk) {
+                        const int half = kk >> 2, kin = kk & 3;
+                        const uint64_t ad = ptx::smem_desc_k_sw128(sk + half * (kKTileBytes / 2) + kin * 32);
+                        const uint64_t bd = ptx::smem_desc_k_sw128(sq + half * Npad * 128 + kin * 32);
+                        ptx::mma_bf16(d, ad, bd, idesc, kk > 0 ? 1u : 0u);
+                    }
+                    ptx::mma_commit(&bars->empty[st]);
+                    if (!(fault && it == 0)) ptx::mma_commit(&bars->acc_full[b]);
                 }
-                ptx::mma_commit(&bars->empty[st]);
-                if (!(fault && hh == 0)) ptx::mma_commit(&bars->acc_full[b]);
             }
             ptx::mma_commit(&bars->mma_done);
         }
-    } else {
+    } else if (warp < 2 + 4 * NA) {
         // ------------------------------------------------------------ epilogue
-        const int e = threadIdx.x - 64;                   // 0 .. kEpiThreads - 1
-        const int qt = (warp - 2) >> 2;                   // quarter of the window rows
+        const int grp = (warp - 2) >> 2;                  // accumulator / item group
+        const int gtid = threadIdx.x - 64 - grp * 128;    // 0 .. 127 within the group
         const int quad = warp & 3;                        // TMEM lanes 32*quad .. +31
-        const int tokl = quad * 32 + lane;
-        const int t = jt * kTileT + tokl;
-        const int qmin = t - (L - G.w);   // > 0 only for tokens in the window part
-        const int q_lo = (qt * G.w) >> 2, q_hi = ((qt + 1) * G.w) >> 2;
+        const int tok = quad * 32 + lane;                 // token within the tile
+        const int bar_id = 1 + grp;                       // named barrier of the group (128 threads)
         const int qO = G.w - G.O, qOe = G.w - G.Oe;
         const float invO = 1.f / (float)G.O, invOe = 1.f / (float)G.Oe;
-        // Row statistics of every head of the group: A = 2^(s * sl2 - (m_r + log2 Z_r)).
-        // They come from the launch this grid is a programmatic dependent of: wait
-        // for it here, after the set-up and the first operand loads.
+        const uint32_t tbase = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(grp * Npad);
+        float* rs_g = rsm + grp * 2 * 256;
+        // Row statistics come from the launch this grid is a programmatic
+        // dependent of: wait for it before the first read.
         asm volatile("griddepcontrol.wait;\n" ::: "memory");
-        for (int i = e; i < nh * R; i += kEpiThreads) {
-            const int hh = i / R, r = i - hh * R;
-            const float2 ms = __ldcg(&sc.rowstat[((size_t)s * G.Hkv + h0 + hh) * R + r]);
-            rs[hh * kRsRows + r] = ms.x + __log2f(ms.y);
-        }
-        ptx::named_bar_sync(1, kEpiThreads);
-        // The warps run through the heads independently: each waits for the
-        // accumulator itself and leaves its partial sums in xfer.
-        for (int hh = 0; hh < nh; ++hh) {
-            const int b = hh % NB, ub = hh / NB;
-            int got = 1;
-            if (lane == 0)
-                got = !bars->abort_flag &&
-                      ptx::mbar_wait(&bars->acc_full[b], ub & 1, fault && hh == 0 ? kFaultWaitNs : 200000000ull);
-            got = __shfl_sync(0xffffffffu, got, 0);
-            if (!got) {
+        // This thread's rows (gtid, gtid + 128) of an item's statistics.
+        auto fetch = [&](int s, int h, float& a, float& b) {
+            const float2* src = sc.rowstat + ((size_t)s * G.Hkv + h) * R;
+            a = b = 0.f;
+            if (gtid < R) {
+                const float2 m = __ldcg(src + gtid);
+                a = m.x + __log2f(m.y);
+            }
+            if (gtid + 128 < R) {
+                const float2 m = __ldcg(src + gtid + 128);
+                b = m.x + __log2f(m.y);
+            }
+        };
+        int it = 0, k = 0;   // it: CTA item index; k: this group's items so far
+        bool failed = false;
+        for (int u = u0, ul = 0; u < units; u += ustep, ++ul) {
+            WinUnit wu;
+            decode_unit(G, cu_dev, u, wu);
+            const int h0 = wu.ng * G.HG, nh = min(G.HG, G.Hkv - h0);
+            const int t = wu.jt * kTileT + tok;                  // token within the sequence
+            const int qmin = t - (wu.L - G.w);                   // > 0 only for tokens in the window part
+            const int buf = ul & 1;
+            int* mg = maxg + buf * G.O * kTileT;
+            // The head maxima buffer of this unit parity is free once the unit two
+            // before has been folded into I (bounded wait on a flag of this CTA).
+            if (!failed && ul >= 2) {
+                int ok = 1;
                 if (lane == 0) {
-                    bars->epi_fail = 1;
-                    win_abort(bars, sc.err);
-                }
-                break;
-            }
-            ptx::tc_fence_after();
-            const uint32_t taddr = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(b * Npad);
-            float po = 0.f, poe = 0.f;
-            head_rows<GG>(taddr, rs + hh * kRsRows, G.g, q_lo, q_hi, qmin, G.sl2, qO, qOe, maxg + tokl, hh == 0, po,
-                          poe);
-            ptx::tc_fence_before();
-            __syncwarp();
-            if (lane == 0) ptx::mbar_arrive(&bars->acc_empty[b]);
-            xfer[(hh * 4 + qt) * kTileT + tokl] = make_float2(po, poe);
-        }
-        // Every epilogue warp arrives here, failed or not; epi_fail is only written
-        // before this barrier, so the branch below is uniform.
-        ptx::named_bar_sync(1, kEpiThreads);
-        const bool aborted = bars->epi_fail != 0;
-        if (!aborted) {
-            // P_O and P_O' of every head of the group: the four quarters' sums.
-            for (int i = e; i < nh * kTileT; i += kEpiThreads) {
-                const int hh = i >> 7, tk = i & (kTileT - 1);
-                const int tt = jt * kTileT + tk;
-                if (tt < Lc) {
-                    float so = 0.f, soe = 0.f;
-#pragma unroll
-                    for (int k = 0; k < 4; ++k) {
-                        const float2 x = xfer[(hh * 4 + k) * kTileT + tk];
-                        so += x.x;
-                        soe += x.y;
+                    const long long c0 = clock64();
+                    while (bars->ready[buf] != ul) {
+                        if (bars->abort_flag || clock64() - c0 > 600000000ll) {
+                            ok = 0;
+                            break;
+                        }
+                        __nanosleep(64);
                     }
-                    const size_t row = (size_t)s * G.Hkv + h0 + hh;
-                    sl.rawO[row * G.ML + tt] = so * invO;
-                    sl.rawOe[row * G.ML + tt] = soe * invOe;
+                }
+                if (!__shfl_sync(0xffffffffu, ok, 0)) {
+                    if (lane == 0) win_abort(bars, sc.err);
+                    failed = true;
+                }
+                __threadfence_block();
+            }
+            float pa = 0.f, pb = 0.f;
+            int hh = (grp - it % NA + NA) % NA;   // the unit's first item for this group
+            if (!failed && hh < nh) fetch(wu.s, h0 + hh, pa, pb);
+            for (; hh < nh && !failed; hh += NA, ++k) {
+                // gtid 0 waits for the accumulator and publishes the outcome to the
+                // group with the statistics (one barrier per item).
+                if (gtid == 0) {
+                    const bool ok = !bars->abort_flag &&
+                                    ptx::mbar_wait_abortable(&bars->acc_full[grp], k & 1, &bars->abort_flag,
+                                                             fault && it + hh == 0 ? kFaultWaitNs : 200000000ull);
+                    if (!ok) win_abort(bars, sc.err);
+                    bars->gok[grp] = ok ? 1 : 0;
+                }
+                float* rsb = rs_g + (k & 1) * 256;
+                rsb[gtid] = pa;
+                rsb[gtid + 128] = pb;
+                ptx::named_bar_sync(bar_id, 128);
+                if (!bars->gok[grp]) {
+                    failed = true;
+                    break;
+                }
+                if (hh + NA < nh) fetch(wu.s, h0 + hh + NA, pa, pb);   // next item's rows, in flight
+                ptx::tc_fence_after();
+                float po = 0.f, poe = 0.f;
+                head_rows<GG>(tbase, rsb, G.g, G.w, qmin, G.sl2, qO, qOe, mg + tok, po, poe);
+                ptx::tc_fence_before();
+                __syncwarp();
+                if (lane == 0) ptx::mbar_arrive(&bars->acc_empty[grp]);
+                if (t < wu.Lc) {
+                    const size_t row = (size_t)wu.s * G.Hkv + h0 + hh;
+                    sl.rawO[row * G.ML + t] = po * invO;
+                    sl.rawOe[row * G.ML + t] = poe * invOe;
                 }
             }
-        }
-        if (!aborted) {
-            // I[t] = (1/O) sum over q >= w - O of the maxima over every KV head.  With
-            // the heads in one CTA it is complete here; otherwise each group leaves its
-            // maxima and the heads kernel takes the maximum over the groups.
-            const int n_el = G.O * kTileT;
-            if (G.NG > 1) {
-                float* wp = sl.wpart + ((size_t)tg * G.NG + ng) * n_el;
-                for (int i = e; i < n_el; i += kEpiThreads) wp[i] = maxg[i];
-            } else if (e < kTileT && jt * kTileT + e < Lc) {
-                float ip = 0.f;
-                for (int qi = 0; qi < G.O; ++qi) ip += maxg[qi * kTileT + e];
-                sl.rawI[(size_t)s * G.ML + jt * kTileT + e] = ip * invO;
+            it += nh;
+            if (failed) break;
+            // This group is done with the unit: the last of the NA groups folds the
+            // head maxima into I and frees the buffer for the unit two ahead.
+            ptx::named_bar_sync(bar_id, 128);
+            if (gtid == 0) {
+                __threadfence_block();
+                bars->last[grp] = atomicAdd(&bars->done[buf], 1) == NA - 1;
+                __threadfence_block();
+            }
+            ptx::named_bar_sync(bar_id, 128);
+            if (bars->last[grp]) {
+                __threadfence_block();
+                if (G.NG > 1) {
+                    float* wp = sl.wpart + ((size_t)wu.tg * G.NG + wu.ng) * G.O * kTileT;
+                    for (int q = 0; q < G.O; ++q) wp[q * kTileT + tok] = __int_as_float(mg[q * kTileT + tok]);
+                } else if (t < wu.Lc) {
+                    float ip = 0.f;
+                    for (int q = 0; q < G.O; ++q) ip += __int_as_float(mg[q * kTileT + tok]);
+                    sl.rawI[(size_t)wu.s * G.ML + t] = ip * invO;
+                }
+                for (int q = 0; q < G.O; ++q) mg[q * kTileT + tok] = 0;
+                ptx::named_bar_sync(bar_id, 128);
+                if (gtid == 0) {
+                    bars->done[buf] = 0;
+                    __threadfence_block();
+                    bars->ready[buf] = ul + 2;
+                }
             }
         }
     }
@@ -367,7 +434,14 @@ __global__ void __launch_bounds__(kWinThreads, 1)
 
 int npad_of(int R) { return (R + 15) & ~15; }
 
-int kst_for(int Npad, int O) { return win_smem_bytes(Npad, O, 2) <= (size_t)kMaxSmemWin ? 2 : 1; }
+int kst_for(int Npad, int O) {
+    int k = kMaxStages;
+    while (k > 1 && win_smem_bytes(Npad, O, k) > (size_t)kMaxSmemWin) --k;
+    return k;
+}
+
+// Units of a launch: (sequence, candidate tile, head group).
+int units_of(const Geometry& g) { return g.win_tiles * g.NG; }
 
 }  // namespace
 
@@ -377,17 +451,13 @@ size_t window_smem_bytes(const Geometry& g) {
 }
 
 cudaError_t configure_window(const Geometry& g) {
-    // Per-function attribute shared by every handle: the largest supported geometry.
-    size_t need = 0;
-    for (int R = 16; R <= 256; R += 16) {
-        const size_t b = win_smem_bytes(R, kMaxObsWindow, kst_for(R, kMaxObsWindow));
-        if (b > need) need = b;
-    }
+    // Per-function attribute shared by every handle: the opt-in maximum (every
+    // geometry's stage count is chosen to fit it).
     (void)g;
     cudaError_t e = cudaSuccess;
     for (auto fn : {window_kernel<0>, window_kernel<1>, window_kernel<2>, window_kernel<4>, window_kernel<7>,
                     window_kernel<8>})
-        if (e == cudaSuccess) e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)need);
+        if (e == cudaSuccess) e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmemWin);
     return e;
 }
 
@@ -401,13 +471,15 @@ cudaError_t launch_window(const ScorePlan& sp, const Geometry& g, const LayerIO&
     a.cu = io.cu;
     a.Npad = npad_of(g.R);
     a.kst = kst_for(a.Npad, g.O);
-    a.nacc = 2 * a.Npad + 32 <= 512 ? 2 : 1;
+    a.nacc = a.Npad <= 128 ? 4 : 2;   // nacc * Npad <= 512 TMEM columns
+    a.units = units_of(g);
     a.fault = test_fault() == 1 ? 1 : 0;
-    uint32_t need = a.nacc == 2 ? (uint32_t)(2 * a.Npad + 32) : 512u, cols = 32;
-    while (cols < need) cols <<= 1;
-    a.tmem_cols = cols;
+    a.tmem_cols = 512;   // one CTA per SM; a 32-column load past the last group's columns stays inside
     const size_t smem = win_smem_bytes(a.Npad, g.O, a.kst);
-    const int grid = g.win_tiles * g.NG;
+    // Persistent: at most one CTA per SM, leaving a few SMs to the selection
+    // chain and the other layers' kernels.
+    const int usable = sp.num_sms > 2 * kWinReserveSms ? sp.num_sms - kWinReserveSms : sp.num_sms;
+    const int grid = a.units < usable ? a.units : usable;
     // after_own_launch: the previous kernel on the stream is this layer's
     // row-statistics launch and no event wait stands between them; the launch is
     // then its programmatic dependent and waits (griddepcontrol.wait) right

@@ -9,11 +9,12 @@
 //               a ring of 128-token K tiles, both 128-byte swizzled;
 //   warp 1      one thread issues tcgen05.mma (M = 128 query rows per M-block,
 //               N = 128 tokens, K = 128 = d) into TMEM accumulators;
-//   warps 2..17 epilogue, one thread per (query row, column split of the
-//               tile): tcgen05.ld of its logits, their max and sum of
-//               2^(s - max), merged online into the thread's running
+//   warps 2..17 epilogue: groups of warps, one per TMEM accumulator, each
+//               taking every NB-th item; one thread per query row and all
+//               128 columns of the item: tcgen05.ld of its logits, their sum
+//               of 2^(s - max), merged online into the thread's running
 //               (max, sum) of the CTA's contiguous segment of (s, h).
-// At the end of a segment the column splits merge in shared memory and the CTA
+// At the end of a segment the groups merge in shared memory and the CTA
 // writes one (max, sum) partial per row, keyed by the segment's first item;
 // rowstat_kernel then merges the partials of a (s, h) into (m_r, Z_r).
 // The window kernel recomputes the logits with these statistics.
@@ -101,7 +102,7 @@ struct __align__(8) Barriers {
     uint64_t mma_done;
     uint32_t tmem_base;
     volatile int abort_flag;
-    float2 xf[512];            // a segment's (max, sum) per column split and row, merged at its end
+    float2 xf[512];            // a segment's (max, sum) per epilogue group and row, merged at its end
 };
 
 __device__ __forceinline__ void raise_abort(Barriers* bars, int* err) {
@@ -109,8 +110,8 @@ __device__ __forceinline__ void raise_abort(Barriers* bars, int* err) {
     atomicExch(err, 3);
 }
 
-// MB: 128-row M-blocks per KV head (R <= 128 * MB).  The 16 epilogue warps cover
-// 4 lane quarters x MB M-blocks x CS = 4 / MB column splits of COLS = 32 * MB.
+// MB: 128-row M-blocks per KV head (R <= 128 * MB).  The 16 epilogue warps form
+// NB = 4 / MB groups of 4 * MB warps, one group per TMEM accumulator.
 template <int MB>
 __global__ void __launch_bounds__(kScoreThreads, 1)
     score_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap qmap,
@@ -124,7 +125,6 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     const Scratch sc = A.sc;
     const int W = A.W, kst = A.kst;
     const int* const cu_dev = A.cu;
-    constexpr int CS = 4 / MB, COLS = 32 * MB;
     const int Rpad = 128 * MB, R = G.R;
     uint8_t* sQ = smem;                                   // 2 halves x Rpad rows x 128 B
     uint8_t* sK = sQ + 2 * Rpad * 128;                    // kst x 32 KB
@@ -151,7 +151,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         ptx::mbar_init(&bars->q_empty, 1);
         for (int b = 0; b < 4; ++b) {
             ptx::mbar_init(&bars->acc_full[b], 1);
-            ptx::mbar_init(&bars->acc_empty[b], kEpiWarps);  // one arrival per epilogue warp
+            ptx::mbar_init(&bars->acc_empty[b], 4 * MB);  // one arrival per warp of the group
         }
         ptx::mbar_init(&bars->mma_done, 1);
         bars->abort_flag = 0;
@@ -251,13 +251,16 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         }
     } else {
         // ------------------------------------------------------------ epilogue
-        // Warp ew = warp - 2 reads TMEM lanes 32*(warp % 4) .. +31 (the lane
-        // quarter its warp id allows) of M-block m, columns [COLS*split, +COLS).
-        // Each warp waits for the accumulators itself; the warps meet only when a
-        // segment ends.
+        // NB groups of GW = 4 * MB warps; group a takes the CTA's items a, a + NB,
+        // ... from its own accumulator, so the groups work on different items at
+        // once (one group's TMEM loads and barrier waits overlap the others' ex2).
+        // Warp k of a group reads TMEM lanes 32*(warp % 4) .. +31 (the lane
+        // quadrant its warp id allows) of M-block k / 4: one thread per query row,
+        // all 128 columns of the item.
+        constexpr int GW = 4 * MB;
         const int ew = warp - 2;
-        const int m = (ew >> 2) % MB;
-        const int split = (ew >> 2) / MB;
+        const int grp = ew / GW;
+        const int m = (ew % GW) >> 2;
         const int quad = warp & 3;
         const int row = m * 128 + quad * 32 + lane;
         const bool vrow = row < R;
@@ -276,19 +279,53 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
             }
         };
         // Every epilogue thread calls this at the same segment boundaries (aborted
-        // warps included), so the named barriers always complete.  The column
-        // splits merge here; rowstat_kernel merges the CTAs' partials of a
+        // warps included), so the named barriers always complete.  The groups'
+        // partials merge here; rowstat_kernel merges the CTAs' partials of a
         // (sequence, head) into (m_r, Z_r).
         auto flush_segment = [&]() {
-            bars->xf[split * Rpad + row] = make_float2(seg_m, seg_z);
+            bars->xf[grp * Rpad + row] = make_float2(seg_m, seg_z);
             ptx::named_bar_sync(1, kEpiThreads);
-            if (split == 0) {
+            if (grp == 0) {
                 float M = seg_m, Z = seg_z;
 #pragma unroll
-                for (int c = 1; c < CS; ++c) merge(M, Z, bars->xf[c * Rpad + row]);
+                for (int c = 1; c < NB; ++c) merge(M, Z, bars->xf[c * Rpad + row]);
                 if (vrow) sc.segpart[(size_t)seg_first * R + row] = make_float2(M, Z);
             }
             ptx::named_bar_sync(1, kEpiThreads);   // xf is free for the next segment
+        };
+        // 32 columns of the row, `lim` of them visible (<= 0: none).  Relative to
+        // the segment's running reference seg_m, 2^(s - seg_m) sums the same mass
+        // as an online max/rescale without a max pass; a chunk far above the
+        // reference (sum not below 2^64) and the segment's first chunk take the
+        // exact path.
+        auto chunk = [&](const float* v, int lim) {
+            if (lim <= 0) return;
+            if (lim >= 32 && seg_m != -INFINITY) {
+                float z4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+                for (int c = 0; c < 32; ++c) z4[c & 3] += ptx::ex2(fmaf(v[c], G.sl2, -seg_m));
+                const float z = (z4[0] + z4[1]) + (z4[2] + z4[3]);
+                if (z < 0x1p64f) {
+                    seg_z += z;
+                    if (seg_z >= 0x1p40f) {
+                        // Keep the sum bounded: move a power of two into the reference.
+                        const int k = ilogbf(seg_z);
+                        seg_m += (float)k;
+                        seg_z = ldexpf(seg_z, -k);
+                    }
+                    return;
+                }
+            }
+            float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+            for (int c = 0; c < 32; ++c)
+                if (c < lim) m4[c & 3] = fmaxf(m4[c & 3], v[c]);
+            const float mu = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * G.sl2;
+            float z4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+            for (int c = 0; c < 32; ++c)
+                if (c < lim) z4[c & 3] += ptx::ex2(fmaf(v[c], G.sl2, -mu));
+            merge(seg_m, seg_z, make_float2(mu, (z4[0] + z4[1]) + (z4[2] + z4[3])));
         };
 
         ItemWalker p;
@@ -302,11 +339,11 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                 seg_z = 0.f;
                 seg_first = i;
             }
-            if (aborted) continue;   // keep walking the items for the segment barriers
-            const int buf = it % NB, nb = it / NB;
+            if (it % NB != grp || aborted) continue;   // another group's item (or keep walking for the barriers)
+            const int nb = it / NB;
             int ok = 1;
             if (lane == 0) {
-                ok = !bars->abort_flag && ptx::mbar_wait(&bars->acc_full[buf], nb & 1);
+                ok = !bars->abort_flag && ptx::mbar_wait(&bars->acc_full[grp], nb & 1);
                 if (!ok) raise_abort(bars, sc.err);
             }
             ok = __shfl_sync(0xffffffffu, ok, 0);
@@ -315,60 +352,29 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                 continue;
             }
             ptx::tc_fence_after();
-            const uint32_t taddr = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(buf * 128 * MB + m * 128);
+            const uint32_t taddr = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(grp * 128 * MB + m * 128);
             const int L = p.L;
             const int t0 = p.j * kTileT;
             const int last = vrow ? min(L - 1, L - G.w + q) : -1;   // causal on the window part
             const int nvalid = max(0, min(kTileT, last - t0 + 1));
-            const int c0 = split * COLS;
-            float v[COLS];
-#pragma unroll
-            for (int c = 0; c < COLS; c += 32) ptx::tmem_ld32(taddr + c0 + c, v + c);
+            // Four 32-column chunks; the next chunk's TMEM load is in flight while
+            // this one is reduced.
+            float va[32], vb[32];
+            ptx::tmem_ld32(taddr, va);
+            ptx::tmem_wait_ld();
+            ptx::tmem_ld32(taddr + 32, vb);
+            chunk(va, nvalid);
+            ptx::tmem_wait_ld();
+            ptx::tmem_ld32(taddr + 64, va);
+            chunk(vb, nvalid - 32);
+            ptx::tmem_wait_ld();
+            ptx::tmem_ld32(taddr + 96, vb);
+            chunk(va, nvalid - 64);
             ptx::tmem_wait_ld();
             ptx::tc_fence_before();
             __syncwarp();
-            if (lane == 0) ptx::mbar_arrive(&bars->acc_empty[buf]);
-            const int lim = nvalid - c0;
-            if (lim <= 0) continue;
-            if (lim >= COLS && seg_m != -INFINITY) {
-                // Relative to the segment's running reference seg_m: 2^(s - seg_m) sums
-                // the same mass as the online max/rescale, without a max pass.  A tile
-                // far above the reference (sum not below 2^64) takes the exact path.
-                float z4[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-                for (int c = 0; c < COLS; ++c) z4[c & 3] += ptx::ex2(fmaf(v[c], G.sl2, -seg_m));
-                const float z = (z4[0] + z4[1]) + (z4[2] + z4[3]);
-                if (z < 0x1p64f) {
-                    seg_z += z;
-                    if (seg_z >= 0x1p40f) {
-                        // Keep the sum bounded: move a power of two into the reference.
-                        const int k = ilogbf(seg_z);
-                        seg_m += (float)k;
-                        seg_z = ldexpf(seg_z, -k);
-                    }
-                    continue;
-                }
-            }
-            float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-            if (lim >= COLS) {
-#pragma unroll
-                for (int c = 0; c < COLS; ++c) m4[c & 3] = fmaxf(m4[c & 3], v[c]);
-            } else {
-#pragma unroll
-                for (int c = 0; c < COLS; ++c)
-                    if (c < lim) m4[c & 3] = fmaxf(m4[c & 3], v[c]);
-            }
-            const float mu = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * G.sl2;
-            float z4[4] = {0.f, 0.f, 0.f, 0.f};
-            if (lim >= COLS) {
-#pragma unroll
-                for (int c = 0; c < COLS; ++c) z4[c & 3] += ptx::ex2(fmaf(v[c], G.sl2, -mu));
-            } else {
-#pragma unroll
-                for (int c = 0; c < COLS; ++c)
-                    if (c < lim) z4[c & 3] += ptx::ex2(fmaf(v[c], G.sl2, -mu));
-            }
-            merge(seg_m, seg_z, make_float2(mu, (z4[0] + z4[1]) + (z4[2] + z4[3])));
+            if (lane == 0) ptx::mbar_arrive(&bars->acc_empty[grp]);   // the accumulator is in registers
+            chunk(vb, nvalid - 96);
         }
         if (cur_sh >= 0) flush_segment();
     }

@@ -432,6 +432,386 @@ __global__ void __launch_bounds__(kWinThreads, 1)
     if (warp == 1) ptx::tmem_dealloc(tmem, tmem_cols);
 }
 
+// ---------------------------------------------------------------------------
+// Tile-owning variant for O <= 16 and a group size with a straight-line epilogue
+// (g in {1, 2, 4, 7, 8}): a unit is T = 4 (or, with N > 128, 2) consecutive
+// candidate tiles of one sequence and one head group, and epilogue group j owns
+// tile j of the unit for every head.  The query block Q_h is loaded once per
+// (unit, head) into its own two-slot ring and serves the T tiles of the head, so
+// the K ring holds 32 KB stages only (4 in flight instead of 3 stages of K and
+// Q).  A thread keeps the running maxima over heads of its token's O last-row
+// group sums in registers, so the groups never synchronise; it adds its rows in
+// the same order as window_kernel, and the results are the same bits.
+// ---------------------------------------------------------------------------
+constexpr int kTileOMax = 16;     // largest O of the tile-owning variant (register maxima)
+constexpr int kMaxKStages = 6;
+
+struct TileArgs {
+    Geometry G;
+    Scratch sc;
+    Slot sl;
+    const int* cu;
+    int Npad, kst, nacc, units, fault;
+};
+
+struct __align__(8) TileBars {
+    uint64_t k_full[kMaxKStages], k_empty[kMaxKStages], q_full[2], q_empty[2], acc_full[4], acc_empty[4];
+    uint64_t mma_done;
+    uint32_t tmem_base;
+    volatile int abort_flag;
+    volatile int gok[4];
+};
+
+__host__ __device__ inline size_t tile_smem_bytes(int Npad, int kst) {
+    return 1024 + (size_t)kst * kKTileBytes + 2 * (size_t)Npad * 256 + 4 * 2 * 256 * sizeof(float) + sizeof(TileBars);
+}
+
+// Unit u -> sequence s, first candidate tile j0 of the unit, its tile count nt,
+// head group ng, global candidate tile of j0.
+struct TileUnit {
+    int s, j0, nt, ng, tg0, L, Lc, row0;
+};
+
+__device__ __forceinline__ bool decode_tile_unit(const Geometry& G, const int* cu, int T, int u, TileUnit& w) {
+    int base = 0, tbase = 0;
+    for (int b = 0; b < G.batch; ++b) {
+        const int c0 = __ldg(&cu[b]), c1 = __ldg(&cu[b + 1]);
+        const int Lc = c1 - c0 - G.wk;
+        const int ntile = Lc > 0 ? (Lc + kTileT - 1) / kTileT : 0;
+        const int ngrp = (ntile + T - 1) / T;
+        if (u < base + ngrp * G.NG) {
+            const int local = u - base;
+            const int tgi = local / G.NG;
+            w.s = b;
+            w.ng = local - tgi * G.NG;
+            w.j0 = tgi * T;
+            w.nt = min(T, ntile - w.j0);
+            w.tg0 = tbase + w.j0;
+            w.L = c1 - c0;
+            w.Lc = Lc;
+            w.row0 = c0 + w.j0 * kTileT;
+            return true;
+        }
+        base += ngrp * G.NG;
+        tbase += ntile;
+    }
+    return false;
+}
+
+// One head of this thread's token: rows [qOe, qO) add to poe only, rows [qO, w)
+// to po, to poe when q >= qOe, and to the running maxima mx[q - qO] (ascending q
+// in both parts, as head_rows).
+template <int GG>
+__device__ __forceinline__ void head_rows_tile(uint32_t taddr, const float* __restrict__ rsb, int w, int qmin,
+                                               float sl2, int qO, int qOe, float* mx, float& po, float& poe) {
+    constexpr int QPC = 32 / GG, CW = QPC * GG;
+    for (int qb = qOe; qb < qO; qb += QPC) {
+        const int c0 = qb * GG;
+        float v[32];
+        ptx::tmem_ld32(taddr + (uint32_t)c0, v);
+        ptx::tmem_wait_ld();
+        float pr[CW];
+#pragma unroll
+        for (int i = 0; i < CW; ++i) pr[i] = ptx::ex2(fmaf(v[i], sl2, -rsb[c0 + i]));
+#pragma unroll
+        for (int k = 0; k < QPC; ++k) {
+            float gs = 0.f;
+#pragma unroll
+            for (int j = 0; j < GG; ++j) gs += pr[k * GG + j];
+            const int q = qb + k;
+            gs = q >= qmin ? gs : 0.f;
+            if (q < qO) poe += gs;
+        }
+    }
+#pragma unroll
+    for (int c = 0; c < (kTileOMax + QPC - 1) / QPC; ++c) {
+        const int qb = qO + c * QPC;
+        if (qb >= w) break;
+        const int c0 = qb * GG;
+        float v[32];
+        ptx::tmem_ld32(taddr + (uint32_t)c0, v);
+        ptx::tmem_wait_ld();
+        float pr[CW];
+#pragma unroll
+        for (int i = 0; i < CW; ++i) pr[i] = ptx::ex2(fmaf(v[i], sl2, -rsb[c0 + i]));
+#pragma unroll
+        for (int k = 0; k < QPC; ++k) {
+            const int idx = c * QPC + k;
+            if (idx < kTileOMax) {
+                float gs = 0.f;
+#pragma unroll
+                for (int j = 0; j < GG; ++j) gs += pr[k * GG + j];
+                const int q = qb + k;
+                gs = q >= qmin ? gs : 0.f;
+                if (q < w) {
+                    if (q >= qOe) poe += gs;
+                    po += gs;
+                    mx[idx] = fmaxf(mx[idx], gs);
+                }
+            }
+        }
+    }
+}
+
+template <int GG>
+__global__ void __launch_bounds__(kWinThreads, 1)
+    window_tiles_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap qmap,
+                        const __grid_constant__ TileArgs A) {
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    if (threadIdx.x == 0) {
+        ptx::prefetch_tensormap(&kmap);
+        ptx::prefetch_tensormap(&qmap);
+        // The next launch on this stream (the next layer's row statistics) reads
+        // nothing this grid writes and does not wait for it: let it be scheduled.
+        asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
+    }
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const Geometry G = A.G;
+    const Scratch sc = A.sc;
+    const Slot sl = A.sl;
+    const int* const cu_dev = A.cu;
+    const int kst = A.kst, NA = A.nacc, units = A.units, fault = A.fault;
+    const int Npad = A.Npad, R = G.R;
+    const int T = NA;                                        // tiles per unit = epilogue groups
+    uint8_t* sK = smem;                                      // kst x 32 KB
+    uint8_t* sQ = sK + (size_t)kst * kKTileBytes;            // 2 slots x Npad x 256 B
+    float* rsm = reinterpret_cast<float*>(sQ + 2 * (size_t)Npad * 256);   // [4][2][256]
+    TileBars* bars = reinterpret_cast<TileBars*>(rsm + 4 * 2 * 256);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int u0 = blockIdx.x, ustep = gridDim.x;
+
+    if (threadIdx.x == 32) {
+        for (int i = 0; i < kst; ++i) {
+            ptx::mbar_init(&bars->k_full[i], 1);
+            ptx::mbar_init(&bars->k_empty[i], 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            ptx::mbar_init(&bars->q_full[i], 1);
+            ptx::mbar_init(&bars->q_empty[i], 1);
+        }
+        for (int i = 0; i < 4; ++i) {
+            ptx::mbar_init(&bars->acc_full[i], 1);
+            ptx::mbar_init(&bars->acc_empty[i], 4);   // one arrival per warp of the group
+        }
+        ptx::mbar_init(&bars->mma_done, 1);
+        bars->abort_flag = 0;
+        ptx::fence_barrier_init();
+    }
+    if (warp == 1) {
+        ptx::tmem_alloc(&bars->tmem_base, 512);
+        ptx::tmem_relinquish();
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    const uint32_t tmem = bars->tmem_base;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ TMA producer
+        if (lane == 0) {
+            const uint64_t policy = ptx::policy_evict_first();   // the K tiles' last use
+            int qi = 0, ki = 0;
+            int kfills[kMaxKStages] = {0, 0, 0, 0, 0, 0};
+            int qfills[2] = {0, 0};
+            bool stop = false;
+            for (int u = u0; u < units && !stop; u += ustep) {
+                TileUnit tu;
+                decode_tile_unit(G, cu_dev, T, u, tu);
+                const int h0 = tu.ng * G.HG, nh = min(G.HG, G.Hkv - h0);
+                for (int hh = 0; hh < nh && !stop; ++hh) {
+                    const int h = h0 + hh;
+                    const int qs = qi & 1, nq = qi >> 1;
+                    if (nq > 0 && !ptx::mbar_wait_abortable(&bars->q_empty[qs], (nq - 1) & 1, &bars->abort_flag)) {
+                        bars->abort_flag = 1;
+                        atomicExch(sc.err, 3);
+                        stop = true;
+                        break;
+                    }
+                    if (bars->abort_flag) {
+                        stop = true;
+                        break;
+                    }
+                    uint8_t* q = sQ + (size_t)qs * Npad * 256;
+                    ptx::mbar_arrive_expect_tx(&bars->q_full[qs], 2u * (uint32_t)R * 128u);
+                    ptx::tma_load_4d(q, &qmap, &bars->q_full[qs], 0, h * G.g, 0, tu.s);
+                    ptx::tma_load_4d(q + Npad * 128, &qmap, &bars->q_full[qs], 64, h * G.g, 0, tu.s);
+                    ++qfills[qs];
+                    ++qi;
+                    for (int j = 0; j < tu.nt; ++j) {
+                        const int st = ki % kst, nk = ki / kst;
+                        if (nk > 0 && !ptx::mbar_wait_abortable(&bars->k_empty[st], (nk - 1) & 1, &bars->abort_flag)) {
+                            bars->abort_flag = 1;
+                            atomicExch(sc.err, 3);
+                            stop = true;
+                            break;
+                        }
+                        uint8_t* sk = sK + (size_t)st * kKTileBytes;
+                        const int row = tu.row0 + j * kTileT;
+                        ptx::mbar_arrive_expect_tx(&bars->k_full[st], (uint32_t)kKTileBytes);
+                        ptx::tma_load_3d(sk, &kmap, &bars->k_full[st], 0, h, row, policy);
+                        ptx::tma_load_3d(sk + kKTileBytes / 2, &kmap, &bars->k_full[st], 64, h, row, policy);
+                        ++kfills[st];
+                        ++ki;
+                    }
+                }
+            }
+            // Drain: every issued copy lands before the CTA may exit.
+            for (int st = 0; st < kst; ++st)
+                if (kfills[st] > 0) ptx::mbar_wait(&bars->k_full[st], (kfills[st] - 1) & 1, 50000000ull);
+            for (int qs = 0; qs < 2; ++qs)
+                if (qfills[qs] > 0) ptx::mbar_wait(&bars->q_full[qs], (qfills[qs] - 1) & 1, 50000000ull);
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            const uint32_t idesc = ptx::idesc_bf16_f32(128, Npad);
+            int qi = 0, ki = 0, first = 1;
+            int cnt[4] = {0, 0, 0, 0};
+            bool stop = false;
+            for (int u = u0; u < units && !stop; u += ustep) {
+                TileUnit tu;
+                decode_tile_unit(G, cu_dev, T, u, tu);
+                const int nh = min(G.HG, G.Hkv - tu.ng * G.HG);
+                for (int hh = 0; hh < nh && !stop; ++hh) {
+                    const int qs = qi & 1;
+                    if (bars->abort_flag ||
+                        !ptx::mbar_wait_abortable(&bars->q_full[qs], (qi >> 1) & 1, &bars->abort_flag)) {
+                        bars->abort_flag = 1;
+                        atomicExch(sc.err, 3);
+                        stop = true;
+                        break;
+                    }
+                    const uint32_t sq = ptx::smem_u32(sQ + (size_t)qs * Npad * 256);
+                    for (int j = 0; j < tu.nt; ++j) {
+                        const int st = ki % kst;
+                        // Giving up on a stage in flight is safe: the producer drains its own loads.
+                        if (!ptx::mbar_wait_abortable(&bars->k_full[st], (ki / kst) & 1, &bars->abort_flag) ||
+                            (cnt[j] > 0 &&
+                             !ptx::mbar_wait_abortable(&bars->acc_empty[j], (cnt[j] - 1) & 1, &bars->abort_flag))) {
+                            bars->abort_flag = 1;
+                            atomicExch(sc.err, 3);
+                            stop = true;
+                            break;
+                        }
+                        ptx::tc_fence_after();
+                        const uint32_t sk = ptx::smem_u32(sK + (size_t)st * kKTileBytes);
+                        const uint32_t d = tmem + (uint32_t)(j * Npad);
+#pragma unroll
+                        for (int kk = 0; kk < 8; ++kk) {
+                            const int half = kk >> 2, kin = kk & 3;
+                            const uint64_t ad = ptx::smem_desc_k_sw128(sk + half * (kKTileBytes / 2) + kin * 32);
+                            const uint64_t bd = ptx::smem_desc_k_sw128(sq + half * Npad * 128 + kin * 32);
+                            ptx::mma_bf16(d, ad, bd, idesc, kk > 0 ? 1u : 0u);
+                        }
+                        ptx::mma_commit(&bars->k_empty[st]);
+                        if (!(fault && first)) ptx::mma_commit(&bars->acc_full[j]);
+                        first = 0;
+                        ++ki;
+                        ++cnt[j];
+                    }
+                    ptx::mma_commit(&bars->q_empty[qs]);
+                    ++qi;
+                }
+            }
+            ptx::mma_commit(&bars->mma_done);
+        }
+    } else if (warp < 2 + 4 * NA) {
+        // ------------------------------------------------------------ epilogue
+        const int grp = (warp - 2) >> 2;                  // the tile of the unit this group owns
+        const int gtid = threadIdx.x - 64 - grp * 128;
+        const int quad = warp & 3;
+        const int tok = quad * 32 + lane;
+        const int bar_id = 1 + grp;
+        const int qO = G.w - G.O, qOe = G.w - G.Oe;
+        const float invO = 1.f / (float)G.O, invOe = 1.f / (float)G.Oe;
+        const uint32_t tbase = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(grp * Npad);
+        float* rs_g = rsm + grp * 2 * 256;
+        asm volatile("griddepcontrol.wait;\n" ::: "memory");
+        auto fetch = [&](int s, int h, float& a, float& b) {
+            const float2* src = sc.rowstat + ((size_t)s * G.Hkv + h) * R;
+            a = b = 0.f;
+            if (gtid < R) {
+                const float2 m = __ldcg(src + gtid);
+                a = m.x + __log2f(m.y);
+            }
+            if (gtid + 128 < R) {
+                const float2 m = __ldcg(src + gtid + 128);
+                b = m.x + __log2f(m.y);
+            }
+        };
+        int k = 0;
+        bool failed = false;
+        for (int u = u0; u < units && !failed; u += ustep) {
+            TileUnit tu;
+            decode_tile_unit(G, cu_dev, T, u, tu);
+            if (grp >= tu.nt) continue;   // this group's tile is past the sequence's last
+            const int h0 = tu.ng * G.HG, nh = min(G.HG, G.Hkv - h0);
+            const int t = (tu.j0 + grp) * kTileT + tok;
+            const int qmin = t - (tu.L - G.w);
+            float mx[kTileOMax];
+#pragma unroll
+            for (int i = 0; i < kTileOMax; ++i) mx[i] = 0.f;
+            float pa, pb;
+            fetch(tu.s, h0, pa, pb);
+            for (int hh = 0; hh < nh; ++hh, ++k) {
+                if (gtid == 0) {
+                    const bool ok = !bars->abort_flag &&
+                                    ptx::mbar_wait_abortable(&bars->acc_full[grp], k & 1, &bars->abort_flag,
+                                                             fault && k == 0 && grp == 0 ? kFaultWaitNs
+                                                                                         : 200000000ull);
+                    if (!ok) {
+                        bars->abort_flag = 1;
+                        atomicExch(sc.err, 3);
+                    }
+                    bars->gok[grp] = ok ? 1 : 0;
+                }
+                float* rsb = rs_g + (k & 1) * 256;
+                rsb[gtid] = pa;
+                rsb[gtid + 128] = pb;
+                ptx::named_bar_sync(bar_id, 128);
+                if (!bars->gok[grp]) {
+                    failed = true;
+                    break;
+                }
+                if (hh + 1 < nh) fetch(tu.s, h0 + hh + 1, pa, pb);   // the next head's rows, in flight
+                ptx::tc_fence_after();
+                float po = 0.f, poe = 0.f;
+                head_rows_tile<GG>(tbase, rsb, G.w, qmin, G.sl2, qO, qOe, mx, po, poe);
+                ptx::tc_fence_before();
+                __syncwarp();
+                if (lane == 0) ptx::mbar_arrive(&bars->acc_empty[grp]);
+                if (t < tu.Lc) {
+                    const size_t row = (size_t)tu.s * G.Hkv + h0 + hh;
+                    sl.rawO[row * G.ML + t] = po * invO;
+                    sl.rawOe[row * G.ML + t] = poe * invOe;
+                }
+            }
+            if (failed) break;
+            // I[t] = (1/O) sum over the last O rows of the maxima over the heads (or
+            // this head group's maxima, combined by the heads kernel).
+            if (G.NG > 1) {
+                float* wp = sl.wpart + ((size_t)(tu.tg0 + grp) * G.NG + tu.ng) * G.O * kTileT;
+#pragma unroll
+                for (int i = 0; i < kTileOMax; ++i)
+                    if (i < G.O) wp[i * kTileT + tok] = mx[i];
+            } else if (t < tu.Lc) {
+                float ip = 0.f;
+#pragma unroll
+                for (int i = 0; i < kTileOMax; ++i)
+                    if (i < G.O) ip += mx[i];
+                sl.rawI[(size_t)tu.s * G.ML + t] = ip * invO;
+            }
+        }
+    }
+
+    // ---------------------------------------------------------------- teardown
+    if (warp == 1 && lane == 0) ptx::mbar_wait(&bars->mma_done, 0, 50000000ull);
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    if (warp == 1) ptx::tmem_dealloc(tmem, 512);
+}
+
 int npad_of(int R) { return (R + 15) & ~15; }
 
 int kst_for(int Npad, int O) {
@@ -458,12 +838,95 @@ cudaError_t configure_window(const Geometry& g) {
     for (auto fn : {window_kernel<0>, window_kernel<1>, window_kernel<2>, window_kernel<4>, window_kernel<7>,
                     window_kernel<8>})
         if (e == cudaSuccess) e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmemWin);
+    for (auto fn : {window_tiles_kernel<1>, window_tiles_kernel<2>, window_tiles_kernel<4>, window_tiles_kernel<7>,
+                    window_tiles_kernel<8>})
+        if (e == cudaSuccess) e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmemWin);
     return e;
 }
+
+namespace {
+
+int tile_kst_for(int Npad) {
+    int k = kMaxKStages;
+    while (k > 1 && tile_smem_bytes(Npad, k) > (size_t)kMaxSmemWin) --k;
+    return k;
+}
+
+// The tile variant applies to O <= 16 with a straight-line group size, when every
+// 32-column TMEM load of its epilogue (chunks starting at rows w - O' and w - O)
+// stays inside the 512 allocated columns.
+bool tile_variant_fits(const Geometry& g) {
+    if (g.O > kTileOMax || !(g.g == 1 || g.g == 2 || g.g == 4 || g.g == 7 || g.g == 8)) return false;
+    const int qpc = 32 / g.g, qO = g.w - g.O, qOe = g.w - g.Oe;
+    const int Npad = npad_of(g.R), nacc = Npad <= 128 ? 4 : 2;
+    int maxcol = 0;
+    for (int qb = qOe; qb < qO; qb += qpc) maxcol = maxcol > qb * g.g + 32 ? maxcol : qb * g.g + 32;
+    for (int c = 0; c < (kTileOMax + qpc - 1) / qpc; ++c) {
+        const int qb = qO + c * qpc;
+        if (qb >= g.w) break;
+        maxcol = maxcol > qb * g.g + 32 ? maxcol : qb * g.g + 32;
+    }
+    return (nacc - 1) * Npad + maxcol <= 512;
+}
+
+// Units of the tile-owning variant: groups of T candidate tiles per sequence and head group.
+int tile_units_of(const Geometry& g, const int* cu_host, int T) {
+    int units = 0;
+    for (int b = 0; b < g.batch; ++b) {
+        const int Lc = cu_host[b + 1] - cu_host[b] - g.wk;
+        const int nt = Lc > 0 ? (Lc + kTileT - 1) / kTileT : 0;
+        units += (nt + T - 1) / T * g.NG;
+    }
+    return units;
+}
+
+cudaError_t launch_window_tiles(const ScorePlan& sp, const Geometry& g, const LayerIO& io, const Scratch& sc,
+                                const Slot& sl, cudaStream_t st, bool after_own_launch) {
+    TileArgs a{};
+    a.G = g;
+    a.sc = sc;
+    a.sl = sl;
+    a.cu = io.cu;
+    a.Npad = npad_of(g.R);
+    a.nacc = a.Npad <= 128 ? 4 : 2;   // nacc * Npad <= 512 TMEM columns
+    a.kst = tile_kst_for(a.Npad);
+    a.units = tile_units_of(g, g.cu_host, a.nacc);
+    a.fault = test_fault() == 1 ? 1 : 0;
+    const size_t smem = tile_smem_bytes(a.Npad, a.kst);
+    const int usable = sp.num_sms > 2 * kWinReserveSms ? sp.num_sms - kWinReserveSms : sp.num_sms;
+    const int grid = a.units < usable ? a.units : usable;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(kWinThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = after_own_launch ? 1 : 0;
+    switch (g.g) {
+        case 1: return cudaLaunchKernelEx(&cfg, window_tiles_kernel<1>, sp.kmap, sp.qmap, a);
+        case 2: return cudaLaunchKernelEx(&cfg, window_tiles_kernel<2>, sp.kmap, sp.qmap, a);
+        case 4: return cudaLaunchKernelEx(&cfg, window_tiles_kernel<4>, sp.kmap, sp.qmap, a);
+        case 7: return cudaLaunchKernelEx(&cfg, window_tiles_kernel<7>, sp.kmap, sp.qmap, a);
+        default: return cudaLaunchKernelEx(&cfg, window_tiles_kernel<8>, sp.kmap, sp.qmap, a);
+    }
+}
+
+}  // namespace
 
 cudaError_t launch_window(const ScorePlan& sp, const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl,
                           cudaStream_t st, bool after_own_launch) {
     if (g.win_tiles == 0) return cudaSuccess;
+    // The tile-owning variant where it applies and its units still give every
+    // usable SM one (it has T times fewer units than the per-tile kernel, whose
+    // CTAs finish sooner when there are few tiles).
+    if (tile_variant_fits(g)) {
+        const int T = npad_of(g.R) <= 128 ? 4 : 2;
+        const int usable = sp.num_sms > 2 * kWinReserveSms ? sp.num_sms - kWinReserveSms : sp.num_sms;
+        if (tile_units_of(g, g.cu_host, T) >= usable) return launch_window_tiles(sp, g, io, sc, sl, st, after_own_launch);
+    }
     WinArgs a{};
     a.G = g;
     a.sc = sc;

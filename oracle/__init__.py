@@ -45,6 +45,7 @@ class _Params(ctypes.Structure):
         ("pool_kernel", ctypes.c_int), ("num_ext_heads", ctypes.c_int),
         ("lam", ctypes.c_double), ("beta", ctypes.c_double), ("softmax_scale", ctypes.c_double),
         ("pool_mode", ctypes.c_int), ("head_criterion", ctypes.c_int), ("all_positions", ctypes.c_int),
+        ("head_budget", ctypes.c_int), ("ada_floor", ctypes.c_double),
     ]
 
 
@@ -70,6 +71,8 @@ def _load():
             lib.kvo_state_bytes.restype = ctypes.c_size_t
             lib.kvo_state_bytes.argtypes = [ctypes.c_int]
             lib.kvo_num_threads.restype = ctypes.c_int
+            lib.kvo_head_capacity.restype = ctypes.c_int
+            lib.kvo_head_capacity.argtypes = [ctypes.POINTER(_Params), ctypes.c_int]
             lib.kvo_select_layer.restype = ctypes.c_int
             lib.kvo_select_layer.argtypes = [
                 ctypes.POINTER(_Params), ctypes.c_int, ctypes.c_void_p, ctypes.c_int,
@@ -95,6 +98,8 @@ class OracleParams:
     pool_mode: int = 0        # 0 max-pool, 1 average pool
     head_criterion: int = 0   # 0 standard deviation, 1 entropy
     all_positions: int = 0    # 0 keep the window tail, 1 every position is a candidate
+    head_budget: int = 0      # 0 uniform fill, 1 head-wise adaptive fill
+    ada_floor: float = 1.0    # share of a head's fill it keeps by its own ranking (adaptive fill)
 
     @classmethod
     def from_workload(cls, wl, **over) -> "OracleParams":
@@ -103,7 +108,8 @@ class OracleParams:
                   pool_kernel=wl.pool_kernel, num_ext_heads=wl.num_ext_heads,
                   lam=float(np.float32(wl.lam)), beta=float(np.float32(wl.beta)),
                   pool_mode=getattr(wl, "pool_mode", 0), head_criterion=getattr(wl, "head_criterion", 0),
-                  all_positions=getattr(wl, "all_positions", 0))
+                  all_positions=getattr(wl, "all_positions", 0), head_budget=getattr(wl, "head_budget", 0),
+                  ada_floor=float(np.float32(getattr(wl, "ada_floor", 1.0))))
         kw.update(over)
         return cls(**kw)
 
@@ -111,7 +117,16 @@ class OracleParams:
         return _Params(self.num_q_heads, self.num_kv_heads, self.head_dim, self.window,
                        self.obs_window, self.ext_window, self.pool_kernel, self.num_ext_heads,
                        float(self.lam), float(self.beta), float(self.softmax_scale), int(self.pool_mode),
-                       int(self.head_criterion), int(self.all_positions))
+                       int(self.head_criterion), int(self.all_positions), int(self.head_budget),
+                       float(self.ada_floor))
+
+
+def head_capacity(params: OracleParams, budget: int) -> int:
+    """Rows per KV head of the outputs (budget for the uniform fill)."""
+    cap = int(_load().kvo_head_capacity(ctypes.byref(params._c()), int(budget)))
+    if cap < 1:
+        raise ValueError("invalid parameters for the output capacity")
+    return cap
 
 
 def state_bytes(max_seqlen: int) -> int:
@@ -159,7 +174,8 @@ def select_layer(params: OracleParams, cu_seqlens, q_obs, k, v, state: np.ndarra
                  max_seqlen: Optional[int] = None, debug: bool = True) -> Dict[str, np.ndarray]:
     """Runs one layer of the oracle.  ``state`` (uint8 [batch][state_bytes]) is updated in place.
 
-    Returns out_idx [batch][Hkv][B] int32, out_k / out_v [batch][Hkv][B][d] uint16 (bf16 bits),
+    Returns out_idx [batch][Hkv][cap] int32, out_k / out_v [batch][Hkv][cap][d] uint16 (bf16 bits),
+    cap = head_capacity(params, budget) (= budget for the uniform fill),
     and, with ``debug``, every intermediate listed in ``kvo_debug``.
     """
     lib = _load()
@@ -170,9 +186,10 @@ def select_layer(params: OracleParams, cu_seqlens, q_obs, k, v, state: np.ndarra
     Hq, Hkv, d, w = params.num_q_heads, params.num_kv_heads, params.head_dim, params.window
     qa, ka, va = _as_u16(q_obs), _as_u16(k), _as_u16(v)
     assert state.dtype == np.uint8 and state.shape == (batch, state_bytes(ML)) and state.flags.c_contiguous
-    out_idx = np.empty((batch, Hkv, budget), np.int32)
-    out_k = np.empty((batch, Hkv, budget, d), np.uint16)
-    out_v = np.empty((batch, Hkv, budget, d), np.uint16)
+    cap = head_capacity(params, budget)
+    out_idx = np.empty((batch, Hkv, cap), np.int32)
+    out_k = np.empty((batch, Hkv, cap, d), np.uint16)
+    out_v = np.empty((batch, Hkv, cap, d), np.uint16)
     res: Dict[str, np.ndarray] = {}
     dbg = None
     if debug:

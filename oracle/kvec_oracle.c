@@ -25,6 +25,13 @@
  *    the budget goes to the highest P' among the other candidates.
  *  - Every top-k orders by higher score, then lower position.
  *  - coverage_t = n_t / (l+1) with l the number of layers already processed.
+ *  - Head-wise adaptive fill (head_budget = 1; Section 2 names AdaKV's head-wise
+ *    budget allocation as a plug-and-play addition without defining it): each
+ *    head keeps its window and preserved tokens and its own floor(a * F) best
+ *    other candidates by P' (F = B - w - K, a = ada_floor); the rest of the
+ *    layer's fill, H_kv * (F - floor(a * F)) slots, goes to the best P' among all
+ *    heads' remaining candidates ranked together (higher P', then lower head,
+ *    then lower position).  a = 1 is the uniform fill.
  */
 #include "kvec_oracle.h"
 
@@ -110,6 +117,27 @@ static void max_pool(const double* x, int n, int kernel, double* y) {
     }
 }
 
+/* Preserved tokens and fill per head: K = min(floor(beta * B), B - wk), F = B - wk - K. */
+static void budget_split(const kvo_params* p, int budget, int* Kp, int* F, int* f0) {
+    const int wk = p->all_positions ? 0 : p->window;
+    int k = (int)floor(p->beta * (double)budget);
+    if (k > budget - wk) k = budget - wk;
+    *Kp = k;
+    *F = budget - wk - k;
+    *f0 = p->head_budget ? (int)floor(p->ada_floor * (double)*F) : *F;
+}
+
+int kvo_head_capacity(const kvo_params* p, int budget) {
+    if (!p || budget < 1 || p->num_kv_heads < 1) return -1;
+    if (p->head_budget != 0 && p->head_budget != 1) return -1;
+    if (p->head_budget && !(p->ada_floor >= 0.0 && p->ada_floor <= 1.0)) return -1;
+    const int wk = p->all_positions ? 0 : p->window;
+    if (budget < wk) return -1;
+    int Kp, F, f0;
+    budget_split(p, budget, &Kp, &F, &f0);
+    return budget + (p->num_kv_heads - 1) * (F - f0);
+}
+
 int kvo_select_layer(const kvo_params* p, int batch, const int32_t* cu_seqlens, int max_seqlen,
                      const uint16_t* q_obs, const uint16_t* k, const uint16_t* v,
                      uint8_t* state, int budget,
@@ -130,6 +158,9 @@ int kvo_select_layer(const kvo_params* p, int batch, const int32_t* cu_seqlens, 
     /* wk: the tail kept unconditionally (the window, or nothing). */
     const int wk = p->all_positions ? 0 : w;
     if (budget < wk || budget < 1) return -7;
+    if (p->head_budget != 0 && p->head_budget != 1) return -4;
+    if (p->head_budget && !(p->ada_floor >= 0.0 && p->ada_floor <= 1.0)) return -6;
+    const int cap = kvo_head_capacity(p, budget);
     for (int b = 0; b < batch; ++b) {
         int L = cu_seqlens[b + 1] - cu_seqlens[b];
         if (L < w || L > max_seqlen) return -8;
@@ -276,9 +307,8 @@ int kvo_select_layer(const kvo_params* p, int batch, const int32_t* cu_seqlens, 
 
         /* Steps 6-8 (Section 4.2): preserve top-K of P, add lambda*focus, fill the rest. */
         const int keep_all = L <= budget;
-        int Kp = (int)floor(p->beta * (double)budget);
-        if (Kp > budget - wk) Kp = budget - wk;
-        const int k2 = budget - wk - Kp;
+        int Kp, k2, f0;
+        budget_split(p, budget, &Kp, &k2, &f0);
         uint8_t* pres = (uint8_t*)calloc((size_t)Hkv * (Lc > 0 ? Lc : 1), 1);
         double* Pp = (double*)calloc((size_t)Hkv * (Lc > 0 ? Lc : 1), sizeof(double));
         uint8_t* keep = (uint8_t*)calloc((size_t)Hkv * L, 1);   /* S_h as a mask over [0, L) */
@@ -299,11 +329,11 @@ int kvo_select_layer(const kvo_params* p, int batch, const int32_t* cu_seqlens, 
             top_k(Ph, NULL, Lc, Kp, ph);
             uint8_t* others = (uint8_t*)malloc((size_t)Lc);
             for (int t = 0; t < Lc; ++t) others[t] = !ph[t];
-            top_k(pph, others, Lc, k2, kh);
+            top_k(pph, others, Lc, f0, kh);   /* the whole fill (uniform) or the head's floor */
             for (int t = 0; t < Lc; ++t) if (ph[t]) kh[t] = 1;
             for (int t = Lc; t < L; ++t) kh[t] = 1;
             /* Literal reading: P' = 1.0 on preserved tokens, then top-(B-w) of P'. */
-            if (dbg) {
+            if (dbg && !p->head_budget) {
                 double* lit = (double*)malloc(sizeof(double) * (size_t)Lc);
                 uint8_t* lsel = (uint8_t*)calloc((size_t)Lc, 1);
                 for (int t = 0; t < Lc; ++t) lit[t] = ph[t] ? 1.0 : pph[t];
@@ -317,11 +347,34 @@ int kvo_select_layer(const kvo_params* p, int batch, const int32_t* cu_seqlens, 
             free(others);
         }
 
+        /* Adaptive fill: the rest of the layer's fill to the best P' over all
+         * heads' remaining candidates, ranked together (entry h * Lc + t, so ties
+         * go to the lower head, then the lower position). */
+        if (p->head_budget && !keep_all && Lc > 0) {
+            const size_t n = (size_t)Hkv * Lc;
+            double* jk = (double*)malloc(sizeof(double) * n);
+            uint8_t* ja = (uint8_t*)calloc(n, 1);
+            uint8_t* js = (uint8_t*)calloc(n, 1);
+            for (int h = 0; h < Hkv; ++h)
+                for (int t = 0; t < Lc; ++t) {
+                    const size_t i = (size_t)h * Lc + t;
+                    jk[i] = Pp[i];
+                    ja[i] = !pres[i] && !keep[(size_t)h * L + t];
+                }
+            top_k(jk, ja, (int)n, Hkv * (k2 - f0), js);
+            for (int h = 0; h < Hkv; ++h)
+                for (int t = 0; t < Lc; ++t)
+                    if (js[(size_t)h * Lc + t]) keep[(size_t)h * L + t] = 1;
+            free(jk);
+            free(ja);
+            free(js);
+        }
+
         /* Outputs: ascending positions per head, then gather of K and V rows. */
         for (int h = 0; h < Hkv; ++h) {
-            int32_t* oi = out_idx + ((size_t)b * Hkv + h) * budget;
-            uint16_t* ok = out_k + ((size_t)b * Hkv + h) * budget * d;
-            uint16_t* ov = out_v + ((size_t)b * Hkv + h) * budget * d;
+            int32_t* oi = out_idx + ((size_t)b * Hkv + h) * cap;
+            uint16_t* ok = out_k + ((size_t)b * Hkv + h) * cap * d;
+            uint16_t* ov = out_v + ((size_t)b * Hkv + h) * cap * d;
             int j = 0;
             for (int t = 0; t < L; ++t) {
                 if (!keep[(size_t)h * L + t]) continue;
@@ -330,7 +383,7 @@ int kvo_select_layer(const kvo_params* p, int batch, const int32_t* cu_seqlens, 
                 memcpy(ov + (size_t)j * d, vb + ((size_t)t * Hkv + h) * d, sizeof(uint16_t) * d);
                 ++j;
             }
-            for (; j < budget; ++j) {
+            for (; j < cap; ++j) {
                 oi[j] = -1;
                 memset(ok + (size_t)j * d, 0, sizeof(uint16_t) * d);
                 memset(ov + (size_t)j * d, 0, sizeof(uint16_t) * d);

@@ -39,6 +39,15 @@ typedef struct {
                             candidates are [0, L-w) (default); 1: every position
                             [0, L) is a candidate and each head keeps the top B of
                             them (Section 4.1's top-B over the T input tokens) */
+    int head_budget;     /* 0: every KV head keeps B tokens (default); 1: head-wise
+                            adaptive fill (the AdaKV-style allocation Section 2 calls
+                            plug-and-play): each head keeps its window and preserved
+                            tokens and the floor(ada_floor * F) best of its own other
+                            candidates by P', F = B - w - K; the layer's remaining
+                            H_kv * F - H_kv * floor(ada_floor * F) fill slots go to the
+                            best P' over all heads' remaining candidates together
+                            (ties: lower head, then lower position) */
+    double ada_floor;    /* in [0, 1]; 1 gives the uniform fill */
 } kvo_params;
 
 /* Optional debug outputs.  Any pointer may be NULL.  Sizes use the caller's
@@ -61,6 +70,11 @@ typedef struct {
     int64_t literal_override_differs; /* heads where setting P'=1.0 literally would change S_h */
 } kvo_debug;
 
+/* Rows per KV head of the outputs: budget for the uniform fill; with the
+ * adaptive fill a head may keep up to budget + (H_kv - 1) * (F - floor(ada_floor * F))
+ * tokens.  -1 for invalid parameters. */
+int kvo_head_capacity(const kvo_params* p, int budget);
+
 /* Bytes of coverage state per sequence for a given max_seqlen.  Layout:
  *   u32 layers_done, u32 seqlen, u32 reserved[2],
  *   u8  n[round_up(max_seqlen, 16)],
@@ -71,8 +85,8 @@ size_t kvo_state_bytes(int max_seqlen);
 /* One layer of eviction selection for a packed (varlen) batch.
  *   cu_seqlens [batch+1]; q_obs [batch][w][H_q][d]; k, v [total][H_kv][d];
  *   state: batch consecutive per-sequence states (stride kvo_state_bytes);
- *   out_idx [batch][H_kv][budget] (ascending, -1 padded);
- *   out_k, out_v [batch][H_kv][budget][d] (zero padded).
+ *   out_idx [batch][H_kv][cap] (ascending, -1 padded), cap = kvo_head_capacity;
+ *   out_k, out_v [batch][H_kv][cap][d] (zero padded).
  * Returns 0 on success, a negative code on invalid arguments. */
 int kvo_select_layer(const kvo_params* p, int batch, const int32_t* cu_seqlens, int max_seqlen,
                      const uint16_t* q_obs, const uint16_t* k, const uint16_t* v,

@@ -47,6 +47,8 @@ class Workload:
     pool_mode: int = 0        # 0 max-pool, 1 average pool (variant)
     head_criterion: int = 0   # 0 standard deviation, 1 entropy (variant)
     all_positions: int = 0    # 0 keep the window tail, 1 every position is a candidate (variant)
+    head_budget: int = 0      # 0 uniform fill, 1 head-wise adaptive fill (variant)
+    ada_floor: float = 0.2    # adaptive fill: share of a head's fill it keeps by its own ranking
     budget: int = 512         # B per KV head, window included
     num_ext_heads: int = 3    # delta
     lam: float = 1.0          # lambda

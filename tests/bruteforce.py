@@ -38,7 +38,7 @@ def _ranked(score: np.ndarray, positions: np.ndarray) -> np.ndarray:
 
 def select(q_full, k, *, num_kv_heads, window, obs_window, ext_window, pool_kernel,
            num_ext_heads, lam, beta, budget, n_counts, layers_done, scale=None, pool_mode=0,
-           head_criterion=0, all_positions=0) -> Dict[str, np.ndarray]:
+           head_criterion=0, all_positions=0, head_budget=0, ada_floor=1.0) -> Dict[str, np.ndarray]:
     """Algorithm 1 followed by per-head top-B for one sequence of length T = q_full.shape[0]."""
     T, Hq, d = q_full.shape
     Hkv = num_kv_heads
@@ -86,6 +86,9 @@ def select(q_full, k, *, num_kv_heads, window, obs_window, ext_window, pool_kern
     coverage = n_counts[:Lc].astype(np.float64) / (layers_done + 1)
     Pprime = P + lam * (I * (1.0 - coverage))[None, :]
     Kp = min(int(math.floor(beta * budget)), budget - wk)
+    F = budget - wk - Kp
+    own = int(math.floor(ada_floor * F)) if head_budget else F   # fill slots ranked within the head
+    cap = budget + (Hkv - 1) * (F - own)
     cand = np.arange(Lc)
     keep = np.zeros((Hkv, T), bool)
     pres = np.zeros((Hkv, max(Lc, 0)), bool)
@@ -96,11 +99,18 @@ def select(q_full, k, *, num_kv_heads, window, obs_window, ext_window, pool_kern
             top = _ranked(P[h], cand)[:Kp]
             pres[h, top] = True
             rest = cand[~pres[h]]
-            fill = _ranked(Pprime[h], rest)[:budget - wk - Kp]
+            fill = _ranked(Pprime[h], rest)[:own]
             keep[h, top] = True
             keep[h, fill] = True
             keep[h, Lc:] = True
-    out_idx = np.full((Hkv, budget), -1, np.int64)
+        if head_budget:
+            # The layer's other fill slots: every head's remaining candidates in one
+            # list, higher P' first, then lower head, then lower position.
+            pool_ = [(-Pprime[h, t], h, t) for h in range(Hkv) for t in range(Lc) if not keep[h, t]]
+            pool_.sort()
+            for _, h, t in pool_[:Hkv * (F - own)]:
+                keep[h, t] = True
+    out_idx = np.full((Hkv, cap), -1, np.int64)
     for h in range(Hkv):
         sel = np.flatnonzero(keep[h])
         out_idx[h, :sel.size] = sel

@@ -476,3 +476,103 @@ def test_all_positions_without_coverage_is_plain_topB_of_every_position(beta):
         r = oracle.select_layer(p, wl.cu_seqlens, x["q_obs"], x["k"], x["v"], st, wl.budget)
         for h in range(wl.num_kv_heads):
             assert (r["out_idx"][0, h] == _top_positions(r["P_O"][0, h, :400], wl.budget)).all()
+
+
+# ---- head-wise adaptive fill (head_budget = 1) ----
+
+ADA_CASES = [
+    # (seed, T, Hq, Hkv, d, w, O, O', pool, delta, lam, beta, B, ada_floor)
+    (21, 16, 4, 2, 8, 4, 2, 4, 3, 1, 1.0, 0.25, 8, 0.0),
+    (22, 16, 8, 4, 4, 5, 2, 5, 1, 2, 0.5, 0.34, 9, 0.5),
+    (23, 15, 6, 3, 8, 4, 2, 4, 3, 1, 1.0, 0.25, 10, 0.2),
+    (24, 12, 4, 4, 8, 3, 2, 3, 5, 3, 2.0, 0.0, 7, 0.3),
+    (25, 10, 4, 2, 8, 4, 2, 4, 3, 1, 1.0, 0.25, 12, 0.2),   # L <= B: keep everything
+]
+
+
+@pytest.mark.parametrize("case", ADA_CASES)
+def test_adaptive_fill_matches_bruteforce_over_layers(case):
+    seed, T, Hq, Hkv, d, w, O, Oe, pool, delta, lam, beta, B, a = case
+    params = oracle.OracleParams(num_q_heads=Hq, num_kv_heads=Hkv, head_dim=d, window=w, obs_window=O,
+                                 ext_window=Oe, pool_kernel=pool, num_ext_heads=delta, lam=lam, beta=beta,
+                                 head_budget=1, ada_floor=a)
+    state = oracle.new_state(1, T)
+    n_bf = np.zeros(T, np.int64)
+    for layer in range(3):
+        x = synth.tiny_full_inputs(seed * 100 + layer, T, Hq, Hkv, d)
+        q_obs = x["q_full"][T - w:].reshape(1, w, Hq, d)
+        r = _run_oracle(params, q_obs, x["k"], x["v"], state, B)
+        bf = bf_select(_f64(x["q_full"]), _f64(x["k"]), num_kv_heads=Hkv, window=w, obs_window=O,
+                       ext_window=Oe, pool_kernel=pool, num_ext_heads=delta, lam=lam, beta=beta,
+                       budget=B, n_counts=n_bf, layers_done=layer, head_budget=1, ada_floor=a)
+        assert r["out_idx"].shape[2] == bf["out_idx"].shape[1] == oracle.head_capacity(params, B)
+        assert (r["out_idx"][0] == bf["out_idx"]).all()
+        n_bf = bf["n"]
+        assert (oracle.state_fields(state, T)["n"][0].astype(np.int64) == n_bf).all()
+
+
+@pytest.mark.parametrize("seed", [31, 32])
+def test_adaptive_fill_with_floor_one_is_the_uniform_fill(seed):
+    wl = synth.small_workload(seqlens=(300, 200), layers=3, budget=64, seed=seed)
+    p_u = oracle.OracleParams.from_workload(wl)
+    p_a = oracle.OracleParams.from_workload(wl, head_budget=1, ada_floor=1.0)
+    assert oracle.head_capacity(p_a, wl.budget) == wl.budget
+    su, sa = oracle.new_state(wl.batch, wl.max_seqlen), oracle.new_state(wl.batch, wl.max_seqlen)
+    for x in synth.make_layers(wl, 3):
+        ru = oracle.select_layer(p_u, wl.cu_seqlens, x["q_obs"], x["k"], x["v"], su, wl.budget, max_seqlen=wl.max_seqlen)
+        ra = oracle.select_layer(p_a, wl.cu_seqlens, x["q_obs"], x["k"], x["v"], sa, wl.budget, max_seqlen=wl.max_seqlen)
+        assert (ru["out_idx"] == ra["out_idx"]).all()
+        assert (su == sa).all()
+
+
+@pytest.mark.parametrize("a", [0.0, 0.3])
+def test_adaptive_fill_of_identical_heads_is_the_uniform_fill(a):
+    """Heads with identical rows rank every position the same way: the joint
+    ranking takes one position of each head in turn, so every head gets the same
+    share and the selection is the uniform one (no pooling and no cross-head
+    window, so that the rows are identical and free of ties)."""
+    T, Hq, Hkv, d, w, B = 64, 8, 4, 16, 8, 24
+    x = synth.tiny_full_inputs(41, T, Hq, Hkv, d)
+    k = x["k"].clone()
+    k[:] = k[:, :1]                                   # every KV head the same keys
+    q = x["q_full"][T - w:].clone().reshape(w, Hkv, Hq // Hkv, d)
+    q[:] = q[:, :1]                                   # every group the same queries
+    q_obs = q.reshape(1, w, Hq, d)
+    common = dict(num_q_heads=Hq, num_kv_heads=Hkv, head_dim=d, window=w, obs_window=4, ext_window=8,
+                  pool_kernel=1, num_ext_heads=0, lam=1.0, beta=0.25)
+    p_u = oracle.OracleParams(**common)
+    p_a = oracle.OracleParams(**common, head_budget=1, ada_floor=a)
+    su, sa = oracle.new_state(1, T), oracle.new_state(1, T)
+    for _ in range(2):
+        ru = _run_oracle(p_u, q_obs, k, x["v"], su, B)
+        ra = _run_oracle(p_a, q_obs, k, x["v"], sa, B)
+        cap = oracle.head_capacity(p_a, B)
+        assert cap > B
+        assert (ra["out_idx"][0, :, :B] == ru["out_idx"][0]).all()
+        assert (ra["out_idx"][0, :, B:] == -1).all()
+        assert (su == sa).all()
+
+
+def test_adaptive_fill_budget_bookkeeping():
+    """Section 4's budget is kept per layer: the heads keep H_kv * B tokens in
+    total, each at least its window, preserved tokens and own floor, at most the
+    capacity; the preserved tokens and the window are always among them."""
+    wl = synth.small_workload(seqlens=(500, 333), layers=2, budget=64, num_kv_heads=4, num_q_heads=16,
+                              num_ext_heads=1, head_budget=1, ada_floor=0.25)
+    p = oracle.OracleParams.from_workload(wl)
+    cap = oracle.head_capacity(p, wl.budget)
+    Kp = int(math.floor(np.float32(wl.beta) * wl.budget))
+    F = wl.budget - wl.window - Kp
+    own = int(math.floor(np.float32(wl.ada_floor) * F))
+    assert cap == wl.budget + (wl.num_kv_heads - 1) * (F - own)
+    st = oracle.new_state(wl.batch, wl.max_seqlen)
+    for x in synth.make_layers(wl, 2):
+        r = oracle.select_layer(p, wl.cu_seqlens, x["q_obs"], x["k"], x["v"], st, wl.budget, max_seqlen=wl.max_seqlen)
+        for b, L in enumerate(wl.seqlens):
+            counts = (r["out_idx"][b] >= 0).sum(axis=1)
+            assert counts.sum() == wl.num_kv_heads * wl.budget
+            assert (counts >= wl.window + Kp + own).all() and (counts <= cap).all()
+            for h in range(wl.num_kv_heads):
+                kept = set(r["out_idx"][b, h][r["out_idx"][b, h] >= 0].tolist())
+                assert set(range(L - wl.window, L)) <= kept
+                assert set(np.flatnonzero(r["pres"][b, h, :L - wl.window]).tolist()) <= kept

@@ -84,6 +84,19 @@ typedef struct {
                              candidate, the window part scored by its causal attention, and
                              each head keeps the top B of them (Section 4.1's top-B over
                              the T input tokens); budget >= 1 instead of >= window */
+    int   head_budget;    /* 0: every KV head keeps B tokens (default).  1: head-wise
+                             adaptive fill (the AdaKV-style allocation Section 2 names
+                             as a plug-and-play addition): each head keeps its window,
+                             its preserved tokens and the floor(ada_floor * F) best of
+                             its own other candidates by P' (F = B - w - K, K the
+                             preserved count); the layer's other H_kv * (F - that)
+                             fill slots go to the best P' over all its heads'
+                             remaining candidates together (ties: lower head, then
+                             lower position), so heads keep different numbers of
+                             tokens, H_kv * B in total.  Not available through
+                             kvec_select_layer_noalloc. */
+    float ada_floor;      /* 0..1, with head_budget = 1: the share of its fill a head
+                             ranks on its own (1 gives the uniform fill) */
 } kvec_params;
 
 /* Creates a handle and allocates its device workspace on the current device.
@@ -93,6 +106,12 @@ KVEC_API kvec_status kvec_create(const kvec_params* params, kvec_handle** out);
 
 /* Frees the workspace; waits for the handle's pending work first. */
 KVEC_API kvec_status kvec_destroy(kvec_handle* h);
+
+/* Rows per KV head of every selection output (out_idx, out_k, out_v below):
+ * budget, or with head_budget = 1 the most tokens one head can keep,
+ * budget + (H_kv - 1) * (F - floor(ada_floor * F)).  -1 if params or budget are
+ * invalid.  Host only; needs no device. */
+KVEC_API int kvec_output_capacity(const kvec_params* params, int budget);
 
 /* Bytes of coverage state per sequence (Section 4.2's counters n_t).  The
  * caller allocates batch * kvec_state_bytes(max_seqlen) bytes of device memory.
@@ -118,9 +137,10 @@ KVEC_API kvec_status kvec_reset(kvec_handle* h, void* coverage_state, int batch,
  *   coverage_state  device, batch states (kvec_state_bytes each); read and updated.
  *   budget B: tokens kept per KV head, the w window tokens included; B >= w
  *          (with all_positions = 1 nothing is kept by rule and B >= 1).
- *   out_idx device int32 [batch][H_kv][B]: kept positions (0-based within the
- *          sequence), ascending; -1 after the last one when L_s < B.
- *   out_k, out_v device bf16 [batch][H_kv][B][d]: gathered rows, zero padded.
+ *   out_idx device int32 [batch][H_kv][C]: kept positions (0-based within the
+ *          sequence), ascending; -1 after a head's last one.  C is
+ *          kvec_output_capacity(params, B): B for the uniform fill.
+ *   out_k, out_v device bf16 [batch][H_kv][C][d]: gathered rows, zero padded.
  * When L_s <= B every token is kept.  All device pointers must be 16-byte aligned. */
 KVEC_API kvec_status kvec_select_layer(kvec_handle* h, int batch,
                               const int32_t* cu_seqlens_host, const int32_t* cu_seqlens_dev,

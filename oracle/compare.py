@@ -9,12 +9,17 @@ Tolerances (bf16 inputs, fp32 accumulation on the GPU, fp64 in the oracle):
   within that tolerance of the selection threshold (the tie band), for the final
   fill and for the preserved set.  A head whose cross-head choice sits on a sigma
   near-tie is compared only for validity.
+* with the head-wise adaptive fill (f0 given) a head's fill has two thresholds,
+  its own f0-th key and the joint threshold over every head's remaining
+  candidates; a near-tie at the joint one can move a slot from one head to
+  another, so per-head list lengths are checked against their bounds and the
+  total over heads against the oracle's.
 * given the GPU's own indices, the gathered K/V rows and the coverage-state
   update must be bit-exact.
 """
 from __future__ import annotations
 
-from typing import Dict, List
+from typing import Dict, List, Optional
 
 import numpy as np
 
@@ -35,14 +40,30 @@ def _threshold_band(key: np.ndarray, cand: np.ndarray, k: int, tol: float):
     return thr, tol * (abs(thr) + np.abs(key[cand]).mean())
 
 
+def _joint_band(orc: Dict[str, np.ndarray], b: int, Lc: int, f0: int, extras: int, tol: float):
+    """Adaptive fill: the oracle's joint threshold (the extras-th largest key among
+    every head's candidates left after its own best f0) and its tie band."""
+    pool = []
+    for h in range(orc["out_idx"].shape[1]):
+        key = orc["Pprime"][b, h, :Lc]
+        free = np.sort(key[~orc["pres"][b, h, :Lc].astype(bool)])[::-1]
+        pool.append(free[f0:])
+    return _threshold_band(np.concatenate(pool), np.arange(sum(x.size for x in pool)), extras, tol)
+
+
 def check_layer(gpu: Dict[str, np.ndarray], orc: Dict[str, np.ndarray], seqlens, window: int, budget: int,
-                Kp: int, num_ext_heads: int, tol: float = TOL) -> List[str]:
+                Kp: int, num_ext_heads: int, tol: float = TOL, f0: Optional[int] = None) -> List[str]:
     """Returns a list of human-readable mismatches (empty when the layer passes).
 
     window: the tail kept unconditionally (w, or 0 when every position is a
-    candidate); the candidates are [0, L - window)."""
+    candidate); the candidates are [0, L - window).  f0: the fill slots a head
+    ranks itself under the head-wise adaptive fill (None for the uniform fill)."""
     errs: List[str] = []
     H = orc["out_idx"].shape[1]
+    F = budget - window - Kp
+    ada = f0 is not None
+    own = f0 if ada else F
+    extras = H * (F - own)
     for b, L in enumerate(seqlens):
         Lc = L - window
         if Lc > 0:
@@ -72,12 +93,23 @@ def check_layer(gpu: Dict[str, np.ndarray], orc: Dict[str, np.ndarray], seqlens,
             lo, hi = order[num_ext_heads - 1], order[num_ext_heads]
             if hi - lo <= tol * max(abs(hi), 1e-30):
                 ambiguous = {h for h in range(H) if abs(sig[h] - lo) <= tol * abs(lo) or abs(sig[h] - hi) <= tol * abs(hi)}
+        joint = (None, 0.0)
+        if ada and L > budget:
+            joint = _joint_band(orc, b, L - window, own, extras, tol)
+            g_tot = int((gpu["out_idx"][b] >= 0).sum())
+            o_tot = int((orc["out_idx"][b] >= 0).sum())
+            if g_tot != o_tot:
+                errs.append(f"seq {b}: {g_tot} kept rows over the heads, the oracle keeps {o_tot}")
         for h in range(H):
             gi = gpu["out_idx"][b, h]
             oi = orc["out_idx"][b, h]
             g_sel = gi[gi >= 0]
             o_sel = oi[oi >= 0]
-            if g_sel.size != o_sel.size or not np.all(np.diff(g_sel) > 0) or np.any(g_sel >= L):
+            if ada and L > budget:
+                size_ok = budget - F + own <= g_sel.size <= budget - F + own + extras
+            else:
+                size_ok = g_sel.size == o_sel.size
+            if not size_ok or not np.all(np.diff(g_sel) > 0) or np.any(g_sel >= L):
                 errs.append(f"seq {b} head {h}: invalid index list (size {g_sel.size} vs {o_sel.size})")
                 continue
             if np.any(gi[g_sel.size:] != -1):
@@ -101,12 +133,17 @@ def check_layer(gpu: Dict[str, np.ndarray], orc: Dict[str, np.ndarray], seqlens,
             pres = orc["pres"][b, h, :Lc].astype(bool)
             thr_p, band_p = _threshold_band(P, cand, Kp, tol)
             key = orc["Pprime"][b, h, :Lc]
-            thr_f, band_f = _threshold_band(key, cand[~pres], budget - window - Kp, tol)
+            thr_f, band_f = _threshold_band(key, cand[~pres], own, tol)
+            thr_j, band_j = joint
             bad = []
             for t in diff:
+                if t >= Lc:   # a window position: reported above
+                    bad.append(t)
+                    continue
                 near_fill = thr_f is not None and abs(key[t] - thr_f) <= band_f
+                near_joint = thr_j is not None and abs(key[t] - thr_j) <= band_j
                 near_pres = thr_p is not None and abs(P[t] - thr_p) <= band_p
-                if not (near_fill or near_pres):
+                if not (near_fill or near_joint or near_pres):
                     bad.append(t)
             if bad:
                 errs.append(f"seq {b} head {h}: {len(bad)} kept positions differ outside the tie band, e.g. {bad[:5]}")

@@ -173,7 +173,20 @@ kvec_status validate_params(const kvec_params* p) {
         return fail(KVEC_ERR_INVALID_ARG, "need max_batch >= 1 and 1 <= max_seqlen <= 131072");
     if (p->max_layers < 1 || p->max_layers > 255)
         return fail(KVEC_ERR_INVALID_ARG, "max_layers must be in [1, 255]");
+    if (p->head_budget != 0 && p->head_budget != 1) return fail(KVEC_ERR_INVALID_ARG, "head_budget must be 0 or 1");
+    if (p->head_budget && !(p->ada_floor >= 0.f && p->ada_floor <= 1.f))
+        return fail(KVEC_ERR_INVALID_ARG, "ada_floor must be in [0, 1]");
     return KVEC_OK;
+}
+
+// Preserved tokens K, fill F = B - wk - K and the fill a head ranks itself.
+void budget_split(const kvec_params& p, int budget, int* Kp, int* F, int* f0) {
+    const int wk = p.all_positions ? 0 : p.window;
+    int k = (int)floor((double)p.beta * (double)budget);
+    if (k > budget - wk) k = budget - wk;
+    *Kp = k;
+    *F = budget - wk - k;
+    *f0 = p.head_budget ? (int)floor((double)p.ada_floor * (double)*F) : *F;
 }
 
 kvec_status set_device(kvec_handle* h, int* prev) {
@@ -243,10 +256,10 @@ Geometry make_geometry(const kvec_handle* h, int batch, int budget, int tiles, i
     G.batch = batch;
     G.budget = budget;
     G.wk = p.all_positions ? 0 : p.window;
-    int Kp = (int)floor((double)p.beta * (double)budget);
-    if (Kp > budget - G.wk) Kp = budget - G.wk;
-    G.Kp = Kp;
-    G.k2 = budget - G.wk - Kp;
+    budget_split(p, budget, &G.Kp, &G.k2, &G.f0);
+    G.ada = p.head_budget;
+    G.extras = p.num_kv_heads * (G.k2 - G.f0);
+    G.cap = budget + (p.num_kv_heads - 1) * (G.k2 - G.f0);
     G.total_tiles = tiles;
     G.win_tiles = chunks;
     G.HG = p.num_kv_heads < kWinHeadsPerCta ? p.num_kv_heads : kWinHeadsPerCta;
@@ -410,6 +423,16 @@ kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* io
             h->prog_nodes.emplace_back(node, prev_select);
             prev_select = node;
         }
+        if (G.ada) {
+            se = launch_ada(G, io, sc, sl, h->s_chain, h->prio_hi, n);
+            if (se != cudaSuccess) return cuda_fail(se, "adaptive fill launch");
+            if (h->capturing) {
+                cudaGraphNode_t node = captured_tail(h->s_chain);
+                if (!node) return fail(KVEC_ERR_CUDA, "adaptive fill: no captured node");
+                h->prog_nodes.emplace_back(node, prev_select);
+                prev_select = node;
+            }
+        }
         KV_CHECK(cudaEventRecord(h->ev_sel[l], h->s_chain));
         KV_CHECK(cudaStreamWaitEvent(h->s_gather, h->ev_sel[l], 0));
         timed_launch(h, 4, h->s_gather, [&] { launch_gather(G, io, sl, h->s_gather); });
@@ -481,6 +504,15 @@ size_t kvec_state_bytes(int max_seqlen) {
     return round_up(16 + ns + 4 * words, 16);
 }
 
+int kvec_output_capacity(const kvec_params* params, int budget) {
+    if (validate_params(params) != KVEC_OK) return -1;
+    const int wk = params->all_positions ? 0 : params->window;
+    if (budget < 1 || budget < wk) return -1;
+    int Kp, F, f0;
+    budget_split(*params, budget, &Kp, &F, &f0);
+    return budget + (params->num_kv_heads - 1) * (F - f0);
+}
+
 kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
     if (!out) return fail(KVEC_ERR_INVALID_ARG, "out is NULL");
     *out = nullptr;
@@ -516,6 +548,7 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
         {(void**)&h->sc.nbuf, MB * round_up((size_t)p.max_seqlen, 16)},
         {(void**)&h->sc.err, sizeof(int)},
         {(void**)&h->sc.keys_sel, MB * Hkv * ML * sizeof(uint32_t)},
+        {(void**)&h->sc.jkeys, p.head_budget ? MB * Hkv * ML * sizeof(uint32_t) : 0},
     };
     for (int k = 0; k < kScoreBufs; ++k) {
         Scratch& b = h->score_buf[k];
@@ -556,6 +589,7 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
     for (Scratch& b : h->score_buf) {
         b.keys = h->sc.keys;
         b.keys_sel = h->sc.keys_sel;
+        b.jkeys = h->sc.jkeys;
         b.nbuf = h->sc.nbuf;
         b.err = h->sc.err;
     }
@@ -826,6 +860,8 @@ kvec_status kvec_select_layer_noalloc(const kvec_params* params, int batch, cons
                                       void* out_k, void* out_v, kvec_stream_t stream) {
     kvec_status s = validate_params(params);
     if (s != KVEC_OK) return s;
+    if (params->head_budget)
+        return fail(KVEC_ERR_UNSUPPORTED, "the head-wise adaptive fill needs a handle (kvec_create)");
     // A stack handle carries the geometry; its vectors stay empty and nothing is allocated.
     kvec_handle tmp;
     tmp.p = *params;

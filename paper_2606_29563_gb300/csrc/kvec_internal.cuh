@@ -28,6 +28,10 @@ struct Geometry {
     int ML;            // max_seqlen: row stride of per-position workspace arrays
     int words;         // ceil(ML / 32)
     int batch, budget, Kp, k2;
+    int ada;           // 1: head-wise adaptive fill (a head ranks f0 of its k2 fill slots itself)
+    int f0;            // fill slots a head takes by its own ranking (k2 for the uniform fill)
+    int extras;        // fill slots ranked over all heads of a sequence together: Hkv * (k2 - f0)
+    int cap;           // rows per KV head of the outputs: budget + (Hkv - 1) * (k2 - f0)
     int total_tiles;   // sum over sequences of ceil(L_s / kTileT)
     int win_tiles;     // sum over sequences of ceil((L_s - wk) / kTileT): candidate tiles
     int HG, NG;        // KV heads per window CTA, window CTAs per candidate tile
@@ -59,6 +63,7 @@ struct Scratch {
     float2* rowstat;      // [max_batch][Hkv][R]    (row max in log2 units, softmax denominator), for inspection
     uint32_t* keys;       // [max_batch][Hkv][ML]   radix-select keys of the heads kernel
     uint32_t* keys_sel;   // [max_batch][Hkv][ML]   radix-select keys of the select kernel
+    uint32_t* jkeys;      // [max_batch][Hkv * ML]  adaptive fill: every head's remaining fill keys, transposed
     uint8_t* nbuf;        // [max_batch][nlen]      second copy of n_t (the coverage counts alternate)
     int* err;             // device error word
 };
@@ -177,6 +182,11 @@ cudaError_t launch_select(const Geometry& g, const LayerIO& io, const Scratch& s
                           cudaStream_t st, int priority, int lcall, int ncall, bool programmatic);
 cudaError_t launch_finalize(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& last, cudaStream_t st,
                             int priority, int ncall);
+// Adaptive fill: the layer's extra fill slots over every head of a sequence,
+// ranked together, ORed into the heads' kept bits.  A programmatic dependent of
+// the layer's selection (it waits for it).
+cudaError_t launch_ada(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st,
+                       int priority, int ncall);
 // out_idx from the slot's kept-position bits, then the K/V rows.
 cudaError_t launch_decode(const DecodeIO& io, cudaStream_t st);
 void launch_gather(const Geometry& g, const LayerIO& io, const Slot& sl, cudaStream_t st);

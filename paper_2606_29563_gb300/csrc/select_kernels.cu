@@ -897,7 +897,21 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
         // The next layer's selection may be scheduled now: its staging overlaps
         // this top-k, then it waits for this grid.
         asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
-        block_topk(keys, kw, Lc, G.k2, bits, sm);
+        block_topk(keys, kw, Lc, G.f0, bits, sm);
+        if (G.ada) {
+            // Head-wise adaptive fill: the head keeps its own best f0; every other
+            // fill candidate goes to the joint ranking over the sequence's heads
+            // (ada_kernel), position t of head h at joint index h * 32 words + t,
+            // so that ties go to the lower head, then the lower position.  Thread
+            // i takes bit lane i / words of word i % words: the stores coalesce.
+            uint32_t* jk = sc.jkeys + (size_t)s * G.Hkv * G.words * 32;
+            const int kwj = G.Hkv * G.words;
+            for (int i = tid; i < 32 * G.words; i += NT) {
+                const int wd = i % G.words, b = i / G.words, t = 32 * wd + b;
+                const uint32_t key = (t < Lc && !((bits[wd] >> b) & 1u)) ? keys[key_index(t, kw)] : 0u;
+                jk[(size_t)b * kwj + (size_t)h * G.words + wd] = key;
+            }
+        }
         for (int wd = tid; wd < wordsL; wd += NT) bits[wd] |= spres[wd] | range_bits(wd, Lc, L);
     } else {
         // Every token is kept; the slice's counts still move to the next array.
@@ -920,6 +934,26 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
             for (int i = 0; t4 + i < L; ++i) nB[t4 + i] = c4[i];
         }
     }
+}
+
+// Head-wise adaptive fill, second step: the Hkv * (k2 - f0) largest of the
+// sequence's exported fill keys (every head's candidates left after its own f0,
+// ranked together) join the heads' kept positions.  The joint index h * 32 words
+// + t puts the bit of (h, t) at word h * words + t / 32 of the sequence's kept
+// rows, so the radix select ORs its winners straight into them.  Grid (batch);
+// a programmatic dependent of the layer's select_kernel.
+__global__ void __launch_bounds__(kSelectThreads) ada_kernel(Geometry G, LayerIO io, Scratch sc, Slot sl, int ncall) {
+    __shared__ TopkShared sm;
+    const int s = blockIdx.x;
+    // The next kernel on this stream (the next layer's selection or the
+    // finalize) waits for this grid itself: let it stage now.
+    asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
+    asm volatile("griddepcontrol.wait;\n" ::: "memory");
+    const int L = io.cu[s + 1] - io.cu[s];
+    const uint32_t ell0 = __ldcg(reinterpret_cast<const uint32_t*>(io.state + (size_t)s * G.state_stride));
+    if (L <= G.budget || ell0 + (uint32_t)ncall > 255u) return;   // all kept, or a refused call
+    const size_t nw = (size_t)G.Hkv * G.words;
+    block_topk(sc.jkeys + (size_t)s * nw * 32, (int)nw, (int)(32 * nw), G.extras, sl.sel + (size_t)s * nw, sm);
 }
 
 // After the last layer of a call: n_t of the state = the last count array plus
@@ -963,9 +997,10 @@ __global__ void __launch_bounds__(kSelectThreads) finalize_kernel(Geometry G, La
     }
 }
 
-// out_idx[s,h,j] = position of the j-th kept bit of (s, h) (-1 past the last);
+// out_idx[s,h,j] = position of the j-th kept bit of (s, h) (-1 past the last),
+// j < cap (the budget, or the head capacity of the adaptive fill);
 // out_k[s,h,j,:] = K[cu[s] + idx, h, :] (zeros for idx = -1); the same for V.
-// Grid (ceil(B/16), Hkv, batch), 256 threads: the block finds its 16 ranks from
+// Grid (ceil(cap/16), Hkv, batch), 256 threads: the block finds its 16 ranks from
 // a prefix count over the row's bits words, then a half-warp moves one 256-byte row.
 __global__ void __launch_bounds__(256) gather_kernel(Geometry G, LayerIO io, Slot sl) {
     __shared__ int wsum[32];
@@ -1000,8 +1035,8 @@ __global__ void __launch_bounds__(256) gather_kernel(Geometry G, LayerIO io, Slo
     __syncthreads();
     const int rloc = warp * 2 + (lane >> 4), sub = lane & 15;
     const int j = r0 + rloc;
-    if (j >= G.budget) return;
-    const size_t orow = srow * G.budget + j;
+    if (j >= G.cap) return;
+    const size_t orow = srow * G.cap + j;
     const int idx = spos[rloc];
     if (sub == 0) io.out_idx[orow] = idx;
     uint4 kv = make_uint4(0, 0, 0, 0), vv = make_uint4(0, 0, 0, 0);
@@ -1065,8 +1100,14 @@ cudaError_t launch_finalize(const Geometry& g, const LayerIO& io, const Scratch&
                        io, sc, last, ncall);
 }
 
+cudaError_t launch_ada(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st,
+                       int priority, int ncall) {
+    return launch_prio(ada_kernel, dim3(g.batch), dim3(kSelectThreads), 0, st, priority, /*programmatic=*/true, g, io,
+                       sc, sl, ncall);
+}
+
 void launch_gather(const Geometry& g, const LayerIO& io, const Slot& sl, cudaStream_t st) {
-    gather_kernel<<<dim3((g.budget + 15) / 16, g.Hkv, g.batch), 256, 0, st>>>(g, io, sl);
+    gather_kernel<<<dim3((g.cap + 15) / 16, g.Hkv, g.batch), 256, 0, st>>>(g, io, sl);
 }
 
 }  // namespace kvec

@@ -29,7 +29,7 @@ EXPORTED = ("kvec_create", "kvec_destroy", "kvec_state_bytes", "kvec_reset", "kv
             "kvec_select_layers", "kvec_debug_scores", "kvec_sync_status", "kvec_set_profiling",
             "kvec_kernel_time", "kvec_status_string", "kvec_last_error", "kvec_select_layer_noalloc",
             "kvec_select_layer_lse", "kvec_select_layers_lse", "kvec_decode_attention",
-            "kvec_noalloc_sync_status", "kvec_set_test_fault")
+            "kvec_noalloc_sync_status", "kvec_set_test_fault", "kvec_output_capacity")
 
 
 class KvecUnavailable(ImportError):
@@ -50,6 +50,7 @@ class kvec_params(ctypes.Structure):
         ("lam", ctypes.c_float), ("beta", ctypes.c_float), ("softmax_scale", ctypes.c_float),
         ("max_batch", ctypes.c_int), ("max_seqlen", ctypes.c_int), ("max_layers", ctypes.c_int),
         ("pool_mode", ctypes.c_int), ("head_criterion", ctypes.c_int), ("all_positions", ctypes.c_int),
+        ("head_budget", ctypes.c_int), ("ada_floor", ctypes.c_float),
     ]
 
 
@@ -99,6 +100,7 @@ def load() -> ctypes.CDLL:
             "kvec_decode_attention": ([_vp, i, _vp, _vp, _vp, _vp, i, _vp, _vp], st),
             "kvec_noalloc_sync_status": ([_vp], st),
             "kvec_set_test_fault": ([i], None),
+            "kvec_output_capacity": ([ctypes.POINTER(kvec_params), i], i),
         }
         for name, (args, res) in sig.items():
             fn = getattr(lib, name)
@@ -180,6 +182,14 @@ def kvec_noalloc_sync_status(stream: int = 0) -> None:
     _check(load().kvec_noalloc_sync_status(stream))
 
 
+def kvec_output_capacity(params: kvec_params, budget: int) -> int:
+    """Rows per KV head of the selection outputs (the budget for the uniform fill)."""
+    cap = int(load().kvec_output_capacity(ctypes.byref(params), int(budget)))
+    if cap < 1:
+        raise KvecError(KVEC_ERR_INVALID_ARG, "invalid parameters or budget for the output capacity")
+    return cap
+
+
 def kvec_set_test_fault(fault: int) -> None:
     """Test hook of the error path (1: window kernels give up on a withheld accumulator; 0: off)."""
     load().kvec_set_test_fault(int(fault))
@@ -218,10 +228,10 @@ def make_params(num_q_heads: int, num_kv_heads: int, head_dim: int = 128, window
                 ext_window: int = 32, pool_kernel: int = 7, num_ext_heads: int = 3, lam: float = 1.0,
                 beta: float = 0.25, softmax_scale: float = 0.0, max_batch: int = 1, max_seqlen: int = 8192,
                 max_layers: int = 32, pool_mode: int = 0, head_criterion: int = 0,
-                all_positions: int = 0) -> kvec_params:
+                all_positions: int = 0, head_budget: int = 0, ada_floor: float = 1.0) -> kvec_params:
     return kvec_params(num_q_heads, num_kv_heads, head_dim, window, obs_window, ext_window, pool_kernel,
                        num_ext_heads, lam, beta, softmax_scale, max_batch, max_seqlen, max_layers, pool_mode,
-                       head_criterion, all_positions)
+                       head_criterion, all_positions, head_budget, ada_floor)
 
 
 def params_from_workload(wl, max_batch: Optional[int] = None, max_seqlen: Optional[int] = None,
@@ -230,7 +240,8 @@ def params_from_workload(wl, max_batch: Optional[int] = None, max_seqlen: Option
                        wl.pool_kernel, wl.num_ext_heads, wl.lam, wl.beta, 0.0,
                        max_batch or wl.batch, max_seqlen or wl.max_seqlen, max_layers or max(wl.layers, 1),
                        getattr(wl, "pool_mode", 0), getattr(wl, "head_criterion", 0),
-                       getattr(wl, "all_positions", 0))
+                       getattr(wl, "all_positions", 0), getattr(wl, "head_budget", 0),
+                       getattr(wl, "ada_floor", 1.0))
 
 
 class _DeviceArray:
@@ -272,11 +283,13 @@ class KvecSelector:
         return st
 
     def alloc_outputs(self, batch: int, budget: int, device="cuda"):
+        """out_idx, out_k, out_v with kvec_output_capacity rows per head."""
         t = self._torch
         p = self.params
-        return (t.empty((batch, p.num_kv_heads, budget), dtype=t.int32, device=device),
-                t.empty((batch, p.num_kv_heads, budget, p.head_dim), dtype=t.bfloat16, device=device),
-                t.empty((batch, p.num_kv_heads, budget, p.head_dim), dtype=t.bfloat16, device=device))
+        cap = kvec_output_capacity(p, budget)
+        return (t.empty((batch, p.num_kv_heads, cap), dtype=t.int32, device=device),
+                t.empty((batch, p.num_kv_heads, cap, p.head_dim), dtype=t.bfloat16, device=device),
+                t.empty((batch, p.num_kv_heads, cap, p.head_dim), dtype=t.bfloat16, device=device))
 
     def select_layer(self, cu_host, cu_dev, q_obs, k, v, state, budget: int, outs=None, stream=None, lse=None):
         """lse: optional fp32 [batch][w][H_q] window-row log-sum-exp (kvec_select_layer_lse)."""

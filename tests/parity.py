@@ -67,6 +67,9 @@ def run_parity(wl: synth.Workload, layers: Optional[int] = None, device: str = "
     oparams = oracle.OracleParams.from_workload(wl)
     kept_tail = 0 if getattr(wl, "all_positions", 0) else wl.window
     Kp = min(int(math.floor(float(np.float32(wl.beta)) * budget)), budget - kept_tail)
+    f0 = None
+    if getattr(wl, "head_budget", 0):
+        f0 = int(math.floor(float(np.float32(wl.ada_floor)) * (budget - kept_tail - Kp)))
     cu_host = torch.tensor(wl.cu_seqlens, dtype=torch.int32)
     cu_dev = cu_host.to(device)
     state = sel.new_state(wl.batch, device)
@@ -89,7 +92,7 @@ def run_parity(wl: synth.Workload, layers: Optional[int] = None, device: str = "
                                 budget, max_seqlen=ML)
         g = dict(gdbg)
         g["out_idx"] = out_idx.cpu().numpy()
-        layer_errs = compare.check_layer(g, r, wl.seqlens, kept_tail, budget, Kp, wl.num_ext_heads, tol)
+        layer_errs = compare.check_layer(g, r, wl.seqlens, kept_tail, budget, Kp, wl.num_ext_heads, tol, f0=f0)
         layer_errs += compare.check_state_and_gather(
             g["out_idx"], _bits(out_k), _bits(out_v), _bits(inputs[l]["k"]), _bits(inputs[l]["v"]), wl.cu_seqlens,
             oracle.state_fields(before, ML), oracle.state_fields(after, ML))

@@ -60,6 +60,10 @@ BAD_PARAMS = [
     (dict(num_q_heads=72, num_kv_heads=8), kvec.KVEC_ERR_UNSUPPORTED),   # 9 x 32 rows > 256
     (dict(num_q_heads=264, num_kv_heads=33), kvec.KVEC_ERR_UNSUPPORTED),
     (dict(all_positions=2), kvec.KVEC_ERR_INVALID_ARG),
+    (dict(head_budget=2), kvec.KVEC_ERR_INVALID_ARG),
+    (dict(head_budget=1, ada_floor=-0.1), kvec.KVEC_ERR_INVALID_ARG),
+    (dict(head_budget=1, ada_floor=1.5), kvec.KVEC_ERR_INVALID_ARG),
+    (dict(head_budget=1, ada_floor=float("nan")), kvec.KVEC_ERR_INVALID_ARG),
 ]
 
 
@@ -88,6 +92,39 @@ def test_calls_on_null_handle_are_rejected(lib):
 def test_status_strings(lib):
     for code in range(6):
         assert kvec.kvec_status_string(code)
+
+
+@pytest.mark.parametrize("budget", [32, 33, 64, 128, 333, 2048])
+@pytest.mark.parametrize("head_budget,ada_floor", [(0, 1.0), (1, 0.0), (1, 0.2), (1, 0.5), (1, 1.0)])
+@pytest.mark.parametrize("all_positions", [0, 1])
+def test_output_capacity_matches_oracle(lib, budget, head_budget, ada_floor, all_positions):
+    p = kvec.make_params(num_q_heads=32, num_kv_heads=8, head_budget=head_budget, ada_floor=ada_floor,
+                         all_positions=all_positions)
+    op = oracle.OracleParams(num_q_heads=32, num_kv_heads=8, head_dim=128, window=p.window, obs_window=p.obs_window,
+                             ext_window=p.ext_window, pool_kernel=p.pool_kernel, num_ext_heads=p.num_ext_heads,
+                             beta=float(p.beta), lam=float(p.lam), head_criterion=p.head_criterion,
+                             all_positions=all_positions, head_budget=head_budget, ada_floor=float(p.ada_floor))
+    cap = kvec.kvec_output_capacity(p, budget)
+    assert cap == oracle.head_capacity(op, budget)
+    assert cap >= budget
+    if head_budget == 0 or ada_floor == 1.0:
+        assert cap == budget
+
+
+def test_output_capacity_rejects_a_budget_below_the_window(lib):
+    p = kvec.make_params(num_q_heads=32, num_kv_heads=8)
+    with pytest.raises(kvec.KvecError):
+        kvec.kvec_output_capacity(p, p.window - 1)
+
+
+def test_noalloc_refuses_the_adaptive_fill_before_cuda(lib):
+    p = kvec.make_params(num_q_heads=32, num_kv_heads=8, head_budget=1, ada_floor=0.2)
+    cu = (ctypes.c_int32 * 2)(0, 4096)
+    fake = 256
+    with pytest.raises(kvec.KvecError) as e:
+        kvec.kvec_select_layer_noalloc(p, 1, ctypes.addressof(cu), ctypes.addressof(cu), fake, fake, fake, fake,
+                                       512, fake, fake, fake, None)
+    assert e.value.status == kvec.KVEC_ERR_UNSUPPORTED
 
 
 def test_noalloc_refuses_oversize_calls_before_cuda(lib):

@@ -335,3 +335,45 @@ def test_all_positions_multi_layer_call_matches_layer_by_layer():
             assert torch.equal(x, y)
     assert torch.equal(st1, st2)
     sel.close()
+
+
+# ---- head-wise adaptive fill (a floor per head, the rest ranked over the heads) ----
+
+@pytest.mark.parametrize("kw", [dict(seqlens=(900,), ada_floor=0.25),
+                                dict(seqlens=(40, 1100, 64, 700), budget=96, ada_floor=0.2),
+                                dict(seqlens=(523,), num_q_heads=28, num_kv_heads=4, ada_floor=0.0),
+                                dict(seqlens=(640,), num_q_heads=16, num_kv_heads=8, ada_floor=0.5, budget=48),
+                                dict(seqlens=(700, 333), ada_floor=0.2, all_positions=1)])
+def test_adaptive_fill_matches_the_oracle(kw):
+    kw.setdefault("num_q_heads", 16)
+    kw.setdefault("num_kv_heads", 4)
+    _assert_parity(synth.small_workload(head_budget=1, layers=3, **kw))
+
+
+def test_adaptive_fill_with_floor_one_is_the_uniform_fill():
+    """ada_floor = 1: every head ranks its whole fill itself, so indices, K/V and
+    state equal the uniform fill's bit for bit."""
+    wl = synth.small_workload(seqlens=(1100, 300, 700), num_q_heads=16, num_kv_heads=4, layers=2, budget=96)
+    outs = []
+    for hb in (0, 1):
+        w = wl.replace(head_budget=hb, ada_floor=1.0)
+        sel = kvec.KvecSelector(kvec.params_from_workload(w))
+        cu = torch.tensor(w.cu_seqlens, dtype=torch.int32)
+        st = sel.new_state(w.batch)
+        res = [[t.cpu() for t in sel.select_layer(cu, cu.cuda(), x["q_obs"].cuda(), x["k"].cuda(), x["v"].cuda(),
+                                                  st, w.budget)] for x in synth.make_layers(w, 2)]
+        torch.cuda.synchronize()
+        outs.append((res, st.cpu()))
+        sel.close()
+    for a, b in zip(outs[0][0], outs[1][0]):
+        for x, y in zip(a, b):
+            assert torch.equal(x, y)
+    assert torch.equal(outs[0][1], outs[1][1])
+
+
+def test_adaptive_fill_llama8b_l8192_b512_first_layers():
+    _assert_parity(synth.WORKLOADS["llama8b_l8192_b512"].replace(head_budget=1, ada_floor=0.2), layers=3)
+
+
+def test_adaptive_fill_llama8b_ragged8_b256_first_layers():
+    _assert_parity(synth.WORKLOADS["llama8b_ragged8_b256"].replace(head_budget=1, ada_floor=0.2), layers=2)

@@ -108,3 +108,9 @@ def test_full_call_llama8b_l8192_b512_all_positions():
 def test_full_call_qwen7b_l16384_b2048():
     # 28 layers, 4 KV heads (group 7), the largest budget of the sweep.
     _check_full_call(synth.WORKLOADS["qwen7b_l16384_b512"].replace(budget=2048))
+
+
+def test_full_call_llama8b_l8192_b512_adaptive_fill():
+    # The joint ranking of every head's fill runs after each layer's selection
+    # on the chain stream, in the captured graph as a programmatic dependent.
+    _check_full_call(synth.WORKLOADS["llama8b_l8192_b512"].replace(head_budget=1, ada_floor=0.2))

@@ -372,34 +372,47 @@ def run_ours(args, wl):
                        "api": "kvec_select_layers_lse: window-row log-sum-exp from the caller's prefill attention",
                        "path_roofline_frac": by["layer_total"] * L_layers / (ms_lse / 1e3) / 1e9 / peak}
 
-    # The same step with every position a candidate (kvec_params.all_positions = 1:
-    # Section 4.1's top-B over the T input tokens, no retained window), own handle.
-    all_positions_variant = None
-    if args.all_positions_variant:
-        sel_ap = kvec.KvecSelector(kvec.params_from_workload(wl.replace(all_positions=1)))
-        state_ap = sel_ap.new_state(wl.batch, dev)
+    def timed_variant(wl_v, api):
+        """The same step through a handle made for the variant's parameters (own
+        outputs: the adaptive fill has more rows per head)."""
+        sel_v = kvec.KvecSelector(kvec.params_from_workload(wl_v))
+        state_v = sel_v.new_state(wl.batch, dev)
+        outs_v = [sel_v.alloc_outputs(wl.batch, wl.budget, dev) for _ in range(L_layers)]
 
-        def step_ap():
-            kvec.kvec_reset(sel_ap.handle, state_ap.data_ptr(), wl.batch, stream.cuda_stream)
-            sel_ap.select_layers(cu_host, cu_dev, qs, ks, vs, state_ap, wl.budget, outs, stream)
+        def step_v():
+            kvec.kvec_reset(sel_v.handle, state_v.data_ptr(), wl.batch, stream.cuda_stream)
+            sel_v.select_layers(cu_host, cu_dev, qs, ks, vs, state_v, wl.budget, outs_v, stream)
 
         for _ in range(max(args.warmup, 3)):
-            step_ap()
-        n_ap = min(args.steps, 500)
+            step_v()
+        n_v = min(args.steps, 500)
         torch.cuda.synchronize()
         start.record(stream)
-        for _ in range(n_ap):
-            step_ap()
+        for _ in range(n_v):
+            step_v()
         stop.record(stream)
         torch.cuda.synchronize()
-        kvec.kvec_sync_status(sel_ap.handle)
-        sel_ap.close()
-        ms_ap = max_over_ranks(start.elapsed_time(stop), dev) / n_ap
-        all_positions_variant = {
-            "metric": METRIC, "value": world * evicted_per_step / (ms_ap / 1e3), "unit": "tokens/s",
-            "ms_per_step": ms_ap, "steps": n_ap,
-            "api": "kvec_select_layers with kvec_params.all_positions = 1: top-B over every position",
-            "path_roofline_frac": by["layer_total"] * L_layers / (ms_ap / 1e3) / 1e9 / peak}
+        kvec.kvec_sync_status(sel_v.handle)
+        sel_v.close()
+        del outs_v, state_v
+        ms_v = max_over_ranks(start.elapsed_time(stop), dev) / n_v
+        return {"metric": METRIC, "value": world * evicted_per_step / (ms_v / 1e3), "unit": "tokens/s",
+                "ms_per_step": ms_v, "steps": n_v, "api": api,
+                "path_roofline_frac": by["layer_total"] * L_layers / (ms_v / 1e3) / 1e9 / peak}
+
+    # Every position a candidate (kvec_params.all_positions = 1: Section 4.1's
+    # top-B over the T input tokens, no retained window).
+    all_positions_variant = None
+    if args.all_positions_variant:
+        all_positions_variant = timed_variant(
+            wl.replace(all_positions=1), "kvec_select_layers with kvec_params.all_positions = 1: top-B over every position")
+    # Head-wise adaptive fill (kvec_params.head_budget = 1): each head ranks a
+    # fifth of its fill itself, the rest is ranked over the heads of a sequence.
+    adaptive_variant = None
+    if args.adaptive_variant:
+        adaptive_variant = timed_variant(
+            wl.replace(head_budget=1, ada_floor=0.2),
+            "kvec_select_layers with kvec_params.head_budget = 1, ada_floor = 0.2: head-wise adaptive fill")
 
     decode = run_decode(args, wl, sel, layers, outs, dev, peak) if args.decode else None
 
@@ -432,6 +445,7 @@ def run_ours(args, wl):
         "gpu_launches": gpu_launches,
         "lse_variant": lse_variant,
         "all_positions_variant": all_positions_variant,
+        "adaptive_variant": adaptive_variant,
         "decode": decode,
         "e2e": e2e,
         "other_configs": other,
@@ -703,6 +717,8 @@ def main(argv=None):
                     help="skip timing the kvec_select_layers_lse variant")
     ap.add_argument("--no-all-positions-variant", dest="all_positions_variant", action="store_false",
                     help="skip timing the top-B-over-every-position variant")
+    ap.add_argument("--no-adaptive-variant", dest="adaptive_variant", action="store_false",
+                    help="skip timing the head-wise adaptive fill (kvec_params.head_budget = 1)")
     ap.add_argument("--no-clock-probe", dest="clock_probe", action="store_false",
                     help="do not extend a short timed region by a second of steps to read the clocks")
     ap.add_argument("--no-other-configs", dest="other_configs", action="store_false",

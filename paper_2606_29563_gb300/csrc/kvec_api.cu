@@ -5,6 +5,7 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <algorithm>
 #include <atomic>
 #include <mutex>
 #include <string>
@@ -260,6 +261,8 @@ Geometry make_geometry(const kvec_handle* h, int batch, int budget, int tiles, i
     G.ada = p.head_budget;
     G.extras = p.num_kv_heads * (G.k2 - G.f0);
     G.cap = budget + (p.num_kv_heads - 1) * (G.k2 - G.f0);
+    G.jpool = G.ada ? std::min(G.extras, 32 * G.words) : 0;
+    G.jstride = p.num_kv_heads * G.ML + 32;
     G.total_tiles = tiles;
     G.win_tiles = chunks;
     G.HG = p.num_kv_heads < kWinHeadsPerCta ? p.num_kv_heads : kWinHeadsPerCta;
@@ -548,7 +551,9 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
         {(void**)&h->sc.nbuf, MB * round_up((size_t)p.max_seqlen, 16)},
         {(void**)&h->sc.err, sizeof(int)},
         {(void**)&h->sc.keys_sel, MB * Hkv * ML * sizeof(uint32_t)},
-        {(void**)&h->sc.jkeys, p.head_budget ? MB * Hkv * ML * sizeof(uint32_t) : 0},
+        {(void**)&h->sc.jkeys, p.head_budget ? MB * (Hkv * ML + 32) * sizeof(uint32_t) : 0},
+        {(void**)&h->sc.jpos, p.head_budget ? MB * (Hkv * ML + 32) * sizeof(int32_t) : 0},
+        {(void**)&h->sc.jbits, p.head_budget ? MB * (Hkv * ML + 32) / 32 * sizeof(uint32_t) : 0},
     };
     for (int k = 0; k < kScoreBufs; ++k) {
         Scratch& b = h->score_buf[k];
@@ -590,6 +595,8 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
         b.keys = h->sc.keys;
         b.keys_sel = h->sc.keys_sel;
         b.jkeys = h->sc.jkeys;
+        b.jpos = h->sc.jpos;
+        b.jbits = h->sc.jbits;
         b.nbuf = h->sc.nbuf;
         b.err = h->sc.err;
     }

@@ -32,6 +32,8 @@ struct Geometry {
     int f0;            // fill slots a head takes by its own ranking (k2 for the uniform fill)
     int extras;        // fill slots ranked over all heads of a sequence together: Hkv * (k2 - f0)
     int cap;           // rows per KV head of the outputs: budget + (Hkv - 1) * (k2 - f0)
+    int jpool;         // adaptive fill: candidates a head offers the joint ranking, min(extras, 32 * words)
+    int jstride;       // adaptive fill: per-sequence stride of the joint candidate arrays
     int total_tiles;   // sum over sequences of ceil(L_s / kTileT)
     int win_tiles;     // sum over sequences of ceil((L_s - wk) / kTileT): candidate tiles
     int HG, NG;        // KV heads per window CTA, window CTAs per candidate tile
@@ -63,7 +65,9 @@ struct Scratch {
     float2* rowstat;      // [max_batch][Hkv][R]    (row max in log2 units, softmax denominator), for inspection
     uint32_t* keys;       // [max_batch][Hkv][ML]   radix-select keys of the heads kernel
     uint32_t* keys_sel;   // [max_batch][Hkv][ML]   radix-select keys of the select kernel
-    uint32_t* jkeys;      // [max_batch][Hkv * ML]  adaptive fill: every head's remaining fill keys, transposed
+    uint32_t* jkeys;      // [max_batch][jstride]   adaptive fill: the heads' joint candidates' keys, transposed
+    int32_t* jpos;        // [max_batch][jstride]   their positions (candidate i belongs to head i / jpool)
+    uint32_t* jbits;      // [max_batch][jstride / 32] winners of the joint ranking, one bit per candidate
     uint8_t* nbuf;        // [max_batch][nlen]      second copy of n_t (the coverage counts alternate)
     int* err;             // device error word
 };
@@ -112,7 +116,7 @@ __device__ __forceinline__ bool locate_item(int batch, int gi, CountFn count, in
     return false;
 }
 
-__device__ __forceinline__ int tiles_of(int L) { return (L + kTileT - 1) / kTileT; }
+__host__ __device__ __forceinline__ int tiles_of(int L) { return (L + kTileT - 1) / kTileT; }
 
 // ---------------------------------------------------------------- launchers
 

@@ -774,11 +774,12 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
     const int wordsL = (L + 31) >> 5;
     const int kw = key_stride(G);
     const bool cached = scores_in_smem(G.ML) && L > G.budget;
-    // Shared memory: bits[words] | preserved bits[words] | union[words] | keys |
-    // P row | I row (P and I 16-byte aligned for float4 stores).
+    // Shared memory: bits[words] | preserved bits[words] | union[words] |
+    // adaptive-fill candidate bits[words] | keys | P row | I row (P and I
+    // 16-byte aligned for float4 stores).
     uint32_t* spres = bits + G.words;
     uint32_t* suni = spres + G.words;
-    const size_t sp_off = ((size_t)3 * G.words + (keys_in_smem(G.ML) ? 32 * (size_t)kw : 0) + 3) & ~(size_t)3;
+    const size_t sp_off = ((size_t)4 * G.words + (keys_in_smem(G.ML) ? 32 * (size_t)kw : 0) + 3) & ~(size_t)3;
     float* sP = reinterpret_cast<float*>(bits + sp_off);
     float* sI = sP + G.ML;
     const size_t row = (size_t)s * G.Hkv + h;
@@ -792,6 +793,7 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
     for (int wd = tid; wd < G.words; wd += NT) {
         bits[wd] = 0u;
         spres[wd] = __ldcg(&pres[wd]);
+        suni[G.words + wd] = 0u;   // adaptive-fill candidate bits
     }
     if (cached) {
         for (int t4 = 4 * tid; t4 < Lc; t4 += 4 * NT) {
@@ -851,7 +853,7 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
     if (select) {
         // P' of the last layer of a call is kept for inspection (kvec_debug_scores).
         float* Pp = lcall + 1 == ncall ? sl.Pprime + row * G.ML : nullptr;
-        uint32_t* keys = keys_in_smem(G.ML) ? suni + G.words : sc.keys_sel + row * G.ML;
+        uint32_t* keys = keys_in_smem(G.ML) ? suni + 2 * G.words : sc.keys_sel + row * G.ML;
         const float* Pr = cached ? sP : P;
         const float* Ir = cached ? sI : I;
         // coverage = n_t / (l + 1) as n_t times the rounded reciprocal: a divide
@@ -899,17 +901,49 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
         asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
         block_topk(keys, kw, Lc, G.f0, bits, sm);
         if (G.ada) {
-            // Head-wise adaptive fill: the head keeps its own best f0; every other
-            // fill candidate goes to the joint ranking over the sequence's heads
-            // (ada_kernel), position t of head h at joint index h * 32 words + t,
-            // so that ties go to the lower head, then the lower position.  Thread
-            // i takes bit lane i / words of word i % words: the stores coalesce.
-            uint32_t* jk = sc.jkeys + (size_t)s * G.Hkv * G.words * 32;
-            const int kwj = G.Hkv * G.words;
-            for (int i = tid; i < 32 * G.words; i += NT) {
-                const int wd = i % G.words, b = i / G.words, t = 32 * wd + b;
-                const uint32_t key = (t < Lc && !((bits[wd] >> b) & 1u)) ? keys[key_index(t, kw)] : 0u;
-                jk[(size_t)b * kwj + (size_t)h * G.words + wd] = key;
+            // Head-wise adaptive fill: the head keeps its own best f0.  A head
+            // can win at most extras = Hkv * (k2 - f0) slots of the joint ranking
+            // over the sequence's heads, and only its best ones: it offers its
+            // nC best remaining candidates (ties to the lower position), in
+            // position order, as candidates h * jpool + r of the joint ranking
+            // (ada_kernel), so that ties there go to the lower head, then the
+            // lower position.  The preserved tokens are exactly Kp of the Lc
+            // candidates, so Lc - Kp - f0 remain.
+            uint32_t* cbits = suni + G.words;   // after the union words: see select_smem_bytes
+            for (int wd = tid; wd < wordsL; wd += NT) {
+                uint32_t a = bits[wd];
+                while (a) {
+                    const int t = 32 * wd + __ffs(a) - 1;
+                    a &= a - 1u;
+                    keys[key_index(t, kw)] = 0u;
+                }
+            }
+            __syncthreads();
+            const int nC = min(G.jpool, Lc - G.Kp - G.f0);
+            block_topk(keys, kw, Lc, nC, cbits, sm);
+            uint32_t* jk = sc.jkeys + (size_t)s * G.jstride;
+            int32_t* jp = sc.jpos + (size_t)s * G.jstride;
+            const int kwj = (G.Hkv * G.jpool + 31) >> 5;
+            const int wpt = (wordsL + NT - 1) / NT;
+            const int w_lo = min(tid * wpt, wordsL), w_hi = min(w_lo + wpt, wordsL);
+            int mine = 0;
+            for (int wd = w_lo; wd < w_hi; ++wd) mine += __popc(cbits[wd]);
+            int total;
+            int r = block_exclusive_sum(mine, sm.wsum, total);
+            for (int wd = w_lo; wd < w_hi; ++wd) {
+                uint32_t c = cbits[wd];
+                while (c) {
+                    const int t = 32 * wd + __ffs(c) - 1;
+                    c &= c - 1u;
+                    const int i = h * G.jpool + r++;
+                    jk[key_index(i, kwj)] = keys[key_index(t, kw)];
+                    jp[i] = t;
+                }
+            }
+            for (int r2 = total + tid; r2 < G.jpool; r2 += NT) {
+                const int i = h * G.jpool + r2;
+                jk[key_index(i, kwj)] = 0u;
+                jp[i] = -1;
             }
         }
         for (int wd = tid; wd < wordsL; wd += NT) bits[wd] |= spres[wd] | range_bits(wd, Lc, L);
@@ -936,15 +970,22 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
     }
 }
 
-// Head-wise adaptive fill, second step: the Hkv * (k2 - f0) largest of the
-// sequence's exported fill keys (every head's candidates left after its own f0,
-// ranked together) join the heads' kept positions.  The joint index h * 32 words
-// + t puts the bit of (h, t) at word h * words + t / 32 of the sequence's kept
-// rows, so the radix select ORs its winners straight into them.  Grid (batch);
-// a programmatic dependent of the layer's select_kernel.
+constexpr int kAdaSmemKeys = 40960;   // joint candidates staged in shared memory (160 KB)
+__host__ __device__ inline bool ada_keys_in_smem(const Geometry& g) { return g.Hkv * g.jpool <= kAdaSmemKeys; }
+
+// Head-wise adaptive fill, second step: the extras = Hkv * (k2 - f0) best of
+// the candidates the sequence's heads offered (select_kernel), ranked together
+// (larger P', then lower head, then lower position), join their heads' kept
+// positions.  Grid (batch); a programmatic dependent of the layer's
+// select_kernel.
 __global__ void __launch_bounds__(kSelectThreads) ada_kernel(Geometry G, LayerIO io, Scratch sc, Slot sl, int ncall) {
     __shared__ TopkShared sm;
-    const int s = blockIdx.x;
+    const int s = blockIdx.x, tid = threadIdx.x, NT = blockDim.x;
+    const int n = G.Hkv * G.jpool, nwords = (n + 31) >> 5;
+    uint32_t* jb = sc.jbits + (size_t)s * (G.jstride / 32);
+    // The previous layer's ada_kernel completed before this layer's selection
+    // started, so the winner bits can be cleared before the wait.
+    for (int wd = tid; wd < nwords; wd += NT) jb[wd] = 0u;
     // The next kernel on this stream (the next layer's selection or the
     // finalize) waits for this grid itself: let it stage now.
     asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
@@ -952,8 +993,35 @@ __global__ void __launch_bounds__(kSelectThreads) ada_kernel(Geometry G, LayerIO
     const int L = io.cu[s + 1] - io.cu[s];
     const uint32_t ell0 = __ldcg(reinterpret_cast<const uint32_t*>(io.state + (size_t)s * G.state_stride));
     if (L <= G.budget || ell0 + (uint32_t)ncall > 255u) return;   // all kept, or a refused call
-    const size_t nw = (size_t)G.Hkv * G.words;
-    block_topk(sc.jkeys + (size_t)s * nw * 32, (int)nw, (int)(32 * nw), G.extras, sl.sel + (size_t)s * nw, sm);
+    // The radix select sweeps the keys once per digit: stage them in shared
+    // memory when they fit (the launch gave ada_smem_bytes).
+    const uint32_t* keys = sc.jkeys + (size_t)s * G.jstride;
+    if (ada_keys_in_smem(G)) {
+        extern __shared__ __align__(16) uint32_t skeys[];
+        for (int i = 4 * tid; i < 32 * nwords; i += 4 * NT)
+            *reinterpret_cast<uint4*>(skeys + i) = __ldcg(reinterpret_cast<const uint4*>(keys + i));
+        keys = skeys;
+    }
+    __syncthreads();
+    block_topk(keys, nwords, n, G.extras, jb, sm);
+    // A thread takes a word of winner bits and loads the 32 positions behind it
+    // at once (independent 16-byte loads, not one L2 round trip per winner).
+    const int32_t* jp = sc.jpos + (size_t)s * G.jstride;
+    uint32_t* sel = sl.sel + (size_t)s * G.Hkv * G.words;
+    for (int wd = tid; wd < nwords; wd += NT) {
+        const uint32_t b = jb[wd];
+        if (!b) continue;
+        int4 pos[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) pos[j] = __ldcg(reinterpret_cast<const int4*>(jp + 32 * wd) + j);
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+            if (!((b >> j) & 1u)) continue;
+            const int4 q = pos[j >> 2];
+            const int t = (j & 3) == 0 ? q.x : (j & 3) == 1 ? q.y : (j & 3) == 2 ? q.z : q.w;
+            atomicOr(&sel[(size_t)((32 * wd + j) / G.jpool) * G.words + (t >> 5)], 1u << (t & 31));
+        }
+    }
 }
 
 // After the last layer of a call: n_t of the state = the last count array plus
@@ -1052,7 +1120,7 @@ __global__ void __launch_bounds__(256) gather_kernel(Geometry G, LayerIO io, Slo
 }  // namespace
 
 size_t select_smem_bytes(const Geometry& g) {
-    const size_t head = ((size_t)3 * g.words + (keys_in_smem(g.ML) ? 32 * (size_t)key_stride(g) : 0) + 3) & ~(size_t)3;
+    const size_t head = ((size_t)4 * g.words + (keys_in_smem(g.ML) ? 32 * (size_t)key_stride(g) : 0) + 3) & ~(size_t)3;
     return sizeof(uint32_t) * (head + (scores_in_smem(g.ML) ? 2 * (size_t)g.ML : 0));
 }
 
@@ -1064,15 +1132,18 @@ cudaError_t configure_select() {
     const int need = (int)(sizeof(uint32_t) * (kSmemKeys / 32 + 32 * ((kSmemKeys / 32) | 1)));
     // The select kernel also keeps the preserved bits and caches P and I rows
     // up to kSmemScores positions.
-    const int need_sel_keys = need + (int)(sizeof(uint32_t) * (2 * (kSmemKeys / 32) + 4));
+    const int need_sel_keys = need + (int)(sizeof(uint32_t) * (3 * (kSmemKeys / 32) + 4));
     const int need_sel_scores =
-        (int)(sizeof(uint32_t) * (3 * (kSmemScores / 32) + 32 * ((kSmemScores / 32) | 1) + 2 * kSmemScores + 64));
+        (int)(sizeof(uint32_t) * (4 * (kSmemScores / 32) + 32 * ((kSmemScores / 32) | 1) + 2 * kSmemScores + 64));
     const int need_sel = need_sel_keys > need_sel_scores ? need_sel_keys : need_sel_scores;
     cudaError_t e = cudaFuncSetAttribute(heads_topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, need);
     if (e == cudaSuccess)
         e = cudaFuncSetAttribute(heads_pool_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kPoolSmemBytes);
     if (e == cudaSuccess)
         e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, need_sel);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(ada_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)(sizeof(uint32_t) * (kAdaSmemKeys + 32)));
     return e;
 }
 
@@ -1102,8 +1173,10 @@ cudaError_t launch_finalize(const Geometry& g, const LayerIO& io, const Scratch&
 
 cudaError_t launch_ada(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st,
                        int priority, int ncall) {
-    return launch_prio(ada_kernel, dim3(g.batch), dim3(kSelectThreads), 0, st, priority, /*programmatic=*/true, g, io,
-                       sc, sl, ncall);
+    // The staged keys: 32 * ceil(n / 32) words, the transposed layout's extent.
+    const size_t smem = ada_keys_in_smem(g) ? sizeof(uint32_t) * 32 * (((size_t)g.Hkv * g.jpool + 31) / 32) : 0;
+    return launch_prio(ada_kernel, dim3(g.batch), dim3(kSelectThreads), smem, st, priority, /*programmatic=*/true, g,
+                       io, sc, sl, ncall);
 }
 
 void launch_gather(const Geometry& g, const LayerIO& io, const Slot& sl, cudaStream_t st) {

@@ -451,7 +451,7 @@ struct TileArgs {
     Scratch sc;
     Slot sl;
     const int* cu;
-    int Npad, kst, nacc, units, fault;   // units: W, the (sequence, head group, tile) triples
+    int Npad, kst, nacc, units, fault;
 };
 
 struct __align__(8) TileBars {
@@ -466,48 +466,35 @@ __host__ __device__ inline size_t tile_smem_bytes(int Npad, int kst) {
     return 1024 + (size_t)kst * kKTileBytes + 2 * (size_t)Npad * 256 + 4 * 2 * 256 * sizeof(float) + sizeof(TileBars);
 }
 
-// The work of a launch is the flat list of (sequence s, head group ng, candidate
-// tile j) triples, sequence-major, then head group, then tile: W = NG * sum_s
-// ntile(s).  CTA b of Gc owns the contiguous range [start(b), start(b + 1)),
-// start(b) = b*q + min(b, r) with W = q*Gc + r, so every CTA has q or q + 1
-// tiles whatever the sequence lengths; its units are the runs of at most T
-// consecutive tiles of one (sequence, head group) inside the range.
+// Unit u -> sequence s, first candidate tile j0 of the unit, its tile count nt,
+// head group ng, global candidate tile of j0.
 struct TileUnit {
     int s, j0, nt, ng, tg0, L, Lc, row0;
 };
 
-__device__ __forceinline__ void tile_range(int W, int b, int Gc, int& f0, int& f1) {
-    const int q = W / Gc, r = W - q * Gc;
-    f0 = b * q + min(b, r);
-    f1 = f0 + q + (b < r ? 1 : 0);
-}
-
-// The unit that starts at flat index f (< f1): sequence, head group, first tile
-// j0, tile count nt, global candidate tile of j0; advances f past it.
-__device__ __forceinline__ bool next_tile_unit(const Geometry& G, const int* cu, int T, int& f, int f1, TileUnit& w) {
-    if (f >= f1) return false;
+__device__ __forceinline__ bool decode_tile_unit(const Geometry& G, const int* cu, int T, int u, TileUnit& w) {
     int base = 0, tbase = 0;
     for (int b = 0; b < G.batch; ++b) {
         const int c0 = __ldg(&cu[b]), c1 = __ldg(&cu[b + 1]);
         const int Lc = c1 - c0 - G.wk;
         const int ntile = Lc > 0 ? (Lc + kTileT - 1) / kTileT : 0;
-        if (f < base + ntile * G.NG) {
-            const int local = f - base;
+        const int ngrp = (ntile + T - 1) / T;
+        if (u < base + ngrp * G.NG) {
+            const int local = u - base;
+            const int tgi = local / G.NG;
             w.s = b;
-            w.ng = local / ntile;
-            w.j0 = local - w.ng * ntile;
-            w.nt = min(T, min(f1 - f, ntile - w.j0));
+            w.ng = local - tgi * G.NG;
+            w.j0 = tgi * T;
+            w.nt = min(T, ntile - w.j0);
             w.tg0 = tbase + w.j0;
             w.L = c1 - c0;
             w.Lc = Lc;
             w.row0 = c0 + w.j0 * kTileT;
-            f += w.nt;
             return true;
         }
-        base += ntile * G.NG;
+        base += ngrp * G.NG;
         tbase += ntile;
     }
-    f = f1;
     return false;
 }
 
@@ -591,8 +578,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
     float* rsm = reinterpret_cast<float*>(sQ + 2 * (size_t)Npad * 256);   // [4][2][256]
     TileBars* bars = reinterpret_cast<TileBars*>(rsm + 4 * 2 * 256);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    int fbeg, fend;
-    tile_range(units, blockIdx.x, gridDim.x, fbeg, fend);
+    const int u0 = blockIdx.x, ustep = gridDim.x;
 
     if (threadIdx.x == 32) {
         for (int i = 0; i < kst; ++i) {
@@ -628,9 +614,9 @@ __global__ void __launch_bounds__(kWinThreads, 1)
             int kfills[kMaxKStages] = {0, 0, 0, 0, 0, 0};
             int qfills[2] = {0, 0};
             bool stop = false;
-            int f = fbeg;
-            TileUnit tu;
-            while (!stop && next_tile_unit(G, cu_dev, T, f, fend, tu)) {
+            for (int u = u0; u < units && !stop; u += ustep) {
+                TileUnit tu;
+                decode_tile_unit(G, cu_dev, T, u, tu);
                 const int h0 = tu.ng * G.HG, nh = min(G.HG, G.Hkv - h0);
                 for (int hh = 0; hh < nh && !stop; ++hh) {
                     const int h = h0 + hh;
@@ -682,9 +668,9 @@ __global__ void __launch_bounds__(kWinThreads, 1)
             int qi = 0, ki = 0, first = 1;
             int cnt[4] = {0, 0, 0, 0};
             bool stop = false;
-            int f = fbeg;
-            TileUnit tu;
-            while (!stop && next_tile_unit(G, cu_dev, T, f, fend, tu)) {
+            for (int u = u0; u < units && !stop; u += ustep) {
+                TileUnit tu;
+                decode_tile_unit(G, cu_dev, T, u, tu);
                 const int nh = min(G.HG, G.Hkv - tu.ng * G.HG);
                 for (int hh = 0; hh < nh && !stop; ++hh) {
                     const int qs = qi & 1;
@@ -755,10 +741,10 @@ __global__ void __launch_bounds__(kWinThreads, 1)
         };
         int k = 0;
         bool failed = false;
-        int f = fbeg;
-        TileUnit tu;
-        while (!failed && next_tile_unit(G, cu_dev, T, f, fend, tu)) {
-            if (grp >= tu.nt) continue;   // the unit has fewer tiles than this group's
+        for (int u = u0; u < units && !failed; u += ustep) {
+            TileUnit tu;
+            decode_tile_unit(G, cu_dev, T, u, tu);
+            if (grp >= tu.nt) continue;   // this group's tile is past the sequence's last
             const int h0 = tu.ng * G.HG, nh = min(G.HG, G.Hkv - h0);
             const int t = (tu.j0 + grp) * kTileT + tok;
             const int qmin = t - (tu.L - G.w);
@@ -883,6 +869,16 @@ bool tile_variant_fits(const Geometry& g) {
     return (nacc - 1) * Npad + maxcol <= 512;
 }
 
+// Units of the tile-owning variant: groups of T candidate tiles per sequence and head group.
+int tile_units_of(const Geometry& g, const int* cu_host, int T) {
+    int units = 0;
+    for (int b = 0; b < g.batch; ++b) {
+        const int Lc = cu_host[b + 1] - cu_host[b] - g.wk;
+        const int nt = Lc > 0 ? (Lc + kTileT - 1) / kTileT : 0;
+        units += (nt + T - 1) / T * g.NG;
+    }
+    return units;
+}
 
 cudaError_t launch_window_tiles(const ScorePlan& sp, const Geometry& g, const LayerIO& io, const Scratch& sc,
                                 const Slot& sl, cudaStream_t st, bool after_own_launch) {
@@ -894,7 +890,7 @@ cudaError_t launch_window_tiles(const ScorePlan& sp, const Geometry& g, const La
     a.Npad = npad_of(g.R);
     a.nacc = a.Npad <= 128 ? 4 : 2;   // nacc * Npad <= 512 TMEM columns
     a.kst = tile_kst_for(a.Npad);
-    a.units = units_of(g);
+    a.units = tile_units_of(g, g.cu_host, a.nacc);
     a.fault = test_fault() == 1 ? 1 : 0;
     const size_t smem = tile_smem_bytes(a.Npad, a.kst);
     const int usable = sp.num_sms > 2 * kWinReserveSms ? sp.num_sms - kWinReserveSms : sp.num_sms;
@@ -923,12 +919,13 @@ cudaError_t launch_window_tiles(const ScorePlan& sp, const Geometry& g, const La
 cudaError_t launch_window(const ScorePlan& sp, const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl,
                           cudaStream_t st, bool after_own_launch) {
     if (g.win_tiles == 0) return cudaSuccess;
-    // The tile-owning variant where it applies and every usable SM gets at
-    // least T tiles (with fewer, the per-tile kernel's CTAs finish sooner).
+    // The tile-owning variant where it applies and its units still give every
+    // usable SM one (it has T times fewer units than the per-tile kernel, whose
+    // CTAs finish sooner when there are few tiles).
     if (tile_variant_fits(g)) {
         const int T = npad_of(g.R) <= 128 ? 4 : 2;
         const int usable = sp.num_sms > 2 * kWinReserveSms ? sp.num_sms - kWinReserveSms : sp.num_sms;
-        if (units_of(g) >= T * usable) return launch_window_tiles(sp, g, io, sc, sl, st, after_own_launch);
+        if (tile_units_of(g, g.cu_host, T) >= usable) return launch_window_tiles(sp, g, io, sc, sl, st, after_own_launch);
     }
     WinArgs a{};
     a.G = g;

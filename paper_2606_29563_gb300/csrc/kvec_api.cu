@@ -74,6 +74,7 @@ struct kvec_handle {
     size_t state_stride = 0, n_off = 16, union_off = 0;
     void* ws = nullptr;
     size_t ws_bytes = 0;
+    int* claims = nullptr;   // [max_layers] the score launches' chunk counters (zero between launches)
     Scratch sc{};
     Scratch score_buf[kScoreBufs]{};   // segment partials and row statistics, one per layer in flight
     Slot slots[kSlots]{};
@@ -280,9 +281,9 @@ kvec_status run_layer_sequential(kvec_handle* h, const Geometry& G, const LayerI
     ScorePlan plan;
     cudaError_t se = plan_score(G, io, h->sc, h->num_sms, &plan);
     if (se != cudaSuccess) return cuda_fail(se, "score kernel tensor maps");
-    se = launch_score(plan, st, false);
+    se = launch_score(plan, h->claims, st, false);
     if (se != cudaSuccess) return cuda_fail(se, "score kernel launch");
-    se = launch_rowstat(plan, G, io, h->sc, st, /*programmatic=*/true, /*after_score=*/true);
+    se = launch_rowstat(plan, G, io, h->sc, h->claims, st, /*programmatic=*/true, /*after_score=*/true);
     if (se != cudaSuccess) return cuda_fail(se, "row statistics launch");
     se = launch_window(plan, G, io, h->sc, h->slots[0], st, false);
     if (se != cudaSuccess) return cuda_fail(se, "window kernel launch");
@@ -369,7 +370,7 @@ kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* io
         // l - 1's (it reads none of its results); the event wait above stays a
         // full dependency (restore_full_edges when captured).
         if (!io.lse) {
-            timed_launch(h, 0, h->s_score, [&] { se = launch_score(plan, h->s_score, l > 0); });
+            timed_launch(h, 0, h->s_score, [&] { se = launch_score(plan, h->claims + l, h->s_score, l > 0); });
             if (se != cudaSuccess) return cuda_fail(se, "score kernel launch");
             if (h->capturing) {
                 cudaGraphNode_t node = captured_tail(h->s_score);
@@ -393,7 +394,7 @@ kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* io
         // overwrite was last read by layer l - 2's window grid, which this
         // layer's score grid waited for.  So consecutive window grids overlap.
         se = io.lse ? launch_rowstat_lse(G, io, sc, h->s_win, l > 0)
-                    : launch_rowstat(plan, G, io, sc, h->s_win, l > 0, /*after_score=*/false);
+                    : launch_rowstat(plan, G, io, sc, h->claims + l, h->s_win, l > 0, /*after_score=*/false);
         if (se != cudaSuccess) return cuda_fail(se, "row statistics launch");
         if (h->capturing) {
             cudaGraphNode_t node = captured_tail(h->s_win);
@@ -554,6 +555,7 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
         {(void**)&h->sc.jkeys, p.head_budget ? MB * (Hkv * ML + 32) * sizeof(uint32_t) : 0},
         {(void**)&h->sc.jpos, p.head_budget ? MB * (Hkv * ML + 32) * sizeof(int32_t) : 0},
         {(void**)&h->sc.jbits, p.head_budget ? MB * (Hkv * ML + 32) / 32 * sizeof(uint32_t) : 0},
+        {(void**)&h->claims, (size_t)p.max_layers * sizeof(int)},
     };
     for (int k = 0; k < kScoreBufs; ++k) {
         Scratch& b = h->score_buf[k];
@@ -899,6 +901,7 @@ kvec_status kvec_select_layer_noalloc(const kvec_params* params, int batch, cons
     const size_t NGv = (Hkv + HGv - 1) / HGv;
     Part parts[] = {
         {(void**)&tmp.sc.err, sizeof(int)},                   // error word, first: see noalloc_setup
+        {(void**)&tmp.claims, sizeof(int)},
         {(void**)&tmp.sc.nbuf, nb * round_up((size_t)params->max_seqlen, 16)},
         {(void**)&tmp.sc.segpart, nt * Hkv * R * sizeof(float2)},
         {(void**)&tmp.slots[0].wpart, nt * NGv * (size_t)params->obs_window * kTileT * sizeof(float)},

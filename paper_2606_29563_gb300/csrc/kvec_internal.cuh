@@ -125,6 +125,7 @@ struct ScorePlan {
     CUtensorMap kmap, qmap;
     alignas(16) unsigned char args[512];
     int grid, threads, mb;   // mb: 128-row M-blocks per KV head
+    int chunk;               // work items per claim of the score kernel (segment boundaries of its partials)
     size_t smem;
     int num_sms;             // SMs of the device (persistent grids are sized from it)
 };
@@ -132,14 +133,17 @@ cudaError_t plan_score(const Geometry& g, const LayerIO& io, const Scratch& sc, 
 // after_own_launch: the stream's previous kernel is the previous layer's launch
 // of the same kernel (the multi-stream layer pipeline); the launch may then
 // overlap it (programmatic stream serialization), as it reads none of its results.
-cudaError_t launch_score(const ScorePlan& plan, cudaStream_t st, bool after_own_launch);
+// claim: an int in device memory, zero before the launch (the CTAs count the
+// work chunks they claim on it; the layer's launch_rowstat sets it back to
+// zero once the score grid has completed); a distinct one for every launch in flight.
+cudaError_t launch_score(const ScorePlan& plan, int* claim, cudaStream_t st, bool after_own_launch);
 // (m_r, Z_r) from the score launch's partials.  programmatic: a programmatic
 // dependent of the stream's previous kernel.  after_score: that kernel is this
 // layer's score launch, waited for (griddepcontrol.wait) before the partials
 // are read; without it the partials must come through a full dependency and the
 // previous kernel (the layer pipeline's previous window grid) is not waited for.
 cudaError_t launch_rowstat(const ScorePlan& plan, const Geometry& g, const LayerIO& io, const Scratch& sc,
-                           cudaStream_t st, bool programmatic, bool after_score);
+                           int* claim, cudaStream_t st, bool programmatic, bool after_score);
 // (m_r, Z_r) = (lse * log2(e), 1) from the caller's log-sum-exp (io.lse), in place
 // of the score and row-statistics launches.  programmatic: as for launch_rowstat
 // without after_score (it reads only the caller's input).

@@ -3,8 +3,10 @@
 // row r of KV head h, the row max m_r of s = <q_r, k_t> * scale (log2 units)
 // and Z_r = sum_t 2^(s_rt - m_r), causal on the window part.
 //
-// Persistent, warp-specialised, one CTA per SM; a CTA walks a contiguous range
-// of work items (sequence s, KV head h, 128-token tile j):
+// Persistent, warp-specialised, one CTA per SM; CTAs claim chunks of
+// consecutive work items (sequence s, KV head h, 128-token tile j)
+// from a per-launch counter, so a CTA that starts late (its SM held by other
+// kernels) takes fewer chunks instead of delaying the launch:
 //   warp 0      TMA producer: the KV head's g*w query rows (once per (s,h)) and
 //               a ring of 128-token K tiles, both 128-byte swizzled;
 //   warp 1      one thread issues tcgen05.mma (M = 128 query rows per M-block,
@@ -14,9 +16,11 @@
 //               128 columns of the item: tcgen05.ld of its logits, their sum
 //               of 2^(s - max), merged online into the thread's running
 //               (max, sum) of the CTA's contiguous segment of (s, h).
-// At the end of a segment the groups merge in shared memory and the CTA
-// writes one (max, sum) partial per row, keyed by the segment's first item;
-// rowstat_kernel then merges the partials of a (s, h) into (m_r, Z_r).
+// At the end of a segment (a run of one (s, h) inside a chunk) the groups merge
+// in shared memory and the CTA writes one (max, sum) partial per row, keyed by
+// the segment's first item; rowstat_kernel then merges the partials of a (s, h)
+// into (m_r, Z_r).  The segments are fixed by the chunk boundaries, not by which
+// CTA claimed a chunk, so the results do not depend on the schedule.
 // The window kernel recomputes the logits with these statistics.
 #include <cudaTypedefs.h>
 
@@ -74,14 +78,10 @@ struct ItemWalker {
     }
 };
 
-// CTA b of G owns items [start(b), start(b+1)) with start(b) = b*q + min(b, r), W = q*G + r.
-__device__ __forceinline__ int range_start(int b, int W, int G) {
-    const int q = W / G, r = W % G;
-    return b * q + min(b, r);
-}
-
 constexpr int kScoreReserveSms = 8;      // SMs a score launch leaves to the other kernels
-constexpr int kScoreItemsPerCta = 8;     // fewest (sequence, head, tile) items a score CTA takes
+constexpr int kChunkLarge = 12;          // (sequence, head, tile) items per claim when there are enough
+constexpr int kChunkSmall = 8;           // items per claim otherwise
+constexpr int kChunkSlots = 4;           // claimed chunks in flight inside a CTA
 
 struct ScoreArgs {
     Geometry G;
@@ -89,6 +89,8 @@ struct ScoreArgs {
     Scratch sc;
     int W;        // total work items
     int kst;      // K ring depth
+    int* claim;   // the launch's chunk counter, zero before the launch
+    int chunk;    // items per claim
 };
 
 constexpr int kEpiWarps = 16;
@@ -99,9 +101,12 @@ struct __align__(8) Barriers {
     uint64_t k_full[kKStages], k_empty[kKStages];
     uint64_t q_full, q_empty;
     uint64_t acc_full[4], acc_empty[4];
+    uint64_t c_full[kChunkSlots], c_empty[kChunkSlots];
     uint64_t mma_done;
     uint32_t tmem_base;
     volatile int abort_flag;
+    volatile int chunk[kChunkSlots];   // claimed chunk (-1: no more work)
+    volatile int cur_chunk[2];         // the epilogue's current chunk (-2: gave up), double-buffered
     float2 xf[512];            // a segment's (max, sum) per epilogue group and row, merged at its end
 };
 
@@ -124,6 +129,9 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     const Geometry G = A.G;
     const Scratch sc = A.sc;
     const int W = A.W, kst = A.kst;
+    const int chunk_items = A.chunk;
+    const int nchunks = (W + chunk_items - 1) / chunk_items;
+    int* const claim = A.claim;
     const int* const cu_dev = A.cu;
     const int Rpad = 128 * MB, R = G.R;
     uint8_t* sQ = smem;                                   // 2 halves x Rpad rows x 128 B
@@ -132,8 +140,6 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     constexpr int NB = 4 / MB;                             // TMEM accumulator buffers
-    const int Gc = gridDim.x;
-    const int i0 = range_start(blockIdx.x, W, Gc), i1 = range_start(blockIdx.x + 1, W, Gc);
 
     if (warp == 0 && lane == 0) {
         ptx::prefetch_tensormap(&kmap);
@@ -153,6 +159,10 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
             ptx::mbar_init(&bars->acc_full[b], 1);
             ptx::mbar_init(&bars->acc_empty[b], 4 * MB);  // one arrival per warp of the group
         }
+        for (int c = 0; c < kChunkSlots; ++c) {
+            ptx::mbar_init(&bars->c_full[c], 1);
+            ptx::mbar_init(&bars->c_empty[c], 2);         // the MMA issuer and the epilogue's leader
+        }
         ptx::mbar_init(&bars->mma_done, 1);
         bars->abort_flag = 0;
         ptx::fence_barrier_init();
@@ -170,33 +180,53 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         // ------------------------------------------------------------ TMA producer
         if (lane == 0) {
             const uint64_t policy = ptx::policy_evict_normal();   // the window kernel reads K again
-            int prev_sh = -1, qloads = 0, issued = 0;
-            ItemWalker p;
-            p.init(cu_dev, G.batch, G.Hkv, i0);
-            for (int i = i0, it = 0; i < i1 && !bars->abort_flag; ++i, ++it, p.next()) {
-                const int sh = p.s * G.Hkv + p.h;
-                if (sh != prev_sh) {
-                    if (qloads > 0 && !ptx::mbar_wait(&bars->q_empty, (qloads - 1) & 1)) {
-                        raise_abort(bars, sc.err);
-                        break;
-                    }
-                    ptx::mbar_arrive_expect_tx(&bars->q_full, 2u * R * 128u);
-                    ptx::tma_load_4d(sQ, &qmap, &bars->q_full, 0, p.h * G.g, 0, p.s);
-                    ptx::tma_load_4d(sQ + Rpad * 128, &qmap, &bars->q_full, 64, p.h * G.g, 0, p.s);
-                    ++qloads;
-                    prev_sh = sh;
-                }
-                const int st = it % kst, n = it / kst;
-                if (n > 0 && !ptx::mbar_wait(&bars->k_empty[st], (n - 1) & 1)) {
+            int qloads = 0, issued = 0, it = 0, di = 0;
+            for (;;) {
+                // Claim a chunk and hand it to the MMA issuer and the epilogue.
+                const int c = bars->abort_flag ? nchunks : atomicAdd(claim, 1);
+                const int ds = di % kChunkSlots, nd = di / kChunkSlots;
+                if (nd > 0 && !ptx::mbar_wait(&bars->c_empty[ds], (nd - 1) & 1)) {
                     raise_abort(bars, sc.err);
                     break;
                 }
-                uint8_t* dst = sK + st * kKStageBytes;
-                const int row = p.row0 + p.j * kTileT;
-                ptx::mbar_arrive_expect_tx(&bars->k_full[st], (uint32_t)kKStageBytes);
-                ptx::tma_load_3d(dst, &kmap, &bars->k_full[st], 0, p.h, row, policy);
-                ptx::tma_load_3d(dst + kKHalfBytes, &kmap, &bars->k_full[st], 64, p.h, row, policy);
-                ++issued;
+                bars->chunk[ds] = c < nchunks ? c : -1;
+                ptx::mbar_arrive(&bars->c_full[ds]);
+                ++di;
+                if (c >= nchunks) break;
+                const int i0 = c * chunk_items, i1 = min(W, i0 + chunk_items);
+                int prev_sh = -1;   // the query rows are loaded again at every chunk's start
+                ItemWalker p;
+                p.init(cu_dev, G.batch, G.Hkv, i0);
+                bool stop = false;
+                for (int i = i0; i < i1; ++i, ++it, p.next()) {
+                    const int sh = p.s * G.Hkv + p.h;
+                    if (sh != prev_sh) {
+                        if (qloads > 0 && !ptx::mbar_wait(&bars->q_empty, (qloads - 1) & 1)) {
+                            stop = true;
+                            break;
+                        }
+                        ptx::mbar_arrive_expect_tx(&bars->q_full, 2u * R * 128u);
+                        ptx::tma_load_4d(sQ, &qmap, &bars->q_full, 0, p.h * G.g, 0, p.s);
+                        ptx::tma_load_4d(sQ + Rpad * 128, &qmap, &bars->q_full, 64, p.h * G.g, 0, p.s);
+                        ++qloads;
+                        prev_sh = sh;
+                    }
+                    const int st = it % kst, n = it / kst;
+                    if (n > 0 && !ptx::mbar_wait(&bars->k_empty[st], (n - 1) & 1)) {
+                        stop = true;
+                        break;
+                    }
+                    uint8_t* dst = sK + st * kKStageBytes;
+                    const int row = p.row0 + p.j * kTileT;
+                    ptx::mbar_arrive_expect_tx(&bars->k_full[st], (uint32_t)kKStageBytes);
+                    ptx::tma_load_3d(dst, &kmap, &bars->k_full[st], 0, p.h, row, policy);
+                    ptx::tma_load_3d(dst + kKHalfBytes, &kmap, &bars->k_full[st], 64, p.h, row, policy);
+                    ++issued;
+                }
+                if (stop) {
+                    raise_abort(bars, sc.err);
+                    break;
+                }
             }
             // Drain: every issued copy lands before the CTA may exit (stage st was
             // filled ceil((issued - st) / kst) times).
@@ -211,41 +241,57 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         if (lane == 0) {
             const uint32_t idesc = ptx::idesc_bf16_f32(128, kTileT);
             const uint32_t sQa = ptx::smem_u32(sQ), sKa = ptx::smem_u32(sK);
-            int prev_sh = -1, qk = 0;
-            ItemWalker p;
-            p.init(cu_dev, G.batch, G.Hkv, i0);
-            for (int i = i0, it = 0; i < i1 && !bars->abort_flag; ++i, ++it, p.next()) {
-                const int sh = p.s * G.Hkv + p.h;
-                if (sh != prev_sh) {
-                    if (!ptx::mbar_wait(&bars->q_full, qk & 1)) {
-                        raise_abort(bars, sc.err);
-                        break;
-                    }
-                    ++qk;
-                    prev_sh = sh;
-                }
-                const int st = it % kst, n = it / kst;
-                const int buf = it % NB, nb = it / NB;
-                if (!ptx::mbar_wait(&bars->k_full[st], n & 1) ||
-                    (nb > 0 && !ptx::mbar_wait(&bars->acc_empty[buf], (nb - 1) & 1))) {
+            int qk = 0, it = 0, di = 0;
+            bool stop = false;
+            while (!stop && !bars->abort_flag) {
+                const int ds = di % kChunkSlots;
+                if (!ptx::mbar_wait(&bars->c_full[ds], (di / kChunkSlots) & 1)) {
                     raise_abort(bars, sc.err);
                     break;
                 }
-                ptx::tc_fence_after();
-                const uint32_t kst = sKa + st * kKStageBytes;
-                for (int m = 0; m < MB; ++m) {
-                    const uint32_t d = tmem + (uint32_t)(buf * 128 * MB + m * 128);
-#pragma unroll
-                    for (int kk = 0; kk < 8; ++kk) {
-                        const int half = kk >> 2, kin = kk & 3;
-                        const uint64_t ad = ptx::smem_desc_k_sw128(sQa + half * Rpad * 128 + m * 16384 + kin * 32);
-                        const uint64_t bd = ptx::smem_desc_k_sw128(kst + half * kKHalfBytes + kin * 32);
-                        ptx::mma_bf16(d, ad, bd, idesc, kk > 0 ? 1u : 0u);
+                const int c = bars->chunk[ds];
+                ptx::mbar_arrive(&bars->c_empty[ds]);
+                ++di;
+                if (c < 0) break;
+                const int i0 = c * chunk_items, i1 = min(W, i0 + chunk_items);
+                int prev_sh = -1;
+                ItemWalker p;
+                p.init(cu_dev, G.batch, G.Hkv, i0);
+                for (int i = i0; i < i1 && !bars->abort_flag; ++i, ++it, p.next()) {
+                    const int sh = p.s * G.Hkv + p.h;
+                    if (sh != prev_sh) {
+                        if (!ptx::mbar_wait(&bars->q_full, qk & 1)) {
+                            raise_abort(bars, sc.err);
+                            stop = true;
+                            break;
+                        }
+                        ++qk;
+                        prev_sh = sh;
                     }
+                    const int st = it % kst, n = it / kst;
+                    const int buf = it % NB, nb = it / NB;
+                    if (!ptx::mbar_wait(&bars->k_full[st], n & 1) ||
+                        (nb > 0 && !ptx::mbar_wait(&bars->acc_empty[buf], (nb - 1) & 1))) {
+                        raise_abort(bars, sc.err);
+                        stop = true;
+                        break;
+                    }
+                    ptx::tc_fence_after();
+                    const uint32_t kst = sKa + st * kKStageBytes;
+                    for (int m = 0; m < MB; ++m) {
+                        const uint32_t d = tmem + (uint32_t)(buf * 128 * MB + m * 128);
+    #pragma unroll
+                        for (int kk = 0; kk < 8; ++kk) {
+                            const int half = kk >> 2, kin = kk & 3;
+                            const uint64_t ad = ptx::smem_desc_k_sw128(sQa + half * Rpad * 128 + m * 16384 + kin * 32);
+                            const uint64_t bd = ptx::smem_desc_k_sw128(kst + half * kKHalfBytes + kin * 32);
+                            ptx::mma_bf16(d, ad, bd, idesc, kk > 0 ? 1u : 0u);
+                        }
+                    }
+                    ptx::mma_commit(&bars->k_empty[st]);
+                    ptx::mma_commit(&bars->acc_full[buf]);
+                    if (i + 1 >= i1 || p.last_of_head()) ptx::mma_commit(&bars->q_empty);
                 }
-                ptx::mma_commit(&bars->k_empty[st]);
-                ptx::mma_commit(&bars->acc_full[buf]);
-                if (i + 1 >= i1 || p.last_of_head()) ptx::mma_commit(&bars->q_empty);
             }
             ptx::mma_commit(&bars->mma_done);
         }
@@ -328,55 +374,77 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
             merge(seg_m, seg_z, make_float2(mu, (z4[0] + z4[1]) + (z4[2] + z4[3])));
         };
 
-        ItemWalker p;
-        p.init(cu_dev, G.batch, G.Hkv, i0);
-        for (int i = i0, it = 0; i < i1; ++i, ++it, p.next()) {
-            const int sh = p.s * G.Hkv + p.h;
-            if (sh != cur_sh) {
-                if (cur_sh >= 0) flush_segment();
-                cur_sh = sh;
-                seg_m = -INFINITY;
-                seg_z = 0.f;
-                seg_first = i;
+        int it = 0, di = 0;
+        for (;;) {
+            // The epilogue's leader takes the next claimed chunk; the barrier
+            // hands it to every epilogue thread (-1: no more work, -2: gave up).
+            const int ds = di % kChunkSlots;
+            if (threadIdx.x == 64) {
+                int c = -2;
+                if (ptx::mbar_wait(&bars->c_full[ds], (di / kChunkSlots) & 1)) {
+                    c = bars->chunk[ds];
+                    ptx::mbar_arrive(&bars->c_empty[ds]);
+                } else {
+                    raise_abort(bars, sc.err);
+                }
+                bars->cur_chunk[di & 1] = c;
             }
-            if (it % NB != grp || aborted) continue;   // another group's item (or keep walking for the barriers)
-            const int nb = it / NB;
-            int ok = 1;
-            if (lane == 0) {
-                ok = !bars->abort_flag && ptx::mbar_wait(&bars->acc_full[grp], nb & 1);
-                if (!ok) raise_abort(bars, sc.err);
+            ptx::named_bar_sync(1, kEpiThreads);
+            const int c = bars->cur_chunk[di & 1];
+            ++di;
+            if (c < 0) break;
+            const int i0 = c * chunk_items, i1 = min(W, i0 + chunk_items);
+            ItemWalker p;
+            p.init(cu_dev, G.batch, G.Hkv, i0);
+            for (int i = i0; i < i1; ++i, ++it, p.next()) {
+                const int sh = p.s * G.Hkv + p.h;
+                if (sh != cur_sh) {
+                    if (cur_sh >= 0) flush_segment();
+                    cur_sh = sh;
+                    seg_m = -INFINITY;
+                    seg_z = 0.f;
+                    seg_first = i;
+                }
+                if (it % NB != grp || aborted) continue;   // another group's item (or keep walking for the barriers)
+                const int nb = it / NB;
+                int ok = 1;
+                if (lane == 0) {
+                    ok = !bars->abort_flag && ptx::mbar_wait(&bars->acc_full[grp], nb & 1);
+                    if (!ok) raise_abort(bars, sc.err);
+                }
+                ok = __shfl_sync(0xffffffffu, ok, 0);
+                if (!ok) {
+                    aborted = true;
+                    continue;
+                }
+                ptx::tc_fence_after();
+                const uint32_t taddr = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(grp * 128 * MB + m * 128);
+                const int L = p.L;
+                const int t0 = p.j * kTileT;
+                const int last = vrow ? min(L - 1, L - G.w + q) : -1;   // causal on the window part
+                const int nvalid = max(0, min(kTileT, last - t0 + 1));
+                // Four 32-column chunks; the next chunk's TMEM load is in flight while
+                // this one is reduced.
+                float va[32], vb[32];
+                ptx::tmem_ld32(taddr, va);
+                ptx::tmem_wait_ld();
+                ptx::tmem_ld32(taddr + 32, vb);
+                chunk(va, nvalid);
+                ptx::tmem_wait_ld();
+                ptx::tmem_ld32(taddr + 64, va);
+                chunk(vb, nvalid - 32);
+                ptx::tmem_wait_ld();
+                ptx::tmem_ld32(taddr + 96, vb);
+                chunk(va, nvalid - 64);
+                ptx::tmem_wait_ld();
+                ptx::tc_fence_before();
+                __syncwarp();
+                if (lane == 0) ptx::mbar_arrive(&bars->acc_empty[grp]);   // the accumulator is in registers
+                chunk(vb, nvalid - 96);
             }
-            ok = __shfl_sync(0xffffffffu, ok, 0);
-            if (!ok) {
-                aborted = true;
-                continue;
-            }
-            ptx::tc_fence_after();
-            const uint32_t taddr = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(grp * 128 * MB + m * 128);
-            const int L = p.L;
-            const int t0 = p.j * kTileT;
-            const int last = vrow ? min(L - 1, L - G.w + q) : -1;   // causal on the window part
-            const int nvalid = max(0, min(kTileT, last - t0 + 1));
-            // Four 32-column chunks; the next chunk's TMEM load is in flight while
-            // this one is reduced.
-            float va[32], vb[32];
-            ptx::tmem_ld32(taddr, va);
-            ptx::tmem_wait_ld();
-            ptx::tmem_ld32(taddr + 32, vb);
-            chunk(va, nvalid);
-            ptx::tmem_wait_ld();
-            ptx::tmem_ld32(taddr + 64, va);
-            chunk(vb, nvalid - 32);
-            ptx::tmem_wait_ld();
-            ptx::tmem_ld32(taddr + 96, vb);
-            chunk(va, nvalid - 64);
-            ptx::tmem_wait_ld();
-            ptx::tc_fence_before();
-            __syncwarp();
-            if (lane == 0) ptx::mbar_arrive(&bars->acc_empty[grp]);   // the accumulator is in registers
-            chunk(vb, nvalid - 96);
+            if (cur_sh >= 0) flush_segment();   // a chunk's end closes its last segment
+            cur_sh = -1;
         }
-        if (cur_sh >= 0) flush_segment();
     }
 
     // ---------------------------------------------------------------- teardown
@@ -387,11 +455,12 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     if (warp == 1) ptx::tmem_dealloc(tmem, kTmemCols);
 }
 
-// (m_r, Z_r) of every row of (s, h) from the score CTAs' segment partials: one
-// at the head's first item, then one at every score CTA's first item inside
-// the head's range of items.  Grid (Hkv, batch), one thread per row.
-__global__ void __launch_bounds__(256) rowstat_kernel(Geometry G, Scratch sc, const int* __restrict__ cu, int W,
-                                                      int Gc, int wait_prev) {
+// (m_r, Z_r) of every row of (s, h) from the score kernel's segment partials:
+// one at the head's first item, then one at every chunk boundary inside the
+// head's range of items, merged in item order.  Grid (Hkv, batch), one thread
+// per row.
+__global__ void __launch_bounds__(256) rowstat_kernel(Geometry G, Scratch sc, const int* __restrict__ cu,
+                                                      int chunk, int* claim, int wait_prev) {
     // The window launch that follows may start; it waits for this grid.
     if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
     // wait_prev: a programmatic dependent of the score launch right before it on
@@ -400,16 +469,17 @@ __global__ void __launch_bounds__(256) rowstat_kernel(Geometry G, Scratch sc, co
     // previous kernel (if a programmatic predecessor at all) is not waited for.
     if (wait_prev) asm volatile("griddepcontrol.wait;\n" ::: "memory");
     const int h = blockIdx.x, s = blockIdx.y, r = threadIdx.x;
+    // The score grid has completed: its chunk counter is free for the next launch.
+    if (h == 0 && s == 0 && r == 0) *claim = 0;
     if (r >= G.R) return;
     int ib = 0;
     for (int b = 0; b < s; ++b) ib += tiles_of(__ldg(&cu[b + 1]) - __ldg(&cu[b])) * G.Hkv;
     const int nt = tiles_of(__ldg(&cu[s + 1]) - __ldg(&cu[s]));
     ib += h * nt;
     const int iend = ib + nt;
-    const int qW = W / Gc, rW = W % Gc;
-    const int cta = ib < rW * (qW + 1) ? ib / (qW + 1) : rW + (ib - rW * (qW + 1)) / qW;
     float M = -INFINITY, Z = 0.f;
-    int next = ib, b = cta + 1;
+    // Segment starts: the head's first item, then every chunk boundary inside it.
+    int next = ib, bnd = (ib / chunk + 1) * chunk;
     while (next < iend) {
         float2 pz[16];
 #pragma unroll
@@ -417,8 +487,8 @@ __global__ void __launch_bounds__(256) rowstat_kernel(Geometry G, Scratch sc, co
             pz[k] = make_float2(-INFINITY, 0.f);
             if (next < iend) {
                 pz[k] = __ldcg(&sc.segpart[(size_t)next * G.R + r]);
-                next = b * qW + min(b, rW);
-                ++b;
+                next = bnd;
+                bnd += chunk;
             }
         }
 #pragma unroll
@@ -528,14 +598,17 @@ cudaError_t plan_score(const Geometry& g, const LayerIO& io, const Scratch& sc, 
     a.sc = sc;
     a.W = g.total_tiles * g.Hkv;
     a.kst = kstages_for(g);
-    // At least kScoreItemsPerCta items per CTA (the CTA's set-up and merge are paid
-    // once and its K stream overlaps the epilogue), on at most all but
-    // kScoreReserveSms SMs: the rest run the window, heads and selection kernels of
-    // neighbouring layers, which cannot share an SM with a score CTA.
+    // At most all but kScoreReserveSms SMs (the rest run the window, heads and
+    // selection kernels of neighbouring layers, which cannot share an SM with a
+    // score CTA) and at most one CTA per chunk.
     const int usable = num_sms > 2 * kScoreReserveSms ? num_sms - kScoreReserveSms : num_sms;
-    int per_cta = (a.W + usable - 1) / usable;
-    if (per_cta < kScoreItemsPerCta) per_cta = kScoreItemsPerCta;
-    plan->grid = (a.W + per_cta - 1) / per_cta;
+    // Chunks of kChunkLarge items when that still gives every usable SM one, else
+    // of kChunkSmall (measured: larger chunks reload the query rows less often,
+    // smaller ones leave fewer SMs idle on small layers).
+    a.chunk = a.W / kChunkLarge >= usable ? kChunkLarge : kChunkSmall;
+    const int nchunks = (a.W + a.chunk - 1) / a.chunk;
+    plan->grid = nchunks < usable ? nchunks : usable;
+    plan->chunk = a.chunk;
     plan->threads = kScoreThreads;
     plan->mb = mblocks(g);
     plan->smem = smem_bytes_for(g);
@@ -544,8 +617,8 @@ cudaError_t plan_score(const Geometry& g, const LayerIO& io, const Scratch& sc, 
 }
 
 cudaError_t launch_rowstat(const ScorePlan& plan, const Geometry& g, const LayerIO& io, const Scratch& sc,
-                           cudaStream_t st, bool programmatic, bool after_score) {
-    const ScoreArgs& a = *reinterpret_cast<const ScoreArgs*>(plan.args);
+                           int* claim, cudaStream_t st, bool programmatic, bool after_score) {
+    (void)plan;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(g.Hkv, g.batch);
     cfg.blockDim = dim3(256);
@@ -555,7 +628,7 @@ cudaError_t launch_rowstat(const ScorePlan& plan, const Geometry& g, const Layer
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = programmatic ? 1 : 0;
-    return cudaLaunchKernelEx(&cfg, rowstat_kernel, g, sc, io.cu, a.W, plan.grid, after_score ? 1 : 0);
+    return cudaLaunchKernelEx(&cfg, rowstat_kernel, g, sc, io.cu, plan.chunk, claim, after_score ? 1 : 0);
 }
 
 cudaError_t launch_rowstat_lse(const Geometry& g, const LayerIO& io, const Scratch& sc, cudaStream_t st,
@@ -572,8 +645,9 @@ cudaError_t launch_rowstat_lse(const Geometry& g, const LayerIO& io, const Scrat
     return cudaLaunchKernelEx(&cfg, rowstat_lse_kernel, g, sc, io.lse);
 }
 
-cudaError_t launch_score(const ScorePlan& plan, cudaStream_t st, bool after_own_launch) {
-    const ScoreArgs& a = *reinterpret_cast<const ScoreArgs*>(plan.args);
+cudaError_t launch_score(const ScorePlan& plan, int* claim, cudaStream_t st, bool after_own_launch) {
+    ScoreArgs a = *reinterpret_cast<const ScoreArgs*>(plan.args);
+    a.claim = claim;
     // after_own_launch: the previous kernel on the stream is the previous
     // layer's launch, whose results this grid does not read; the launch is then
     // its programmatic dependent and never executes griddepcontrol.wait.

@@ -291,6 +291,7 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
                     }
                     int at = off + incl - mc;
                     const int pos0 = sg * kTopkSeg + lane * kTopkKPL;
+                    uint32_t half = 0u;   // this lane's positions above the bucket: selected for certain
 #pragma unroll
                     for (int j = 0; j < kTopkKPL; ++j) {
                         const uint32_t v = key_at(sg, j);
@@ -300,8 +301,14 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
                             sm.cpos[at] = pos0 + j;
                         }
                         at += m ? 1 : 0;
+                        half |= (v != 0u && (v & mask) > prefix ? 1u : 0u) << j;
                     }
                     off += __shfl_sync(0xffffffffu, incl, 31);
+                    // Lanes 2m and 2m + 1 hold the low and high halves of the segment's word m.
+                    const uint32_t high = __shfl_xor_sync(0xffffffffu, half, 1);
+                    const int wd = sg * (kTopkSeg / 32) + (lane >> 1);
+                    const uint32_t word = half | (high << 16);
+                    if ((lane & 1) == 0 && wd < nwords && word) bits[wd] |= word;
                 }
                 mlist = cnt;
                 topk_bar();
@@ -341,6 +348,47 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
             }
         }
         const bool ties = !whole_bin && !few;
+        if (mlist >= 0) {
+            // The compaction sweep marked every key above its bucket; the list
+            // holds that bucket in position order, a thread the four entries
+            // [4 tid, 4 tid + 4).  Mark the entries above the final threshold, the
+            // whole final bucket when it is taken whole, and with ties its equal
+            // entries at the kk lowest positions (the few path ranks its bucket below).
+            constexpr int kPer = kTopkCap / kTopkThreads;
+            uint32_t v4[kPer];
+            int eq = 0;
+#pragma unroll
+            for (int r = 0; r < kPer; ++r) {
+                const int j = kPer * tid + r;
+                v4[r] = j < mlist ? sm.ckey[j] : 0u;
+                eq += (v4[r] != 0u && (v4[r] & mask) == prefix) ? 1 : 0;
+            }
+            int before = 0;   // equal entries in lower positions (ties only)
+            if (ties) {
+                int incl = eq;
+#pragma unroll
+                for (int o = 1; o < 32; o <<= 1) {
+                    const int y = __shfl_up_sync(0xffffffffu, incl, o);
+                    if (lane >= o) incl += y;
+                }
+                if (lane == 31) sm.weq[warp] = incl;
+                topk_bar();
+                for (int x = 0; x < warp; ++x) before += sm.weq[x];
+                before += incl - eq;
+            }
+#pragma unroll
+            for (int r = 0; r < kPer; ++r) {
+                const int j = kPer * tid + r;
+                const uint32_t um = v4[r] & mask;
+                const bool isq = v4[r] != 0u && um == prefix;
+                const bool sel = (v4[r] != 0u && um > prefix) || (whole_bin && isq) || (ties && isq && before < kk);
+                before += isq ? 1 : 0;
+                if (sel) {
+                    const int pos = sm.cpos[j];
+                    atomicOr(&bits[pos >> 5], 1u << (pos & 31));
+                }
+            }
+        } else {
         if (ties) {
             // More equal keys straddle the threshold than kTopkFew: rank by position.
             int eqc = 0;
@@ -400,6 +448,7 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
             const int wd = sg * (kTopkSeg / 32) + (lane >> 1);
             const uint32_t word = half | (high << 16);
             if ((lane & 1) == 0 && wd < nwords && word) bits[wd] |= word;
+        }
         }
         if (few) {
             topk_bar();   // the sweep's plain stores are done before warp 0 adds bits

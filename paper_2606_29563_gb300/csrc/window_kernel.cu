@@ -63,7 +63,7 @@ struct __align__(8) WinBars {
     uint64_t mma_done;
     uint32_t tmem_base;
     volatile int abort_flag;
-    volatile int gok[4];        // per group: the outcome of its last accumulator wait
+    volatile int gok[4][2];     // per group: the outcome of its accumulator wait, by item parity
     int done[2];                // per unit parity: groups finished with the unit
     volatile int ready[2];      // per unit parity: the local unit index whose maxima may use the buffer
     int last[4];                // per group: 1 if it finished a unit last
@@ -369,13 +369,13 @@ __global__ void __launch_bounds__(kWinThreads, 1)
                                     ptx::mbar_wait_abortable(&bars->acc_full[grp], k & 1, &bars->abort_flag,
                                                              fault && it + hh == 0 ? kFaultWaitNs : 200000000ull);
                     if (!ok) win_abort(bars, sc.err);
-                    bars->gok[grp] = ok ? 1 : 0;
+                    bars->gok[grp][k & 1] = ok ? 1 : 0;
                 }
                 float* rsb = rs_g + (k & 1) * 256;
                 rsb[gtid] = pa;
                 rsb[gtid + 128] = pb;
                 ptx::named_bar_sync(bar_id, 128);
-                if (!bars->gok[grp]) {
+                if (!bars->gok[grp][k & 1]) {
                     failed = true;
                     break;
                 }
@@ -459,7 +459,7 @@ struct __align__(8) TileBars {
     uint64_t mma_done;
     uint32_t tmem_base;
     volatile int abort_flag;
-    volatile int gok[4];
+    volatile int gok[4][2];     // per group: the outcome of its accumulator wait, by item parity
 };
 
 __host__ __device__ inline size_t tile_smem_bytes(int Npad, int kst) {
@@ -763,13 +763,13 @@ __global__ void __launch_bounds__(kWinThreads, 1)
                         bars->abort_flag = 1;
                         atomicExch(sc.err, 3);
                     }
-                    bars->gok[grp] = ok ? 1 : 0;
+                    bars->gok[grp][k & 1] = ok ? 1 : 0;
                 }
                 float* rsb = rs_g + (k & 1) * 256;
                 rsb[gtid] = pa;
                 rsb[gtid + 128] = pb;
                 ptx::named_bar_sync(bar_id, 128);
-                if (!bars->gok[grp]) {
+                if (!bars->gok[grp][k & 1]) {
                     failed = true;
                     break;
                 }

@@ -131,7 +131,7 @@ __device__ __forceinline__ int warp_digit_counts(const uint32_t* pair, int lane)
 // later passes read only them; once it holds at most kTopkFew keys one warp
 // ranks them directly (larger key first, then lower position).  If more equal
 // keys than that straddle the threshold they are ranked by position.
-template <bool kCached>
+template <int NS>
 __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ keys, int kw, int n, int k, uint32_t* bits,
                                                 TopkShared& sm) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, tid = threadIdx.x;
@@ -140,26 +140,40 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
         const int nseg = (n + kTopkSeg - 1) / kTopkSeg;
         const int spw = (nseg + kTopkWarps - 1) / kTopkWarps;   // segments per warp
         const int seg0 = min(warp * spw, nseg), seg1 = min(seg0 + spw, nseg);
-        // Key j of this lane's positions in segment sg (0 past the row).  With one
-        // segment per warp (kCached) a lane's keys stay in registers.
+        // Key j of this lane's positions in segment sg (0 past the row).  With at
+        // most NS > 0 segments per warp a lane's keys stay in registers (segment
+        // seg0 + si in ureg[16 si ..]); with NS = 0 every sweep reads them again.
         auto fetch_key = [&](int sg, int j) -> uint32_t {
             const int t = sg * kTopkSeg + lane * kTopkKPL + j;
             return t < n ? keys[key_index(t, kw)] : 0u;
         };
-        uint32_t ureg[kCached ? kTopkKPL : 1];
-        if (kCached) {
+        uint32_t ureg[NS > 0 ? NS * kTopkKPL : 1];
+        if constexpr (NS > 0) {
 #pragma unroll
-            for (int j = 0; j < kTopkKPL; ++j) ureg[kCached ? j : 0] = fetch_key(seg0 < seg1 ? seg0 : nseg, j);
+            for (int si = 0; si < NS; ++si) {
+#pragma unroll
+                for (int j = 0; j < kTopkKPL; ++j)
+                    ureg[si * kTopkKPL + j] = seg0 + si < seg1 ? fetch_key(seg0 + si, j) : 0u;
+            }
         }
-        auto key_at = [&](int sg, int j) -> uint32_t { return kCached ? ureg[kCached ? j : 0] : fetch_key(sg, j); };
+        auto key_at = [&](int si, int sg, int j) -> uint32_t {
+            if constexpr (NS > 0) return ureg[si * kTopkKPL + j];
+            return fetch_key(sg, j);
+        };
+        // Segment loops: si counts the warp's segments (a constant trip count when
+        // the keys are in registers, so that ureg is indexed statically).
+        const int nsi = NS > 0 ? NS : seg1 - seg0;
 
         // Bits shared by every eligible key.
         {
             uint32_t kor = 0u, kand = 0xffffffffu;
-            for (int sg = seg0; sg < seg1; ++sg) {
+#pragma unroll
+            for (int si = 0; si < nsi; ++si) {
+                const int sg = seg0 + si;
+                if (sg >= seg1) break;
 #pragma unroll
                 for (int j = 0; j < kTopkKPL; ++j) {
-                    const uint32_t v = key_at(sg, j);
+                    const uint32_t v = key_at(si, sg, j);
                     kor |= v;
                     kand &= v != 0u ? v : 0xffffffffu;
                 }
@@ -207,14 +221,17 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
             int mine;   // lane d < 16: this warp's count of digit d
             if (mlist < 0) {
                 uint32_t pair[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
-                for (int sg = seg0; sg < seg1; ++sg) {
+#pragma unroll
+                for (int si = 0; si < nsi; ++si) {
+                    const int sg = seg0 + si;
+                    if (sg >= seg1) break;
                     DigitBytes db;
 #pragma unroll
                     for (int j0 = 0; j0 < kTopkKPL; j0 += 15) {
                         unsigned long long nib = 0ull;
 #pragma unroll
                         for (int j = j0; j < j0 + 15 && j < kTopkKPL; ++j)
-                            nib += digit_nibble(key_at(sg, j), mask, prefix, lo, wmask);
+                            nib += digit_nibble(key_at(si, sg, j), mask, prefix, lo, wmask);
                         db.add(nib);
                     }
                     db.to_pairs(pair);
@@ -276,11 +293,14 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
                 // matches of its segment's lower lanes and earlier segments.
                 int off = 0;
                 for (int x = 0; x < warp; ++x) off += sm.wcnt[buf][x][D];
-                for (int sg = seg0; sg < seg1; ++sg) {
+#pragma unroll
+                for (int si = 0; si < nsi; ++si) {
+                    const int sg = seg0 + si;
+                    if (sg >= seg1) break;
                     int mc = 0;
 #pragma unroll
                     for (int j = 0; j < kTopkKPL; ++j) {
-                        const uint32_t v = key_at(sg, j);
+                        const uint32_t v = key_at(si, sg, j);
                         mc += (v != 0u && (v & mask) == prefix) ? 1 : 0;
                     }
                     int incl = mc;
@@ -294,7 +314,7 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
                     uint32_t half = 0u;   // this lane's positions above the bucket: selected for certain
 #pragma unroll
                     for (int j = 0; j < kTopkKPL; ++j) {
-                        const uint32_t v = key_at(sg, j);
+                        const uint32_t v = key_at(si, sg, j);
                         const bool m = v != 0u && (v & mask) == prefix;
                         if (m && at < kTopkCap) {
                             sm.ckey[at] = v;
@@ -331,11 +351,14 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
                     }
                 }
             } else {
-                for (int sg = seg0; sg < seg1; ++sg) {
+#pragma unroll
+                for (int si = 0; si < nsi; ++si) {
+                    const int sg = seg0 + si;
+                    if (sg >= seg1) break;
                     const int pos0 = sg * kTopkSeg + lane * kTopkKPL;
 #pragma unroll
                     for (int j = 0; j < kTopkKPL; ++j) {
-                        const uint32_t v = key_at(sg, j);
+                        const uint32_t v = key_at(si, sg, j);
                         if (v != 0u && (v & mask) == prefix) {
                             const int slot = atomicAdd(&sm.fcount, 1);
                             if (slot < kTopkFew) {
@@ -392,10 +415,13 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
         if (ties) {
             // More equal keys straddle the threshold than kTopkFew: rank by position.
             int eqc = 0;
-            for (int sg = seg0; sg < seg1; ++sg) {
+#pragma unroll
+            for (int si = 0; si < nsi; ++si) {
+                const int sg = seg0 + si;
+                if (sg >= seg1) break;
 #pragma unroll
                 for (int j = 0; j < kTopkKPL; ++j) {
-                    const uint32_t v = key_at(sg, j);
+                    const uint32_t v = key_at(si, sg, j);
                     eqc += (v != 0u && (v & mask) == prefix) ? 1 : 0;
                 }
             }
@@ -408,12 +434,15 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
             for (int x = 0; x < warp; ++x) base += sm.weq[x];
         // Mark the keys above the threshold prefix (all of the bucket when it is
         // taken whole; with ties, the equal keys at the kk lowest positions).
-        for (int sg = seg0; sg < seg1; ++sg) {
+#pragma unroll
+        for (int si = 0; si < nsi; ++si) {
+            const int sg = seg0 + si;
+            if (sg >= seg1) break;
             uint32_t half = 0u;   // this lane's 16 positions
             if (!ties) {
 #pragma unroll
                 for (int j = 0; j < kTopkKPL; ++j) {
-                    const uint32_t v = key_at(sg, j);
+                    const uint32_t v = key_at(si, sg, j);
                     const uint32_t um = v & mask;
                     const bool sel = v != 0u && (um > prefix || (whole_bin && um == prefix));
                     half |= (sel ? 1u : 0u) << j;
@@ -422,7 +451,7 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
                 int ec = 0;
 #pragma unroll
                 for (int j = 0; j < kTopkKPL; ++j) {
-                    const uint32_t v = key_at(sg, j);
+                    const uint32_t v = key_at(si, sg, j);
                     ec += (v != 0u && (v & mask) == prefix) ? 1 : 0;
                 }
                 int incl = ec;
@@ -434,7 +463,7 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
                 int rank = base + incl - ec;
 #pragma unroll
                 for (int j = 0; j < kTopkKPL; ++j) {
-                    const uint32_t v = key_at(sg, j);
+                    const uint32_t v = key_at(si, sg, j);
                     const uint32_t um = v & mask;
                     const bool eq = v != 0u && um == prefix;
                     const bool sel = (v != 0u && um > prefix) || (eq && rank < kk);
@@ -468,13 +497,18 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
     }
 }
 
+// NSMAX: the most 512-position segments per warp kept in registers (2 where the
+// caller has the registers to spare).
+template <int NSMAX = 1>
 __device__ void block_topk(const uint32_t* __restrict__ keys, int kw, int n, int k, uint32_t* bits, TopkShared& sm) {
     if (k > 0 && n > 0 && (threadIdx.x >> 5) < kTopkWarps) {
         const int nseg = (n + kTopkSeg - 1) / kTopkSeg;
         if (nseg <= kTopkWarps)
-            block_topk_impl<true>(keys, kw, n, k, bits, sm);
+            block_topk_impl<1>(keys, kw, n, k, bits, sm);
+        else if (NSMAX >= 2 && nseg <= 2 * kTopkWarps)
+            block_topk_impl<NSMAX >= 2 ? 2 : 1>(keys, kw, n, k, bits, sm);
         else
-            block_topk_impl<false>(keys, kw, n, k, bits, sm);
+            block_topk_impl<0>(keys, kw, n, k, bits, sm);
     }
     __syncthreads();
 }
@@ -746,7 +780,7 @@ __global__ void __launch_bounds__(kSelectThreads) heads_pool_kernel(Geometry G, 
 // per (KV head, sequence), launched after heads_pool_kernel: every CTA ranks the
 // sequence's sigmas the same way, the delta lowest-sigma heads take the O'
 // scores, then the top-K preserved tokens of the chosen row by radix select.
-__global__ void __launch_bounds__(kSelectThreads) heads_topk_kernel(Geometry G, LayerIO io, Scratch sc, Slot sl) {
+__global__ void __launch_bounds__(kSelectThreads, 2) heads_topk_kernel(Geometry G, LayerIO io, Scratch sc, Slot sl) {
     __shared__ TopkShared sm;
     __shared__ int top_flag;
     extern __shared__ uint32_t bits[];
@@ -948,7 +982,7 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
         // The next layer's selection may be scheduled now: its staging overlaps
         // this top-k, then it waits for this grid.
         asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
-        block_topk(keys, kw, Lc, G.f0, bits, sm);
+        block_topk<2>(keys, kw, Lc, G.f0, bits, sm);
         if (G.ada) {
             // Head-wise adaptive fill: the head keeps its own best f0.  A head
             // can win at most extras = Hkv * (k2 - f0) slots of the joint ranking

@@ -1003,7 +1003,7 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
             }
             __syncthreads();
             const int nC = min(G.jpool, Lc - G.Kp - G.f0);
-            block_topk(keys, kw, Lc, nC, cbits, sm);
+            block_topk<2>(keys, kw, Lc, nC, cbits, sm);
             uint32_t* jk = sc.jkeys + (size_t)s * G.jstride;
             int32_t* jp = sc.jpos + (size_t)s * G.jstride;
             const int kwj = (G.Hkv * G.jpool + 31) >> 5;

@@ -104,6 +104,49 @@ def test_uniform_keys_tie_to_lowest_positions():
     sel.close()
 
 
+@pytest.mark.parametrize("plateau,budget", [((4500, 5800), 1024), ((4800, 12000), 1024), ((5100, 5140), 64)])
+def test_equal_keys_across_row_slices_tie_to_lowest_positions(plateau, budget):
+    """Positions [a, b) of a 20000-position row share one key vector that every
+    (constant) query favours, so their scores are equal and above every other
+    candidate; B - w of them are kept, and equal keys must go to the lowest
+    positions, across the warps' segments of the radix select (the row has more
+    512-position segments than its 16 warps keep in registers): the kept
+    candidates are one run of B - w consecutive positions starting at the
+    plateau (pooling may widen it by 3).  The cases reach the threshold through
+    the compacted list, the full sweep and the few-key ranking."""
+    L = 20000
+    wl = synth.small_workload(seqlens=(L,), budget=budget, layers=1)
+    params = kvec.params_from_workload(wl)
+    sel = kvec.KvecSelector(params)
+    x = synth.make_layer(wl, 0)
+    q = torch.full_like(x["q_obs"], 0.1).cuda()
+    k = torch.zeros_like(x["k"])
+    a, b = plateau
+    k[a:b] = 0.5
+    k = k.cuda()
+    cu = torch.tensor(wl.cu_seqlens, dtype=torch.int32)
+    st = sel.new_state(1)
+    idx, _, _ = sel.select_layer(cu, cu.cuda(), q, k, x["v"].cuda(), st, budget)
+    torch.cuda.synchronize()
+    for h in range(wl.num_kv_heads):
+        got = idx[0, h].cpu().tolist()
+        assert got[-wl.window:] == list(range(L - wl.window, L))
+        run = got[:budget - wl.window]
+        assert a - 3 <= run[0] <= a + 3 and run == list(range(run[0], run[0] + len(run))), (h, run[:5], run[-5:])
+    sel.close()
+
+
+@pytest.mark.parametrize("kw", [dict(seqlens=(9000,), layers=3),
+                                dict(seqlens=(30000,), layers=2, budget=128),
+                                dict(seqlens=(17000, 600, 40), layers=3, budget=256),
+                                dict(seqlens=(16384,), num_q_heads=28, num_kv_heads=4, layers=2, budget=512)])
+def test_long_rows_of_small_batches_match_the_oracle(kw):
+    """Few (sequence, KV head) rows of 9000 to 30000 positions over several
+    layers: one to four 512-position segments per warp in the radix
+    select; the ragged case adds a short sequence and one that fits the budget."""
+    _assert_parity(synth.small_workload(**kw))
+
+
 def test_deterministic_rerun():
     wl = synth.small_workload(seqlens=(900, 450), layers=2)
     outs = []

@@ -63,7 +63,7 @@ struct TimedLaunch {
 int kvec::test_fault() { return g_test_fault.load(std::memory_order_relaxed); }
 
 constexpr int kSlots = 8;   // per-layer score arrays in flight between the score and select stages
-constexpr int kScoreBufs = 2;   // score-statistics buffers in flight between the score and window stages
+constexpr int kScoreBufs = 2;   // segment-partial buffers in flight between the score and row-statistics stages
 constexpr size_t kGraphCache = 16;  // captured multi-layer calls kept per handle
 
 struct kvec_handle {
@@ -76,9 +76,10 @@ struct kvec_handle {
     size_t ws_bytes = 0;
     int* claims = nullptr;   // [max_layers] the score launches' chunk counters (zero between launches)
     Scratch sc{};
-    Scratch score_buf[kScoreBufs]{};   // segment partials and row statistics, one per layer in flight
+    Scratch score_buf[kScoreBufs]{};   // segment partials, one per layer in flight
     Slot slots[kSlots]{};
-    int last_slot = 0, last_parity = 0;
+    float2* rowstat_slot[kSlots]{};    // row statistics of the layer in slot k (read by its window grid)
+    int last_slot = 0;
     int last_batch = 0;
     bool profiling = false;
     std::vector<TimedLaunch> timed;
@@ -87,7 +88,7 @@ struct kvec_handle {
     // layer, so consecutive layers' head passes overlap) | coverage select | gather.
     cudaStream_t s_score = nullptr, s_win = nullptr, s_heads = nullptr, s_heads2 = nullptr, s_chain = nullptr,
                  s_gather = nullptr, s_cap = nullptr;
-    std::vector<cudaEvent_t> ev_score, ev_win, ev_heads, ev_sel, ev_gather;
+    std::vector<cudaEvent_t> ev_score, ev_rs, ev_win, ev_heads, ev_sel, ev_gather;
     cudaEvent_t ev_fork = nullptr, ev_join[5] = {nullptr, nullptr, nullptr, nullptr, nullptr};
     // Scheduling priorities: the heads and coverage-select kernels (the serial
     // chain of the pipeline) take SMs before the score, window and gather kernels.
@@ -350,7 +351,14 @@ cudaError_t restore_full_edges(cudaGraph_t graph, const std::vector<std::pair<cu
 // Layers 0..n-1 as a five-stream pipeline.  Only the coverage-adjusted select
 // is serial across layers (it carries n_t); the score, window and heads work of
 // later layers runs ahead of it, bounded by the double-buffered score scratch
-// and by the kSlots ring of per-layer score arrays.
+// and by the kSlots ring of per-layer score arrays.  The row statistics live
+// with the slot (for the window grid); a layer's score grid reuses the segment
+// partials of layer l - kScoreBufs after that layer's window grid, or, when the
+// score and window grids fit on the SMs together, as soon as its row
+// statistics are done with them (else an early score grid only takes SMs that
+// the window and heads kernels of the layers ahead need: measured slower).
+// With the caller's log-sum-exp there is no score grid, and the same wait
+// keeps at most two layers' window grids in flight.
 kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* ios, int n, cudaStream_t origin) {
     KV_CHECK(cudaEventRecord(h->ev_fork, origin));
     for (cudaStream_t st : {h->s_score, h->s_win, h->s_heads, h->s_heads2, h->s_chain, h->s_gather})
@@ -358,14 +366,17 @@ kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* io
     cudaGraphNode_t prev_score = nullptr, prev_window = nullptr, prev_select = nullptr;   // captured (h->capturing)
     for (int l = 0; l < n; ++l) {
         const Slot& sl = h->slots[l % kSlots];
-        const Scratch& sc = h->score_buf[l % kScoreBufs];
+        Scratch sc = h->score_buf[l % kScoreBufs];
+        sc.rowstat = h->rowstat_slot[l % kSlots];
         const LayerIO& io = ios[l];
-        // Statistics buffer reuse: layer l - kScoreBufs's row statistics and window
-        // (window stream) are done with it.
-        if (l >= kScoreBufs) KV_CHECK(cudaStreamWaitEvent(h->s_score, h->ev_win[l - kScoreBufs], 0));
         ScorePlan plan;
         cudaError_t se = plan_score(G, io, sc, h->num_sms, &plan);
         if (se != cudaSuccess) return cuda_fail(se, "score kernel tensor maps");
+        // Partials buffer reuse (window stream).
+        if (l >= kScoreBufs) {
+            const bool early = !io.lse && plan.grid + window_grid_size(plan, G) <= h->num_sms;
+            KV_CHECK(cudaStreamWaitEvent(h->s_score, early ? h->ev_rs[l - kScoreBufs] : h->ev_win[l - kScoreBufs], 0));
+        }
         // The score grid of layer l > 0 is a programmatic dependent of layer
         // l - 1's (it reads none of its results); the event wait above stays a
         // full dependency (restore_full_edges when captured).
@@ -391,8 +402,8 @@ kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* io
         // The row statistics are a programmatic dependent of the previous layer's
         // window grid, which they do not wait for: they read only this layer's
         // partials (full dependency above), and the statistics buffer they
-        // overwrite was last read by layer l - 2's window grid, which this
-        // layer's score grid waited for.  So consecutive window grids overlap.
+        // overwrite belongs to this layer's slot, last read by layer l - kSlots's
+        // window grid (the waits above).  So consecutive window grids overlap.
         se = io.lse ? launch_rowstat_lse(G, io, sc, h->s_win, l > 0)
                     : launch_rowstat(plan, G, io, sc, h->claims + l, h->s_win, l > 0, /*after_score=*/false);
         if (se != cudaSuccess) return cuda_fail(se, "row statistics launch");
@@ -401,6 +412,7 @@ kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* io
             if (!node) return fail(KVEC_ERR_CUDA, "row statistics: no captured node");
             if (l > 0) h->prog_nodes.emplace_back(node, prev_window);
         }
+        KV_CHECK(cudaEventRecord(h->ev_rs[l], h->s_win));
         timed_launch(h, 1, h->s_win, [&] { se = launch_window(plan, G, io, sc, sl, h->s_win, true); });
         if (se != cudaSuccess) return cuda_fail(se, "window kernel launch");
         if (h->capturing) {
@@ -458,7 +470,6 @@ kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* io
     KV_CHECK(cudaStreamWaitEvent(origin, h->ev_fork, 0));
     for (cudaEvent_t e : h->ev_join) KV_CHECK(cudaStreamWaitEvent(origin, e, 0));
     h->last_slot = (n - 1) % kSlots;
-    h->last_parity = (n - 1) % kScoreBufs;
     return KVEC_OK;
 }
 
@@ -485,7 +496,7 @@ void release_handle(kvec_handle* h) {
     h->graphs.clear();
     for (cudaStream_t st : {h->s_score, h->s_win, h->s_heads, h->s_heads2, h->s_chain, h->s_gather, h->s_cap})
         if (st) cudaStreamDestroy(st);
-    for (auto* v : {&h->ev_score, &h->ev_win, &h->ev_heads, &h->ev_sel, &h->ev_gather})
+    for (auto* v : {&h->ev_score, &h->ev_rs, &h->ev_win, &h->ev_heads, &h->ev_sel, &h->ev_gather})
         for (cudaEvent_t ev : *v)
             if (ev) cudaEventDestroy(ev);
     if (h->ev_fork) cudaEventDestroy(h->ev_fork);
@@ -561,7 +572,6 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
         Scratch& b = h->score_buf[k];
         std::vector<Part> sp = {
             {(void**)&b.segpart, max_tiles * Hkv * R * sizeof(float2)},
-            {(void**)&b.rowstat, MB * Hkv * R * sizeof(float2)},
         };
         parts.insert(parts.end(), sp.begin(), sp.end());
     }
@@ -575,6 +585,7 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
             {(void**)&sl.pres, MB * Hkv * W * sizeof(uint32_t)}, {(void**)&sl.Pprime, MB * Hkv * ML * sizeof(float)},
             {(void**)&sl.sel, MB * Hkv * W * sizeof(uint32_t)},
             {(void**)&sl.wpart, max_tiles * NGmax * p.obs_window * kTileT * sizeof(float)},
+            {(void**)&h->rowstat_slot[k], MB * Hkv * R * sizeof(float2)},
         };
         parts.insert(parts.end(), sp.begin(), sp.end());
     }
@@ -616,11 +627,12 @@ kvec_status kvec_create(const kvec_params* params, kvec_handle** out) {
     for (cudaStream_t* st : {&h->s_heads, &h->s_heads2, &h->s_chain})
         if (e == cudaSuccess) e = cudaStreamCreateWithPriority(st, cudaStreamNonBlocking, h->prio_hi);
     h->ev_score.assign(p.max_layers, nullptr);
+    h->ev_rs.assign(p.max_layers, nullptr);
     h->ev_win.assign(p.max_layers, nullptr);
     h->ev_heads.assign(p.max_layers, nullptr);
     h->ev_sel.assign(p.max_layers, nullptr);
     h->ev_gather.assign(p.max_layers, nullptr);
-    for (auto* v : {&h->ev_score, &h->ev_win, &h->ev_heads, &h->ev_sel, &h->ev_gather})
+    for (auto* v : {&h->ev_score, &h->ev_rs, &h->ev_win, &h->ev_heads, &h->ev_sel, &h->ev_gather})
         for (auto& ev : *v)
             if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
     if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming);
@@ -729,7 +741,6 @@ kvec_status select_layers_impl(kvec_handle* h, int num_layers, int batch, const 
             if (h->graphs[i].key != key) continue;
             KV_CHECK(cudaGraphLaunch(h->graphs[i].exec, st));
             h->last_slot = (num_layers - 1) % kSlots;
-            h->last_parity = (num_layers - 1) % kScoreBufs;
             h->last_batch = batch;
             return KVEC_OK;
         }
@@ -1025,7 +1036,7 @@ kvec_status kvec_debug_scores(kvec_handle* h, kvec_debug_view* out) {
     out->htop = sl.htop;
     out->pres_bits = sl.pres;
     out->Pprime = sl.Pprime;
-    out->row_stats = reinterpret_cast<const float*>(h->score_buf[h->last_parity].rowstat);
+    out->row_stats = reinterpret_cast<const float*>(h->rowstat_slot[h->last_slot]);
     out->max_seqlen = (int)row_stride(h->p.max_seqlen);
     out->words_per_row = h->words;
     return KVEC_OK;

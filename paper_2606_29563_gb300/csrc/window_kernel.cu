@@ -916,6 +916,13 @@ cudaError_t launch_window_tiles(const ScorePlan& sp, const Geometry& g, const La
 
 }  // namespace
 
+int window_grid_size(const ScorePlan& sp, const Geometry& g) {
+    if (g.win_tiles == 0) return 0;
+    const int usable = sp.num_sms > 2 * kWinReserveSms ? sp.num_sms - kWinReserveSms : sp.num_sms;
+    if (tile_variant_fits(g) && tile_units_of(g, g.cu_host, npad_of(g.R) <= 128 ? 4 : 2) >= usable) return usable;
+    return units_of(g) < usable ? units_of(g) : usable;
+}
+
 cudaError_t launch_window(const ScorePlan& sp, const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl,
                           cudaStream_t st, bool after_own_launch) {
     if (g.win_tiles == 0) return cudaSuccess;

@@ -19,11 +19,18 @@ __host__ __device__ inline bool keys_in_smem(int ML) { return ML <= kSmemKeys; }
 constexpr int kSmemScores = 16448;  // row stride up to which the select kernel caches P and I in shared memory
 __host__ __device__ inline bool scores_in_smem(int ML) { return ML <= kSmemScores; }
 
-// Key rows are stored transposed, key t at keys[(t & 31) * kw + (t >> 5)]: a lane
-// that owns the 32 positions of one bits word then reads them from consecutive
-// words of its warp's neighbours (an odd stride keeps the writers' banks apart).
-__host__ __device__ inline int key_stride(const Geometry& g) { return keys_in_smem(g.ML) ? (g.words | 1) : g.words; }
-__device__ __forceinline__ int key_index(int t, int kw) { return (t & 31) * kw + (t >> 5); }
+// Key rows are stored in position order in 16-byte chunks of four keys, chunk c
+// at c ^ ((c >> 3) & 7): a radix-select lane reads its 16 consecutive keys as
+// four 16-byte loads, and the eight lanes of a quarter-warp (64 bytes apart)
+// then hit eight different 16-byte bank groups, as do eight threads storing
+// eight consecutive chunks.  The permutation stays inside each group of 32
+// keys, so a row of n keys takes round_up(n, 32) words (32 * words per row).
+__device__ __forceinline__ int key_chunk(int t4) {   // t4 a multiple of 4
+    const int c = t4 >> 2;
+    return (c ^ ((c >> 3) & 7)) << 2;
+}
+__device__ __forceinline__ int key_index(int t) { return key_chunk(t & ~3) | (t & 3); }
+__host__ __device__ inline size_t key_row_words(const Geometry& g) { return 32 * (size_t)g.words; }
 
 constexpr int kPoolSmemBytes = 96 * 1024;     // raw-I chunk of the heads pooling kernel
 constexpr int kTopkWarps = 16;                 // warps that run the radix select
@@ -115,7 +122,7 @@ __device__ __forceinline__ int warp_digit_counts(const uint32_t* pair, int lane)
 }
 
 // ORs into bits[] (shared, one bit per position) the k largest keys of a row of
-// n keys stored transposed with stride kw; every thread of the block calls it
+// n keys (stored as key_index lays them out); every thread of the block calls it
 // and the bits are complete on return.  Key 0 marks an ineligible position;
 // the caller guarantees k <= #eligible.
 //
@@ -132,7 +139,7 @@ __device__ __forceinline__ int warp_digit_counts(const uint32_t* pair, int lane)
 // ranks them directly (larger key first, then lower position).  If more equal
 // keys than that straddle the threshold they are ranked by position.
 template <int NS>
-__device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ keys, int kw, int n, int k, uint32_t* bits,
+__device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ keys, int n, int k, uint32_t* bits,
                                                 TopkShared& sm) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, tid = threadIdx.x;
     {
@@ -140,25 +147,50 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
         const int nseg = (n + kTopkSeg - 1) / kTopkSeg;
         const int spw = (nseg + kTopkWarps - 1) / kTopkWarps;   // segments per warp
         const int seg0 = min(warp * spw, nseg), seg1 = min(seg0 + spw, nseg);
-        // Key j of this lane's positions in segment sg (0 past the row).  With at
-        // most NS > 0 segments per warp a lane's keys stay in registers (segment
-        // seg0 + si in ureg[16 si ..]); with NS = 0 every sweep reads them again.
-        auto fetch_key = [&](int sg, int j) -> uint32_t {
-            const int t = sg * kTopkSeg + lane * kTopkKPL + j;
-            return t < n ? keys[key_index(t, kw)] : 0u;
+        // This lane's 16 keys of segment sg (0 past the row): four 16-byte loads.
+        // With at most NS > 0 segments per warp a lane's keys stay in registers
+        // (segment seg0 + si in ureg[16 si ..]); with NS = 0 every sweep reads
+        // them again, once per segment.
+        auto load16 = [&](int sg, uint32_t* kv) {
+            const int t0 = sg * kTopkSeg + lane * kTopkKPL;
+            if (t0 + kTopkKPL <= n) {
+#pragma unroll
+                for (int q = 0; q < kTopkKPL / 4; ++q) {
+                    const uint4 v = *reinterpret_cast<const uint4*>(keys + key_chunk(t0 + 4 * q));
+                    kv[4 * q] = v.x;
+                    kv[4 * q + 1] = v.y;
+                    kv[4 * q + 2] = v.z;
+                    kv[4 * q + 3] = v.w;
+                }
+            } else {
+#pragma unroll
+                for (int j = 0; j < kTopkKPL; ++j) kv[j] = t0 + j < n ? keys[key_index(t0 + j)] : 0u;
+            }
         };
         uint32_t ureg[NS > 0 ? NS * kTopkKPL : 1];
         if constexpr (NS > 0) {
 #pragma unroll
             for (int si = 0; si < NS; ++si) {
+                if (seg0 + si < seg1) {
+                    load16(seg0 + si, ureg + si * kTopkKPL);
+                } else {
 #pragma unroll
-                for (int j = 0; j < kTopkKPL; ++j)
-                    ureg[si * kTopkKPL + j] = seg0 + si < seg1 ? fetch_key(seg0 + si, j) : 0u;
+                    for (int j = 0; j < kTopkKPL; ++j) ureg[si * kTopkKPL + j] = 0u;
+                }
             }
         }
-        auto key_at = [&](int si, int sg, int j) -> uint32_t {
-            if constexpr (NS > 0) return ureg[si * kTopkKPL + j];
-            return fetch_key(sg, j);
+        struct Keys16 {
+            uint32_t v[kTopkKPL];
+        };
+        auto seg_keys = [&](int si, int sg) -> Keys16 {
+            Keys16 r;
+            if constexpr (NS > 0) {
+#pragma unroll
+                for (int j = 0; j < kTopkKPL; ++j) r.v[j] = ureg[si * kTopkKPL + j];
+            } else {
+                load16(sg, r.v);
+            }
+            return r;
         };
         // Segment loops: si counts the warp's segments (a constant trip count when
         // the keys are in registers, so that ureg is indexed statically).
@@ -171,9 +203,10 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
             for (int si = 0; si < nsi; ++si) {
                 const int sg = seg0 + si;
                 if (sg >= seg1) break;
+                const Keys16 kv = seg_keys(si, sg);
 #pragma unroll
                 for (int j = 0; j < kTopkKPL; ++j) {
-                    const uint32_t v = key_at(si, sg, j);
+                    const uint32_t v = kv.v[j];
                     kor |= v;
                     kand &= v != 0u ? v : 0xffffffffu;
                 }
@@ -225,13 +258,14 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
                 for (int si = 0; si < nsi; ++si) {
                     const int sg = seg0 + si;
                     if (sg >= seg1) break;
+                    const Keys16 kv = seg_keys(si, sg);
                     DigitBytes db;
 #pragma unroll
                     for (int j0 = 0; j0 < kTopkKPL; j0 += 15) {
                         unsigned long long nib = 0ull;
 #pragma unroll
                         for (int j = j0; j < j0 + 15 && j < kTopkKPL; ++j)
-                            nib += digit_nibble(key_at(si, sg, j), mask, prefix, lo, wmask);
+                            nib += digit_nibble(kv.v[j], mask, prefix, lo, wmask);
                         db.add(nib);
                     }
                     db.to_pairs(pair);
@@ -297,10 +331,11 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
                 for (int si = 0; si < nsi; ++si) {
                     const int sg = seg0 + si;
                     if (sg >= seg1) break;
+                    const Keys16 kv = seg_keys(si, sg);
                     int mc = 0;
 #pragma unroll
                     for (int j = 0; j < kTopkKPL; ++j) {
-                        const uint32_t v = key_at(si, sg, j);
+                        const uint32_t v = kv.v[j];
                         mc += (v != 0u && (v & mask) == prefix) ? 1 : 0;
                     }
                     int incl = mc;
@@ -314,7 +349,7 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
                     uint32_t half = 0u;   // this lane's positions above the bucket: selected for certain
 #pragma unroll
                     for (int j = 0; j < kTopkKPL; ++j) {
-                        const uint32_t v = key_at(si, sg, j);
+                        const uint32_t v = kv.v[j];
                         const bool m = v != 0u && (v & mask) == prefix;
                         if (m && at < kTopkCap) {
                             sm.ckey[at] = v;
@@ -355,10 +390,11 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
                 for (int si = 0; si < nsi; ++si) {
                     const int sg = seg0 + si;
                     if (sg >= seg1) break;
+                    const Keys16 kv = seg_keys(si, sg);
                     const int pos0 = sg * kTopkSeg + lane * kTopkKPL;
 #pragma unroll
                     for (int j = 0; j < kTopkKPL; ++j) {
-                        const uint32_t v = key_at(si, sg, j);
+                        const uint32_t v = kv.v[j];
                         if (v != 0u && (v & mask) == prefix) {
                             const int slot = atomicAdd(&sm.fcount, 1);
                             if (slot < kTopkFew) {
@@ -419,9 +455,10 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
             for (int si = 0; si < nsi; ++si) {
                 const int sg = seg0 + si;
                 if (sg >= seg1) break;
+                const Keys16 kv = seg_keys(si, sg);
 #pragma unroll
                 for (int j = 0; j < kTopkKPL; ++j) {
-                    const uint32_t v = key_at(si, sg, j);
+                    const uint32_t v = kv.v[j];
                     eqc += (v != 0u && (v & mask) == prefix) ? 1 : 0;
                 }
             }
@@ -438,11 +475,12 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
         for (int si = 0; si < nsi; ++si) {
             const int sg = seg0 + si;
             if (sg >= seg1) break;
+            const Keys16 kv = seg_keys(si, sg);
             uint32_t half = 0u;   // this lane's 16 positions
             if (!ties) {
 #pragma unroll
                 for (int j = 0; j < kTopkKPL; ++j) {
-                    const uint32_t v = key_at(si, sg, j);
+                    const uint32_t v = kv.v[j];
                     const uint32_t um = v & mask;
                     const bool sel = v != 0u && (um > prefix || (whole_bin && um == prefix));
                     half |= (sel ? 1u : 0u) << j;
@@ -451,7 +489,7 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
                 int ec = 0;
 #pragma unroll
                 for (int j = 0; j < kTopkKPL; ++j) {
-                    const uint32_t v = key_at(si, sg, j);
+                    const uint32_t v = kv.v[j];
                     ec += (v != 0u && (v & mask) == prefix) ? 1 : 0;
                 }
                 int incl = ec;
@@ -463,7 +501,7 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
                 int rank = base + incl - ec;
 #pragma unroll
                 for (int j = 0; j < kTopkKPL; ++j) {
-                    const uint32_t v = key_at(si, sg, j);
+                    const uint32_t v = kv.v[j];
                     const uint32_t um = v & mask;
                     const bool eq = v != 0u && um == prefix;
                     const bool sel = (v != 0u && um > prefix) || (eq && rank < kk);
@@ -500,15 +538,15 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
 // NSMAX: the most 512-position segments per warp kept in registers (2 where the
 // caller has the registers to spare).
 template <int NSMAX = 1>
-__device__ void block_topk(const uint32_t* __restrict__ keys, int kw, int n, int k, uint32_t* bits, TopkShared& sm) {
+__device__ void block_topk(const uint32_t* __restrict__ keys, int n, int k, uint32_t* bits, TopkShared& sm) {
     if (k > 0 && n > 0 && (threadIdx.x >> 5) < kTopkWarps) {
         const int nseg = (n + kTopkSeg - 1) / kTopkSeg;
         if (nseg <= kTopkWarps)
-            block_topk_impl<1>(keys, kw, n, k, bits, sm);
+            block_topk_impl<1>(keys, n, k, bits, sm);
         else if (NSMAX >= 2 && nseg <= 2 * kTopkWarps)
-            block_topk_impl<NSMAX >= 2 ? 2 : 1>(keys, kw, n, k, bits, sm);
+            block_topk_impl<NSMAX >= 2 ? 2 : 1>(keys, n, k, bits, sm);
         else
-            block_topk_impl<0>(keys, kw, n, k, bits, sm);
+            block_topk_impl<0>(keys, n, k, bits, sm);
     }
     __syncthreads();
 }
@@ -783,7 +821,7 @@ __global__ void __launch_bounds__(kSelectThreads) heads_pool_kernel(Geometry G, 
 __global__ void __launch_bounds__(kSelectThreads, 2) heads_topk_kernel(Geometry G, LayerIO io, Scratch sc, Slot sl) {
     __shared__ TopkShared sm;
     __shared__ int top_flag;
-    extern __shared__ uint32_t bits[];
+    extern __shared__ __align__(16) uint32_t bits[];
     const int h = blockIdx.x, s = blockIdx.y;
     const int tid = threadIdx.x, NT = blockDim.x;
     const int L = io.cu[s + 1] - io.cu[s];
@@ -807,8 +845,7 @@ __global__ void __launch_bounds__(kSelectThreads, 2) heads_topk_kernel(Geometry 
     const int top = top_flag;
     if (L > G.budget && G.Kp > 0) {
         const float* __restrict__ P = (top ? sl.POe : sl.PO) + row * G.ML;
-        uint32_t* keys = keys_in_smem(G.ML) ? bits + G.words : sc.keys + row * G.ML;
-        const int kw = key_stride(G);
+        uint32_t* keys = keys_in_smem(G.ML) ? bits + ((G.words + 3) & ~3) : sc.keys + row * G.ML;
         for (int b0 = 4 * tid; b0 < Lc; b0 += 16 * NT) {
             float4 pv[4];
 #pragma unroll
@@ -819,14 +856,17 @@ __global__ void __launch_bounds__(kSelectThreads, 2) heads_topk_kernel(Geometry 
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
                 const int t4 = b0 + 4 * u * NT;
-                const float x[4] = {pv[u].x, pv[u].y, pv[u].z, pv[u].w};
+                if (t4 < Lc) {   // positions from Lc on get key 0 (never read)
+                    const float x[4] = {pv[u].x, pv[u].y, pv[u].z, pv[u].w};
+                    uint32_t kq[4];
 #pragma unroll
-                for (int i = 0; i < 4; ++i)
-                    if (t4 + i < Lc) keys[key_index(t4 + i, kw)] = float_order_key(x[i]);
+                    for (int i = 0; i < 4; ++i) kq[i] = t4 + i < Lc ? float_order_key(x[i]) : 0u;
+                    *reinterpret_cast<uint4*>(keys + key_chunk(t4)) = make_uint4(kq[0], kq[1], kq[2], kq[3]);
+                }
             }
         }
         __syncthreads();
-        block_topk(keys, kw, Lc, G.Kp, bits, sm);
+        block_topk(keys, Lc, G.Kp, bits, sm);
     }
     uint32_t* pres = sl.pres + row * G.words;
     for (int wd = tid; wd < G.words; wd += NT) pres[wd] = bits[wd];
@@ -855,14 +895,13 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
     const int L = io.cu[s + 1] - io.cu[s];
     const int Lc = L - G.wk;
     const int wordsL = (L + 31) >> 5;
-    const int kw = key_stride(G);
     const bool cached = scores_in_smem(G.ML) && L > G.budget;
     // Shared memory: bits[words] | preserved bits[words] | union[words] |
     // adaptive-fill candidate bits[words] | keys | P row | I row (P and I
     // 16-byte aligned for float4 stores).
     uint32_t* spres = bits + G.words;
     uint32_t* suni = spres + G.words;
-    const size_t sp_off = ((size_t)4 * G.words + (keys_in_smem(G.ML) ? 32 * (size_t)kw : 0) + 3) & ~(size_t)3;
+    const size_t sp_off = ((size_t)4 * G.words + (keys_in_smem(G.ML) ? key_row_words(G) : 0) + 3) & ~(size_t)3;
     float* sP = reinterpret_cast<float*>(bits + sp_off);
     float* sI = sP + G.ML;
     const size_t row = (size_t)s * G.Hkv + h;
@@ -966,6 +1005,7 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
                 const float i4[4] = {iv[u].x, iv[u].y, iv[u].z, iv[u].w};
                 const uint8_t n4[4] = {c.x, c.y, c.z, c.w};
                 float out[4];
+                uint32_t kq[4];   // positions from Lc on get key 0 (never read)
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
                     const int t = t4 + i;
@@ -973,8 +1013,9 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
                     const float pp = p4[i] + G.lambda * (i4[i] * (1.f - coverage));
                     out[i] = pp;
                     const bool kept = (pw[u] >> (t & 31)) & 1u;
-                    if (t < Lc) keys[key_index(t, kw)] = kept ? 0u : float_order_key(pp);
+                    kq[i] = (t < Lc && !kept) ? float_order_key(pp) : 0u;
                 }
+                *reinterpret_cast<uint4*>(keys + key_chunk(t4)) = make_uint4(kq[0], kq[1], kq[2], kq[3]);
                 if (Pp) *reinterpret_cast<float4*>(Pp + t4) = make_float4(out[0], out[1], out[2], out[3]);
             }
         }
@@ -982,7 +1023,7 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
         // The next layer's selection may be scheduled now: its staging overlaps
         // this top-k, then it waits for this grid.
         asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
-        block_topk<2>(keys, kw, Lc, G.f0, bits, sm);
+        block_topk<2>(keys, Lc, G.f0, bits, sm);
         if (G.ada) {
             // Head-wise adaptive fill: the head keeps its own best f0.  A head
             // can win at most extras = Hkv * (k2 - f0) slots of the joint ranking
@@ -998,15 +1039,14 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
                 while (a) {
                     const int t = 32 * wd + __ffs(a) - 1;
                     a &= a - 1u;
-                    keys[key_index(t, kw)] = 0u;
+                    keys[key_index(t)] = 0u;
                 }
             }
             __syncthreads();
             const int nC = min(G.jpool, Lc - G.Kp - G.f0);
-            block_topk<2>(keys, kw, Lc, nC, cbits, sm);
+            block_topk<2>(keys, Lc, nC, cbits, sm);
             uint32_t* jk = sc.jkeys + (size_t)s * G.jstride;
             int32_t* jp = sc.jpos + (size_t)s * G.jstride;
-            const int kwj = (G.Hkv * G.jpool + 31) >> 5;
             const int wpt = (wordsL + NT - 1) / NT;
             const int w_lo = min(tid * wpt, wordsL), w_hi = min(w_lo + wpt, wordsL);
             int mine = 0;
@@ -1019,13 +1059,13 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(Geometry G, Laye
                     const int t = 32 * wd + __ffs(c) - 1;
                     c &= c - 1u;
                     const int i = h * G.jpool + r++;
-                    jk[key_index(i, kwj)] = keys[key_index(t, kw)];
+                    jk[key_index(i)] = keys[key_index(t)];
                     jp[i] = t;
                 }
             }
             for (int r2 = total + tid; r2 < G.jpool; r2 += NT) {
                 const int i = h * G.jpool + r2;
-                jk[key_index(i, kwj)] = 0u;
+                jk[key_index(i)] = 0u;
                 jp[i] = -1;
             }
         }
@@ -1086,7 +1126,7 @@ __global__ void __launch_bounds__(kSelectThreads) ada_kernel(Geometry G, LayerIO
         keys = skeys;
     }
     __syncthreads();
-    block_topk(keys, nwords, n, G.extras, jb, sm);
+    block_topk(keys, n, G.extras, jb, sm);
     // A thread takes a word of winner bits and loads the 32 positions behind it
     // at once (independent 16-byte loads, not one L2 round trip per winner).
     const int32_t* jp = sc.jpos + (size_t)s * G.jstride;
@@ -1203,21 +1243,21 @@ __global__ void __launch_bounds__(256) gather_kernel(Geometry G, LayerIO io, Slo
 }  // namespace
 
 size_t select_smem_bytes(const Geometry& g) {
-    const size_t head = ((size_t)4 * g.words + (keys_in_smem(g.ML) ? 32 * (size_t)key_stride(g) : 0) + 3) & ~(size_t)3;
+    const size_t head = ((size_t)4 * g.words + (keys_in_smem(g.ML) ? key_row_words(g) : 0) + 3) & ~(size_t)3;
     return sizeof(uint32_t) * (head + (scores_in_smem(g.ML) ? 2 * (size_t)g.ML : 0));
 }
 
 size_t heads_smem_bytes(const Geometry& g) {
-    return sizeof(uint32_t) * ((size_t)g.words + (keys_in_smem(g.ML) ? 32 * (size_t)key_stride(g) : 0));
+    return sizeof(uint32_t) * ((((size_t)g.words + 3) & ~(size_t)3) + (keys_in_smem(g.ML) ? key_row_words(g) : 0));
 }
 
 cudaError_t configure_select() {
-    const int need = (int)(sizeof(uint32_t) * (kSmemKeys / 32 + 32 * ((kSmemKeys / 32) | 1)));
+    const int need = (int)(sizeof(uint32_t) * (kSmemKeys / 32 + kSmemKeys));   // bits + one key row
     // The select kernel also keeps the preserved bits and caches P and I rows
     // up to kSmemScores positions.
     const int need_sel_keys = need + (int)(sizeof(uint32_t) * (3 * (kSmemKeys / 32) + 4));
     const int need_sel_scores =
-        (int)(sizeof(uint32_t) * (4 * (kSmemScores / 32) + 32 * ((kSmemScores / 32) | 1) + 2 * kSmemScores + 64));
+        (int)(sizeof(uint32_t) * (4 * (kSmemScores / 32) + kSmemScores + 2 * kSmemScores + 64));
     const int need_sel = need_sel_keys > need_sel_scores ? need_sel_keys : need_sel_scores;
     cudaError_t e = cudaFuncSetAttribute(heads_topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, need);
     if (e == cudaSuccess)

@@ -42,6 +42,8 @@ constexpr int kTopkCap = 2048;                 // keys a compacted candidate lis
 static_assert(kTopkKPL == 16, "two lanes share a bits word");
 static_assert(kTopkCap % kTopkThreads == 0, "the compacted list is split evenly over the select threads");
 constexpr int kTopkFew = 32;                   // a threshold bucket this small is ranked directly
+constexpr int kTopkSampleK = 4;                // sampled threshold for k <= kTopkCap / kTopkSampleK
+constexpr int kTopkSampleN = 32;               // and k <= n / kTopkSampleN (measured: slower for larger k / n)
 
 struct TopkShared {
     int wcnt[2][kTopkWarps][16];   // per-warp digit counts, double-buffered across passes
@@ -196,8 +198,170 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
         // the keys are in registers, so that ureg is indexed statically).
         const int nsi = NS > 0 ? NS : seg1 - seg0;
 
-        // Bits shared by every eligible key.
-        {
+        int cnt = 0x7fffffff;   // keys matching the prefix (unknown before the first pass)
+        int mlist = -1;         // length of the compacted list, -1 while counting all keys
+        if (tid == 0) sm.fcount = 0;   // read only after the next barrier
+        // Sampled threshold, when k is small against the row and every warp holds
+        // a segment (taken with at most 1/32 of the row selected): T, the lower edge of the 8-bit bin of two sample keys per
+        // lane in which the sample's count from the top reaches about twice its
+        // share of k; one compare sweep counts the keys >= T and, when there are
+        // k to kTopkCap of them, a second one compacts them (in position order)
+        // into the list, whose digit passes then finish the selection.  Exact:
+        // the list holds every key >= T and at least k keys.  Otherwise (too few
+        // or too many) the full sweeps below run as if nothing happened.
+        bool listed = false;
+        uint32_t gor = 0u, gand = 0xffffffffu;
+        if (kTopkSampleK * k <= kTopkCap && kTopkSampleN * k <= n && nseg >= kTopkWarps) {
+            int* hist = reinterpret_cast<int*>(sm.ckey);   // 256 bins; the list overwrites it later
+            if (tid < 256) hist[tid] = 0;
+            uint32_t s0, s1;   // this lane's samples: its first key in its first two segments (or key 8)
+            {
+                const Keys16 kv = seg_keys(0, seg0);
+                s0 = kv.v[0];
+                s1 = kv.v[8];
+                if constexpr (NS >= 2) {
+                    if (seg0 + 1 < seg1) s1 = ureg[kTopkKPL];
+                }
+            }
+            uint32_t sor = s0 | s1, sand = (s0 != 0u ? s0 : 0xffffffffu) & (s1 != 0u ? s1 : 0xffffffffu);
+            const int se = (s0 != 0u ? 1 : 0) + (s1 != 0u ? 1 : 0);
+            const int wse = __reduce_add_sync(0xffffffffu, se);
+            sor = __reduce_or_sync(0xffffffffu, sor);
+            sand = __reduce_and_sync(0xffffffffu, sand);
+            if (lane == 0) {
+                sm.wor[warp] = sor;
+                sm.wand[warp] = sand;
+                sm.weq[warp] = wse;
+            }
+            topk_bar();
+            uint32_t qor = 0u, qand = 0xffffffffu;
+            int S = 0;
+#pragma unroll
+            for (int x = 0; x < kTopkWarps; ++x) {
+                qor |= sm.wor[x];
+                qand &= sm.wand[x];
+                S += sm.weq[x];
+            }
+            // Bins: the 8 bits below the sample's highest differing bit (its
+            // common bits above fixed); all sample keys equal: T is that key.
+            const uint32_t qdiff = qor ^ qand;
+            const int qhb = qdiff ? 31 - __clz(qdiff) : 0;
+            const int qsh = max(qhb - 7, 0);
+            if (qdiff) {
+                if (s0 != 0u) atomicAdd(&hist[(s0 >> qsh) & 255u], 1);
+                if (s1 != 0u) atomicAdd(&hist[(s1 >> qsh) & 255u], 1);
+            }
+            topk_bar();
+            uint32_t T = qand;
+            if (qdiff) {
+                // Lane l holds bins 255 - 8 l .. 248 - 8 l (from the top); the bin in
+                // which the count from the top reaches ks.
+                const int ks = min(S, (2 * k * S + n - 1) / n + 2);
+                int c8[8], csum = 0;
+#pragma unroll
+                for (int b = 0; b < 8; ++b) {
+                    c8[b] = hist[255 - 8 * lane - b];
+                    csum += c8[b];
+                }
+                int incl = csum;
+#pragma unroll
+                for (int o = 1; o < 32; o <<= 1) {
+                    const int y = __shfl_up_sync(0xffffffffu, incl, o);
+                    if (lane >= o) incl += y;
+                }
+                const unsigned hit = __ballot_sync(0xffffffffu, incl >= ks);
+                const int hl = hit ? __ffs(hit) - 1 : 31;
+                int run = __shfl_sync(0xffffffffu, incl - csum, hl);
+                int bin = 248 - 8 * hl;
+#pragma unroll
+                for (int b = 0; b < 8; ++b) {
+                    const int cb = __shfl_sync(0xffffffffu, c8[b], hl);
+                    if (run < ks) {
+                        run += cb;
+                        bin = 255 - 8 * hl - b;
+                    }
+                }
+                const uint32_t above = qhb >= 31 ? 0u : ~((2u << qhb) - 1u);
+                T = (qand & above) | ((uint32_t)bin << qsh);
+            }
+            // Count the keys >= T (T > 0: eligible keys only).
+            if (T != 0u) {
+                int c = 0;
+#pragma unroll
+                for (int si = 0; si < nsi; ++si) {
+                    const int sg = seg0 + si;
+                    if (sg >= seg1) break;
+                    const Keys16 kv = seg_keys(si, sg);
+#pragma unroll
+                    for (int j = 0; j < kTopkKPL; ++j) c += kv.v[j] >= T ? 1 : 0;
+                }
+                c = __reduce_add_sync(0xffffffffu, c);
+                if (lane == 0) sm.wcnt[0][warp][0] = c;
+            }
+            topk_bar();
+            int total = 0, off = 0;
+            if (T != 0u) {
+#pragma unroll
+                for (int x = 0; x < kTopkWarps; ++x) {
+                    const int cx = sm.wcnt[0][x][0];
+                    total += cx;
+                    off += x < warp ? cx : 0;
+                }
+            }
+            if (T != 0u && total >= k && total <= kTopkCap) {
+                // Compact them in position order: warp w after warps 0..w-1, a lane
+                // after its segment's lower lanes and the warp's earlier segments.
+#pragma unroll
+                for (int si = 0; si < nsi; ++si) {
+                    const int sg = seg0 + si;
+                    if (sg >= seg1) break;
+                    const Keys16 kv = seg_keys(si, sg);
+                    int mc = 0;
+#pragma unroll
+                    for (int j = 0; j < kTopkKPL; ++j) mc += kv.v[j] >= T ? 1 : 0;
+                    int incl = mc;
+#pragma unroll
+                    for (int o = 1; o < 32; o <<= 1) {
+                        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+                        if (lane >= o) incl += y;
+                    }
+                    int at = off + incl - mc;
+                    const int pos0 = sg * kTopkSeg + lane * kTopkKPL;
+#pragma unroll
+                    for (int j = 0; j < kTopkKPL; ++j) {
+                        if (kv.v[j] >= T && at < kTopkCap) {
+                            sm.ckey[at] = kv.v[j];
+                            sm.cpos[at] = pos0 + j;
+                            ++at;
+                        }
+                    }
+                    off += __shfl_sync(0xffffffffu, incl, 31);
+                }
+                topk_bar();
+                // The list's own shared bits start the digit passes.
+                uint32_t kor = 0u, kand = 0xffffffffu;
+#pragma unroll
+                for (int r = 0; r < kTopkCap / kTopkThreads; ++r) {
+                    const int j = tid + r * kTopkThreads;
+                    if (j < total) {
+                        kor |= sm.ckey[j];
+                        kand &= sm.ckey[j];
+                    }
+                }
+                kor = __reduce_or_sync(0xffffffffu, kor);
+                kand = __reduce_and_sync(0xffffffffu, kand);
+                if (lane == 0) {
+                    sm.wor[warp] = kor;
+                    sm.wand[warp] = kand;
+                }
+                topk_bar();
+                mlist = total;
+                cnt = total;
+                listed = true;
+            }
+        }
+        if (!listed) {
+            // Bits shared by every eligible key.
             uint32_t kor = 0u, kand = 0xffffffffu;
 #pragma unroll
             for (int si = 0; si < nsi; ++si) {
@@ -217,10 +381,8 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
                 sm.wor[warp] = kor;
                 sm.wand[warp] = kand;
             }
-            if (tid == 0) sm.fcount = 0;
+            topk_bar();
         }
-        topk_bar();
-        uint32_t gor = 0u, gand = 0xffffffffu;
 #pragma unroll
         for (int x = 0; x < kTopkWarps; ++x) {
             gor |= sm.wor[x];
@@ -230,8 +392,6 @@ __device__ __forceinline__ void block_topk_impl(const uint32_t* __restrict__ key
 
         uint32_t prefix = 0u, mask = 0u;
         int kk = k;
-        int cnt = 0x7fffffff;   // keys matching the prefix (unknown before the first pass)
-        int mlist = -1;         // length of the compacted list, -1 while counting all keys
         bool whole_bin = false;
         int lo = 32;            // lowest bit resolved so far
         for (int pass = 0;; ++pass) {

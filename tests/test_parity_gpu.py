@@ -104,6 +104,27 @@ def test_uniform_keys_tie_to_lowest_positions():
     sel.close()
 
 
+def test_uniform_keys_long_row_tie_to_lowest_positions():
+    """K = 0 on a 20000-position row: every candidate scores the same, so the
+    radix select's sampled threshold finds all keys above it (far more than the
+    list holds) and falls back to the full digit passes; the preserved tokens
+    and the fill must still be the lowest positions."""
+    L, budget = 20000, 64
+    wl = synth.small_workload(seqlens=(L,), budget=budget, layers=1)
+    params = kvec.params_from_workload(wl)
+    sel = kvec.KvecSelector(params)
+    x = synth.make_layer(wl, 0)
+    k = torch.zeros_like(x["k"]).cuda()
+    cu = torch.tensor(wl.cu_seqlens, dtype=torch.int32)
+    st = sel.new_state(1)
+    idx, _, _ = sel.select_layer(cu, cu.cuda(), x["q_obs"].cuda(), k, x["v"].cuda(), st, budget)
+    torch.cuda.synchronize()
+    expect = list(range(budget - wl.window)) + list(range(L - wl.window, L))
+    for h in range(wl.num_kv_heads):
+        assert idx[0, h].cpu().tolist() == expect
+    sel.close()
+
+
 @pytest.mark.parametrize("plateau,budget", [((4500, 5800), 1024), ((4800, 12000), 1024), ((5100, 5140), 64)])
 def test_equal_keys_across_row_slices_tie_to_lowest_positions(plateau, budget):
     """Positions [a, b) of a 20000-position row share one key vector that every

@@ -65,7 +65,7 @@ struct Scratch {
     float2* rowstat;      // [max_batch][Hkv][R]    (row max in log2 units, softmax denominator), for inspection
     uint32_t* keys;       // [max_batch][Hkv][ML]   radix-select keys of the heads kernel
     uint32_t* keys_sel;   // [max_batch][Hkv][ML]   radix-select keys of the select kernel
-    uint32_t* jkeys;      // [max_batch][jstride]   adaptive fill: the heads' joint candidates' keys, transposed
+    uint32_t* jkeys;      // [max_batch][jstride]   adaptive fill: the heads' joint candidates' keys (a key row)
     int32_t* jpos;        // [max_batch][jstride]   their positions (candidate i belongs to head i / jpool)
     uint32_t* jbits;      // [max_batch][jstride / 32] winners of the joint ranking, one bit per candidate
     uint8_t* nbuf;        // [max_batch][nlen]      second copy of n_t (the coverage counts alternate)

@@ -1456,7 +1456,7 @@ cudaError_t launch_finalize(const Geometry& g, const LayerIO& io, const Scratch&
 
 cudaError_t launch_ada(const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl, cudaStream_t st,
                        int priority, int ncall) {
-    // The staged keys: 32 * ceil(n / 32) words, the transposed layout's extent.
+    // The staged keys: 32 * ceil(n / 32) words, the extent of a key row of n keys.
     const size_t smem = ada_keys_in_smem(g) ? sizeof(uint32_t) * 32 * (((size_t)g.Hkv * g.jpool + 31) / 32) : 0;
     return launch_prio(ada_kernel, dim3(g.batch), dim3(kSelectThreads), smem, st, priority, /*programmatic=*/true, g,
                        io, sc, sl, ncall);

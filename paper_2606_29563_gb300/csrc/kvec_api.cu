@@ -374,7 +374,7 @@ kvec_status launch_pipeline(kvec_handle* h, const Geometry& G, const LayerIO* io
         if (se != cudaSuccess) return cuda_fail(se, "score kernel tensor maps");
         // Partials buffer reuse (window stream).
         if (l >= kScoreBufs) {
-            const bool early = !io.lse && plan.grid + window_grid_size(plan, G) <= h->num_sms;
+            const bool early = !io.lse && plan.grid + window_grid_size(plan, G, false) <= h->num_sms;
             KV_CHECK(cudaStreamWaitEvent(h->s_score, early ? h->ev_rs[l - kScoreBufs] : h->ev_win[l - kScoreBufs], 0));
         }
         // The score grid of layer l > 0 is a programmatic dependent of layer

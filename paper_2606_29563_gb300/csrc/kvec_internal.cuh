@@ -151,8 +151,9 @@ cudaError_t launch_rowstat_lse(const Geometry& g, const LayerIO& io, const Scrat
                                bool programmatic);
 cudaError_t launch_window(const ScorePlan& sp, const Geometry& g, const LayerIO& io, const Scratch& sc, const Slot& sl,
                           cudaStream_t st, bool after_own_launch);
-// CTAs of the grid launch_window starts for this layer (0 without candidates).
-int window_grid_size(const ScorePlan& sp, const Geometry& g);
+// CTAs of the grid launch_window starts for this layer (0 without candidates);
+// lse: the layer comes with the caller's log-sum-exp (io.lse).
+int window_grid_size(const ScorePlan& sp, const Geometry& g, bool lse);
 // Launches kernel<<<grid, block, smem, st>>> with a scheduling priority (lower
 // numbers first; the range comes from cudaDeviceGetStreamPriorityRange) and,
 // with `programmatic`, as a programmatic dependent of the stream's previous

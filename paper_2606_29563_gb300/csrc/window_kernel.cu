@@ -869,6 +869,14 @@ bool tile_variant_fits(const Geometry& g) {
     return (nacc - 1) * Npad + maxcol <= 512;
 }
 
+// Candidate tiles per unit of the tile-owning variant: one TMEM accumulator and
+// epilogue group each (nacc * Npad <= 512 columns).  With the caller's
+// log-sum-exp no score grid runs beside the window grids, and units of three
+// tiles (more units, a shorter tail) were faster than four there (ragged batch
+// of 8: 2.09 -> 1.90 ms per step), while beside the score grids they were
+// slower (3.02 -> 3.06 ms); two tiles were slower in both.
+int tile_unit_tiles(const Geometry& g, bool lse) { return npad_of(g.R) <= 128 ? (lse ? 3 : 4) : 2; }
+
 // Units of the tile-owning variant: groups of T candidate tiles per sequence and head group.
 int tile_units_of(const Geometry& g, const int* cu_host, int T) {
     int units = 0;
@@ -888,7 +896,7 @@ cudaError_t launch_window_tiles(const ScorePlan& sp, const Geometry& g, const La
     a.sl = sl;
     a.cu = io.cu;
     a.Npad = npad_of(g.R);
-    a.nacc = a.Npad <= 128 ? 4 : 2;   // nacc * Npad <= 512 TMEM columns
+    a.nacc = tile_unit_tiles(g, io.lse != nullptr);
     a.kst = tile_kst_for(a.Npad);
     a.units = tile_units_of(g, g.cu_host, a.nacc);
     a.fault = test_fault() == 1 ? 1 : 0;
@@ -916,10 +924,10 @@ cudaError_t launch_window_tiles(const ScorePlan& sp, const Geometry& g, const La
 
 }  // namespace
 
-int window_grid_size(const ScorePlan& sp, const Geometry& g) {
+int window_grid_size(const ScorePlan& sp, const Geometry& g, bool lse) {
     if (g.win_tiles == 0) return 0;
     const int usable = sp.num_sms > 2 * kWinReserveSms ? sp.num_sms - kWinReserveSms : sp.num_sms;
-    if (tile_variant_fits(g) && tile_units_of(g, g.cu_host, npad_of(g.R) <= 128 ? 4 : 2) >= usable) return usable;
+    if (tile_variant_fits(g) && tile_units_of(g, g.cu_host, tile_unit_tiles(g, lse)) >= usable) return usable;
     return units_of(g) < usable ? units_of(g) : usable;
 }
 
@@ -930,7 +938,7 @@ cudaError_t launch_window(const ScorePlan& sp, const Geometry& g, const LayerIO&
     // usable SM one (it has T times fewer units than the per-tile kernel, whose
     // CTAs finish sooner when there are few tiles).
     if (tile_variant_fits(g)) {
-        const int T = npad_of(g.R) <= 128 ? 4 : 2;
+        const int T = tile_unit_tiles(g, io.lse != nullptr);
         const int usable = sp.num_sms > 2 * kWinReserveSms ? sp.num_sms - kWinReserveSms : sp.num_sms;
         if (tile_units_of(g, g.cu_host, T) >= usable) return launch_window_tiles(sp, g, io, sc, sl, st, after_own_launch);
     }

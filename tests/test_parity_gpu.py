@@ -245,6 +245,12 @@ def test_lse_input_llama8b_l8192_b512_first_layers():
     _assert_parity(synth.WORKLOADS["llama8b_l8192_b512"], layers=2, with_lse=True)
 
 
+def test_lse_input_llama8b_ragged8_b256_first_layers():
+    # The ragged batch of 8 runs the tile-owning window kernel, which takes units
+    # of three candidate tiles when the caller supplies the log-sum-exp.
+    _assert_parity(synth.WORKLOADS["llama8b_ragged8_b256"], layers=2, with_lse=True)
+
+
 def test_lse_multi_layer_call_matches_layer_by_layer():
     wl = synth.small_workload(seqlens=(1100, 700), layers=3, budget=96)
     cpu_layers = synth.make_layers(wl, 3)

@@ -101,6 +101,10 @@ def test_full_call_llama8b_l8192_b512_with_caller_lse():
     _check_full_call(synth.WORKLOADS["llama8b_l8192_b512"], with_lse=True)
 
 
+def test_full_call_llama8b_ragged8_b256_with_caller_lse():
+    _check_full_call(synth.WORKLOADS["llama8b_ragged8_b256"], with_lse=True)
+
+
 def test_full_call_llama8b_l8192_b512_all_positions():
     _check_full_call(synth.WORKLOADS["llama8b_l8192_b512"].replace(all_positions=1))
 

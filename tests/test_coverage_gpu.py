@@ -1,7 +1,6 @@
 """Coverage read from the GPU's coverage state (paper_2606_29563_gb300.coverage)
 against the fp64 oracle's count of covered tokens, one layer per method and
 budget so that both sides start from the same state."""
-import numpy as np
 import pytest
 import torch
 

@@ -31,11 +31,16 @@ def build(force: bool = False) -> str:
     if fresh and not force:
         return _LIB_PATH
     tmp = _LIB_PATH + f".tmp{os.getpid()}"
-    cmd = ["gcc", "-O2", "-std=c99", "-fPIC", "-shared", "-fopenmp", "-ffp-contract=off",
-           "-o", tmp, src, "-lm"]
-    subprocess.run(cmd, check=True)
+    compile_source(src, tmp)
     os.replace(tmp, _LIB_PATH)
     return _LIB_PATH
+
+
+def compile_source(src: str, out: str) -> None:
+    """gcc -O2 (OpenMP, no FMA contraction) of an oracle source into a shared library."""
+    cmd = ["gcc", "-O2", "-std=c99", "-fPIC", "-shared", "-fopenmp", "-ffp-contract=off",
+           "-I", _HERE, "-o", out, src, "-lm"]
+    subprocess.run(cmd, check=True)
 
 
 class _Params(ctypes.Structure):
@@ -66,8 +71,10 @@ def _load():
     global _lib
     with _lock:
         if _lib is None:
-            build()
-            lib = ctypes.CDLL(_LIB_PATH)
+            # KVEC_ORACLE_LIB: another build of kvec_oracle.c to load instead (the
+            # test that plants mistakes in copies of the oracle runs the pins on them).
+            path = os.environ.get("KVEC_ORACLE_LIB") or build()
+            lib = ctypes.CDLL(path)
             lib.kvo_state_bytes.restype = ctypes.c_size_t
             lib.kvo_state_bytes.argtypes = [ctypes.c_int]
             lib.kvo_num_threads.restype = ctypes.c_int

@@ -141,6 +141,47 @@ def test_noalloc_refuses_oversize_calls_before_cuda(lib):
     assert "scratch" in str(e.value)
 
 
+@pytest.mark.parametrize("case,needle", [
+    ("empty_batch", "batch 0"), ("batch_over_max", "batch 3"), ("cu_not_from_zero", "cu_seqlens[0]"),
+    ("sequence_shorter_than_window", "length 31"), ("sequence_over_max_seqlen", "length 4097"),
+    ("budget_below_window", "budget 31"), ("zero_budget", "budget 0"), ("null_k", "NULL"),
+    ("misaligned_k", "aligned")])
+def test_noalloc_validates_calls_before_cuda(lib, case, needle):
+    # Degenerate and malformed calls: every one is refused by the host checks,
+    # before any CUDA call (the placeholder pointers are never dereferenced).
+    p = kvec.make_params(num_q_heads=32, num_kv_heads=8, max_batch=2, max_seqlen=4096)
+    batch, budget, lens, first = 2, 256, [1000, 2000], 0
+    fake = {n: 256 for n in ("q", "k", "v", "state", "out_idx", "out_k", "out_v")}
+    if case == "empty_batch":
+        batch = 0
+    elif case == "batch_over_max":
+        batch, lens = 3, [1000, 2000, 500]
+    elif case == "cu_not_from_zero":
+        first = 1
+    elif case == "sequence_shorter_than_window":
+        lens = [1000, p.window - 1]
+    elif case == "sequence_over_max_seqlen":
+        lens = [4097, 100]
+    elif case == "budget_below_window":
+        budget = p.window - 1
+    elif case == "zero_budget":
+        budget = 0
+    elif case == "null_k":
+        fake["k"] = 0
+    elif case == "misaligned_k":
+        fake["k"] = 256 + 2
+    cu_vals = [first]
+    for L in lens:
+        cu_vals.append(cu_vals[-1] + L)
+    cu = (ctypes.c_int32 * len(cu_vals))(*cu_vals)
+    with pytest.raises(kvec.KvecError) as e:
+        kvec.kvec_select_layer_noalloc(p, batch, ctypes.addressof(cu), ctypes.addressof(cu), fake["q"], fake["k"],
+                                       fake["v"], fake["state"], budget, fake["out_idx"], fake["out_k"],
+                                       fake["out_v"], None)
+    assert e.value.status == kvec.KVEC_ERR_INVALID_ARG
+    assert needle in str(e.value), str(e.value)
+
+
 @pytest.mark.parametrize("struct", [kvec.kvec_params, kvec.kvec_debug_view])
 def test_binding_structs_match_the_header_layout(tmp_path, struct):
     """Every field of the ctypes mirror sits at the offset (and the struct has the

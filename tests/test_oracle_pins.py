@@ -576,3 +576,56 @@ def test_adaptive_fill_budget_bookkeeping():
                 kept = set(r["out_idx"][b, h][r["out_idx"][b, h] >= 0].tolist())
                 assert set(range(L - wl.window, L)) <= kept
                 assert set(np.flatnonzero(r["pres"][b, h, :L - wl.window]).tolist()) <= kept
+
+
+def _random_case(i):
+    """A random small configuration (shapes, windows, pooling, hyper-parameters and
+    the variants), seeded by i; valid for the oracle's parameter checks."""
+    rng = np.random.default_rng(9000 + i)
+    Hkv = int(rng.choice([1, 2, 4]))
+    g = int(rng.choice([1, 2, 3]))
+    w = int(rng.integers(2, 9))
+    O = int(rng.integers(1, w + 1))
+    Oe = int(rng.integers(O, w + 1))
+    T = int(rng.integers(w + 1, 25))
+    all_positions = int(rng.random() < 0.3)
+    B = int(rng.integers(1 if all_positions else w, T + 2))   # B >= T (keep all) now and then
+    return dict(seed=9000 + i, T=T, Hq=g * Hkv, Hkv=Hkv, d=int(rng.choice([4, 8])), w=w, O=O, Oe=Oe,
+                pool=int(rng.choice([1, 3, 5])), delta=int(rng.integers(0, Hkv + 1)),
+                lam=float(rng.choice([0.0, 0.5, 1.0, 2.0])), beta=float(rng.choice([0.0, 0.25, 0.5, 1.0])), B=B,
+                pool_mode=int(rng.random() < 0.3), head_criterion=int(rng.random() < 0.3),
+                all_positions=all_positions)
+
+
+@pytest.mark.parametrize("i", range(60))
+def test_oracle_matches_bruteforce_on_random_configurations(i):
+    """Sixty seeded random configurations (beyond the hand-picked cases above),
+    two layers each with the state carried: every score row, sigma, the chosen
+    heads, P', the preserved set, the kept indices and n_t equal the brute force."""
+    c = _random_case(i)
+    T, Hq, Hkv, d, w, B = c["T"], c["Hq"], c["Hkv"], c["d"], c["w"], c["B"]
+    variant = dict(pool_mode=c["pool_mode"], head_criterion=c["head_criterion"], all_positions=c["all_positions"])
+    params = oracle.OracleParams(num_q_heads=Hq, num_kv_heads=Hkv, head_dim=d, window=w, obs_window=c["O"],
+                                 ext_window=c["Oe"], pool_kernel=c["pool"], num_ext_heads=c["delta"],
+                                 lam=c["lam"], beta=c["beta"], **variant)
+    state = oracle.new_state(1, T)
+    n_bf = np.zeros(T, np.int64)
+    Lc = T if c["all_positions"] else T - w
+    for layer in range(2):
+        x = synth.tiny_full_inputs(c["seed"] * 10 + layer, T, Hq, Hkv, d)
+        q_obs = x["q_full"][T - w:].reshape(1, w, Hq, d)
+        r = _run_oracle(params, q_obs, x["k"], x["v"], state, B)
+        bf = bf_select(_f64(x["q_full"]), _f64(x["k"]), num_kv_heads=Hkv, window=w, obs_window=c["O"],
+                       ext_window=c["Oe"], pool_kernel=c["pool"], num_ext_heads=c["delta"], lam=c["lam"],
+                       beta=c["beta"], budget=B, n_counts=n_bf, layers_done=layer, **variant)
+        np.testing.assert_allclose(r["P_O"][0, :, :Lc], bf["P_O"], rtol=1e-12, atol=1e-15)
+        np.testing.assert_allclose(r["P_Oext"][0, :, :Lc], bf["P_Oext"], rtol=1e-12, atol=1e-15)
+        np.testing.assert_allclose(r["I"][0, :Lc], bf["I"], rtol=1e-12, atol=1e-15)
+        np.testing.assert_allclose(r["sigma"][0], bf["sigma"], rtol=1e-9, atol=1e-15)
+        assert (r["htop"][0].astype(bool) == bf["htop"]).all(), c
+        np.testing.assert_allclose(r["Pprime"][0, :, :Lc], bf["Pprime"], rtol=1e-12, atol=1e-15)
+        if T > B:
+            assert (r["pres"][0, :, :Lc].astype(bool) == bf["pres"]).all(), c
+        assert (r["out_idx"][0] == bf["out_idx"]).all(), c
+        n_bf = bf["n"]
+        assert (oracle.state_fields(state, T)["n"][0].astype(np.int64) == n_bf).all(), c

@@ -629,3 +629,31 @@ def test_oracle_matches_bruteforce_on_random_configurations(i):
         assert (r["out_idx"][0] == bf["out_idx"]).all(), c
         n_bf = bf["n"]
         assert (oracle.state_fields(state, T)["n"][0].astype(np.int64) == n_bf).all(), c
+
+
+@pytest.mark.parametrize("i", range(30))
+def test_adaptive_fill_matches_bruteforce_on_random_configurations(i):
+    """The head-wise adaptive fill on thirty seeded random configurations (random
+    floor α included), two layers each: kept indices, capacity and n_t equal the
+    brute force."""
+    c = _random_case(1000 + i)
+    a = float(np.random.default_rng(7000 + i).choice([0.0, 0.2, 0.5, 0.8, 1.0]))
+    T, Hq, Hkv, d, w, B = c["T"], c["Hq"], c["Hkv"], c["d"], c["w"], c["B"]
+    variant = dict(pool_mode=c["pool_mode"], head_criterion=c["head_criterion"], all_positions=c["all_positions"])
+    params = oracle.OracleParams(num_q_heads=Hq, num_kv_heads=Hkv, head_dim=d, window=w, obs_window=c["O"],
+                                 ext_window=c["Oe"], pool_kernel=c["pool"], num_ext_heads=c["delta"],
+                                 lam=c["lam"], beta=c["beta"], head_budget=1, ada_floor=a, **variant)
+    state = oracle.new_state(1, T)
+    n_bf = np.zeros(T, np.int64)
+    for layer in range(2):
+        x = synth.tiny_full_inputs(c["seed"] * 10 + layer, T, Hq, Hkv, d)
+        q_obs = x["q_full"][T - w:].reshape(1, w, Hq, d)
+        r = _run_oracle(params, q_obs, x["k"], x["v"], state, B)
+        bf = bf_select(_f64(x["q_full"]), _f64(x["k"]), num_kv_heads=Hkv, window=w, obs_window=c["O"],
+                       ext_window=c["Oe"], pool_kernel=c["pool"], num_ext_heads=c["delta"], lam=c["lam"],
+                       beta=c["beta"], budget=B, n_counts=n_bf, layers_done=layer, head_budget=1, ada_floor=a,
+                       **variant)
+        assert r["out_idx"].shape[2] == bf["out_idx"].shape[1] == oracle.head_capacity(params, B)
+        assert (r["out_idx"][0] == bf["out_idx"]).all(), (c, a)
+        n_bf = bf["n"]
+        assert (oracle.state_fields(state, T)["n"][0].astype(np.int64) == n_bf).all(), (c, a)

@@ -446,3 +446,31 @@ def test_adaptive_fill_llama8b_l8192_b512_first_layers():
 
 def test_adaptive_fill_llama8b_ragged8_b256_first_layers():
     _assert_parity(synth.WORKLOADS["llama8b_ragged8_b256"].replace(head_budget=1, ada_floor=0.2), layers=2)
+
+
+def _random_small_workload(i):
+    """A seeded random configuration inside the kernels' limits (d = 128, g*w a
+    multiple of 8 and <= 256, odd pool width <= 15): batch, lengths, heads,
+    windows, pooling, delta, lambda, beta, budget and the variants at random."""
+    rng = np.random.default_rng(5000 + i)
+    Hkv = int(rng.choice([1, 2, 4, 8]))
+    g = int(rng.choice([1, 2, 3, 4, 7, 8]))
+    w = int(rng.choice([8, 16, 24, 32]))
+    O = int(rng.integers(1, w + 1))
+    Oe = int(rng.integers(O, w + 1))
+    batch = int(rng.integers(1, 4))
+    seqlens = tuple(int(x) for x in rng.integers(w, 1201, size=batch))
+    all_positions = int(rng.random() < 0.25)
+    head_budget = int(rng.random() < 0.25)
+    return synth.small_workload(
+        name=f"random{i}", seqlens=seqlens, num_q_heads=g * Hkv, num_kv_heads=Hkv, window=w, obs_window=O,
+        ext_window=Oe, pool_kernel=int(rng.choice([1, 3, 7, 15])), num_ext_heads=int(rng.integers(0, Hkv + 1)),
+        lam=float(rng.choice([0.0, 1.0, 2.0])), beta=float(rng.choice([0.0, 0.25, 0.5])),
+        budget=int(rng.integers(1 if all_positions else w, 301)), layers=2, seed=5000 + i,
+        pool_mode=int(rng.random() < 0.25), head_criterion=int(rng.random() < 0.25), all_positions=all_positions,
+        head_budget=head_budget, ada_floor=float(rng.choice([0.0, 0.2, 0.5])) if head_budget else 1.0)
+
+
+@pytest.mark.parametrize("i", range(16))
+def test_random_small_configurations_match_the_oracle(i):
+    _assert_parity(_random_small_workload(i))

@@ -700,15 +700,17 @@ def run_reference(args, wl):
 
 def main(argv=None):
     ap = argparse.ArgumentParser()
-    ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=1000)
-    ap.add_argument("--warmup", type=int, default=5)
-    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
-    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
-    ap.add_argument("--budget", type=int, default=None)
+    ap.add_argument("--gpus", type=int, default=1, help="GPUs of one node (N > 1: launched by torch.distributed.run, one replica per GPU)")
+    ap.add_argument("--steps", type=int, default=1000, help="timed steps (one step: every layer of one batch)")
+    ap.add_argument("--warmup", type=int, default=5, help="untimed steps before the timed ones")
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours",
+                    help="reference: time the fp64 oracle on the host cores instead of the CUDA path")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, help="one of synth.WORKLOADS")
+    ap.add_argument("--budget", type=int, default=None, help="tokens kept per KV head (default: the workload's)")
     ap.add_argument("--layers", type=int, default=None, help="run only the first N layers (not a bench line)")
-    ap.add_argument("--no-e2e", dest="e2e", action="store_false")
-    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", dest="e2e", action="store_false",
+                    help="skip the end-to-end measurement with inputs copied from host memory")
+    ap.add_argument("--no-cpu-baseline", action="store_true", help="skip timing the fp64 oracle on a sample")
     ap.add_argument("--coverage-sweep", action="store_true",
                     help="print the token coverage of K-VEC and SnapKV at eviction rates 0.25-0.9 and exit")
     ap.add_argument("--no-decode", dest="decode", action="store_false",
